@@ -1,0 +1,135 @@
+"""Pure-numpy decoder of the library's storage format (test helper).
+
+Written from the format description only; it turns packed activation streams,
+packed weight buffers and MMA planes back into natural-order codes and scales
+so that tests can compare them with the oracle and check the layouts by eye.
+"""
+import numpy as np
+
+
+def slot_blocks(bits):
+    bits = np.asarray(bits)
+    order = [np.flatnonzero(bits == w) for w in (4, 6, 8)]
+    return np.concatenate(order).astype(np.int64), tuple(int(o.size) for o in order)
+
+
+def align256(v):
+    return (v + 255) // 256 * 256
+
+
+def sext4(n):
+    n = n.astype(np.int16)
+    return np.where(n >= 8, n - 16, n).astype(np.int8)
+
+
+def decode_act(bits, pcodes, pscales):
+    """row-major grouped stream -> (scales [R,nb], codes [R,K]) in natural order."""
+    sb, (n4, n6, n8) = slot_blocks(bits)
+    R = pcodes.shape[0]
+    nb = len(bits)
+    K = 32 * nb
+    codes = np.zeros((R, K), np.int8)
+    scales = np.zeros((R, nb), np.uint8)
+    for s, kb in enumerate(sb):
+        scales[:, kb] = pscales[:, s]
+        if s < n4:
+            byts = pcodes[:, 16 * s:16 * s + 16]
+            codes[:, 32 * kb + 0:32 * kb + 32:2] = sext4(byts & 0xF)
+            codes[:, 32 * kb + 1:32 * kb + 32:2] = sext4(byts >> 4)
+        else:
+            off = 16 * n4 + 32 * (s - n4)
+            codes[:, 32 * kb:32 * kb + 32] = pcodes[:, off:off + 32].view(np.int8)
+    return scales, codes
+
+
+def weight_offsets(N, bits):
+    sb, (n4, n6, n8) = slot_blocks(bits)
+    n68 = n6 + n8
+    T = (N + 15) // 16
+    o8 = align256(T * n4 * 256)
+    os_ = align256(o8 + T * n68 * 512)
+    compact = align256(os_ + 16 * T * len(bits))
+    return o8, os_, compact
+
+
+def decode_weight(N, bits, buf):
+    """compact weight buffer -> (scales [N,nb], codes [N,K]) in natural order."""
+    sb, (n4, n6, n8) = slot_blocks(bits)
+    n68 = n6 + n8
+    nb = len(bits)
+    K = 32 * nb
+    T = (N + 15) // 16
+    o8, os_, _ = weight_offsets(N, bits)
+    codes = np.zeros((16 * T, K), np.int8)
+    # lane l = 4g + q; row within tile = g + 8h
+    lanes = np.arange(32)
+    g, q = lanes // 4, lanes % 4
+    for s, kb in enumerate(sb):
+        for t in range(T):
+            if s < n4:
+                ch = buf[(t * n4 + s) * 256:(t * n4 + s + 1) * 256].reshape(32, 2, 4)  # lane, h, j
+                for h in range(2):
+                    for j in range(4):
+                        rows = 16 * t + g + 8 * h
+                        byte = ch[:, h, j]
+                        codes[rows, 32 * kb + 4 * q + j] = sext4(byte >> 4)
+                        codes[rows, 32 * kb + 16 + 4 * q + j] = sext4(byte & 0xF)
+            else:
+                base = o8 + (t * n68 + (s - n4)) * 512
+                ch = buf[base:base + 512].reshape(32, 4, 4).view(np.int8)  # lane, reg, j
+                for reg in range(4):
+                    h = reg % 2
+                    e0 = 16 if reg >= 2 else 0
+                    for j in range(4):
+                        codes[16 * t + g + 8 * h, 32 * kb + e0 + 4 * q + j] = ch[:, reg, j]
+    sc = buf[os_:os_ + 16 * T * nb].reshape(16 * T, nb)
+    scales = np.zeros((16 * T, nb), np.uint8)
+    scales[:, sb] = sc
+    return scales[:N], codes[:N]
+
+
+def e4m3_value(code):
+    code = int(code)
+    s = -1.0 if code & 0x80 else 1.0
+    e = (code >> 3) & 0xF
+    f = code & 7
+    if e == 0xF and f == 7:
+        return float("nan")
+    if e == 0:
+        return s * f / 8.0 * 2.0 ** -6
+    return s * (1 + f / 8.0) * 2.0 ** (e - 7)
+
+
+E4M3_TABLE = np.array([e4m3_value(c) for c in range(256)])
+
+
+def decode_planes(bits, planes, sf):
+    """planes [R,Kp] + scale tiles -> (scales [R,nb], codes [R,K]) natural order."""
+    sb, (n4, n6, n8) = slot_blocks(bits)
+    n68 = n6 + n8
+    st4 = (n4 + 3) // 4
+    nst = st4 + (n68 + 1) // 2
+    R = planes.shape[0]
+    nb = len(bits)
+    codes = np.zeros((R, 32 * nb), np.int8)
+    vals = E4M3_TABLE[planes]
+    for s, kb in enumerate(sb):
+        b = int(bits[kb])
+        if s < n4:
+            v = vals[:, 32 * s:32 * s + 32]
+        else:
+            off = 128 * st4 + 64 * (s - n4)
+            v = vals[:, off:off + 32] + vals[:, off + 32:off + 64]
+        codes[:, 32 * kb:32 * kb + 32] = np.rint(v * 2.0 ** (b - 2)).astype(np.int8)
+    # scale tiles: [tau][st][i][w][q] -> row 128 tau + 32 w + i
+    tiles = sf.reshape(-1, nst, 32, 4, 4)
+    scales = np.zeros((R, nb), np.uint8)
+    for s, kb in enumerate(sb):
+        if s < n4:
+            st, qq = s // 4, s % 4
+        else:
+            st, qq = st4 + (s - n4) // 2, (s - n4) % 2
+        col = tiles[:, st, :, :, qq]            # [tau, i, w]
+        rows = col.transpose(0, 2, 1).reshape(-1)  # row = 128 tau + 32 w + i
+        scales[:, kb] = rows[:R]
+    return scales, codes
