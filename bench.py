@@ -1,0 +1,449 @@
+#!/usr/bin/env python
+"""Benchmark of the MXINT mixed-precision linear layer (MXSens) on GB300.
+
+Default workload (LLaMA-3-8B-shaped decode): for M in {1, 4, 16} tokens, the
+seven projections (q, k, v, o: 4096x4096 / 4096x1024; gate, up: 4096x14336;
+down: 14336x4096) of all 32 decoder layers; width map 85/10/5 % (4/6/8 bits)
+per projection, weights N(0, 0.02), activations N(0, 1) with 1 % outlier
+columns x30.  One step = for every (M, layer, projection): quantize the
+activations (A1) and run the MXINT GEMM (A4); weights are packed once (A2).
+The step is captured in a CUDA graph and replayed.  The 4.2 GB of packed
+weights a step streams is far larger than L2, so no flush is needed.
+
+Metric: GB/s of algorithmic traffic (packed weights + bf16 activations read +
+fp32 outputs written) per second, whole job; TOPS (2*M*N*K per second) is
+reported beside it.
+
+--impl reference times the CPU oracle (the paper publishes no kernel to run)
+on a bounded sample of the same workload, on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_17733_gb300 import inputs as I  # noqa: E402
+
+DECODE_MS = (1, 4, 16)
+MAP = (0.85, 0.10, 0.05)
+W_SIGMA = 0.02
+OUTLIER_FRAC, OUTLIER_SCALE = 0.01, 30.0
+SEED = 2607
+SAMPLE_ROWS = 2048
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--layers", type=int, default=32)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------- helpers
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]),
+                "bf16_tflops_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
+                "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def profile_traffic(kernel_file: str, profile_md: str):
+    """DRAM bytes per launch recorded in a committed ncu summary, if it was taken
+    on the current source of the kernel (sha256 of the .cu file)."""
+    import hashlib
+    try:
+        src = open(os.path.join(ROOT, "paper_2607_17733_gb300", "csrc", kernel_file), "rb").read()
+        text = open(os.path.join(ROOT, "profiles", profile_md)).read()
+    except OSError:
+        return None
+    sha = hashlib.sha256(src).hexdigest()[:16]
+    for line in text.splitlines():
+        if line.startswith("traffic_bytes_per_launch:"):
+            parts = line.split()
+            # traffic_bytes_per_launch: <bytes> kernel_sha: <sha>
+            if len(parts) >= 4 and parts[3] == sha:
+                return float(parts[1])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str | None):
+        self.proc = None
+        self.lines = []
+        self.gpu_id = gpu_id
+
+    def start(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50"]
+        if self.gpu_id:
+            cmd += ["-i", self.gpu_id]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.12)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("gloo", rank=rank, world_size=ws)  # harness barriers / max only
+    return ws, rank, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def allreduce_max(v: float, ws: int) -> float:
+    if ws == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --------------------------------------------------------------- CPU oracle sample
+_SAMPLE = None
+
+
+def _oracle_jobs(seed_rank: int = 0):
+    """Layer 0 of the workload for the oracle, the first min(N, 2048) output
+    rows of every projection: weights quantized once (offline packing is not
+    timed), activations for M = 1, 4, 16."""
+    global _SAMPLE
+    if _SAMPLE is None:
+        from oracle import mxo
+        jobs = []
+        for pi, (name, K, N) in enumerate(I.LLAMA3_8B):
+            g = I.rng(SEED, seed_rank, 0, pi)
+            bits = I.width_map(K // 32, *MAP, g)
+            N = min(N, SAMPLE_ROWS)
+            w = I.normal_bf16((N, K), W_SIGMA, g)
+            w_s, w_c = mxo.quantize_bf16(w, bits)
+            del w
+            for M in DECODE_MS:
+                x = I.activations_bf16(M, bits, I.rng(SEED, seed_rank, 1, pi, M), OUTLIER_FRAC,
+                                       outlier_scale=OUTLIER_SCALE)
+                jobs.append((bits, x, w_s, w_c, K, N, M))
+        _SAMPLE = jobs
+    return _SAMPLE
+
+
+def oracle_sample(min_seconds: float = 10.0):
+    """Time the oracle on a bounded sample of the step: the quantization and
+    exact GEMM of layer 0's seven projections at M = 1, 4, 16 (the first
+    min(N, 2048) output columns of each), passes
+    repeated until min_seconds have elapsed (at least one).  Returns (GB/s of
+    the same algorithmic traffic as the GPU step, seconds, threads, text)."""
+    from oracle import mxo
+    jobs = _oracle_jobs()
+    t0 = time.perf_counter()
+    nbytes = 0
+    passes = 0
+    while True:
+        for bits, x, w_s, w_c, K, N, M in jobs:
+            a_s, a_c = mxo.quantize_bf16(x, bits)
+            mxo.gemm(bits, a_c, a_s, w_c, w_s)
+            n4 = int(np.sum(bits == 4))
+            nbytes += N * (16 * n4 + 32 * (bits.size - n4) + bits.size) + M * K * 2 + M * N * 4
+        passes += 1
+        if time.perf_counter() - t0 >= min_seconds:
+            break
+    dt = time.perf_counter() - t0
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    desc = (f"layer 0 (q/k/v/o/gate/up/down, first min(N,{SAMPLE_ROWS}) output columns) at M=1,4,16, "
+            f"{passes} pass(es): oracle "
+            f"activation quantization + exact GEMM, OpenMP over output rows")
+    return nbytes / dt / 1e9, dt, threads, desc
+
+
+def run_reference(args):
+    ws, rank, _ = dist_setup()
+    if rank != 0:
+        return
+    for _ in range(args.warmup):
+        oracle_sample(min_seconds=0.0)
+    vals, secs = [], []
+    for _ in range(args.steps):
+        v, dt, threads, desc = oracle_sample(min_seconds=0.0)
+        vals.append(v)
+        secs.append(dt)
+    value = statistics.median(vals)
+    line = {
+        "impl": "reference", "metric": "mxint_decode_gemm_gbps", "value": value, "unit": "GB/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * statistics.median(secs), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int64+f64", "data": "synthetic",
+        "config": {"workload": "llama3-8b-decode (sample)", "layers": 1, "M": list(DECODE_MS)},
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": threads, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------- GPU arm
+def run_ours(args):
+    import torch
+
+    ws, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_17733_gb300 import build as B
+    from paper_2607_17733_gb300 import mxs
+    from paper_2607_17733_gb300.runtime import MxLinear
+    if not os.path.exists(mxs.LIB_PATH):
+        B.build()
+    mxs.lib()
+
+    L = args.layers
+    # ---- weights: drawn on the GPU (seeded per layer/projection), packed once
+    layers = []
+    gen = torch.Generator(device=dev)
+    for l in range(L):
+        projs = []
+        for pi, (name, K, N) in enumerate(I.LLAMA3_8B):
+            bits = I.width_map(K // 32, *MAP, I.rng(SEED, rank, l, pi))
+            gen.manual_seed(SEED * 1_000_003 + rank * 10_007 + l * 101 + pi)
+            w = (torch.randn((N, K), generator=gen, device=dev, dtype=torch.float32) * W_SIGMA).to(torch.bfloat16)
+            projs.append(MxLinear(w, bits))
+            del w
+        layers.append(projs)
+    torch.cuda.synchronize()
+
+    # ---- inputs: one contiguous pinned host block and one device block per step
+    items = []  # (M, lin, x_dev, bufs)
+    x_sizes = []
+    for M in DECODE_MS:
+        for l in range(L):
+            for pi, lin in enumerate(layers[l]):
+                x_sizes.append(M * lin.K)
+    x_host = torch.empty(sum(x_sizes), dtype=torch.bfloat16, pin_memory=True)
+    x_dev = torch.empty_like(x_host, device=dev)
+    y_sizes = []
+    off = 0
+    xi = 0
+    for M in DECODE_MS:
+        for l in range(L):
+            for pi, lin in enumerate(layers[l]):
+                xb = I.activations_bf16(M, lin.bits, I.rng(SEED, rank, 2, M, l, pi), OUTLIER_FRAC,
+                                        outlier_scale=OUTLIER_SCALE)
+                n = M * lin.K
+                x_host[off:off + n].copy_(torch.from_numpy(xb.view(np.int16).ravel()).view(torch.bfloat16))
+                bufs = lin.buffers(M, dev)
+                items.append((M, lin, x_dev[off:off + n].view(M, lin.K), bufs))
+                y_sizes.append(M * lin.N)
+                off += n
+                xi += 1
+    y_dev = torch.empty(sum(y_sizes), dtype=torch.float32, device=dev)
+    y_host = torch.empty_like(y_dev, device="cpu", pin_memory=True)
+    off = 0
+    for (M, lin, x, bufs), n in zip(items, y_sizes):
+        bufs["y"] = y_dev[off:off + n].view(M, lin.N)
+        off += n
+    x_dev.copy_(x_host)
+    torch.cuda.synchronize()
+
+    # ---- algorithmic work per step
+    step_bytes = sum(lin.weight_bytes + M * lin.K * 2 + M * lin.N * 4 for M, lin, _, _ in items)
+    step_ops = sum(2 * M * lin.N * lin.K for M, lin, _, _ in items)
+    gemm_bytes = sum(lin.weight_bytes + M * (mxs.act_row_bytes(lin.K, lin.bits) + lin.K // 32) + M * lin.N * 4
+                     for M, lin, _, _ in items)
+    launches_per_step = 2 * len(items)
+
+    # ---- graphs: a plain one (warm-up, e2e) and a few with CUDA events around every GEMM
+    capture_stream = torch.cuda.Stream(device=dev)
+
+    def make_step(events=None):
+        def fn():
+            for i, (M, lin, x, bufs) in enumerate(items):
+                lin.quantize(x, bufs)
+                if events is not None:
+                    events[i][0].record()
+                lin.matmul(bufs)
+                if events is not None:
+                    events[i][1].record()
+        return fn
+
+    def capture(fn):
+        capture_stream.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(capture_stream):
+            fn()
+        capture_stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=capture_stream):
+            fn()
+        torch.cuda.synchronize()
+        return g
+
+    plain = capture(make_step())
+    n_timed_graphs = max(1, min(4, args.steps))
+    try:
+        ev_sets = [[(torch.cuda.Event(enable_timing=True, external=True),
+                     torch.cuda.Event(enable_timing=True, external=True)) for _ in items]
+                   for _ in range(n_timed_graphs)]
+        timed = [capture(make_step(evs)) for evs in ev_sets]
+    except TypeError:  # torch without external events: time the plain graph only
+        ev_sets, timed = None, [plain]
+
+    for _ in range(args.warmup):
+        plain.replay()
+    torch.cuda.synchronize()
+
+    gpu_id = None
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid).replace("GPU-", "")
+    except Exception:
+        pass
+    sampler = ClockSampler(gpu_id)
+
+    # ---- timed region (device time, max over ranks)
+    barrier(ws)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.1)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for k in range(args.steps):
+        timed[k % len(timed)].replay()
+    t1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    barrier(ws)
+    ms = t0.elapsed_time(t1) / args.steps
+    ms = allreduce_max(ms, ws)
+    value = ws * step_bytes / (ms * 1e-3) / 1e9
+    tops = ws * step_ops / (ms * 1e-3) / 1e12
+
+    # ---- the dominant kernel (decode GEMM): per-launch durations from the graphs' events
+    pk = peaks()
+    roofline = None
+    if ev_sets is not None:
+        gemm_ms = sum(s.elapsed_time(e) for evs in ev_sets for s, e in evs) / len(ev_sets)
+        achieved = gemm_bytes / (gemm_ms * 1e-3) / 1e9
+        traffic = profile_traffic("gemm_decode.cu", "gemm_decode_llama3_8b_decode.md")
+        roofline = {"kernel": "gemm_decode_kernel", "bound": "hbm", "achieved": achieved,
+                    "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": achieved / pk["hbm_gbs"],
+                    "peak_source": pk["source"], "traffic": traffic,
+                    "bytes_per_step": gemm_bytes, "gemm_ms_per_step": gemm_ms,
+                    "launches_per_step": len(items), "share_of_step": gemm_ms / ms}
+
+    # ---- end to end through the public API with host buffers
+    barrier(ws)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e2e_steps = max(1, min(args.steps, 50))
+    e0.record()
+    for _ in range(e2e_steps):
+        x_dev.copy_(x_host, non_blocking=True)
+        plain.replay()
+        y_host.copy_(y_dev, non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = allreduce_max(e0.elapsed_time(e1) / e2e_steps, ws)
+    e2e = {"value": ws * step_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
+           "h2d_bytes_per_step": x_host.numel() * 2, "d2h_bytes_per_step": y_host.numel() * 4,
+           "ms_per_step": e2e_ms}
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        v, dt, threads, desc = oracle_sample()
+        cpu = {"value": v, "unit": "GB/s", "cores": threads, "kind": "oracle", "sample": desc, "seconds": dt}
+
+    if rank == 0:
+        line = {
+            "metric": "mxint_decode_gemm_gbps", "value": value, "unit": "GB/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int8+f32",
+            "data": "synthetic (seeded; weights N(0,0.02), activations N(0,1) with 1% outlier columns x30)",
+            "config": {"workload": "llama3-8b-decode", "M": list(DECODE_MS), "layers": L,
+                       "projections": [p[0] for p in I.LLAMA3_8B], "map_4_6_8": list(MAP),
+                       "parallelism": f"replicas x{ws}", "l2": "inputs larger than L2 (packed weights "
+                       f"{sum(lin.weight_bytes for p in layers for lin in p) / 1e9:.2f} GB per step)"},
+            "tops": tops,
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

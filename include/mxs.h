@@ -1,0 +1,191 @@
+/*
+ * mxs.h -- C ABI of libmxs, the MXINT mixed-precision linear layer of MXSens
+ * (arxiv 2607.17733) for NVIDIA GB300 (sm_103a).
+ *
+ * The layer computes y = x W^T where the activations x [M,K] (bf16) and the
+ * weights W [N,K] (bf16) are both quantized to MXINT: every block of 32
+ * consecutive values along K shares one power-of-two scale and holds fixed-point
+ * integer mantissas of 4, 6 or 8 bits (Sec. 2, Sec. 4.1).  The width of each
+ * K-block comes from a per-layer map (the paper's Alg. 3 allocation, produced
+ * offline).  The quantization rules the paper leaves open are read from the OCP
+ * MX MXINT definition it cites:
+ *   scale byte S = clamp(floor(log2 max|x|), -127, 127) + 127 (E8M0);
+ *   element m = clamp(round(x * 2^(b-2-E)), -(2^(b-1)-1), 2^(b-1)-1),
+ *   value = m * 2^(E-(b-2)); rounding ties-to-even (MXS_RNE) or away from
+ *   zero (MXS_RHAZ); a block with a NaN/Inf gets S = 255 and zero codes.
+ * The GEMM returns fp32 y[m,n] = sum_blocks 2^(Ea'+Ew') * (exact integer dot
+ * of the two blocks), E' = E-(b-2), accumulated in fp32.
+ *
+ * Conventions (all entry points):
+ *   - Return MXS_OK (0) or a positive MXS_ERR_* code; never abort, never print.
+ *     mxs_last_error() gives a thread-local message for the last failure.
+ *   - Sizes are int64_t; K must be a positive multiple of 32 and at most
+ *     MXS_MAX_K; M, N >= 1 (M = 0 is accepted and does nothing).
+ *   - `bits` is a HOST array of K/32 bytes, each 4, 6 or 8, read during the
+ *     call.  Blocks are stored grouped by width: slot s < n4 holds the s-th
+ *     4-bit block, then the 6-bit blocks, then the 8-bit ones, each group in
+ *     increasing block order.
+ *   - Every other pointer is DEVICE memory owned by the caller; the library
+ *     allocates nothing.  Buffers must be 16-byte aligned unless stated.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Work is enqueued asynchronously; device pointers must stay
+ *     valid until the stream reaches it.  Errors raised while the kernels run
+ *     surface at the caller's next synchronisation.
+ *   - Outputs are overwritten in full, padding rows and slots included; only
+ *     the alignment gaps between the sections of an activation planes buffer
+ *     are left unwritten.
+ *   - Only sm_103a devices are supported (MXS_ERR_UNSUPPORTED otherwise).
+ *
+ * Storage format (the "packed" layouts; byte offsets are exact):
+ *   Activation codes, per row m (row_bytes = 16*n4 + 32*(n6+n8)):
+ *     4-bit slot s: bytes [16s, 16s+16), element i in byte i/2 (low nibble for
+ *     even i), two's complement; 6/8-bit slot s: bytes [16*n4 + 32(s-n4), +32),
+ *     one int8 per element.  Activation scales: uint8 [M, K/32] by slot.
+ *   Weight buffer (layout MXS_W_COMPACT): rows padded to Np = 16*ceil(N/16),
+ *     cut into tiles of 16 rows; inside a tile one block of all 16 rows is
+ *     stored in the order a warp holds the A operand of a 16x8x32 integer MMA
+ *     (lane l = 4g+q: rows g, g+8; elements 4q..4q+3 and 16+4q..16+4q+3):
+ *       Q4 at 0:             chunk (t,s) of 256 B at (t*n4+s)*256; byte
+ *                            8l+4h+j: row 16t+g+8h, high nibble = element 4q+j,
+ *                            low nibble = element 16+4q+j;
+ *       Q8 at O8 = align256(T*n4*256): chunk (t,j) of 512 B at
+ *                            O8+(t*(n6+n8)+j)*512; byte 16l+4c+j: c=0 row g
+ *                            elem 4q+j, c=1 row g+8 elem 4q+j, c=2 row g elem
+ *                            16+4q+j, c=3 row g+8 elem 16+4q+j;
+ *       SC at OS = align256(O8 + T*(n6+n8)*512): uint8 [Np, K/32] scales by slot;
+ *       compact size = align256(OS + Np*K/32).
+ *   MMA planes (layout MXS_W_COMPACT_AND_PLANES for weights, the `planes`
+ *     output of mxs_quantize_act for activations), Kp = 128*(ceil(n4/4) +
+ *     ceil((n6+n8)/2)):
+ *       P [rows, Kp] e4m3: 4-bit slot s at bytes [32s, +32) = m/4; padding to
+ *       a multiple of 4 slots is zero; 6/8-bit slot j at 128*ceil(n4/4)+64j:
+ *       high digit then low digit (32 B each); b=6: m = 8h+l, digits h/2, l/16;
+ *       b=8: m = 16h+l, digits h/4, l/64 (l >= 0), so that the two digits add
+ *       up to m*2^-(b-2) and the block scale S applies to both unchanged.
+ *       SF at align256(P + rows*Kp): per 128-row tile and 128-byte K' stage,
+ *       512 B ordered [i<32][w<4][q<4] = S of row 128*tile+32w+i, slot 4*st+q
+ *       (4-bit stages) or 2*(st-ceil(n4/4))+q for q<2 (6/8-bit stages); every
+ *       other byte 0.
+ *     For weights P and SF follow the compact part inside the same buffer.
+ */
+#ifndef MXS_H_
+#define MXS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define MXS_API __attribute__((visibility("default")))
+#else
+#define MXS_API
+#endif
+
+#define MXS_VERSION 1
+#define MXS_MAX_K 65536 /* K/32 <= 2048 blocks */
+
+enum mxs_status {
+    MXS_OK = 0,
+    MXS_ERR_INVALID_ARG = 1, /* NULL pointer, bad enum, bad leading dimension */
+    MXS_ERR_SHAPE = 2,       /* K not a positive multiple of 32, K > MXS_MAX_K, M/N < 0 */
+    MXS_ERR_BITS = 3,        /* a map entry outside {4, 6, 8} */
+    MXS_ERR_ALIGN = 4,       /* a device pointer not 16-byte aligned */
+    MXS_ERR_BUFFER = 5,      /* a caller buffer smaller than required */
+    MXS_ERR_CUDA = 6,        /* a CUDA runtime call failed (message has the name) */
+    MXS_ERR_TIMEOUT = 7,     /* a kernel gave up waiting (see mxs_device_status) */
+    MXS_ERR_UNSUPPORTED = 8  /* not an sm_103a device, or a feature not built */
+};
+
+enum mxs_rounding { MXS_RNE = 0, MXS_RHAZ = 1 };
+enum mxs_weight_layout { MXS_W_COMPACT = 0, MXS_W_COMPACT_AND_PLANES = 1 };
+
+/* Thread-local description of the last failure of a call on this thread. */
+MXS_API const char *mxs_last_error(void);
+/* MXS_VERSION of the built library. */
+MXS_API int mxs_version(void);
+
+/* ---------------------------------------------------------------- sizes
+ * Bytes the caller must provide.  They touch no device and return a negative
+ * mxs_status (e.g. -MXS_ERR_BITS) for invalid arguments. */
+MXS_API int64_t mxs_act_row_bytes(int64_t K, const uint8_t *bits);
+MXS_API int64_t mxs_act_codes_bytes(int64_t M, int64_t K, const uint8_t *bits);
+/* activation planes + their scale tiles (one buffer; SF at align256(M*Kp)) */
+MXS_API int64_t mxs_act_planes_bytes(int64_t M, int64_t K, const uint8_t *bits);
+MXS_API int64_t mxs_weight_bytes(int64_t N, int64_t K, const uint8_t *bits, int layout);
+/* scratch for mxs_gemm / mxs_gemm_decode: split-K partial sums (fp32). */
+MXS_API int64_t mxs_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K, const uint8_t *bits);
+
+/* ---------------------------------------------------------------- A1: activation quantization
+ * Quantizes x (bf16 [M,K], row stride ld_x elements, ld_x >= K and a multiple
+ * of 8) block by block with widths `bits` (Sec. 4.1 one width per block;
+ * Appendix A.2 activations quantized on the fly) and writes
+ *   codes  [M, mxs_act_row_bytes]  packed codes (may be NULL)
+ *   scales [M, K/32]               scale bytes by slot (NULL iff codes NULL)
+ *   planes mxs_act_planes_bytes    MMA planes + scale tiles (may be NULL)
+ * At least one of codes / planes must be non-NULL. */
+MXS_API int mxs_quantize_act(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x,
+                     const uint8_t *bits, int rounding,
+                     void *codes, uint8_t *scales, void *planes, void *stream);
+
+/* ---------------------------------------------------------------- A2: weight packing (offline)
+ * Quantizes W (bf16 [N,K] row stride ld_w, the nn.Linear convention) with the
+ * same rules and writes the weight buffer (mxs_weight_bytes(N,K,bits,layout)
+ * bytes).  Run once per layer. */
+MXS_API int mxs_pack_weight(const void *w_bf16, int64_t N, int64_t K, int64_t ld_w,
+                    const uint8_t *bits, int rounding, int layout,
+                    void *packed, void *stream);
+
+/* ---------------------------------------------------------------- A3/A4: GEMM
+ * y [M,N] fp32 (row stride ld_y >= N, elements) = x W^T over the quantized
+ * operands.  act_bits must equal w_bits (the paper allocates one map per
+ * linear layer and applies it to W and A); other pairs return
+ * MXS_ERR_UNSUPPORTED.  `w_layout` is the layout W was packed with.
+ * mxs_gemm picks the decode kernel for M <= 16 (needs codes/scales) and the
+ * tensor-core prefill kernel otherwise (needs act_planes and a weight packed
+ * with MXS_W_COMPACT_AND_PLANES).  workspace may be NULL when
+ * mxs_gemm_workspace_bytes() is 0. */
+MXS_API int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const void *act_planes,
+             const uint8_t *act_bits, const void *packed_w, int w_layout, const uint8_t *w_bits,
+             int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y,
+             void *workspace, size_t ws_bytes, void *stream);
+
+/* Decode path only (M <= 16): weights streamed once from the compact layout,
+ * integer warp MMAs per block, fp32 fold, split-K with a fixed-order reduction. */
+MXS_API int mxs_gemm_decode(const void *act_codes, const uint8_t *act_scales, const uint8_t *bits,
+                    const void *packed_w, int64_t M, int64_t N, int64_t K,
+                    float *y, int64_t ld_y, void *workspace, size_t ws_bytes, void *stream);
+
+/* Prefill path only (any M >= 1, efficient for M >= 128): the tensor-core
+ * kernel over the MMA planes of the activations (mxs_quantize_act `planes`)
+ * and of the weights (packed with MXS_W_COMPACT_AND_PLANES).  Sec. 6: the
+ * mixed widths are executed on a fixed-width tensor core by splitting each
+ * 6/8-bit mantissa into two exactly representable e4m3 digits (4 MMAs per
+ * block pair, 1 for 4-bit blocks); scales are applied per 32-element block by
+ * the block-scaled MMA (UE8M0).  Waits inside the kernel are bounded (about
+ * 2 s); on expiry it records MXS_ERR_TIMEOUT (see mxs_device_status). */
+MXS_API int mxs_gemm_prefill(const void *act_planes, const uint8_t *bits, const void *packed_w,
+                             int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, void *stream);
+
+/* ---------------------------------------------------------------- status
+ * Kernels that wait on barriers give up after a bounded number of polls and
+ * record MXS_ERR_TIMEOUT in a per-device status word instead of hanging.
+ * Reads that word for the current device after synchronising `stream`;
+ * clears it when reset != 0. */
+MXS_API int mxs_device_status(int *status, int reset, void *stream);
+
+/* Test hook for the bounded waits: mxs_gemm_prefill, except that the
+ * producer never loads K' stage `stage` (1-based), so the MMA warp's wait for
+ * it runs out; the kernel then records MXS_ERR_TIMEOUT, drains what it issued,
+ * frees its tensor memory and returns (y is left partly unwritten).  No
+ * device fault or hang is involved; the context stays usable. */
+MXS_API int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits, const void *packed_w,
+                                    int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, int stage,
+                                    void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MXS_H_ */

@@ -1,0 +1,109 @@
+// common.cuh -- shared pieces of libmxs: the grouping plan, the block
+// quantizer, launch helpers.  Device code here is sm_103a only.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/mxs.h"
+
+namespace mxs {
+
+constexpr int kBlock = 32;
+constexpr int kMaxNb = MXS_MAX_K / kBlock;
+
+// Width grouping of a map (step A0).  slot -> original block index, stable
+// inside each width group; passed by value to kernels (__grid_constant__).
+struct Plan {
+    int nb, n4, n6, n8, n68;
+    int st4;  // ceil(n4/4): 128-byte K' stages of 4-bit slots in the plane layout
+    int nst;  // st4 + ceil(n68/2)
+    int64_t row_bytes;  // packed activation row
+    int64_t kp;         // plane row bytes = 128*nst
+    uint16_t slot_block[kMaxNb];
+};
+
+__host__ __device__ inline int slot_width(const Plan &p, int s) {
+    return s < p.n4 ? 4 : (s < p.n4 + p.n6 ? 6 : 8);
+}
+
+__host__ __device__ inline int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
+
+struct WeightOffsets {
+    int64_t T, Np, o8, os, compact, planes, sf, total;
+};
+
+__host__ __device__ inline WeightOffsets weight_offsets(const Plan &p, int64_t N, bool with_planes) {
+    WeightOffsets w;
+    w.T = (N + 15) / 16;
+    w.Np = w.T * 16;
+    w.o8 = align256(w.T * p.n4 * 256);
+    w.os = align256(w.o8 + w.T * p.n68 * 512);
+    w.compact = align256(w.os + w.Np * p.nb);
+    w.planes = w.compact;
+    w.sf = align256(w.planes + N * p.kp);
+    w.total = with_planes ? align256(w.sf + (N + 127) / 128 * p.nst * 512) : w.compact;
+    return w;
+}
+
+// ------------------------------------------------------------ quantizer
+// Integer form of the MXINT rule on bf16 bit patterns: the scale byte is the
+// bf16 exponent field of the block's largest magnitude (floor(log2) of a
+// normal number, 0 for zero/subnormal maxima, 255 for Inf/NaN), and an element
+// with significand sig and exponent field e is sig * 2^-sh in units of the
+// grid step, sh = S - max(e,1) + 9 - b >= 0.  Rounding is done on the bits
+// that shift out, then the magnitude is clamped to 2^(b-1)-1.
+__device__ __forceinline__ int quant_elem(uint32_t h, int S, int b, int rhaz) {
+    const int e = (h >> 7) & 0xFF;
+    const int sig = e ? (int)((h & 0x7F) | 0x80) : (int)(h & 0x7F);
+    int sh = S - (e ? e : 1) + 9 - b;
+    sh = sh > 10 ? 10 : sh;  // beyond 9 the magnitude is below 1/4 step: 0
+    int q;
+    if (sh == 0) {
+        q = sig;
+    } else {
+        q = sig >> sh;
+        const int rem = sig & ((1 << sh) - 1);
+        const int half = 1 << (sh - 1);
+        q += (rem > half) | ((rem == half) & (rhaz | (q & 1)));
+    }
+    const int Q = (1 << (b - 1)) - 1;
+    q = q > Q ? Q : q;
+    return (h & 0x8000) ? -q : q;
+}
+
+// e4m3 byte of an exactly representable value (hardware conversion).
+__device__ __forceinline__ uint16_t e4m3x2(float lo, float hi) {
+    uint16_t r;
+    asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+// 2^e as fp32 for e in [-149, 127] (subnormal below -126), exact.
+__device__ __forceinline__ float pow2f(int e) {
+    return e >= -126 ? __int_as_float((e + 127) << 23) : __int_as_float(1 << (e + 149 < 0 ? 0 : e + 149));
+}
+
+}  // namespace mxs
+
+// ------------------------------------------------------------ host side
+namespace mxs {
+void set_error(const char *fmt, ...);
+int fail(int code, const char *fmt, ...);
+int build_plan(const uint8_t *bits, int64_t K, Plan *p);
+int check_device();
+int cuda_fail(cudaError_t e, const char *what);
+
+// kernel launchers (one translation unit each)
+int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rounding, void *codes,
+                    uint8_t *scales, void *planes, cudaStream_t st);
+int launch_pack_weight(const Plan &p, const void *w, int64_t N, int64_t ld, int rounding, bool planes,
+                       void *packed, cudaStream_t st);
+int64_t decode_workspace_bytes(const Plan &p, int64_t M, int64_t N);
+int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, const void *packed,
+                       int64_t M, int64_t N, float *y, int64_t ld_y, void *ws, size_t ws_bytes,
+                       cudaStream_t st);
+int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N,
+                        float *y, int64_t ld_y, int starve, cudaStream_t st);
+int prefill_status(int *status, int reset, cudaStream_t st);
+}  // namespace mxs

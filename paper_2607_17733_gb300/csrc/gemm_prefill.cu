@@ -1,0 +1,380 @@
+// gemm_prefill.cu -- A3: the MXINT GEMM for prefill shapes on the 5th-generation
+// tensor cores (tcgen05), M > 16 tokens.
+//
+// y[m,n] = sum over 32-element K-blocks of 2^(Ea+Ew) * sum_i (ma_i 2^-(b-2)) *
+// (mw_i 2^-(b-2)): the MXINT product of Sec. 2 with the widths of Sec. 4.1.
+// sm_103a has no integer tcgen05 MMA, so the integer mantissas enter the
+// block-scaled FP8 MMA (kind::mxf8f6f4, e4m3 x e4m3, one UE8M0 scale per 32
+// K-elements) as exact e4m3 "digit planes" -- the decomposition into high- and
+// low-precision parts that Sec. 6 describes for mixed-width execution:
+//   4-bit block:    one plane  m/4;
+//   6/8-bit block:  two planes, m*2^-(b-2) = high + low (both exact in e4m3),
+//                   four MMAs (hi*hi, hi*lo, lo*hi, lo*lo).
+// Every plane product is an exact small integer sum scaled by the block's own
+// scale bytes; the tensor core accumulates it into fp32 TMEM.
+//
+// Structure (one 128x256 output tile per CTA, 192 threads):
+//   warp 0     TMA producer: 128-byte K' stages of A and W planes (128B swizzle)
+//              plus the scale tiles (1-D bulk copies), into a 4-stage ring;
+//   warp 1     TMEM owner and MMA issuer: tcgen05.cp scales -> TMEM, then the
+//              MMAs of the stage, tcgen05.commit frees the stage;
+//   warps 2-5  epilogue: tcgen05.ld the fp32 accumulator, store y.
+// Every mbarrier wait is bounded; on expiry the kernel records MXS_ERR_TIMEOUT
+// in a device status word, stops issuing work, drains what it issued and frees
+// its tensor memory before returning.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+
+namespace mxs {
+
+__device__ int g_prefill_status;  // sticky MXS_ERR_TIMEOUT, read by mxs_device_status
+
+namespace {
+
+constexpr int kBM = 128, kBN = 256, kBK = 128;  // tile rows (A), tile rows (W), K' bytes per stage
+constexpr int kStages = 4;
+constexpr int kABytes = kBM * kBK, kBBytes = kBN * kBK;  // 16 KB, 32 KB
+constexpr int kSfaBytes = 512, kSfbBytes = 1024;
+constexpr int kTmemCols = 512;
+constexpr int kAccCol = 0, kSfCol = 256;  // per stage: SFA 4 columns, SFB 8 columns
+constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on any single wait
+
+struct PrefillArgs {
+    const uint8_t *sfa;  // scale tiles of A: [ceil(M/128)][nst][512]
+    const uint8_t *sfb;  // scale tiles of W: [ceil(N/128)][nst][512]
+    float *y;
+    int64_t ld_y;
+    int M, N, nst, st4, sfb_tiles;
+    int starve;  // test hook: >0 makes the producer skip stage `starve-1` (the wait then times out)
+};
+
+struct Smem {
+    uint8_t a[kStages][kABytes];
+    uint8_t b[kStages][kBBytes];
+    uint8_t sfa[kStages][kSfaBytes];
+    uint8_t sfb[kStages][kSfbBytes];
+    uint64_t full[kStages], empty[kStages], acc_full;
+    uint32_t tmem_base;
+    int abort;
+};
+
+__device__ __forceinline__ uint32_t su32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ uint64_t now_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(su32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait: false if the CTA aborted or the wait ran out (then it aborts).
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = now_ns();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort) return false;
+        if (now_ns() - t0 > kWaitNs) {
+            *abort = 1;
+            atomicExch(&g_prefill_status, MXS_ERR_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, uint64_t *bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+            su32(dst)),
+        "l"(map), "r"(su32(bar)), "r"(x), "r"(y)
+        : "memory");
+}
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     su32(dst)),
+                 "l"(src), "r"(bytes), "r"(su32(bar))
+                 : "memory");
+}
+
+// UMMA shared-memory descriptors (sm_100 family): start>>4 [0,14), LBO>>4 [16,30),
+// SBO>>4 [32,46), version 1 [46,48), layout [61,64) (2 = 128B swizzle, 0 = none).
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t addr) {
+    return (uint64_t)((addr & 0x3FFFF) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+__device__ __forceinline__ uint64_t desc_sf(uint32_t addr) {  // 32 rows x 16 B, no swizzle
+    return (uint64_t)((addr & 0x3FFFF) >> 4) | ((uint64_t)(128 >> 4) << 32) | ((uint64_t)1 << 46);
+}
+
+// Instruction descriptor, kind::mxf8f6f4: A/B e4m3 (0), K-major, N>>3 at 17,
+// UE8M0 scales (bit 23), M>>4 at 24, scale-factor byte ids at [4,6) (B) and [29,31) (A).
+constexpr uint32_t kIdesc = ((uint32_t)(kBN >> 3) << 17) | (1u << 23) | ((uint32_t)(kBM >> 4) << 24);
+__device__ __forceinline__ uint32_t idesc(int sfa_id, int sfb_id) {
+    return kIdesc | ((uint32_t)sfb_id << 4) | ((uint32_t)sfa_id << 29);
+}
+
+__device__ __forceinline__ void mma_mx(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t sfa, uint32_t sfb,
+                                       uint32_t accum) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%5], [%6], p;\n}" ::"r"(d),
+        "l"(a), "l"(b), "r"(id), "r"(accum), "r"(sfa), "r"(sfb)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_cp_sf(uint32_t taddr, uint64_t desc) {
+    asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(desc) : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%"
+        "19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+          "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_constant__ CUtensorMap tmap_a,
+                                                              const __grid_constant__ CUtensorMap tmap_b,
+                                                              const __grid_constant__ PrefillArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    // 1024-byte alignment for the 128B-swizzled operand tiles
+    const uint32_t base = su32(smem_raw);
+    Smem &sm = *reinterpret_cast<Smem *>(smem_raw + (((base + 1023) & ~1023u) - base));
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.y * kBM, n0 = blockIdx.x * kBN;
+    const int nst = a.nst;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&sm.full[s], 1);
+            mbar_init(&sm.empty[s], 1);
+        }
+        mbar_init(&sm.acc_full, 1);
+        sm.abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(&sm.tmem_base)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    fence_before();
+    __syncthreads();
+    fence_after();
+    const uint32_t tmem = sm.tmem_base;
+    volatile int *abort = &sm.abort;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const int tile_a = m0 / 128, tile_b = n0 / 128;
+            const bool two_b = tile_b + 1 < a.sfb_tiles;
+            const uint32_t tx = kABytes + kBBytes + kSfaBytes + (two_b ? 2 : 1) * 512;
+            int issued = 0;
+            for (int ks = 0; ks < nst; ++ks) {
+                const int s = ks % kStages;
+                const uint32_t ph = (ks / kStages) & 1;
+                if (!mbar_wait(&sm.empty[s], ph ^ 1, abort)) break;
+                if (a.starve == ks + 1) continue;  // test hook: this stage never arrives
+                mbar_expect_tx(&sm.full[s], tx);
+                tma_load_2d(sm.a[s], &tmap_a, &sm.full[s], ks * kBK, m0);
+                tma_load_2d(sm.b[s], &tmap_b, &sm.full[s], ks * kBK, n0);
+                bulk_load(sm.sfa[s], a.sfa + ((int64_t)tile_a * nst + ks) * 512, 512, &sm.full[s]);
+                bulk_load(sm.sfb[s], a.sfb + ((int64_t)tile_b * nst + ks) * 512, 512, &sm.full[s]);
+                if (two_b) bulk_load(sm.sfb[s] + 512, a.sfb + ((int64_t)(tile_b + 1) * nst + ks) * 512, 512, &sm.full[s]);
+                issued = ks + 1;
+            }
+            // drain: every stage this thread issued must have landed before the CTA exits
+            for (int ks = (issued > kStages ? issued - kStages : 0); ks < issued; ++ks) {
+                if (a.starve == ks + 1) continue;
+                const int s = ks % kStages;
+                const uint64_t t0 = now_ns();
+                while (!mbar_try_wait(&sm.full[s], (ks / kStages) & 1) && now_ns() - t0 < kWaitNs) {
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            int committed = 0;
+            for (int ks = 0; ks < nst; ++ks) {
+                const int s = ks % kStages;
+                const uint32_t ph = (ks / kStages) & 1;
+                if (!mbar_wait(&sm.full[s], ph, abort)) break;
+                fence_after();
+                const uint32_t sfa_t = tmem + kSfCol + 12 * s, sfb_t = sfa_t + 4;
+                tmem_cp_sf(sfa_t, desc_sf(su32(sm.sfa[s])));
+                tmem_cp_sf(sfb_t, desc_sf(su32(sm.sfb[s])));
+                tmem_cp_sf(sfb_t + 4, desc_sf(su32(sm.sfb[s] + 512)));
+                const uint32_t a_addr = su32(sm.a[s]), b_addr = su32(sm.b[s]);
+                if (ks < a.st4) {  // four 4-bit blocks, one plane each
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        mma_mx(tmem + kAccCol, desc_sw128(a_addr + 32 * q), desc_sw128(b_addr + 32 * q), idesc(q, q),
+                               sfa_t, sfb_t, (ks > 0 || q > 0) ? 1u : 0u);
+                } else {  // two 6/8-bit blocks, high and low plane each
+#pragma unroll
+                    for (int j = 0; j < 2; ++j)
+#pragma unroll
+                        for (int pp = 0; pp < 4; ++pp) {
+                            const int pa = pp >> 1, pb = pp & 1;
+                            mma_mx(tmem + kAccCol, desc_sw128(a_addr + 64 * j + 32 * pa),
+                                   desc_sw128(b_addr + 64 * j + 32 * pb), idesc(j, j), sfa_t, sfb_t,
+                                   (ks > 0 || j > 0 || pp > 0) ? 1u : 0u);
+                        }
+                }
+                mma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
+                committed = ks + 1;
+            }
+            if (committed == nst) mma_commit(&sm.acc_full);
+            // drain: wait (bounded) until the tensor core has finished what was issued
+            if (committed > 0) {
+                const int ks = committed - 1;
+                const uint64_t t0 = now_ns();
+                while (!mbar_try_wait(&sm.empty[ks % kStages], (ks / kStages) & 1) && now_ns() - t0 < kWaitNs) {
+                }
+            }
+        }
+    } else {
+        // ------------------------------------------------ epilogue (warps 2..5)
+        const int quad = warp & 3;  // TMEM lane quadrant this warp may access
+        // warp-uniform decision: tcgen05.ld below is .sync.aligned
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full, 0, abort));
+        if (ok) {
+            fence_after();
+            const int row = m0 + 32 * quad + lane;
+            float *yrow = a.y + (int64_t)row * a.ld_y;
+            const bool vec = ((a.ld_y & 3) == 0) && ((reinterpret_cast<uintptr_t>(a.y) & 15) == 0);
+#pragma unroll 1
+            for (int c = 0; c < kBN / 32; ++c) {
+                uint32_t r[32];
+                tmem_ld32(tmem + ((uint32_t)(32 * quad) << 16) + kAccCol + 32 * c, r);
+                const int n = n0 + 32 * c;
+                if (row < a.M) {
+                    if (vec && n + 32 <= a.N) {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i)
+                            *reinterpret_cast<uint4 *>(yrow + n + 4 * i) =
+                                make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (n + i < a.N) yrow[n + i] = __uint_as_float(r[i]);
+                    }
+                }
+            }
+        }
+    }
+
+    fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+int make_map(CUtensorMap *map, const void *base, int64_t rows, int64_t kp, int box_rows) {
+    auto fn = encode_fn();
+    if (!fn) return fail(MXS_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+    cuuint64_t dims[2] = {(cuuint64_t)kp, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)kp};
+    cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(MXS_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+    return MXS_OK;
+}
+
+}  // namespace
+
+int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N, float *y,
+                        int64_t ld_y, int starve, cudaStream_t st) {
+    if (M > 0x7FFFFFF0 || N > 0x7FFFFFF0) return fail(MXS_ERR_SHAPE, "M or N too large");
+    const uint8_t *ap = static_cast<const uint8_t *>(act_planes);
+    const uint8_t *wb = static_cast<const uint8_t *>(packed_w);
+    const WeightOffsets off = weight_offsets(p, N, true);
+    CUtensorMap ta, tb;
+    int rc = make_map(&ta, ap, M, p.kp, kBM);
+    if (rc) return rc;
+    rc = make_map(&tb, wb + off.planes, N, p.kp, kBN);
+    if (rc) return rc;
+    PrefillArgs a;
+    a.sfa = ap + align256(M * p.kp);
+    a.sfb = wb + off.sf;
+    a.y = y;
+    a.ld_y = ld_y;
+    a.M = (int)M;
+    a.N = (int)N;
+    a.nst = p.nst;
+    a.st4 = p.st4;
+    a.sfb_tiles = (int)((N + 127) / 128);
+    a.starve = starve;
+    const size_t smem = sizeof(Smem) + 1024;
+    cudaError_t e = cudaFuncSetAttribute(gemm_prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(prefill smem)");
+    dim3 grid((unsigned)((N + kBN - 1) / kBN), (unsigned)((M + kBM - 1) / kBM));
+    if (grid.y > 65535) return fail(MXS_ERR_SHAPE, "M too large for the prefill grid");
+    gemm_prefill_kernel<<<grid, 192, smem, st>>>(ta, tb, a);
+    return cuda_fail(cudaGetLastError(), "gemm_prefill_kernel launch");
+}
+
+int prefill_status(int *status, int reset, cudaStream_t st) {
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    int v = 0;
+    e = cudaMemcpyFromSymbol(&v, g_prefill_status, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyFromSymbol(status)");
+    *status = v;
+    if (reset && v != 0) {
+        const int zero = 0;
+        e = cudaMemcpyToSymbol(g_prefill_status, &zero, sizeof(int));
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyToSymbol(status)");
+    }
+    return MXS_OK;
+}
+
+}  // namespace mxs

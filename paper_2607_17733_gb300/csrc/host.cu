@@ -1,0 +1,241 @@
+// host.cu -- the C ABI of libmxs (include/mxs.h): argument validation, the
+// width-grouping plan (step A0), size queries and dispatch to the kernels.
+// Validation happens before any CUDA call, so a bad argument is reported the
+// same way with or without a GPU.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "common.cuh"
+
+namespace mxs {
+
+static thread_local char g_err[512] = "";
+
+void set_error(const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+}
+
+int fail(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char *what) {
+    if (e == cudaSuccess) return MXS_OK;
+    return fail(MXS_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Step A0: validate the map and partition block indices by width, keeping the
+// original order inside each group (Sec. 4.1: one width per block; the 6/8-bit
+// columns come in whole blocks, so every block has exactly one width).
+int build_plan(const uint8_t *bits, int64_t K, Plan *p) {
+    if (K <= 0 || K % kBlock != 0 || K > MXS_MAX_K)
+        return fail(MXS_ERR_SHAPE, "K=%lld must be a positive multiple of 32 and <= %d", (long long)K,
+                    MXS_MAX_K);
+    if (!bits) return fail(MXS_ERR_INVALID_ARG, "bits is NULL");
+    const int nb = (int)(K / kBlock);
+    int counts[3] = {0, 0, 0};
+    for (int kb = 0; kb < nb; ++kb) {
+        const int b = bits[kb];
+        if (b != 4 && b != 6 && b != 8) return fail(MXS_ERR_BITS, "bits[%d]=%d is not 4, 6 or 8", kb, b);
+        counts[(b - 4) / 2]++;
+    }
+    p->nb = nb;
+    p->n4 = counts[0];
+    p->n6 = counts[1];
+    p->n8 = counts[2];
+    p->n68 = counts[1] + counts[2];
+    p->st4 = (p->n4 + 3) / 4;
+    p->nst = p->st4 + (p->n68 + 1) / 2;
+    p->row_bytes = 16 * (int64_t)p->n4 + 32 * (int64_t)p->n68;
+    p->kp = 128 * (int64_t)p->nst;
+    int s = 0;
+    for (int w = 4; w <= 8; w += 2)
+        for (int kb = 0; kb < nb; ++kb)
+            if (bits[kb] == w) p->slot_block[s++] = (uint16_t)kb;
+    for (int i = nb; i < kMaxNb; ++i) p->slot_block[i] = 0;
+    return MXS_OK;
+}
+
+int check_device() {
+    static int cached[64];  // 0 unknown, 1 ok, 2 unsupported
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev >= 0 && dev < 64 && cached[dev] == 1) return MXS_OK;
+    int major = 0, minor = 0;
+    e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    const bool ok = major == 10 && minor == 3;
+    if (dev >= 0 && dev < 64) cached[dev] = ok ? 1 : 2;
+    if (!ok) return fail(MXS_ERR_UNSUPPORTED, "device %d is sm_%d%d; libmxs is built for sm_103a only", dev, major, minor);
+    return MXS_OK;
+}
+
+static bool aligned16(const void *ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15) == 0; }
+
+}  // namespace mxs
+
+using namespace mxs;
+
+extern "C" {
+
+const char *mxs_last_error(void) { return g_err; }
+
+int mxs_version(void) { return MXS_VERSION; }
+
+int64_t mxs_act_row_bytes(int64_t K, const uint8_t *bits) {
+    Plan p;
+    const int rc = build_plan(bits, K, &p);
+    return rc ? -rc : p.row_bytes;
+}
+
+int64_t mxs_act_codes_bytes(int64_t M, int64_t K, const uint8_t *bits) {
+    if (M < 0) return -fail(MXS_ERR_SHAPE, "M=%lld < 0", (long long)M);
+    Plan p;
+    const int rc = build_plan(bits, K, &p);
+    return rc ? -rc : M * p.row_bytes;
+}
+
+int64_t mxs_act_planes_bytes(int64_t M, int64_t K, const uint8_t *bits) {
+    if (M < 0) return -fail(MXS_ERR_SHAPE, "M=%lld < 0", (long long)M);
+    Plan p;
+    const int rc = build_plan(bits, K, &p);
+    return rc ? -rc : align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);
+}
+
+int64_t mxs_weight_bytes(int64_t N, int64_t K, const uint8_t *bits, int layout) {
+    if (N < 0) return -fail(MXS_ERR_SHAPE, "N=%lld < 0", (long long)N);
+    if (layout != MXS_W_COMPACT && layout != MXS_W_COMPACT_AND_PLANES)
+        return -fail(MXS_ERR_INVALID_ARG, "layout=%d", layout);
+    Plan p;
+    const int rc = build_plan(bits, K, &p);
+    return rc ? -rc : weight_offsets(p, N, layout == MXS_W_COMPACT_AND_PLANES).total;
+}
+
+int64_t mxs_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K, const uint8_t *bits) {
+    if (M < 0 || N < 0) return -fail(MXS_ERR_SHAPE, "M/N < 0");
+    Plan p;
+    const int rc = build_plan(bits, K, &p);
+    if (rc) return -rc;
+    return M <= 16 ? decode_workspace_bytes(p, M, N) : 0;
+}
+
+int mxs_quantize_act(const void *x, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits, int rounding,
+                     void *codes, uint8_t *scales, void *planes, void *stream) {
+    Plan p;
+    int rc = build_plan(bits, K, &p);
+    if (rc) return rc;
+    if (M < 0) return fail(MXS_ERR_SHAPE, "M=%lld < 0", (long long)M);
+    if (rounding != MXS_RNE && rounding != MXS_RHAZ) return fail(MXS_ERR_INVALID_ARG, "rounding=%d", rounding);
+    if (!x) return fail(MXS_ERR_INVALID_ARG, "x is NULL");
+    if (!codes && !planes) return fail(MXS_ERR_INVALID_ARG, "both codes and planes are NULL");
+    if (!codes != !scales) return fail(MXS_ERR_INVALID_ARG, "codes and scales must be both set or both NULL");
+    if (ld_x < K || ld_x % 8 != 0) return fail(MXS_ERR_INVALID_ARG, "ld_x=%lld must be >= K and a multiple of 8", (long long)ld_x);
+    if (!aligned16(x) || (codes && !aligned16(codes)) || (planes && !aligned16(planes)))
+        return fail(MXS_ERR_ALIGN, "x, codes and planes must be 16-byte aligned");
+    if (M == 0) return MXS_OK;
+    if ((rc = check_device())) return rc;
+    return launch_quantize(p, x, M, ld_x, rounding, codes, scales, planes, static_cast<cudaStream_t>(stream));
+}
+
+int mxs_pack_weight(const void *w, int64_t N, int64_t K, int64_t ld_w, const uint8_t *bits, int rounding,
+                    int layout, void *packed, void *stream) {
+    Plan p;
+    int rc = build_plan(bits, K, &p);
+    if (rc) return rc;
+    if (N < 0) return fail(MXS_ERR_SHAPE, "N=%lld < 0", (long long)N);
+    if (rounding != MXS_RNE && rounding != MXS_RHAZ) return fail(MXS_ERR_INVALID_ARG, "rounding=%d", rounding);
+    if (layout != MXS_W_COMPACT && layout != MXS_W_COMPACT_AND_PLANES)
+        return fail(MXS_ERR_INVALID_ARG, "layout=%d", layout);
+    if (!w || !packed) return fail(MXS_ERR_INVALID_ARG, "w or packed is NULL");
+    if (ld_w < K || ld_w % 8 != 0) return fail(MXS_ERR_INVALID_ARG, "ld_w=%lld must be >= K and a multiple of 8", (long long)ld_w);
+    if (!aligned16(w) || !aligned16(packed)) return fail(MXS_ERR_ALIGN, "w and packed must be 16-byte aligned");
+    if (N == 0) return MXS_OK;
+    if ((rc = check_device())) return rc;
+    return launch_pack_weight(p, w, N, ld_w, rounding, layout == MXS_W_COMPACT_AND_PLANES, packed,
+                              static_cast<cudaStream_t>(stream));
+}
+
+int mxs_gemm_decode(const void *codes, const uint8_t *scales, const uint8_t *bits, const void *packed_w,
+                    int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, void *ws, size_t ws_bytes,
+                    void *stream) {
+    Plan p;
+    int rc = build_plan(bits, K, &p);
+    if (rc) return rc;
+    if (M < 0 || N < 0) return fail(MXS_ERR_SHAPE, "M=%lld N=%lld", (long long)M, (long long)N);
+    if (M > 16) return fail(MXS_ERR_SHAPE, "decode path takes M <= 16 (M=%lld)", (long long)M);
+    if (!codes || !scales || !packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
+    if (ld_y < N) return fail(MXS_ERR_INVALID_ARG, "ld_y=%lld < N", (long long)ld_y);
+    if (!aligned16(codes) || !aligned16(packed_w) || (reinterpret_cast<uintptr_t>(y) & 3))
+        return fail(MXS_ERR_ALIGN, "codes/packed_w must be 16-byte aligned, y 4-byte aligned");
+    const int64_t need = decode_workspace_bytes(p, M, N);
+    if ((int64_t)ws_bytes < need || (need > 0 && !ws))
+        return fail(MXS_ERR_BUFFER, "workspace of %lld bytes needed, %zu given", (long long)need, ws_bytes);
+    if (ws && !aligned16(ws)) return fail(MXS_ERR_ALIGN, "workspace must be 16-byte aligned");
+    if (M == 0 || N == 0) return MXS_OK;
+    if ((rc = check_device())) return rc;
+    return launch_gemm_decode(p, codes, scales, packed_w, M, N, y, ld_y, ws, ws_bytes,
+                              static_cast<cudaStream_t>(stream));
+}
+
+int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const void *act_planes, const uint8_t *act_bits,
+             const void *packed_w, int w_layout, const uint8_t *w_bits, int64_t M, int64_t N, int64_t K, float *y,
+             int64_t ld_y, void *ws, size_t ws_bytes, void *stream) {
+    Plan p;
+    int rc = build_plan(act_bits, K, &p);
+    if (rc) return rc;
+    if (!w_bits) return fail(MXS_ERR_INVALID_ARG, "w_bits is NULL");
+    if (act_bits != w_bits && std::memcmp(act_bits, w_bits, (size_t)p.nb) != 0)
+        return fail(MXS_ERR_UNSUPPORTED, "activation and weight maps differ; one map per layer is supported");
+    if (w_layout != MXS_W_COMPACT && w_layout != MXS_W_COMPACT_AND_PLANES)
+        return fail(MXS_ERR_INVALID_ARG, "w_layout=%d", w_layout);
+    if (M <= 16)
+        return mxs_gemm_decode(act_codes, act_scales, act_bits, packed_w, M, N, K, y, ld_y, ws, ws_bytes, stream);
+    if (w_layout != MXS_W_COMPACT_AND_PLANES)
+        return fail(MXS_ERR_INVALID_ARG, "M > 16 needs a weight packed with MXS_W_COMPACT_AND_PLANES");
+    return mxs_gemm_prefill(act_planes, act_bits, packed_w, M, N, K, y, ld_y, stream);
+}
+
+static int prefill_checked(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M, int64_t N,
+                           int64_t K, float *y, int64_t ld_y, int starve, void *stream) {
+    Plan p;
+    int rc = build_plan(bits, K, &p);
+    if (rc) return rc;
+    if (M < 0 || N < 0) return fail(MXS_ERR_SHAPE, "M=%lld N=%lld", (long long)M, (long long)N);
+    if (!act_planes || !packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
+    if (ld_y < N) return fail(MXS_ERR_INVALID_ARG, "ld_y=%lld < N", (long long)ld_y);
+    if (!aligned16(act_planes) || !aligned16(packed_w) || (reinterpret_cast<uintptr_t>(y) & 3))
+        return fail(MXS_ERR_ALIGN, "act_planes/packed_w must be 16-byte aligned, y 4-byte aligned");
+    if (M == 0 || N == 0) return MXS_OK;
+    if ((rc = check_device())) return rc;
+    return launch_gemm_prefill(p, act_planes, packed_w, M, N, y, ld_y, starve, static_cast<cudaStream_t>(stream));
+}
+
+int mxs_gemm_prefill(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M, int64_t N,
+                     int64_t K, float *y, int64_t ld_y, void *stream) {
+    return prefill_checked(act_planes, bits, packed_w, M, N, K, y, ld_y, 0, stream);
+}
+
+int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M, int64_t N,
+                            int64_t K, float *y, int64_t ld_y, int stage, void *stream) {
+    if (stage < 1) return fail(MXS_ERR_INVALID_ARG, "stage=%d must be >= 1", stage);
+    return prefill_checked(act_planes, bits, packed_w, M, N, K, y, ld_y, stage, stream);
+}
+
+int mxs_device_status(int *status, int reset, void *stream) {
+    if (!status) return fail(MXS_ERR_INVALID_ARG, "status is NULL");
+    int rc = check_device();
+    if (rc) return rc;
+    return prefill_status(status, reset, static_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

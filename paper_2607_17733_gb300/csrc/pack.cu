@@ -1,0 +1,143 @@
+// pack.cu -- A2: offline quantization and packing of a weight matrix.
+//
+// Same MXINT rule as the activations (Appendix A.2: weights and activations
+// of every linear layer are quantized; Sec. 4.1: one width per 32-element
+// block).  One thread owns one (row, slot) block: it loads the 32 bf16 values
+// with four 128-bit loads and scatters the codes into the 16-row fragment
+// tiles read by the decode kernel, the scale byte, and optionally the e4m3
+// digit planes and scale tiles read by the tensor-core prefill kernel.  The
+// buffer is cleared first, so padding rows and slots read as zero.  This runs
+// once per layer and is not on the timed path.
+#include "common.cuh"
+
+namespace mxs {
+namespace {
+
+struct PackArgs {
+    const uint16_t *w;
+    int64_t N, ld;
+    int rhaz, with_planes;
+    uint8_t *out;
+    WeightOffsets off;
+};
+
+__global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant__ Plan p,
+                                                          const __grid_constant__ PackArgs a) {
+    const int64_t gid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t n = gid / p.nb;
+    const int s = (int)(gid - n * p.nb);
+    if (n >= a.N) return;
+    const int kb = p.slot_block[s];
+    const int b = slot_width(p, s);
+
+    uint32_t h[32];
+    const uint4 *src = reinterpret_cast<const uint4 *>(a.w + n * a.ld + kBlock * kb);
+    uint32_t mag = 0;
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+        const uint4 u = __ldg(src + v);
+        const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            h[8 * v + 2 * i] = w4[i] & 0xFFFF;
+            h[8 * v + 2 * i + 1] = w4[i] >> 16;
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 32; ++i) mag = max(mag, h[i] & 0x7FFF);
+    const int S = (int)(mag >> 7);
+    int m[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) m[i] = S == 255 ? 0 : quant_elem(h[i], S, b, a.rhaz);
+
+    const int64_t t = n >> 4;
+    const int rr = (int)(n & 15), g = rr & 7, hh = rr >> 3;
+    if (b == 4) {
+        uint8_t *chunk = a.out + (t * p.n4 + s) * 256;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint32_t word = 0;
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                word |= (uint32_t)(((m[4 * q + j] & 0xF) << 4) | (m[16 + 4 * q + j] & 0xF)) << (8 * j);
+            *reinterpret_cast<uint32_t *>(chunk + 8 * (4 * g + q) + 4 * hh) = word;
+        }
+    } else {
+        uint8_t *chunk = a.out + a.off.o8 + (t * p.n68 + (s - p.n4)) * 512;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint32_t w0 = 0, w1 = 0;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                w0 |= (uint32_t)(m[4 * q + j] & 0xFF) << (8 * j);
+                w1 |= (uint32_t)(m[16 + 4 * q + j] & 0xFF) << (8 * j);
+            }
+            uint8_t *lane = chunk + 16 * (4 * g + q);
+            *reinterpret_cast<uint32_t *>(lane + 4 * hh) = w0;
+            *reinterpret_cast<uint32_t *>(lane + 4 * (2 + hh)) = w1;
+        }
+    }
+    a.out[a.off.os + n * p.nb + s] = (uint8_t)S;
+
+    if (a.with_planes) {
+        uint8_t *prow = a.out + a.off.planes + n * p.kp;
+        int st, q;
+        if (b == 4) {
+            uint32_t *dst = reinterpret_cast<uint32_t *>(prow + 32 * (int64_t)s);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const uint16_t c0 = e4m3x2(0.25f * m[4 * i], 0.25f * m[4 * i + 1]);
+                const uint16_t c1 = e4m3x2(0.25f * m[4 * i + 2], 0.25f * m[4 * i + 3]);
+                dst[i] = c0 | ((uint32_t)c1 << 16);
+            }
+            st = s >> 2;
+            q = s & 3;
+        } else {
+            const int j = s - p.n4;
+            const int sh = b == 6 ? 3 : 4;
+            const float fh = b == 6 ? 0.5f : 0.25f, fl = b == 6 ? 0.0625f : 0.015625f;
+            uint32_t *hi = reinterpret_cast<uint32_t *>(prow + 128 * (int64_t)p.st4 + 64 * (int64_t)j);
+            uint32_t *lo = hi + 8;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                int hd[4], ld[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    hd[k] = m[4 * i + k] >> sh;
+                    ld[k] = m[4 * i + k] & ((1 << sh) - 1);
+                }
+                hi[i] = e4m3x2(fh * hd[0], fh * hd[1]) | ((uint32_t)e4m3x2(fh * hd[2], fh * hd[3]) << 16);
+                lo[i] = e4m3x2(fl * ld[0], fl * ld[1]) | ((uint32_t)e4m3x2(fl * ld[2], fl * ld[3]) << 16);
+            }
+            st = p.st4 + (j >> 1);
+            q = j & 1;
+        }
+        const int64_t tile = n >> 7;
+        const int r = (int)(n & 127);
+        a.out[a.off.sf + ((tile * p.nst + st) * 32 + (r & 31)) * 16 + 4 * (r >> 5) + q] = (uint8_t)S;
+    }
+}
+
+}  // namespace
+
+int launch_pack_weight(const Plan &p, const void *w, int64_t N, int64_t ld, int rounding, bool planes,
+                       void *packed, cudaStream_t st) {
+    PackArgs a;
+    a.w = static_cast<const uint16_t *>(w);
+    a.N = N;
+    a.ld = ld;
+    a.rhaz = rounding == MXS_RHAZ;
+    a.with_planes = planes;
+    a.out = static_cast<uint8_t *>(packed);
+    a.off = weight_offsets(p, N, planes);
+    cudaError_t e = cudaMemsetAsync(packed, 0, (size_t)a.off.total, st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(packed)");
+    const int64_t threads = N * p.nb;
+    if (threads == 0) return MXS_OK;
+    const int64_t blocks = (threads + 255) / 256;
+    if (blocks > 0x7FFFFFFF) return fail(MXS_ERR_SHAPE, "pack_weight: problem too large");
+    pack_weight_kernel<<<(unsigned)blocks, 256, 0, st>>>(p, a);
+    return cuda_fail(cudaGetLastError(), "pack_weight_kernel launch");
+}
+
+}  // namespace mxs

@@ -1,0 +1,238 @@
+"""Thin ctypes binding of libmxs (include/mxs.h).
+
+Argument marshalling only: every step of the quantize / pack / GEMM path runs
+in the library's CUDA kernels.  torch supplies device memory and the current
+stream.  There is no fallback: if libmxs.so is missing or the device is not
+sm_103a, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+
+MXS_OK = 0
+ERRORS = {1: "INVALID_ARG", 2: "SHAPE", 3: "BITS", 4: "ALIGN", 5: "BUFFER", 6: "CUDA",
+          7: "TIMEOUT", 8: "UNSUPPORTED"}
+RNE, RHAZ = 0, 1
+W_COMPACT, W_COMPACT_AND_PLANES = 0, 1
+MAX_K = 65536
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libmxs.so")
+EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_bytes",
+           "mxs_act_planes_bytes", "mxs_weight_bytes", "mxs_gemm_workspace_bytes",
+           "mxs_quantize_act", "mxs_pack_weight", "mxs_gemm", "mxs_gemm_decode",
+           "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve"]
+
+_lock = threading.Lock()
+_lib = None
+
+
+class MxsError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"MXS_ERR_{ERRORS.get(code, code)}: {msg}")
+        self.code = code
+
+
+def lib() -> ctypes.CDLL:
+    """Load libmxs.so (built by paper_2607_17733_gb300.build)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: run `python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(LIB_PATH)
+        P, I64, I, SZ = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_size_t
+        L.mxs_last_error.restype = ctypes.c_char_p
+        L.mxs_last_error.argtypes = []
+        L.mxs_version.restype = I
+        for name in ("mxs_act_row_bytes",):
+            getattr(L, name).argtypes = [I64, P]
+            getattr(L, name).restype = I64
+        for name in ("mxs_act_codes_bytes", "mxs_act_planes_bytes"):
+            getattr(L, name).argtypes = [I64, I64, P]
+            getattr(L, name).restype = I64
+        L.mxs_weight_bytes.argtypes = [I64, I64, P, I]
+        L.mxs_weight_bytes.restype = I64
+        L.mxs_gemm_workspace_bytes.argtypes = [I64, I64, I64, P]
+        L.mxs_gemm_workspace_bytes.restype = I64
+        L.mxs_quantize_act.argtypes = [P, I64, I64, I64, P, I, P, P, P, P]
+        L.mxs_quantize_act.restype = I
+        L.mxs_pack_weight.argtypes = [P, I64, I64, I64, P, I, I, P, P]
+        L.mxs_pack_weight.restype = I
+        L.mxs_gemm.argtypes = [P, P, P, P, P, I, P, I64, I64, I64, P, I64, P, SZ, P]
+        L.mxs_gemm.restype = I
+        L.mxs_gemm_decode.argtypes = [P, P, P, P, I64, I64, I64, P, I64, P, SZ, P]
+        L.mxs_gemm_decode.restype = I
+        L.mxs_gemm_prefill.argtypes = [P, P, P, I64, I64, I64, P, I64, P]
+        L.mxs_gemm_prefill.restype = I
+        L.mxs_test_prefill_starve.argtypes = [P, P, P, I64, I64, I64, P, I64, I, P]
+        L.mxs_test_prefill_starve.restype = I
+        L.mxs_device_status.argtypes = [ctypes.POINTER(ctypes.c_int), I, P]
+        L.mxs_device_status.restype = I
+        _lib = L
+        return L
+
+
+def last_error() -> str:
+    return lib().mxs_last_error().decode()
+
+
+def check(rc: int) -> None:
+    if rc != MXS_OK:
+        raise MxsError(rc, last_error())
+
+
+def _size(v: int) -> int:
+    if v < 0:
+        raise MxsError(-v, last_error())
+    return int(v)
+
+
+class _Bits:
+    """Host copy of a width map, kept alive for the duration of a call."""
+
+    def __init__(self, bits):
+        self.arr = np.ascontiguousarray(np.asarray(bits, dtype=np.uint8))
+        self.ptr = self.arr.ctypes.data
+
+    def __len__(self):
+        return self.arr.size
+
+
+def _ptr(t) -> int | None:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    import torch
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+# ------------------------------------------------------------------ sizes
+def act_row_bytes(K: int, bits) -> int:
+    b = _Bits(bits)
+    return _size(lib().mxs_act_row_bytes(K, b.ptr))
+
+
+def act_codes_bytes(M: int, K: int, bits) -> int:
+    b = _Bits(bits)
+    return _size(lib().mxs_act_codes_bytes(M, K, b.ptr))
+
+
+def act_planes_bytes(M: int, K: int, bits) -> int:
+    b = _Bits(bits)
+    return _size(lib().mxs_act_planes_bytes(M, K, b.ptr))
+
+
+def weight_bytes(N: int, K: int, bits, layout: int = W_COMPACT) -> int:
+    b = _Bits(bits)
+    return _size(lib().mxs_weight_bytes(N, K, b.ptr, layout))
+
+
+def gemm_workspace_bytes(M: int, N: int, K: int, bits) -> int:
+    b = _Bits(bits)
+    return _size(lib().mxs_gemm_workspace_bytes(M, N, K, b.ptr))
+
+
+# ------------------------------------------------------------------ calls
+def quantize_act(x, bits, rounding: int = RNE, codes=None, scales=None, planes=None,
+                 want_codes: bool = True, want_planes: bool = False, stream=None):
+    """x: bf16 [M, K] CUDA tensor (row stride may exceed K).  Returns
+    (codes uint8 [M, row_bytes] | None, scales uint8 [M, K/32] | None, planes uint8 | None)."""
+    import torch
+    M, K = x.shape
+    b = _Bits(bits)
+    if want_codes and codes is None:
+        codes = torch.empty((M, act_row_bytes(K, b.arr)), dtype=torch.uint8, device=x.device)
+        scales = torch.empty((M, K // 32), dtype=torch.uint8, device=x.device)
+    if want_planes and planes is None:
+        planes = torch.empty(act_planes_bytes(M, K, b.arr), dtype=torch.uint8, device=x.device)
+    check(lib().mxs_quantize_act(_ptr(x), M, K, x.stride(0), b.ptr, rounding, _ptr(codes), _ptr(scales),
+                                 _ptr(planes), _stream(stream)))
+    return codes, scales, planes
+
+
+def pack_weight(w, bits, layout: int = W_COMPACT, rounding: int = RNE, out=None, stream=None):
+    """w: bf16 [N, K] CUDA tensor -> packed uint8 buffer."""
+    import torch
+    N, K = w.shape
+    b = _Bits(bits)
+    if out is None:
+        out = torch.empty(weight_bytes(N, K, b.arr, layout), dtype=torch.uint8, device=w.device)
+    check(lib().mxs_pack_weight(_ptr(w), N, K, w.stride(0), b.ptr, rounding, layout, _ptr(out),
+                                _stream(stream)))
+    return out
+
+
+def gemm(codes, scales, planes, bits, packed_w, N: int, w_layout: int = W_COMPACT, y=None,
+         workspace=None, M: int | None = None, K: int | None = None, stream=None):
+    """y [M, N] fp32 = x W^T on quantized operands (decode kernel for M <= 16)."""
+    import torch
+    b = _Bits(bits)
+    K = 32 * len(b) if K is None else K
+    if M is None:
+        M = (codes if codes is not None else planes).shape[0] if codes is not None else M
+    dev = packed_w.device
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float32, device=dev)
+    ws_need = gemm_workspace_bytes(M, N, K, b.arr)
+    if workspace is None and ws_need > 0:
+        workspace = torch.empty(ws_need, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    check(lib().mxs_gemm(_ptr(codes), _ptr(scales), _ptr(planes), b.ptr, _ptr(packed_w), w_layout, b.ptr,
+                         M, N, K, _ptr(y), y.stride(0), _ptr(workspace), ws_bytes, _stream(stream)))
+    return y
+
+
+def gemm_decode(codes, scales, bits, packed_w, N: int, y=None, workspace=None, stream=None):
+    import torch
+    b = _Bits(bits)
+    M = codes.shape[0]
+    K = 32 * len(b)
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float32, device=packed_w.device)
+    ws_need = gemm_workspace_bytes(M, N, K, b.arr)
+    if workspace is None and ws_need > 0:
+        workspace = torch.empty(ws_need, dtype=torch.uint8, device=packed_w.device)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    check(lib().mxs_gemm_decode(_ptr(codes), _ptr(scales), b.ptr, _ptr(packed_w), M, N, K, _ptr(y),
+                                y.stride(0), _ptr(workspace), ws_bytes, _stream(stream)))
+    return y
+
+
+def gemm_prefill(planes, bits, packed_w, M: int, N: int, y=None, stream=None):
+    """Tensor-core path: planes from quantize_act(want_planes=True), weights
+    packed with W_COMPACT_AND_PLANES."""
+    import torch
+    b = _Bits(bits)
+    K = 32 * len(b)
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float32, device=packed_w.device)
+    check(lib().mxs_gemm_prefill(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), y.stride(0),
+                                 _stream(stream)))
+    return y
+
+
+def test_prefill_starve(planes, bits, packed_w, M: int, N: int, stage: int, y=None, stream=None):
+    """Test hook: the prefill kernel with K' stage `stage` never loaded."""
+    import torch
+    b = _Bits(bits)
+    K = 32 * len(b)
+    if y is None:
+        y = torch.zeros((M, N), dtype=torch.float32, device=packed_w.device)
+    check(lib().mxs_test_prefill_starve(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), y.stride(0),
+                                        int(stage), _stream(stream)))
+    return y
+
+
+def device_status(reset: bool = False, stream=None) -> int:
+    st = ctypes.c_int(0)
+    check(lib().mxs_device_status(ctypes.byref(st), int(reset), _stream(stream)))
+    return st.value

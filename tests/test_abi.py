@@ -1,0 +1,113 @@
+"""The C ABI: exports, size queries and argument validation (no GPU needed).
+
+Validation happens before any CUDA call, so every error path below runs the
+same on a machine without a GPU."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import mxo
+from paper_2607_17733_gb300 import build as B
+from paper_2607_17733_gb300 import mxs
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    B.build()
+    return mxs.lib()
+
+
+def header_functions():
+    text = open(os.path.join(ROOT, "include", "mxs.h")).read()
+    return sorted(set(re.findall(r"MXS_API\s+[\w\s\*]*?\b(mxs_\w+)\s*\(", text)))
+
+
+def test_every_declared_function_is_exported(L):
+    names = header_functions()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(L, n), n
+    assert sorted(mxs.EXPORTS) == names
+    assert L.mxs_version() == 1
+
+
+def _bits(nb, seed=0, p=(0.7, 0.2, 0.1)):
+    rs = np.random.default_rng(seed)
+    return rs.choice(np.array([4, 6, 8], np.uint8), size=nb, p=p)
+
+
+@pytest.mark.parametrize("K", [32, 96, 4096, 14336])
+def test_sizes_match_the_storage_format(L, K):
+    bits = _bits(K // 32, K)
+    n4 = int(np.sum(bits == 4))
+    assert mxs.act_row_bytes(K, bits) == 16 * n4 + 32 * (K // 32 - n4)
+    assert mxs.act_codes_bytes(7, K, bits) == 7 * (16 * n4 + 32 * (K // 32 - n4))
+    for N in (1, 16, 37, 1000):
+        for layout in (0, 1):
+            assert mxs.weight_bytes(N, K, bits, layout) == mxo.weight_bytes(N, K, bits, bool(layout))
+    kp, nst = mxo.plane_shape(bits)
+    M = 130
+    sf_off = (M * kp + 255) // 256 * 256
+    assert mxs.act_planes_bytes(M, K, bits) == (sf_off + 2 * nst * 512 + 255) // 256 * 256
+
+
+def test_size_queries_reject_bad_arguments(L):
+    bits = np.full(4, 4, np.uint8)
+    assert L.mxs_act_row_bytes(100, bits.ctypes.data) == -2  # K not a multiple of 32
+    assert L.mxs_act_row_bytes(0, bits.ctypes.data) == -2
+    assert L.mxs_act_row_bytes(65536 + 32, bits.ctypes.data) == -2
+    bad = np.array([4, 5, 6, 8], np.uint8)
+    assert L.mxs_act_row_bytes(128, bad.ctypes.data) == -3
+    assert "bits[1]=5" in mxs.last_error()
+    assert L.mxs_act_row_bytes(128, None) == -1
+    assert L.mxs_weight_bytes(16, 128, bits.ctypes.data, 7) == -1
+    assert L.mxs_act_codes_bytes(-1, 128, bits.ctypes.data) == -2
+
+
+FAKE = 1 << 20  # an aligned address that is never dereferenced: validation fails first
+
+
+def test_quantize_validation(L):
+    bits = np.full(4, 4, np.uint8)
+    b = bits.ctypes.data
+    q = L.mxs_quantize_act
+    assert q(FAKE, 4, 100, 100, b, 0, FAKE, FAKE, None, None) == 2
+    assert q(FAKE, 4, 128, 128, np.full(4, 7, np.uint8).ctypes.data, 0, FAKE, FAKE, None, None) == 3
+    assert q(FAKE, 4, 128, 120, b, 0, FAKE, FAKE, None, None) == 1   # ld_x < K
+    assert q(FAKE, 4, 128, 132, b, 0, FAKE, FAKE, None, None) == 1   # ld_x not a multiple of 8
+    assert q(FAKE, 4, 128, 128, b, 2, FAKE, FAKE, None, None) == 1   # rounding
+    assert q(FAKE, 4, 128, 128, b, 0, None, None, None, None) == 1   # no output
+    assert q(FAKE, 4, 128, 128, b, 0, FAKE, None, None, None) == 1   # codes without scales
+    assert q(FAKE + 8, 4, 128, 128, b, 0, FAKE, FAKE, None, None) == 4
+    assert q(FAKE, 4, 128, 128, b, 0, FAKE, FAKE, FAKE + 4, None) == 4
+    assert q(FAKE, 0, 128, 128, b, 0, FAKE, FAKE, None, None) == 0   # M = 0: nothing to do
+
+
+def test_pack_and_gemm_validation(L):
+    bits = np.full(4, 4, np.uint8)
+    b = bits.ctypes.data
+    assert L.mxs_pack_weight(FAKE, 16, 128, 128, b, 0, 3, FAKE, None) == 1
+    assert L.mxs_pack_weight(FAKE, 16, 128, 128, b, 0, 0, None, None) == 1
+    assert L.mxs_pack_weight(FAKE, 16, 128, 128, b, 0, 0, FAKE + 2, None) == 4
+    other = np.array([4, 4, 8, 4], np.uint8)
+    g = L.mxs_gemm
+    assert g(FAKE, FAKE, None, b, FAKE, 0, other.ctypes.data, 4, 16, 128, FAKE, 16, None, 0, None) == 8
+    d = L.mxs_gemm_decode
+    assert d(FAKE, FAKE, b, FAKE, 17, 16, 128, FAKE, 16, None, 0, None) == 2   # M > 16
+    assert d(FAKE, FAKE, b, FAKE, 4, 16, 128, FAKE, 8, None, 0, None) == 1     # ld_y < N
+    assert d(FAKE, FAKE, b, None, 4, 16, 128, FAKE, 16, None, 0, None) == 1
+    assert d(FAKE, FAKE, b, FAKE, 4, 16, 128, FAKE + 2, 16, None, 0, None) == 4
+
+
+def test_valid_call_without_gpu_reports_cuda_error(L):
+    torch = pytest.importorskip("torch")
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    bits = np.full(4, 4, np.uint8)
+    rc = L.mxs_quantize_act(FAKE, 4, 128, 128, bits.ctypes.data, 0, FAKE, FAKE, None, None)
+    assert rc == 6 and "cudaGetDevice" in mxs.last_error()

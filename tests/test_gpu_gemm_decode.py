@@ -1,0 +1,116 @@
+"""A4 parity: the decode GEMM (M <= 16) against the exact CPU oracle."""
+import numpy as np
+import pytest
+
+from oracle import mxo
+from paper_2607_17733_gb300 import inputs as I
+from paper_2607_17733_gb300 import mxs
+import gpu_util as U
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    return U.torch_or_skip()
+
+
+def layer(torch, M, K, N, bits, g, w_sigma=0.02, outlier_frac=0.01, outlier_scale=30.0):
+    xb = I.activations_bf16(M, bits, g, outlier_frac, outlier_scale=outlier_scale)
+    wb = I.normal_bf16((N, K), w_sigma, g)
+    codes, scales, _ = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits)
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
+    return xb, wb, codes, scales, packed
+
+
+def oracle_full(xb, wb, bits):
+    a_s, a_c = mxo.quantize_bf16(xb, bits)
+    w_s, w_c = mxo.quantize_bf16(wb, bits)
+    return mxo.gemm(bits, a_c, a_s, w_c, w_s)
+
+
+@pytest.mark.parametrize("M", [1, 2, 4, 7, 8, 9, 16])
+@pytest.mark.parametrize("N,nb", [(16, 1), (37, 5), (200, 40), (1000, 128)])
+def test_decode_small(torch, M, N, nb):
+    g = I.rng(M, N, nb)
+    bits = I.width_map(nb, 0.7, 0.2, 0.1, g)
+    xb, wb, codes, scales, packed = layer(torch, M, 32 * nb, N, bits, g)
+    y = mxs.gemm(codes, scales, None, bits, packed, N)
+    ref, ab = oracle_full(xb, wb, bits)
+    U.check_gemm(y.cpu().numpy(), ref, ab)
+
+
+@pytest.mark.parametrize("p", [(1, 0, 0), (0, 1, 0), (0, 0, 1), (0.5, 0.3, 0.2)])
+def test_decode_uniform_and_mixed_maps(torch, p):
+    g = I.rng(7, int(10 * p[0]))
+    bits = I.width_map(96, *p, g)
+    xb, wb, codes, scales, packed = layer(torch, 16, 3072, 300, bits, g)
+    y = mxs.gemm(codes, scales, None, bits, packed, 300)
+    ref, ab = oracle_full(xb, wb, bits)
+    U.check_gemm(y.cpu().numpy(), ref, ab)
+
+
+def test_decode_output_stride_and_determinism(torch):
+    g = I.rng(8, 8)
+    bits = I.width_map(64, 0.8, 0.15, 0.05, g)
+    xb, wb, codes, scales, packed = layer(torch, 5, 2048, 130, bits, g)
+    y = torch.full((5, 160), -7.0, device="cuda")
+    mxs.gemm(codes, scales, None, bits, packed, 130, y=y[:, :130])
+    y2 = mxs.gemm(codes, scales, None, bits, packed, 130)
+    torch.cuda.synchronize()
+    yh = y.cpu().numpy()
+    assert np.all(yh[:, 130:] == -7.0)
+    assert np.array_equal(yh[:, :130], y2.cpu().numpy())
+    ref, ab = oracle_full(xb, wb, bits)
+    U.check_gemm(yh[:, :130], ref, ab)
+
+
+def test_decode_nan_block(torch):
+    bits = np.array([4, 8, 6, 4], np.uint8)
+    g = I.rng(9)
+    xb = I.activations_bf16(3, bits, g, 0.0)
+    xb[1, 40] = 0x7FC0  # NaN in block 1 of token 1
+    wb = I.normal_bf16((20, 128), 0.02, g)
+    codes, scales, _ = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits)
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
+    y = mxs.gemm(codes, scales, None, bits, packed, 20).cpu().numpy()
+    ref, ab = oracle_full(xb, wb, bits)
+    assert np.all(np.isnan(y[1])) and not np.isnan(y[[0, 2]]).any()
+    U.check_gemm(y, ref, ab)
+
+
+LLAMA3 = {name: (K, N) for name, K, N in I.LLAMA3_8B}
+
+
+@pytest.mark.parametrize("proj", ["q", "k", "o", "gate", "down"])
+@pytest.mark.parametrize("M", [1, 4, 16])
+def test_decode_llama3_8b_full_size(torch, proj, M):
+    """8B decode projections at full size; map 85/10/5, 1% outlier columns x30.
+    Every output is checked for M=1/4, 2048 sampled columns for M=16."""
+    K, N = LLAMA3[proj]
+    g = I.rng(1, K, N, M)
+    bits = I.width_map(K // 32, 0.85, 0.10, 0.05, g)
+    xb, wb, codes, scales, packed = layer(torch, M, K, N, bits, g)
+    y = mxs.gemm(codes, scales, None, bits, packed, N).cpu().numpy()
+    a_s, a_c = mxo.quantize_bf16(xb, bits)
+    cols = np.arange(N) if M < 16 or N <= 2048 else np.sort(np.random.default_rng(0).choice(N, 2048, replace=False))
+    w_s, w_c = mxo.quantize_bf16(wb[cols], bits)
+    ref, ab = mxo.gemm(bits, a_c, a_s, w_c, w_s)
+    U.check_gemm(y[:, cols], ref, ab)
+
+
+@pytest.mark.parametrize("maps", ["u4", "u8", "90/5/5", "50/30/20-clustered"])
+def test_decode_sweep_70b_shape_sampled(torch, maps):
+    """K=8192, N=28672, M=16 (bitwidth sweep shape), 1% outliers x50; 512 columns."""
+    K, N, M = 8192, 28672, 16
+    g = I.rng(4, len(maps))
+    p = {"u4": (1, 0, 0), "u8": (0, 0, 1), "90/5/5": (0.9, 0.05, 0.05),
+         "50/30/20-clustered": (0.5, 0.3, 0.2)}[maps]
+    bits = I.width_map(K // 32, *p, g, clustered=maps.endswith("clustered"))
+    xb, wb, codes, scales, packed = layer(torch, M, K, N, bits, g, outlier_scale=50.0)
+    y = mxs.gemm(codes, scales, None, bits, packed, N).cpu().numpy()
+    cols = np.sort(np.random.default_rng(1).choice(N, 512, replace=False))
+    a_s, a_c = mxo.quantize_bf16(xb, bits)
+    w_s, w_c = mxo.quantize_bf16(wb[cols], bits)
+    ref, ab = mxo.gemm(bits, a_c, a_s, w_c, w_s)
+    U.check_gemm(y[:, cols], ref, ab)

@@ -1,0 +1,101 @@
+"""A3 parity: the tcgen05 prefill GEMM (e4m3 digit planes, block-scaled MMA,
+fp32 TMEM accumulation) against the exact CPU oracle."""
+import numpy as np
+import pytest
+
+from oracle import mxo
+from paper_2607_17733_gb300 import inputs as I
+from paper_2607_17733_gb300 import mxs
+import gpu_util as U
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    return U.torch_or_skip()
+
+
+def prep(torch, xb, wb, bits):
+    _, _, planes = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits, want_codes=False, want_planes=True)
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits, layout=mxs.W_COMPACT_AND_PLANES)
+    return planes, packed
+
+
+def oracle_entries(xb, wb, bits, rows=None, cols=None):
+    if rows is not None:
+        xb = xb[rows]
+    if cols is not None:
+        wb = wb[cols]
+    a_s, a_c = mxo.quantize_bf16(xb, bits)
+    w_s, w_c = mxo.quantize_bf16(wb, bits)
+    return mxo.gemm(bits, a_c, a_s, w_c, w_s)
+
+
+MAPS = {"u4": (1, 0, 0), "u6": (0, 1, 0), "u8": (0, 0, 1), "mix": (0.8, 0.15, 0.05), "heavy": (0.5, 0.3, 0.2)}
+
+
+@pytest.mark.parametrize("M,N,nb", [(128, 256, 4), (17, 16, 1), (130, 300, 9), (300, 520, 40), (256, 1024, 128)])
+@pytest.mark.parametrize("mp", list(MAPS))
+def test_prefill_small(torch, M, N, nb, mp):
+    g = I.rng(M, N, nb, len(mp))
+    bits = I.width_map(nb, *MAPS[mp], g)
+    xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=50.0)
+    wb = I.normal_bf16((N, 32 * nb), 0.02, g)
+    planes, packed = prep(torch, xb, wb, bits)
+    y = mxs.gemm_prefill(planes, bits, packed, M, N).cpu().numpy()
+    ref, ab = oracle_entries(xb, wb, bits)
+    err = U.check_gemm(y, ref, ab)
+    print(f"prefill M={M} N={N} K={32 * nb} map={mp}: max err/abssum {err:.2e}")
+
+
+def test_prefill_through_mxs_gemm_and_stride(torch):
+    g = I.rng(21)
+    bits = I.width_map(32, 0.8, 0.15, 0.05, g)
+    M, N = 200, 384
+    xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=50.0)
+    wb = I.normal_bf16((N, 1024), 0.02, g)
+    planes, packed = prep(torch, xb, wb, bits)
+    y = torch.full((M, N + 64), -3.0, device="cuda")
+    mxs.gemm(None, None, planes, bits, packed, N, w_layout=mxs.W_COMPACT_AND_PLANES, y=y[:, :N], M=M)
+    yh = y.cpu().numpy()
+    assert np.all(yh[:, N:] == -3.0)
+    ref, ab = oracle_entries(xb, wb, bits)
+    U.check_gemm(yh[:, :N], ref, ab)
+
+
+@pytest.mark.parametrize("shape", [("llama3-8b-gate", 2048, 4096, 14336, (0.8, 0.15, 0.05)),
+                                   ("llama3-8b-down", 2048, 14336, 4096, (0.8, 0.15, 0.05)),
+                                   ("single-layer", 128, 4096, 4096, (0.8, 0.15, 0.05))])
+def test_prefill_full_size_sampled(torch, shape):
+    name, M, K, N, p = shape
+    g = I.rng(2, M, K, N)
+    bits = I.width_map(K // 32, *p, g)
+    xb = I.activations_bf16(M, bits, g, 0.005, student_t=True)
+    wb = I.normal_bf16((N, K), 0.02, g)
+    planes, packed = prep(torch, xb, wb, bits)
+    y = mxs.gemm_prefill(planes, bits, packed, M, N).cpu().numpy()
+    rs = np.random.default_rng(0)
+    rows = np.sort(rs.choice(M, min(M, 96), replace=False))
+    cols = np.sort(rs.choice(N, min(N, 512), replace=False))
+    ref, ab = oracle_entries(xb, wb, bits, rows, cols)
+    err = U.check_gemm(y[np.ix_(rows, cols)], ref, ab)
+    print(f"prefill {name}: max err/abssum {err:.2e}")
+
+
+def test_prefill_bounded_wait_reports_timeout(torch):
+    """A stage that is never loaded: the kernel gives up after its wait bound,
+    records MXS_ERR_TIMEOUT, frees its tensor memory and the context stays usable."""
+    g = I.rng(31)
+    bits = I.width_map(16, 1, 0, 0, g)
+    M, N = 128, 256
+    xb = I.activations_bf16(M, bits, g, 0.0)
+    wb = I.normal_bf16((N, 512), 0.02, g)
+    planes, packed = prep(torch, xb, wb, bits)
+    assert mxs.device_status(reset=True) in (0, mxs.MXS_OK, 7)
+    mxs.test_prefill_starve(planes, bits, packed, M, N, stage=2)
+    assert mxs.device_status(reset=True) == 7
+    assert mxs.device_status() == 0
+    y = mxs.gemm_prefill(planes, bits, packed, M, N).cpu().numpy()  # the context still works
+    ref, ab = oracle_entries(xb, wb, bits)
+    U.check_gemm(y, ref, ab)
