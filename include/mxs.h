@@ -41,7 +41,9 @@
  *     4-bit slot s: bytes [16s, 16s+16), element i in byte i/2 (low nibble for
  *     even i), two's complement; 6/8-bit slot s: bytes [16*n4 + 32(s-n4), +32),
  *     one int8 per element.  Activation scales: uint8 [M, K/32] by slot.
- *   Weight buffer (layout MXS_W_COMPACT): rows padded to Np = 16*ceil(N/16),
+ *   Weight buffer (layout MXS_W_COMPACT): codes are sign-magnitude, a 4-bit
+ *     code as (sign<<3)|m and a 6/8-bit code as (sign<<7)|m (the symmetric
+ *     clamp never yields -2^(b-1)); rows padded to Np = 16*ceil(N/16),
  *     cut into tiles of 16 rows; inside a tile one block of all 16 rows is
  *     stored in the order a warp holds the A operand of a 16x8x32 integer MMA
  *     (lane l = 4g+q: rows g, g+8; elements 4q..4q+3 and 16+4q..16+4q+3):

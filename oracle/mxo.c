@@ -317,11 +317,13 @@ int mxo_pack_act(int64_t R, int64_t K, const uint8_t *bits, const uint8_t *scale
     return 0;
 }
 
-/* Weight stream.  Rows are padded to Np = 16*ceil(N/16) and cut into tiles
- * of 16 rows.  Inside a tile, one 32-element block of all 16 rows is stored
- * in the order in which lane l = 4g+q of a warp holds the operand of a
- * 16x8x32 integer warp MMA: row g (and g+8), elements 4q..4q+3 and
- * 16+4q..16+4q+3.
+/* Weight stream.  Codes are stored sign-magnitude: a 4-bit code as
+ * (sign << 3) | |m| and a 6/8-bit code as (sign << 7) | |m| (the symmetric
+ * clamp R4 never produces -2^(b-1), so nothing is lost).  Rows are padded to
+ * Np = 16*ceil(N/16) and cut into tiles of 16 rows.  Inside a tile, one
+ * 32-element block of all 16 rows is stored in the order in which lane
+ * l = 4g+q of a warp holds the operand of a 16x8x32 warp MMA: row g (and g+8),
+ * elements 4q..4q+3 and 16+4q..16+4q+3.
  *   Section Q4 (offset 0): T*n4 chunks of 256 B, chunk (t,s) at (t*n4+s)*256.
  *     byte 8l + 4h + j (h in {0,1}, j<4): row 16t+g+8h;
  *     high nibble = element 4q+j, low nibble = element 16+4q+j.
@@ -485,13 +487,15 @@ int mxo_pack_weight(int64_t N, int64_t K, const uint8_t *bits, const uint8_t *sc
                 const int second = i >= 16;          /* elements 16..31 */
                 const int q = (i % 16) / 4, j = i % 4;
                 const int64_t lane = 4 * g + q;
+                const int mag = c[i] < 0 ? -c[i] : c[i];
                 if (s < n4) {
                     uint8_t *byte = out + (t * n4 + s) * 256 + 8 * lane + 4 * h + j;
-                    uint8_t nib = (uint8_t)c[i] & 0x0F;
+                    uint8_t nib = (uint8_t)(((c[i] < 0) << 3) | mag);
                     *byte |= (uint8_t)(second ? nib : (nib << 4));
                 } else {
                     const int reg = (second ? 2 : 0) + (int)h;
-                    out[o8 + (t * n68 + (s - n4)) * 512 + 16 * lane + 4 * reg + j] = (uint8_t)c[i];
+                    out[o8 + (t * n68 + (s - n4)) * 512 + 16 * lane + 4 * reg + j] =
+                        (uint8_t)(((c[i] < 0) << 7) | mag);
                 }
             }
         }

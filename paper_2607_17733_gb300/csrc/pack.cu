@@ -3,8 +3,9 @@
 // Same MXINT rule as the activations (Appendix A.2: weights and activations
 // of every linear layer are quantized; Sec. 4.1: one width per 32-element
 // block).  One thread owns one (row, slot) block: it loads the 32 bf16 values
-// with four 128-bit loads and scatters the codes into the 16-row fragment
-// tiles read by the decode kernel, the scale byte, and optionally the e4m3
+// with four 128-bit loads and scatters the codes (sign-magnitude) into the
+// 16-row fragment tiles read by the decode kernel, the scale byte, and
+// optionally the e4m3
 // digit planes and scale tiles read by the tensor-core prefill kernel.  The
 // buffer is cleared first, so padding rows and slots read as zero.  This runs
 // once per layer and is not on the timed path.
@@ -50,6 +51,9 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
 #pragma unroll
     for (int i = 0; i < 32; ++i) m[i] = S == 255 ? 0 : quant_elem(h[i], S, b, a.rhaz);
 
+    // sign-magnitude codes: (sign << 3) | |m| for 4 bits, (sign << 7) | |m| for 6/8 bits
+    auto sm4 = [](int v) { return (uint32_t)(((v < 0) << 3) | (v < 0 ? -v : v)); };
+    auto sm8 = [](int v) { return (uint32_t)(((v < 0) << 7) | (v < 0 ? -v : v)); };
     const int64_t t = n >> 4;
     const int rr = (int)(n & 15), g = rr & 7, hh = rr >> 3;
     if (b == 4) {
@@ -59,7 +63,7 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
             uint32_t word = 0;
 #pragma unroll
             for (int j = 0; j < 4; ++j)
-                word |= (uint32_t)(((m[4 * q + j] & 0xF) << 4) | (m[16 + 4 * q + j] & 0xF)) << (8 * j);
+                word |= ((sm4(m[4 * q + j]) << 4) | sm4(m[16 + 4 * q + j])) << (8 * j);
             *reinterpret_cast<uint32_t *>(chunk + 8 * (4 * g + q) + 4 * hh) = word;
         }
     } else {
@@ -69,8 +73,8 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
             uint32_t w0 = 0, w1 = 0;
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                w0 |= (uint32_t)(m[4 * q + j] & 0xFF) << (8 * j);
-                w1 |= (uint32_t)(m[16 + 4 * q + j] & 0xFF) << (8 * j);
+                w0 |= sm8(m[4 * q + j]) << (8 * j);
+                w1 |= sm8(m[16 + 4 * q + j]) << (8 * j);
             }
             uint8_t *lane = chunk + 16 * (4 * g + q);
             *reinterpret_cast<uint32_t *>(lane + 4 * hh) = w0;

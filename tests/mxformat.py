@@ -17,6 +17,16 @@ def align256(v):
     return (v + 255) // 256 * 256
 
 
+def signmag4(n):
+    n = n.astype(np.int16)
+    return np.where(n & 8, -(n & 7), n & 7).astype(np.int8)
+
+
+def signmag8(n):
+    n = n.astype(np.int16)
+    return np.where(n & 0x80, -(n & 0x7F), n & 0x7F).astype(np.int8)
+
+
 def sext4(n):
     n = n.astype(np.int16)
     return np.where(n >= 8, n - 16, n).astype(np.int8)
@@ -72,11 +82,11 @@ def decode_weight(N, bits, buf):
                     for j in range(4):
                         rows = 16 * t + g + 8 * h
                         byte = ch[:, h, j]
-                        codes[rows, 32 * kb + 4 * q + j] = sext4(byte >> 4)
-                        codes[rows, 32 * kb + 16 + 4 * q + j] = sext4(byte & 0xF)
+                        codes[rows, 32 * kb + 4 * q + j] = signmag4(byte >> 4)
+                        codes[rows, 32 * kb + 16 + 4 * q + j] = signmag4(byte & 0xF)
             else:
                 base = o8 + (t * n68 + (s - n4)) * 512
-                ch = buf[base:base + 512].reshape(32, 4, 4).view(np.int8)  # lane, reg, j
+                ch = signmag8(buf[base:base + 512].reshape(32, 4, 4))  # lane, reg, j
                 for reg in range(4):
                     h = reg % 2
                     e0 = 16 if reg >= 2 else 0

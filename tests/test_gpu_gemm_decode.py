@@ -114,3 +114,31 @@ def test_decode_sweep_70b_shape_sampled(torch, maps):
     w_s, w_c = mxo.quantize_bf16(wb[cols], bits)
     ref, ab = mxo.gemm(bits, a_c, a_s, w_c, w_s)
     U.check_gemm(y[:, cols], ref, ab)
+
+
+def wide_range_layer(M, N, nb, bits, g, spread=20):
+    """Blocks scaled by random powers of two over 2*spread binades: the exact
+    results no longer fit fp32, so the kernels' accumulation rounding shows."""
+    xb = I.activations_bf16(M, bits, g, 0.0)
+    wb = I.normal_bf16((N, 32 * nb), 0.02, g)
+    xf = I.bf16_bits_to_f32(xb).reshape(M, nb, 32)
+    wf = I.bf16_bits_to_f32(wb).reshape(N, nb, 32)
+    xf = xf * np.exp2(g.integers(-spread, spread + 1, size=(M, nb, 1))).astype(np.float32)
+    wf = wf * np.exp2(g.integers(-spread, spread + 1, size=(N, nb, 1))).astype(np.float32)
+    return I.f32_to_bf16_bits(xf.reshape(M, -1)), I.f32_to_bf16_bits(wf.reshape(N, -1))
+
+
+@pytest.mark.parametrize("M,nb,p", [(1, 128, (0.85, 0.10, 0.05)), (16, 448, (0.8, 0.15, 0.05)),
+                                    (5, 64, (0, 0, 1))])
+def test_decode_wide_dynamic_range(torch, M, nb, p):
+    g = I.rng(40, M, nb)
+    bits = I.width_map(nb, *p, g)
+    N = 300
+    xb, wb = wide_range_layer(M, N, nb, bits, g)
+    codes, scales, _ = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits)
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
+    y = mxs.gemm(codes, scales, None, bits, packed, N).cpu().numpy()
+    ref, ab = oracle_full(xb, wb, bits)
+    assert np.mean(ref.astype(np.float32).astype(np.float64) == ref) < 0.5  # rounding really happens
+    err = U.check_gemm(y, ref, ab)
+    print(f"decode wide range M={M} K={32 * nb}: max err/abssum {err:.2e}")

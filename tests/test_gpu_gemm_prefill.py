@@ -99,3 +99,18 @@ def test_prefill_bounded_wait_reports_timeout(torch):
     y = mxs.gemm_prefill(planes, bits, packed, M, N).cpu().numpy()  # the context still works
     ref, ab = oracle_entries(xb, wb, bits)
     U.check_gemm(y, ref, ab)
+
+
+@pytest.mark.parametrize("M,nb,p", [(256, 128, (0.8, 0.15, 0.05)), (130, 448, (0.5, 0.3, 0.2))])
+def test_prefill_wide_dynamic_range(torch, M, nb, p):
+    from test_gpu_gemm_decode import wide_range_layer
+    g = I.rng(41, M, nb)
+    bits = I.width_map(nb, *p, g)
+    N = 384
+    xb, wb = wide_range_layer(M, N, nb, bits, g)
+    planes, packed = prep(torch, xb, wb, bits)
+    y = mxs.gemm_prefill(planes, bits, packed, M, N).cpu().numpy()
+    ref, ab = oracle_entries(xb, wb, bits)
+    assert np.mean(ref.astype(np.float32).astype(np.float64) == ref) < 0.5
+    err = U.check_gemm(y, ref, ab)
+    print(f"prefill wide range M={M} K={32 * nb}: max err/abssum {err:.2e}")
