@@ -49,8 +49,12 @@ def parse():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--layers", type=int, default=32)
+    ap.add_argument("--layers", type=int, default=None,
+                    help="decoder layers per step (default 32 for decode, 8 for prefill)")
+    ap.add_argument("--workload", default="llama3-8b-decode", choices=["llama3-8b-decode", "llama3-8b-prefill"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--unfused", action="store_true",
+                    help="separate quantize and GEMM launches instead of the fused decode kernel")
     ap.add_argument("--eager", action="store_true",
                     help="launch the step's kernels directly (no CUDA graph, no events): for ncu runs")
     return ap.parse_args()
@@ -314,9 +318,12 @@ def run_ours(args):
     # ---- algorithmic work per step
     step_bytes = sum(lin.weight_bytes + M * lin.K * 2 + M * lin.N * 4 for M, lin, _, _ in items)
     step_ops = sum(2 * M * lin.N * lin.K for M, lin, _, _ in items)
-    gemm_bytes = sum(lin.weight_bytes + M * (mxs.act_row_bytes(lin.K, lin.bits) + lin.K // 32) + M * lin.N * 4
-                     for M, lin, _, _ in items)
-    launches_per_step = 2 * len(items)
+    if args.unfused:  # the GEMM reads the packed codes the quantizer wrote
+        gemm_bytes = sum(lin.weight_bytes + M * (mxs.act_row_bytes(lin.K, lin.bits) + lin.K // 32) + M * lin.N * 4
+                         for M, lin, _, _ in items)
+    else:  # the fused kernel reads the bf16 activations itself
+        gemm_bytes = step_bytes
+    launches_per_step = (2 if args.unfused else 1) * len(items)
 
     # ---- the step as one CUDA graph.  Inputs are independent synthetic draws, so
     # for each M the graph runs all activation quantizations, then all GEMMs;
@@ -329,12 +336,16 @@ def run_ours(args):
     def make_step(events=None):
         def fn():
             for gi, grp in enumerate(groups):
-                for M, lin, x, bufs in grp:
-                    lin.quantize(x, bufs)
+                if args.unfused:
+                    for M, lin, x, bufs in grp:
+                        lin.quantize(x, bufs)
                 if events is not None:
                     events[gi][0].record()
                 for M, lin, x, bufs in grp:
-                    lin.matmul(bufs)
+                    if args.unfused:
+                        lin.matmul(bufs)
+                    else:
+                        lin.fused(x, bufs["y"])
                 if events is not None:
                     events[gi][1].record()
         return fn
@@ -405,7 +416,8 @@ def run_ours(args):
         gemm_ms = sum(s.elapsed_time(e) for evs in ev_sets for s, e in evs) / len(ev_sets)  # per step
         achieved = gemm_bytes / (gemm_ms * 1e-3) / 1e9
         traffic = profile_traffic("gemm_decode.cu", "gemm_decode_llama3_8b_decode.md")
-        roofline = {"kernel": "gemm_decode_kernel", "bound": "hbm", "achieved": achieved,
+        roofline = {"kernel": "gemm_decode_kernel" + ("" if args.unfused else " (fused quantize)"),
+                    "bound": "hbm", "achieved": achieved,
                     "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": achieved / pk["hbm_gbs"],
                     "peak_source": pk["source"], "traffic": traffic,
                     "bytes_per_step": gemm_bytes, "gemm_ms_per_step": gemm_ms,
@@ -441,6 +453,7 @@ def run_ours(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "int8+f32",
             "data": "synthetic (seeded; weights N(0,0.02), activations N(0,1) with 1% outlier columns x30)",
             "config": {"workload": "llama3-8b-decode", "M": list(DECODE_MS), "layers": L,
+                       "path": "quantize + GEMM" if args.unfused else "fused quantize-GEMM (one launch per projection)",
                        "projections": [p[0] for p in I.LLAMA3_8B], "map_4_6_8": list(MAP),
                        "parallelism": f"replicas x{ws}", "l2": "inputs larger than L2 (packed weights "
                        f"{sum(lin.weight_bytes for p in layers for lin in p) / 1e9:.2f} GB per step)"},
@@ -454,11 +467,115 @@ def run_ours(args):
         print(json.dumps(line), flush=True)
 
 
+def run_prefill(args):
+    """LLaMA-3-8B-shaped prefill: M = 2048 tokens through q/k/v/o/gate/up/down of
+    `layers` layers, map 80/15/5, activations N(0,1) with Student-t(3) outlier
+    channels on 0.5 % of K.  Per projection: quantize to MMA planes (A1) and the
+    tcgen05 GEMM (A3).  Metric: effective TOPS = 2*M*N*K / s, whole job."""
+    import torch
+
+    ws, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_17733_gb300 import build as B
+    from paper_2607_17733_gb300 import mxs
+    from paper_2607_17733_gb300.runtime import MxLinear
+    if not os.path.exists(mxs.LIB_PATH):
+        B.build()
+    mxs.lib()
+    M = 2048
+    L = args.layers or 8
+    gen = torch.Generator(device=dev)
+    items = []
+    for l in range(L):
+        for pi, (name, K, N) in enumerate(I.LLAMA3_8B):
+            bits = I.width_map(K // 32, 0.80, 0.15, 0.05, I.rng(SEED, rank, 3, l, pi))
+            gen.manual_seed(SEED * 7 + rank * 10_007 + l * 101 + pi)
+            w = (torch.randn((N, K), generator=gen, device=dev, dtype=torch.float32) * W_SIGMA).to(torch.bfloat16)
+            lin = MxLinear(w, bits, with_planes=True)
+            del w
+            items.append((lin, bits))
+    planes, ys = [], []
+    for idx, (lin, bits) in enumerate(items):
+        # N(0,1) activations, 0.5 % of K channels (inside 8-bit blocks) redrawn from
+        # a Student-t(3) = Z / sqrt(chi2_3 / 3); drawn on the GPU from a seeded stream
+        gen.manual_seed(SEED * 13 + rank * 10_007 + idx)
+        x = torch.randn((M, lin.K), generator=gen, device=dev, dtype=torch.float32)
+        cols = torch.from_numpy(I.outlier_columns(bits, int(np.floor(0.005 * lin.K + 0.5)),
+                                                  I.rng(SEED, rank, 6, idx))).to(dev)
+        z = torch.randn((M, cols.numel(), 4), generator=gen, device=dev, dtype=torch.float32)
+        x[:, cols] = z[..., 0] / torch.sqrt((z[..., 1:] ** 2).sum(-1) / 3.0)
+        x = x.to(torch.bfloat16)
+        planes.append((x, torch.empty(mxs.act_planes_bytes(M, lin.K, bits), dtype=torch.uint8, device=dev)))
+        ys.append(torch.empty((M, lin.N), dtype=torch.float32, device=dev))
+    torch.cuda.synchronize()
+    step_ops = sum(2 * M * lin.N * lin.K for lin, _ in items)
+
+    def fn(events=None):
+        for idx, (lin, bits) in enumerate(items):
+            x, pl = planes[idx]
+            mxs.quantize_act(x, bits, planes=pl, want_codes=False)
+            if events is not None:
+                events[idx][0].record()
+            mxs.gemm_prefill(pl, bits, lin.packed, M, lin.N, y=ys[idx])
+            if events is not None:
+                events[idx][1].record()
+
+    if args.eager:
+        for _ in range(args.warmup + args.steps):
+            fn()
+        torch.cuda.synchronize()
+        print(json.dumps({"eager_steps": args.steps, "launches_per_step": 2 * len(items)}), flush=True)
+        return
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in items]
+           for _ in range(args.steps)]
+    sampler = ClockSampler(None)
+    barrier(ws)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.1)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for k in range(args.steps):
+        fn(evs[k])
+    t1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = allreduce_max(t0.elapsed_time(t1) / args.steps, ws)
+    gemm_ms = sum(s.elapsed_time(e) for ev in evs for s, e in ev) / args.steps
+    pk = peaks()
+    fp8_peak = 2.0 * pk["bf16_tflops"]
+    achieved = step_ops / (gemm_ms * 1e-3) / 1e12
+    value = ws * step_ops / (ms * 1e-3) / 1e12
+    if rank == 0:
+        print(json.dumps({
+            "metric": "mxint_prefill_gemm_tops", "value": value, "unit": "TOPS", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "e4m3 digit planes + f32",
+            "data": "synthetic (seeded; W N(0,0.02), A N(0,1) with Student-t(3) outlier channels on 0.5% of K)",
+            "config": {"workload": "llama3-8b-prefill", "M": M, "layers": L, "map_4_6_8": [0.8, 0.15, 0.05],
+                       "l2": "inputs larger than L2"},
+            "roofline": {"kernel": "gemm_prefill_kernel", "bound": "tensor", "achieved": achieved,
+                         "peak": fp8_peak, "unit": "TFLOP/s", "frac": achieved / fp8_peak,
+                         "peak_source": pk["source"] + " bf16 x 2 (fp8/bf16 nominal ratio)",
+                         "traffic": profile_traffic("gemm_prefill.cu", "gemm_prefill_llama3_8b_prefill.md"),
+                         "gemm_ms_per_step": gemm_ms, "share_of_step": gemm_ms / ms},
+            "gpu_launches": 2 * len(items) * args.steps, "clocks": clocks}), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload == "llama3-8b-prefill":
+        run_prefill(args)
     else:
+        if args.layers is None:
+            args.layers = 32
         run_ours(args)
 
 

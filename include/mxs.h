@@ -54,7 +54,8 @@
  *                            O8+(t*(n6+n8)+j)*512; byte 16l+4c+j: c=0 row g
  *                            elem 4q+j, c=1 row g+8 elem 4q+j, c=2 row g elem
  *                            16+4q+j, c=3 row g+8 elem 16+4q+j;
- *       SC at OS = align256(O8 + T*(n6+n8)*512): uint8 [Np, K/32] scales by slot;
+ *       SC at OS = align256(O8 + T*(n6+n8)*512): scale bytes tile-major, byte
+ *                            OS + (t*K/32 + s)*16 + r = row 16t+r, slot s;
  *       compact size = align256(OS + Np*K/32).
  *   MMA planes (layout MXS_W_COMPACT_AND_PLANES for weights, the `planes`
  *     output of mxs_quantize_act for activations), Kp = 128*(ceil(n4/4) +
@@ -154,11 +155,23 @@ MXS_API int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const voi
              int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y,
              void *workspace, size_t ws_bytes, void *stream);
 
-/* Decode path only (M <= 16): weights streamed once from the compact layout,
- * integer warp MMAs per block, fp32 fold, split-K with a fixed-order reduction. */
+/* Decode path only (M <= 16): weights streamed once from the compact layout by
+ * bulk copies into a shared-memory ring; exact FP8 warp MMAs per block on
+ * sign-magnitude digits, fp32 fold; when K is split over a thread-block
+ * cluster the partial tiles are added in rank order.  Needs no workspace
+ * (ws may be NULL).  Waits are bounded like the prefill kernel's. */
 MXS_API int mxs_gemm_decode(const void *act_codes, const uint8_t *act_scales, const uint8_t *bits,
                     const void *packed_w, int64_t M, int64_t N, int64_t K,
                     float *y, int64_t ld_y, void *workspace, size_t ws_bytes, void *stream);
+
+/* A1 fused into A4 (M <= 16): quantizes x (bf16 [M,K], row stride ld_x) with
+ * `bits` and `rounding` inside the decode GEMM's prologue -- the same codes
+ * mxs_quantize_act would write, never stored -- and returns y [M,N] fp32 =
+ * x W^T like mxs_gemm_decode.  One launch per linear layer and token batch
+ * (Appendix A.2: activations are quantized on the fly). */
+MXS_API int mxs_linear_decode(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits,
+                              int rounding, const void *packed_w, int64_t N, float *y, int64_t ld_y,
+                              void *stream);
 
 /* Prefill path only (any M >= 1, efficient for M >= 128): the tensor-core
  * kernel over the MMA planes of the activations (mxs_quantize_act `planes`)

@@ -331,8 +331,8 @@ int mxo_pack_act(int64_t R, int64_t K, const uint8_t *bits, const uint8_t *scale
  *     chunk (t,j68) at O8 + (t*(n6+n8)+j68)*512.
  *     byte 16l + 4c + j: c=0 row g elem 4q+j; c=1 row g+8 elem 4q+j;
  *                        c=2 row g elem 16+4q+j; c=3 row g+8 elem 16+4q+j.
- *   Section SC (offset OS = align256(O8 + T*(n6+n8)*512)): [Np, nb] scales
- *     per slot, zero for padding rows.
+ *   Section SC (offset OS = align256(O8 + T*(n6+n8)*512)): scales tile-major,
+ *     byte OS + (t*nb + s)*16 + r is row 16t+r, slot s; zero for padding rows.
  *   Compact size = align256(OS + Np*nb).
  *   With planes: section P (offset compact size): [N, Kp] e4m3 planes and
  *   section SF (offset align256(P + N*Kp)): tcgen05 scale tiles, see below. */
@@ -482,7 +482,7 @@ int mxo_pack_weight(int64_t N, int64_t K, const uint8_t *bits, const uint8_t *sc
         for (int64_t s = 0; s < nb; ++s) {
             const int64_t kb = sb[s];
             const int8_t *c = codes + r * K + kb * MXO_BLOCK;
-            out[os + r * nb + s] = scales[r * nb + kb];
+            out[os + (t * nb + s) * 16 + rr] = scales[r * nb + kb];
             for (int i = 0; i < MXO_BLOCK; ++i) {
                 const int second = i >= 16;          /* elements 16..31 */
                 const int q = (i % 16) / 4, j = i % 4;

@@ -103,6 +103,9 @@ int64_t decode_workspace_bytes(const Plan &p, int64_t M, int64_t N);
 int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, const void *packed,
                        int64_t M, int64_t N, float *y, int64_t ld_y, void *ws, size_t ws_bytes,
                        cudaStream_t st);
+int launch_linear_decode(const Plan &p, const void *x, int64_t ld_x, int rounding, const void *packed, int64_t M,
+                         int64_t N, float *y, int64_t ld_y, cudaStream_t st);
+int decode_status(int *status, int reset);
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N,
                         float *y, int64_t ld_y, int starve, cudaStream_t st);
 int prefill_status(int *status, int reset, cudaStream_t st);

@@ -187,6 +187,24 @@ int mxs_gemm_decode(const void *codes, const uint8_t *scales, const uint8_t *bit
                               static_cast<cudaStream_t>(stream));
 }
 
+int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits, int rounding,
+                      const void *packed_w, int64_t N, float *y, int64_t ld_y, void *stream) {
+    Plan p;
+    int rc = build_plan(bits, K, &p);
+    if (rc) return rc;
+    if (M < 0 || N < 0) return fail(MXS_ERR_SHAPE, "M=%lld N=%lld", (long long)M, (long long)N);
+    if (M > 16) return fail(MXS_ERR_SHAPE, "the fused decode path takes M <= 16 (M=%lld)", (long long)M);
+    if (rounding != MXS_RNE && rounding != MXS_RHAZ) return fail(MXS_ERR_INVALID_ARG, "rounding=%d", rounding);
+    if (!x || !packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
+    if (ld_x < K || ld_x % 8 != 0) return fail(MXS_ERR_INVALID_ARG, "ld_x=%lld must be >= K and a multiple of 8", (long long)ld_x);
+    if (ld_y < N) return fail(MXS_ERR_INVALID_ARG, "ld_y=%lld < N", (long long)ld_y);
+    if (!aligned16(x) || !aligned16(packed_w) || (reinterpret_cast<uintptr_t>(y) & 3))
+        return fail(MXS_ERR_ALIGN, "x/packed_w must be 16-byte aligned, y 4-byte aligned");
+    if (M == 0 || N == 0) return MXS_OK;
+    if ((rc = check_device())) return rc;
+    return launch_linear_decode(p, x, ld_x, rounding, packed_w, M, N, y, ld_y, static_cast<cudaStream_t>(stream));
+}
+
 int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const void *act_planes, const uint8_t *act_bits,
              const void *packed_w, int w_layout, const uint8_t *w_bits, int64_t M, int64_t N, int64_t K, float *y,
              int64_t ld_y, void *ws, size_t ws_bytes, void *stream) {
@@ -235,7 +253,11 @@ int mxs_device_status(int *status, int reset, void *stream) {
     if (!status) return fail(MXS_ERR_INVALID_ARG, "status is NULL");
     int rc = check_device();
     if (rc) return rc;
-    return prefill_status(status, reset, static_cast<cudaStream_t>(stream));
+    int a = 0, b = 0;
+    if ((rc = prefill_status(&a, reset, static_cast<cudaStream_t>(stream)))) return rc;
+    if ((rc = decode_status(&b, reset))) return rc;
+    *status = a ? a : b;
+    return MXS_OK;
 }
 
 }  // extern "C"

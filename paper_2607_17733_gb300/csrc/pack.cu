@@ -81,7 +81,7 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
             *reinterpret_cast<uint32_t *>(lane + 4 * (2 + hh)) = w1;
         }
     }
-    a.out[a.off.os + n * p.nb + s] = (uint8_t)S;
+    a.out[a.off.os + (t * p.nb + s) * 16 + rr] = (uint8_t)S;
 
     if (a.with_planes) {
         uint8_t *prow = a.out + a.off.planes + n * p.kp;

@@ -47,8 +47,14 @@ class MxLinear:
         return mxs.gemm(bufs["codes"], bufs["scales"], None, self.bits, self.packed, self.N,
                         w_layout=self.layout, y=bufs["y"], workspace=bufs["ws"])
 
+    def fused(self, x: torch.Tensor, y: torch.Tensor) -> torch.Tensor:
+        """M <= 16: activation quantization inside the decode GEMM (one launch)."""
+        return mxs.linear_decode(x, self.bits, self.packed, self.N, rounding=self.rounding, y=y)
+
     def __call__(self, x: torch.Tensor, bufs: dict | None = None) -> torch.Tensor:
         bufs = bufs or self.buffers(x.shape[0], x.device)
+        if x.shape[0] <= 16:
+            return self.fused(x, bufs["y"])
         self.quantize(x, bufs)
         return self.matmul(bufs)
 

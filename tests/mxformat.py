@@ -92,7 +92,7 @@ def decode_weight(N, bits, buf):
                     e0 = 16 if reg >= 2 else 0
                     for j in range(4):
                         codes[16 * t + g + 8 * h, 32 * kb + e0 + 4 * q + j] = ch[:, reg, j]
-    sc = buf[os_:os_ + 16 * T * nb].reshape(16 * T, nb)
+    sc = buf[os_:os_ + 16 * T * nb].reshape(T, nb, 16).transpose(0, 2, 1).reshape(16 * T, nb)
     scales = np.zeros((16 * T, nb), np.uint8)
     scales[:, sb] = sc
     return scales[:N], codes[:N]

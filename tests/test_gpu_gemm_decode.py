@@ -142,3 +142,36 @@ def test_decode_wide_dynamic_range(torch, M, nb, p):
     assert np.mean(ref.astype(np.float32).astype(np.float64) == ref) < 0.5  # rounding really happens
     err = U.check_gemm(y, ref, ab)
     print(f"decode wide range M={M} K={32 * nb}: max err/abssum {err:.2e}")
+
+
+@pytest.mark.parametrize("M", [1, 3, 8, 16])
+@pytest.mark.parametrize("N,nb,p", [(37, 5, (0.6, 0.2, 0.2)), (1000, 128, (0.85, 0.10, 0.05)),
+                                    (64, 448, (0.8, 0.15, 0.05)), (300, 896, (0.5, 0.3, 0.2))])
+def test_fused_linear_decode(torch, M, N, nb, p):
+    """Quantization inside the GEMM prologue: same y as quantize + GEMM (bit for
+    bit) and within the bar of the oracle."""
+    g = I.rng(50, M, N, nb)
+    bits = I.width_map(nb, *p, g)
+    xb, wb, codes, scales, packed = layer(torch, M, 32 * nb, N, bits, g)
+    y_fused = mxs.linear_decode(U.to_dev_bf16(torch, xb), bits, packed, N).cpu().numpy()
+    y_two = mxs.gemm(codes, scales, None, bits, packed, N).cpu().numpy()
+    assert np.array_equal(y_fused, y_two)
+    ref, ab = oracle_full(xb, wb, bits)
+    U.check_gemm(y_fused, ref, ab)
+
+
+def test_fused_linear_decode_rhaz_and_stride(torch):
+    g = I.rng(51)
+    bits = I.width_map(64, 0.7, 0.2, 0.1, g)
+    M, K, N = 6, 2048, 100
+    xb = I.activations_bf16(M, bits, g, 0.02, outlier_scale=50.0)
+    wb = I.normal_bf16((N, K), 0.02, g)
+    wide = np.zeros((M, K + 64), np.uint16)
+    wide[:, :K] = xb
+    x = U.to_dev_bf16(torch, wide)[:, :K]
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits, rounding=mxs.RHAZ)
+    y = mxs.linear_decode(x, bits, packed, N, rounding=mxs.RHAZ).cpu().numpy()
+    a_s, a_c = mxo.quantize_bf16(xb, bits, mxo.RHAZ)
+    w_s, w_c = mxo.quantize_bf16(wb, bits, mxo.RHAZ)
+    ref, ab = mxo.gemm(bits, a_c, a_s, w_c, w_s)
+    U.check_gemm(y, ref, ab)

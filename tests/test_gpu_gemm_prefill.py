@@ -112,5 +112,12 @@ def test_prefill_wide_dynamic_range(torch, M, nb, p):
     y = mxs.gemm_prefill(planes, bits, packed, M, N).cpu().numpy()
     ref, ab = oracle_entries(xb, wb, bits)
     assert np.mean(ref.astype(np.float32).astype(np.float64) == ref) < 0.5
-    err = U.check_gemm(y, ref, ab)
-    print(f"prefill wide range M={M} K={32 * nb}: max err/abssum {err:.2e}")
+    # The tensor core adds each MMA's block product into the fp32 accumulator;
+    # with n_mma such adds (one per 4-bit block, four per 6/8-bit block) a
+    # recursive fp32 sum errs by at most n_mma * 2^-23 of sum|terms| even if every
+    # add truncated.  This spread (+-20 binades per block) is far outside the
+    # LLaMA-shaped workloads, which meet the 1e-5 bar exactly (see above).
+    n4 = int(np.sum(bits == 4))
+    n_mma = n4 + 4 * (bits.size - n4)
+    err = U.check_gemm(y, ref, ab, rtol=n_mma * 2.0 ** -23)
+    print(f"prefill wide range M={M} K={32 * nb}: max err/abssum {err:.2e} (bound {n_mma * 2.0 ** -23:.2e})")
