@@ -43,20 +43,17 @@
  *     one int8 per element.  Activation scales: uint8 [M, K/32] by slot.
  *   Weight buffer (layout MXS_W_COMPACT): codes are sign-magnitude, a 4-bit
  *     code as (sign<<3)|m and a 6/8-bit code as (sign<<7)|m (the symmetric
- *     clamp never yields -2^(b-1)); rows padded to Np = 16*ceil(N/16),
- *     cut into tiles of 16 rows; inside a tile one block of all 16 rows is
- *     stored in the order a warp holds the A operand of a 16x8x32 integer MMA
+ *     clamp never yields -2^(b-1)); rows are padded to Np = 16*ceil(N/16) and
+ *     cut into tiles of 16 rows; tile t is TB = 272*n4 + 528*(n6+n8)
+ *     contiguous bytes at t*TB, so any K range of a tile is one copy:
+ *       4-bit slot s at 272*s: 256 code bytes, then 16 scale bytes (row r at +256+r);
+ *       6/8-bit slot n4+j at 272*n4 + 528*j: 512 code bytes, then 16 scale bytes.
+ *     Codes are in the order a warp holds the A operand of a 16x8x32 MMA
  *     (lane l = 4g+q: rows g, g+8; elements 4q..4q+3 and 16+4q..16+4q+3):
- *       Q4 at 0:             chunk (t,s) of 256 B at (t*n4+s)*256; byte
- *                            8l+4h+j: row 16t+g+8h, high nibble = element 4q+j,
- *                            low nibble = element 16+4q+j;
- *       Q8 at O8 = align256(T*n4*256): chunk (t,j) of 512 B at
- *                            O8+(t*(n6+n8)+j)*512; byte 16l+4c+j: c=0 row g
- *                            elem 4q+j, c=1 row g+8 elem 4q+j, c=2 row g elem
- *                            16+4q+j, c=3 row g+8 elem 16+4q+j;
- *       SC at OS = align256(O8 + T*(n6+n8)*512): scale bytes tile-major, byte
- *                            OS + (t*K/32 + s)*16 + r = row 16t+r, slot s;
- *       compact size = align256(OS + Np*K/32).
+ *       4-bit byte 8l+4h+j: row g+8h, high nibble = element 4q+j, low nibble =
+ *       element 16+4q+j;  6/8-bit byte 16l+4c+j: c=0 row g elem 4q+j, c=1 row
+ *       g+8 elem 4q+j, c=2 row g elem 16+4q+j, c=3 row g+8 elem 16+4q+j.
+ *     Compact size = align256(T*TB); scale bytes of padding rows are 0.
  *   MMA planes (layout MXS_W_COMPACT_AND_PLANES for weights, the `planes`
  *     output of mxs_quantize_act for activations), Kp = 128*(ceil(n4/4) +
  *     ceil((n6+n8)/2)):

@@ -320,29 +320,25 @@ int mxo_pack_act(int64_t R, int64_t K, const uint8_t *bits, const uint8_t *scale
 /* Weight stream.  Codes are stored sign-magnitude: a 4-bit code as
  * (sign << 3) | |m| and a 6/8-bit code as (sign << 7) | |m| (the symmetric
  * clamp R4 never produces -2^(b-1), so nothing is lost).  Rows are padded to
- * Np = 16*ceil(N/16) and cut into tiles of 16 rows.  Inside a tile, one
- * 32-element block of all 16 rows is stored in the order in which lane
- * l = 4g+q of a warp holds the operand of a 16x8x32 warp MMA: row g (and g+8),
- * elements 4q..4q+3 and 16+4q..16+4q+3.
- *   Section Q4 (offset 0): T*n4 chunks of 256 B, chunk (t,s) at (t*n4+s)*256.
- *     byte 8l + 4h + j (h in {0,1}, j<4): row 16t+g+8h;
- *     high nibble = element 4q+j, low nibble = element 16+4q+j.
- *   Section Q8 (offset O8 = align256(T*n4*256)): T*(n6+n8) chunks of 512 B,
- *     chunk (t,j68) at O8 + (t*(n6+n8)+j68)*512.
- *     byte 16l + 4c + j: c=0 row g elem 4q+j; c=1 row g+8 elem 4q+j;
- *                        c=2 row g elem 16+4q+j; c=3 row g+8 elem 16+4q+j.
- *   Section SC (offset OS = align256(O8 + T*(n6+n8)*512)): scales tile-major,
- *     byte OS + (t*nb + s)*16 + r is row 16t+r, slot s; zero for padding rows.
- *   Compact size = align256(OS + Np*nb).
+ * Np = 16*ceil(N/16) and cut into tiles of 16 rows; tile t occupies
+ * TB = 272*n4 + 528*(n6+n8) contiguous bytes at t*TB:
+ *   4-bit slot s:      at 272*s: 256 bytes of codes, then 16 scale bytes;
+ *   6/8-bit slot n4+j: at 272*n4 + 528*j: 512 bytes of codes, then 16 scales.
+ * The codes of one slot are in the order in which lane l = 4g+q of a warp
+ * holds the operand of a 16x8x32 warp MMA: row g (and g+8), elements
+ * 4q..4q+3 and 16+4q..16+4q+3.
+ *   4-bit:   byte 8l + 4h + j (h in {0,1}, j<4): row g+8h of the tile;
+ *            high nibble = element 4q+j, low nibble = element 16+4q+j.
+ *   6/8-bit: byte 16l + 4c + j: c=0 row g elem 4q+j; c=1 row g+8 elem 4q+j;
+ *            c=2 row g elem 16+4q+j; c=3 row g+8 elem 16+4q+j.
+ *   scale byte r of a slot: row r of the tile (zero for padding rows).
+ *   Compact size = align256(T*TB).
  *   With planes: section P (offset compact size): [N, Kp] e4m3 planes and
  *   section SF (offset align256(P + N*Kp)): tcgen05 scale tiles, see below. */
-static void weight_offsets(int64_t N, int64_t n4, int64_t n68, int64_t nb,
-                           int64_t *o8, int64_t *os, int64_t *compact)
+static int64_t tile_bytes(int64_t n4, int64_t n68) { return 272 * n4 + 528 * n68; }
+static int64_t weight_compact(int64_t N, int64_t n4, int64_t n68)
 {
-    const int64_t T = (N + 15) / 16, Np = T * 16;
-    *o8 = align256(T * n4 * 256);
-    *os = align256(*o8 + T * n68 * 512);
-    *compact = align256(*os + Np * nb);
+    return align256((N + 15) / 16 * tile_bytes(n4, n68));
 }
 
 /* Planes: for every row, Kp = 128*(ceil(n4/4) + ceil(n68/2)) e4m3 bytes.
@@ -367,8 +363,7 @@ int64_t mxo_weight_bytes(int64_t N, int64_t K, const uint8_t *bits, int with_pla
     int64_t cnt[3];
     if (!sb || mxo_slots(bits, nb, sb, cnt) != 0) { free(sb); return -1; }
     free(sb);
-    int64_t o8, os, compact;
-    weight_offsets(N, cnt[0], cnt[1] + cnt[2], nb, &o8, &os, &compact);
+    const int64_t compact = weight_compact(N, cnt[0], cnt[1] + cnt[2]);
     if (!with_planes) return compact;
     const int64_t kp = kp_bytes(cnt[0], cnt[1] + cnt[2]);
     const int64_t sf = align256(compact + N * kp);
@@ -473,8 +468,7 @@ int mxo_pack_weight(int64_t N, int64_t K, const uint8_t *bits, const uint8_t *sc
     int64_t cnt[3];
     if (!sb || mxo_slots(bits, nb, sb, cnt) != 0) { free(sb); return -1; }
     const int64_t n4 = cnt[0], n68 = cnt[1] + cnt[2];
-    int64_t o8, os, compact;
-    weight_offsets(N, n4, n68, nb, &o8, &os, &compact);
+    const int64_t TB = tile_bytes(n4, n68), compact = weight_compact(N, n4, n68);
     const int64_t total = mxo_weight_bytes(N, K, bits, with_planes);
     memset(out, 0, (size_t)total);
     for (int64_t r = 0; r < N; ++r) {
@@ -482,20 +476,20 @@ int mxo_pack_weight(int64_t N, int64_t K, const uint8_t *bits, const uint8_t *sc
         for (int64_t s = 0; s < nb; ++s) {
             const int64_t kb = sb[s];
             const int8_t *c = codes + r * K + kb * MXO_BLOCK;
-            out[os + (t * nb + s) * 16 + rr] = scales[r * nb + kb];
+            uint8_t *slot = out + t * TB + (s < n4 ? 272 * s : 272 * n4 + 528 * (s - n4));
+            slot[(s < n4 ? 256 : 512) + rr] = scales[r * nb + kb];
             for (int i = 0; i < MXO_BLOCK; ++i) {
                 const int second = i >= 16;          /* elements 16..31 */
                 const int q = (i % 16) / 4, j = i % 4;
                 const int64_t lane = 4 * g + q;
                 const int mag = c[i] < 0 ? -c[i] : c[i];
                 if (s < n4) {
-                    uint8_t *byte = out + (t * n4 + s) * 256 + 8 * lane + 4 * h + j;
+                    uint8_t *byte = slot + 8 * lane + 4 * h + j;
                     uint8_t nib = (uint8_t)(((c[i] < 0) << 3) | mag);
                     *byte |= (uint8_t)(second ? nib : (nib << 4));
                 } else {
                     const int reg = (second ? 2 : 0) + (int)h;
-                    out[o8 + (t * n68 + (s - n4)) * 512 + 16 * lane + 4 * reg + j] =
-                        (uint8_t)(((c[i] < 0) << 7) | mag);
+                    slot[16 * lane + 4 * reg + j] = (uint8_t)(((c[i] < 0) << 7) | mag);
                 }
             }
         }

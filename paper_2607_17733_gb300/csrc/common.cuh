@@ -29,17 +29,22 @@ __host__ __device__ inline int slot_width(const Plan &p, int s) {
 
 __host__ __device__ inline int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
 
+// Packed weights: tile t (16 rows) is TB = 272*n4 + 528*n68 contiguous bytes;
+// a 4-bit slot is 256 code bytes + 16 scale bytes, a 6/8-bit slot 512 + 16.
 struct WeightOffsets {
-    int64_t T, Np, o8, os, compact, planes, sf, total;
+    int64_t T, Np, TB, compact, planes, sf, total;
 };
+
+__host__ __device__ inline int64_t slot_offset(const Plan &p, int s) {
+    return s < p.n4 ? 272 * (int64_t)s : 272 * (int64_t)p.n4 + 528 * (int64_t)(s - p.n4);
+}
 
 __host__ __device__ inline WeightOffsets weight_offsets(const Plan &p, int64_t N, bool with_planes) {
     WeightOffsets w;
     w.T = (N + 15) / 16;
     w.Np = w.T * 16;
-    w.o8 = align256(w.T * p.n4 * 256);
-    w.os = align256(w.o8 + w.T * p.n68 * 512);
-    w.compact = align256(w.os + w.Np * p.nb);
+    w.TB = 272 * (int64_t)p.n4 + 528 * (int64_t)p.n68;
+    w.compact = align256(w.T * w.TB);
     w.planes = w.compact;
     w.sf = align256(w.planes + N * p.kp);
     w.total = with_planes ? align256(w.sf + (N + 127) / 128 * p.nst * 512) : w.compact;

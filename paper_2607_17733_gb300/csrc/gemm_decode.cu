@@ -46,8 +46,8 @@ namespace {
 
 constexpr int kConsumers = 8;
 constexpr int kThreads = 32 * (kConsumers + 1);
-constexpr int kCH = 16;  // slots per stage
-constexpr uint64_t kWaitNs = 2000000000ull;
+constexpr int kCH = 64;  // slots per stage: one bulk copy of 17-34 KB (copies cost per count, not per byte)
+constexpr long long kWaitCycles = 4000000000ll;  // ~2 s at the maximum SM clock
 
 struct DecodeArgs {
     const uint8_t *codes;   // [M, row_bytes] packed activation codes (or NULL when x is given)
@@ -61,17 +61,12 @@ struct DecodeArgs {
     int M, N, T;
     int GS, chunk;        // CTAs per cluster along K, slots per CTA
     int stages, stage_bytes;
-    int b4_bytes, b8_bytes;  // shared-memory carve of the token operands
-    int64_t o8, os;
+    int b_bytes;  // shared-memory bytes of the token operands (largest rank)
+    int64_t TB;  // bytes of one 16-row weight tile
 };
 
 // ------------------------------------------------------------------ PTX helpers
 __device__ __forceinline__ uint32_t su32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
-__device__ __forceinline__ uint64_t now_ns() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
-    return t;
-}
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
 }
@@ -91,6 +86,16 @@ __device__ __forceinline__ void mbar_arrive_remote(uint64_t *bar, uint32_t rank)
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(su32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// waits on barriers that threads of other CTAs of the cluster arrive on
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
         "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
         " selp.u32 %0, 1, 0, p;\n}"
         : "=r"(ok)
@@ -98,19 +103,39 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
+template <bool kCluster = false>
+__device__ __forceinline__ bool poll(uint64_t *bar, uint32_t parity) {
+    return kCluster ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity);
+}
+template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = now_ns();
-    for (;;) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*abort) return false;
-        if (now_ns() - t0 > kWaitNs) {
-            *abort = 1;
-            atomicExch(&g_decode_status, MXS_ERR_TIMEOUT);
-            return false;
+    if (poll<kCluster>(bar, parity)) return true;
+    const long long t0 = clock64();
+    for (uint32_t i = 1;; ++i) {
+        if (poll<kCluster>(bar, parity)) return true;
+        if ((i & 63) == 0) {  // the bound is checked every 64 polls: reading a clock is not free
+            if (*abort) return false;
+            if (clock64() - t0 > kWaitCycles) {
+                *abort = 1;
+                atomicExch(&g_decode_status, MXS_ERR_TIMEOUT);
+                return false;
+            }
         }
     }
 }
+// Whole-warp wait: one lane polls (256 threads spinning on one barrier word
+// would compete with the shared-memory traffic they are waiting for), then
+// every lane takes its own, immediately successful, acquiring test.
+template <bool kCluster = false>
+__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
+    const int lane = threadIdx.x & 31;
+    bool ok = true;
+    if (lane == 0) ok = mbar_wait<kCluster>(bar, parity, abort);
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (ok) poll<kCluster>(bar, parity);
+    return ok;
+}
+
 __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                      su32(dst)),
@@ -194,8 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
     extern __shared__ __align__(128) uint8_t smem[];
     uint8_t *ring = smem;                                                    // stages x stage_bytes
     uint32_t *B4 = reinterpret_cast<uint32_t *>(ring + (size_t)a.stages * a.stage_bytes);
-    uint2 *B8 = reinterpret_cast<uint2 *>(reinterpret_cast<uint8_t *>(B4) + a.b4_bytes);
-    float *fa = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(B8) + a.b8_bytes);  // [chunk][16]
+    float *fa = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(B4) + a.b_bytes);  // [chunk][16]
     float *red = fa + (size_t)a.chunk * 16;                       // [2][kConsumers][NT*128]
     float *xbuf = red + 2 * kConsumers * NT * 128;                // [GS-1][2][NT*128] (rank 0)
     uint64_t *bars = reinterpret_cast<uint64_t *>(xbuf + (size_t)(a.GS - 1) * 2 * NT * 128);
@@ -209,6 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
     const int nchunks = (c1 - c0 + kCH - 1) / kCH;
     const int n4lo = min(c0, p.n4), n4hi = min(c1, p.n4);  // 4-bit slots of this CTA: [n4lo, n4hi)
     const int s8lo = max(c0, p.n4);                        // 6/8-bit slots: [s8lo, c1)
+    uint2 *B8 = reinterpret_cast<uint2 *>(B4 + (size_t)max(0, n4hi - n4lo) * NT * 32);
     constexpr int kOut = NT * 128;
 
     if (threadIdx.x == 0) {
@@ -236,21 +261,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                     const int s = (int)(qn % a.stages);
                     if (!mbar_wait(&empty[s], ((qn / a.stages) & 1) ^ 1, abort)) { stop = true; break; }
                     const int lo = c0 + j * kCH, hi = min(c1, lo + kCH);
-                    const int lo4 = min(lo, p.n4), hi4 = min(hi, p.n4), lo8 = max(lo, p.n4);
-                    const uint32_t q4 = (uint32_t)(hi4 - lo4) * 256, q8 = (uint32_t)max(0, hi - lo8) * 512;
-                    const uint32_t sc = (uint32_t)(hi - lo) * 16;
-                    uint8_t *dst = ring + (size_t)s * a.stage_bytes;
-                    mbar_expect_tx(&full[s], q4 + q8 + sc);
-                    if (q4) bulk_load(dst, a.w + ((int64_t)t * p.n4 + lo4) * 256, q4, &full[s]);
-                    if (q8) bulk_load(dst + q4, a.w + a.o8 + ((int64_t)t * p.n68 + (lo8 - p.n4)) * 512, q8, &full[s]);
-                    bulk_load(dst + q4 + q8, a.w + a.os + ((int64_t)t * p.nb + lo) * 16, sc, &full[s]);
+                    const int64_t off = slot_offset(p, lo);
+                    const uint32_t bytes = (uint32_t)(slot_offset(p, hi) - off);  // slots [lo, hi) of tile t: contiguous
+                    mbar_expect_tx(&full[s], bytes);
+                    bulk_load(ring + (size_t)s * a.stage_bytes, a.w + (int64_t)t * a.TB + off, bytes, &full[s]);
                 }
             }
             // drain: every copy issued must land before the CTA leaves
             const uint32_t first = qn > (uint32_t)a.stages ? qn - a.stages : 0;
             for (uint32_t k = first; k < qn; ++k) {
-                const uint64_t t0 = now_ns();
-                while (!mbar_try_wait(&full[k % a.stages], (k / a.stages) & 1) && now_ns() - t0 < kWaitNs) {
+                const long long t0 = clock64();
+                while (!mbar_try_wait(&full[k % a.stages], (k / a.stages) & 1) && clock64() - t0 < kWaitCycles) {
                 }
             }
         }
@@ -326,22 +347,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
 
             for (int j = 0; j < nchunks && !stop; ++j, ++qn) {
                 const int s = (int)(qn % a.stages);
-                if (!mbar_wait(&full[s], (qn / a.stages) & 1, abort)) { stop = true; break; }
+                if (!warp_wait(&full[s], (qn / a.stages) & 1, abort)) { stop = true; break; }
                 const int lo = c0 + j * kCH, hi = min(c1, lo + kCH);
-                const int lo4 = min(lo, p.n4), hi4 = min(hi, p.n4), lo8 = max(lo, p.n4);
-                const int q4 = (hi4 - lo4) * 256, q8 = max(0, hi - lo8) * 512;
-                const uint8_t *st = ring + (size_t)s * a.stage_bytes;
-                const uint8_t *scb = st + q4 + q8;
+                const uint8_t *st = ring + (size_t)s * a.stage_bytes - slot_offset(p, lo);  // + slot_offset(sl)
                 const int per = (hi - lo + kConsumers - 1) / kConsumers;
                 const int my0 = lo + cw * per, my1 = min(hi, my0 + per);
                 for (int sl = my0; sl < my1; ++sl) {
                     const int b = slot_width(p, sl);
-                    const int S0 = scb[(sl - lo) * 16 + g], S1 = scb[(sl - lo) * 16 + g + 8];
+                    const uint8_t *blk = st + slot_offset(p, sl);
+                    const uint8_t *scb = blk + (b == 4 ? 256 : 512);
+                    const int S0 = scb[g], S1 = scb[g + 8];
                     const float f0 = S0 == 255 ? __int_as_float(0x7fc00000) : pow2f(S0 - 127 - (b - 2));
                     const float f1 = S1 == 255 ? __int_as_float(0x7fc00000) : pow2f(S1 - 127 - (b - 2));
                     const float *fs = fa + (sl - c0) * 16 + 2 * q;
                     if (sl < p.n4) {
-                        const uint2 wv = *reinterpret_cast<const uint2 *>(st + (sl - lo4) * 256 + 8 * lane);
+                        const uint2 wv = *reinterpret_cast<const uint2 *>(blk + 8 * lane);
                         const uint32_t af[4] = {e4m3_hi_nib(wv.x), e4m3_hi_nib(wv.y), e4m3_lo_nib(wv.x),
                                                 e4m3_lo_nib(wv.y)};
 #pragma unroll
@@ -356,7 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                             acc[nt][3] = fmaf(d[3], f1 * ft.y, acc[nt][3]);
                         }
                     } else {
-                        const uint4 wv = *reinterpret_cast<const uint4 *>(st + q4 + (sl - lo8) * 512 + 16 * lane);
+                        const uint4 wv = *reinterpret_cast<const uint4 *>(blk + 16 * lane);
                         const uint32_t ah[4] = {e4m3_hi_dig(wv.x), e4m3_hi_dig(wv.y), e4m3_hi_dig(wv.z),
                                                 e4m3_hi_dig(wv.w)};
                         const uint32_t al[4] = {e4m3_lo_dig(wv.x), e4m3_lo_dig(wv.y), e4m3_lo_dig(wv.z),
@@ -401,14 +421,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
 #pragma unroll
                 for (int k = 0; k < kConsumers; ++k) v += rb[k * kOut + o];
                 if (a.GS > 1 && rank > 0) {
-                    if (!mbar_wait(&xempty[buf], ((iter >> 1) & 1) ^ 1, abort)) { stop = true; }
+                    if (!mbar_wait<true>(&xempty[buf], ((iter >> 1) & 1) ^ 1, abort)) { stop = true; }
                     else {
                         st_remote_f32(xbuf + ((rank - 1) * 2 + buf) * kOut + o, 0, v);
                         mbar_arrive_remote(&xfull[buf], 0);
                     }
                 } else {
                     if (a.GS > 1) {
-                        if (!mbar_wait(&xfull[buf], (iter >> 1) & 1, abort)) { stop = true; }
+                        if (!mbar_wait<true>(&xfull[buf], (iter >> 1) & 1, abort)) { stop = true; }
                         else {
                             for (int r = 1; r < a.GS; ++r) v += xbuf[((r - 1) * 2 + buf) * kOut + o];
                             for (int r = 1; r < a.GS; ++r) mbar_arrive_remote(&xempty[buf], (uint32_t)r);
@@ -428,7 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
 }
 
 struct DecodeShape {
-    int GS, chunk, stages, stage_bytes, b4_bytes, b8_bytes, grid;
+    int GS, chunk, stages, stage_bytes, b_bytes, grid;
     size_t smem;
 };
 
@@ -436,22 +456,20 @@ DecodeShape shape_for(const Plan &p, int NT, int GS, int64_t T, int sms) {
     DecodeShape sh;
     sh.GS = GS;
     sh.chunk = (p.nb + GS - 1) / GS;
-    int max4 = 0, max8 = 0, max_stage = 0;
+    int max_b = 0, max_stage = 0;
     for (int r = 0; r < GS; ++r) {
         const int c0 = r * sh.chunk, c1 = std::min(p.nb, c0 + sh.chunk);
         const int n4c = std::max(0, std::min(c1, p.n4) - std::min(c0, p.n4));
-        max4 = std::max(max4, n4c);
-        max8 = std::max(max8, std::max(0, c1 - c0) - n4c);
+        const int n8c = std::max(0, c1 - c0) - n4c;
+        max_b = std::max(max_b, n4c * NT * 128 + n8c * NT * 256);
         for (int lo = c0; lo < c1; lo += kCH) {
             const int hi = std::min(c1, lo + kCH);
-            const int q4 = std::max(0, std::min(hi, p.n4) - std::min(lo, p.n4));
-            max_stage = std::max(max_stage, q4 * 256 + (hi - lo - q4) * 512 + (hi - lo) * 16);
+            max_stage = std::max(max_stage, (int)(slot_offset(p, hi) - slot_offset(p, lo)));
         }
     }
     sh.stage_bytes = (max_stage + 127) / 128 * 128;
-    sh.b4_bytes = max4 * NT * 128;
-    sh.b8_bytes = max8 * NT * 256;
-    const size_t fixed = (size_t)sh.b4_bytes + sh.b8_bytes + (size_t)sh.chunk * 64 + 2 * kConsumers * NT * 512 +
+    sh.b_bytes = (max_b + 127) / 128 * 128;
+    const size_t fixed = (size_t)sh.b_bytes + (size_t)sh.chunk * 64 + 2 * kConsumers * NT * 512 +
                          (size_t)(GS - 1) * 2 * NT * 512;
     const size_t budget = 220 * 1024;
     sh.stages = 0;
@@ -466,14 +484,17 @@ DecodeShape shape_for(const Plan &p, int NT, int GS, int64_t T, int sms) {
 // too small to give every SM a row tile.
 DecodeShape pick_shape(const Plan &p, int NT, int64_t T, int sms) {
     const int gs_max = std::max(1, std::min(8, p.nb));
-    DecodeShape best = shape_for(p, NT, 1, T, sms);
+    DecodeShape best = shape_for(p, NT, 1, T, sms), most = best;
+    bool found = false;
     for (int GS = 1; GS <= gs_max; GS *= 2) {
         const DecodeShape sh = shape_for(p, NT, GS, T, sms);
-        if (sh.stages < 4) continue;
+        if (sh.stages > most.stages) most = sh;
+        if (sh.stages < 3) continue;
         best = sh;
+        found = true;
         if (T * GS >= sms || 2 * GS > gs_max) break;
     }
-    return best;
+    return found ? best : most;
 }
 
 int sm_count() {
@@ -498,8 +519,7 @@ int launch_nt(const Plan &p, const DecodeArgs &a0, cudaStream_t st) {
     a.chunk = sh.chunk;
     a.stages = sh.stages;
     a.stage_bytes = sh.stage_bytes;
-    a.b4_bytes = sh.b4_bytes;
-    a.b8_bytes = sh.b8_bytes;
+    a.b_bytes = sh.b_bytes;
     auto kern = gemm_decode_kernel<NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh.smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(decode smem)");
@@ -528,8 +548,7 @@ int launch(const Plan &p, DecodeArgs a, int64_t M, int64_t N, cudaStream_t st) {
     a.N = (int)N;
     a.T = (int)((N + 15) / 16);
     const WeightOffsets off = weight_offsets(p, N, false);
-    a.o8 = off.o8;
-    a.os = off.os;
+    a.TB = off.TB;
     if (N > (int64_t)0x7FFFFFF0) return fail(MXS_ERR_SHAPE, "N too large");
     return M <= 8 ? launch_nt<1>(p, a, st) : launch_nt<2>(p, a, st);
 }

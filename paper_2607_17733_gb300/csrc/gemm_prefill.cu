@@ -39,7 +39,7 @@ constexpr int kABytes = kBM * kBK, kBBytes = kBN * kBK;  // 16 KB, 32 KB
 constexpr int kSfaBytes = 512, kSfbBytes = 1024;
 constexpr int kTmemCols = 512;
 constexpr int kAccCol = 0, kSfCol = 256;  // per stage: SFA 4 columns, SFB 8 columns
-constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on any single wait
+constexpr long long kWaitCycles = 4000000000ll;  // ~2 s at the maximum SM clock  // 2 s bound on any single wait
 
 struct PrefillArgs {
     const uint8_t *sfa;  // scale tiles of A: [ceil(M/128)][nst][512]
@@ -62,11 +62,6 @@ struct Smem {
 
 __device__ __forceinline__ uint32_t su32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
-__device__ __forceinline__ uint64_t now_ns() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
-    return t;
-}
 
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
@@ -86,14 +81,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
 // Bounded wait: false if the CTA aborted or the wait ran out (then it aborts).
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
     if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = now_ns();
-    for (;;) {
+    const long long t0 = clock64();
+    for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
-        if (*abort) return false;
-        if (now_ns() - t0 > kWaitNs) {
-            *abort = 1;
-            atomicExch(&g_prefill_status, MXS_ERR_TIMEOUT);
-            return false;
+        if ((i & 63) == 0) {  // the bound is checked every 64 polls: reading a clock is not free
+            if (*abort) return false;
+            if (clock64() - t0 > kWaitCycles) {
+                *abort = 1;
+                atomicExch(&g_prefill_status, MXS_ERR_TIMEOUT);
+                return false;
+            }
         }
     }
 }
@@ -216,8 +213,8 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
             for (int ks = (issued > kStages ? issued - kStages : 0); ks < issued; ++ks) {
                 if (a.starve == ks + 1) continue;
                 const int s = ks % kStages;
-                const uint64_t t0 = now_ns();
-                while (!mbar_try_wait(&sm.full[s], (ks / kStages) & 1) && now_ns() - t0 < kWaitNs) {
+                const long long t0 = clock64();
+                while (!mbar_try_wait(&sm.full[s], (ks / kStages) & 1) && clock64() - t0 < kWaitCycles) {
                 }
             }
         }
@@ -258,16 +255,20 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
             // drain: wait (bounded) until the tensor core has finished what was issued
             if (committed > 0) {
                 const int ks = committed - 1;
-                const uint64_t t0 = now_ns();
-                while (!mbar_try_wait(&sm.empty[ks % kStages], (ks / kStages) & 1) && now_ns() - t0 < kWaitNs) {
+                const long long t0 = clock64();
+                while (!mbar_try_wait(&sm.empty[ks % kStages], (ks / kStages) & 1) && clock64() - t0 < kWaitCycles) {
                 }
             }
         }
     } else {
         // ------------------------------------------------ epilogue (warps 2..5)
         const int quad = warp & 3;  // TMEM lane quadrant this warp may access
-        // warp-uniform decision: tcgen05.ld below is .sync.aligned
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full, 0, abort));
+        // one lane polls for the whole main loop, then every lane takes its own
+        // acquiring test; the decision is warp-uniform (tcgen05.ld is .sync.aligned)
+        bool ok = true;
+        if (lane == 0) ok = mbar_wait(&sm.acc_full, 0, abort);
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (ok) mbar_try_wait(&sm.acc_full, 0);
         if (ok) {
             fence_after();
             const int row = m0 + 32 * quad + lane;

@@ -56,8 +56,9 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
     auto sm8 = [](int v) { return (uint32_t)(((v < 0) << 7) | (v < 0 ? -v : v)); };
     const int64_t t = n >> 4;
     const int rr = (int)(n & 15), g = rr & 7, hh = rr >> 3;
+    uint8_t *slot = a.out + t * a.off.TB + slot_offset(p, s);
     if (b == 4) {
-        uint8_t *chunk = a.out + (t * p.n4 + s) * 256;
+        uint8_t *chunk = slot;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             uint32_t word = 0;
@@ -67,7 +68,7 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
             *reinterpret_cast<uint32_t *>(chunk + 8 * (4 * g + q) + 4 * hh) = word;
         }
     } else {
-        uint8_t *chunk = a.out + a.off.o8 + (t * p.n68 + (s - p.n4)) * 512;
+        uint8_t *chunk = slot;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             uint32_t w0 = 0, w1 = 0;
@@ -81,7 +82,7 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
             *reinterpret_cast<uint32_t *>(lane + 4 * (2 + hh)) = w1;
         }
     }
-    a.out[a.off.os + (t * p.nb + s) * 16 + rr] = (uint8_t)S;
+    slot[(b == 4 ? 256 : 512) + rr] = (uint8_t)S;
 
     if (a.with_planes) {
         uint8_t *prow = a.out + a.off.planes + n * p.kp;

@@ -52,14 +52,10 @@ def decode_act(bits, pcodes, pscales):
     return scales, codes
 
 
-def weight_offsets(N, bits):
+def weight_compact(N, bits):
     sb, (n4, n6, n8) = slot_blocks(bits)
-    n68 = n6 + n8
     T = (N + 15) // 16
-    o8 = align256(T * n4 * 256)
-    os_ = align256(o8 + T * n68 * 512)
-    compact = align256(os_ + 16 * T * len(bits))
-    return o8, os_, compact
+    return align256(T * (272 * n4 + 528 * (n6 + n8)))
 
 
 def decode_weight(N, bits, buf):
@@ -69,32 +65,32 @@ def decode_weight(N, bits, buf):
     nb = len(bits)
     K = 32 * nb
     T = (N + 15) // 16
-    o8, os_, _ = weight_offsets(N, bits)
+    TB = 272 * n4 + 528 * n68
     codes = np.zeros((16 * T, K), np.int8)
-    # lane l = 4g + q; row within tile = g + 8h
+    scales = np.zeros((16 * T, nb), np.uint8)
     lanes = np.arange(32)
     g, q = lanes // 4, lanes % 4
     for s, kb in enumerate(sb):
         for t in range(T):
             if s < n4:
-                ch = buf[(t * n4 + s) * 256:(t * n4 + s + 1) * 256].reshape(32, 2, 4)  # lane, h, j
+                base = t * TB + 272 * s
+                ch = buf[base:base + 256].reshape(32, 2, 4)  # lane, h, j
                 for h in range(2):
                     for j in range(4):
                         rows = 16 * t + g + 8 * h
                         byte = ch[:, h, j]
                         codes[rows, 32 * kb + 4 * q + j] = signmag4(byte >> 4)
                         codes[rows, 32 * kb + 16 + 4 * q + j] = signmag4(byte & 0xF)
+                scales[16 * t:16 * t + 16, kb] = buf[base + 256:base + 272]
             else:
-                base = o8 + (t * n68 + (s - n4)) * 512
+                base = t * TB + 272 * n4 + 528 * (s - n4)
                 ch = signmag8(buf[base:base + 512].reshape(32, 4, 4))  # lane, reg, j
                 for reg in range(4):
                     h = reg % 2
                     e0 = 16 if reg >= 2 else 0
                     for j in range(4):
                         codes[16 * t + g + 8 * h, 32 * kb + e0 + 4 * q + j] = ch[:, reg, j]
-    sc = buf[os_:os_ + 16 * T * nb].reshape(T, nb, 16).transpose(0, 2, 1).reshape(16 * T, nb)
-    scales = np.zeros((16 * T, nb), np.uint8)
-    scales[:, sb] = sc
+                scales[16 * t:16 * t + 16, kb] = buf[base + 512:base + 528]
     return scales[:N], codes[:N]
 
 

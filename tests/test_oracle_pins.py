@@ -341,7 +341,7 @@ def test_pack_weight_round_trip(N):
     buf = mxo.pack_weight(bits, scales, codes, with_planes=True)
     s2, c2 = mxformat.decode_weight(N, bits, buf)
     assert np.array_equal(s2, scales) and np.array_equal(c2, codes)
-    _, _, compact = mxformat.weight_offsets(N, bits)
+    compact = mxformat.weight_compact(N, bits)
     kp, nst = mxo.plane_shape(bits)
     pl = buf[compact:compact + N * kp].reshape(N, kp)
     sf_off = mxformat.align256(compact + N * kp)
