@@ -43,17 +43,15 @@
  *     one int8 per element.  Activation scales: uint8 [M, K/32] by slot.
  *   Weight buffer (layout MXS_W_COMPACT): codes are sign-magnitude, a 4-bit
  *     code as (sign<<3)|m and a 6/8-bit code as (sign<<7)|m (the symmetric
- *     clamp never yields -2^(b-1)); rows are padded to Np = 16*ceil(N/16) and
- *     cut into tiles of 16 rows; tile t is TB = 272*n4 + 528*(n6+n8)
- *     contiguous bytes at t*TB, so any K range of a tile is one copy:
- *       4-bit slot s at 272*s: 256 code bytes, then 16 scale bytes (row r at +256+r);
- *       6/8-bit slot n4+j at 272*n4 + 528*j: 512 code bytes, then 16 scale bytes.
- *     Codes are in the order a warp holds the A operand of a 16x8x32 MMA
- *     (lane l = 4g+q: rows g, g+8; elements 4q..4q+3 and 16+4q..16+4q+3):
- *       4-bit byte 8l+4h+j: row g+8h, high nibble = element 4q+j, low nibble =
- *       element 16+4q+j;  6/8-bit byte 16l+4c+j: c=0 row g elem 4q+j, c=1 row
- *       g+8 elem 4q+j, c=2 row g elem 16+4q+j, c=3 row g+8 elem 16+4q+j.
- *     Compact size = align256(T*TB); scale bytes of padding rows are 0.
+ *     clamp never yields -2^(b-1)); rows are padded to a multiple of 128 and
+ *     cut into groups of 128 rows; group g is GB = 2176*n4 + 4224*(n6+n8)
+ *     contiguous bytes at g*GB, so any K range of a group is one copy:
+ *       4-bit slot s at 2176*s: 128 rows x 16 code bytes (row r at 16r; byte
+ *         4i+j holds element 8i+j in the low nibble, 8i+4+j in the high
+ *         nibble), then the rows' 128 scale bytes;
+ *       6/8-bit slot n4+j at 2176*n4 + 4224*j: 128 rows x 32 code bytes
+ *         (row r at 32r, byte e = element e), then 128 scale bytes.
+ *     Compact size = align256(G*GB); scale bytes of padding rows are 0.
  *   MMA planes (layout MXS_W_COMPACT_AND_PLANES for weights, the `planes`
  *     output of mxs_quantize_act for activations), Kp = 128*(ceil(n4/4) +
  *     ceil((n6+n8)/2)):

@@ -320,25 +320,20 @@ int mxo_pack_act(int64_t R, int64_t K, const uint8_t *bits, const uint8_t *scale
 /* Weight stream.  Codes are stored sign-magnitude: a 4-bit code as
  * (sign << 3) | |m| and a 6/8-bit code as (sign << 7) | |m| (the symmetric
  * clamp R4 never produces -2^(b-1), so nothing is lost).  Rows are padded to
- * Np = 16*ceil(N/16) and cut into tiles of 16 rows; tile t occupies
- * TB = 272*n4 + 528*(n6+n8) contiguous bytes at t*TB:
- *   4-bit slot s:      at 272*s: 256 bytes of codes, then 16 scale bytes;
- *   6/8-bit slot n4+j: at 272*n4 + 528*j: 512 bytes of codes, then 16 scales.
- * The codes of one slot are in the order in which lane l = 4g+q of a warp
- * holds the operand of a 16x8x32 warp MMA: row g (and g+8), elements
- * 4q..4q+3 and 16+4q..16+4q+3.
- *   4-bit:   byte 8l + 4h + j (h in {0,1}, j<4): row g+8h of the tile;
- *            high nibble = element 4q+j, low nibble = element 16+4q+j.
- *   6/8-bit: byte 16l + 4c + j: c=0 row g elem 4q+j; c=1 row g+8 elem 4q+j;
- *            c=2 row g elem 16+4q+j; c=3 row g+8 elem 16+4q+j.
- *   scale byte r of a slot: row r of the tile (zero for padding rows).
- *   Compact size = align256(T*TB).
+ * a multiple of 128 and cut into groups of 128 rows; group g occupies
+ * GB = 2176*n4 + 4224*(n6+n8) contiguous bytes at g*GB:
+ *   4-bit slot s at 2176*s: 128 rows x 16 code bytes (row r at 16r), then
+ *     128 scale bytes (row r at 2048 + r).  In a row, byte 4i+j holds
+ *     element 8i+j in its low nibble and element 8i+4+j in its high nibble;
+ *   6/8-bit slot n4+j at 2176*n4 + 4224*j: 128 rows x 32 code bytes (row r
+ *     at 32r, byte e = element e), then 128 scale bytes (row r at 4096 + r).
+ *   Scale bytes of padding rows are zero.  Compact size = align256(G*GB).
  *   With planes: section P (offset compact size): [N, Kp] e4m3 planes and
  *   section SF (offset align256(P + N*Kp)): tcgen05 scale tiles, see below. */
-static int64_t tile_bytes(int64_t n4, int64_t n68) { return 272 * n4 + 528 * n68; }
+static int64_t group_bytes(int64_t n4, int64_t n68) { return 2176 * n4 + 4224 * n68; }
 static int64_t weight_compact(int64_t N, int64_t n4, int64_t n68)
 {
-    return align256((N + 15) / 16 * tile_bytes(n4, n68));
+    return align256((N + 127) / 128 * group_bytes(n4, n68));
 }
 
 /* Planes: for every row, Kp = 128*(ceil(n4/4) + ceil(n68/2)) e4m3 bytes.
@@ -468,28 +463,29 @@ int mxo_pack_weight(int64_t N, int64_t K, const uint8_t *bits, const uint8_t *sc
     int64_t cnt[3];
     if (!sb || mxo_slots(bits, nb, sb, cnt) != 0) { free(sb); return -1; }
     const int64_t n4 = cnt[0], n68 = cnt[1] + cnt[2];
-    const int64_t TB = tile_bytes(n4, n68), compact = weight_compact(N, n4, n68);
+    const int64_t GB = group_bytes(n4, n68), compact = weight_compact(N, n4, n68);
     const int64_t total = mxo_weight_bytes(N, K, bits, with_planes);
     memset(out, 0, (size_t)total);
     for (int64_t r = 0; r < N; ++r) {
-        const int64_t t = r / 16, rr = r % 16, g = rr % 8, h = rr / 8;
+        const int64_t grp = r / 128, rr = r % 128;
         for (int64_t s = 0; s < nb; ++s) {
             const int64_t kb = sb[s];
             const int8_t *c = codes + r * K + kb * MXO_BLOCK;
-            uint8_t *slot = out + t * TB + (s < n4 ? 272 * s : 272 * n4 + 528 * (s - n4));
-            slot[(s < n4 ? 256 : 512) + rr] = scales[r * nb + kb];
-            for (int i = 0; i < MXO_BLOCK; ++i) {
-                const int second = i >= 16;          /* elements 16..31 */
-                const int q = (i % 16) / 4, j = i % 4;
-                const int64_t lane = 4 * g + q;
-                const int mag = c[i] < 0 ? -c[i] : c[i];
-                if (s < n4) {
-                    uint8_t *byte = slot + 8 * lane + 4 * h + j;
-                    uint8_t nib = (uint8_t)(((c[i] < 0) << 3) | mag);
-                    *byte |= (uint8_t)(second ? nib : (nib << 4));
-                } else {
-                    const int reg = (second ? 2 : 0) + (int)h;
-                    slot[16 * lane + 4 * reg + j] = (uint8_t)(((c[i] < 0) << 7) | mag);
+            uint8_t *slot = out + grp * GB + (s < n4 ? 2176 * s : 2176 * n4 + 4224 * (s - n4));
+            if (s < n4) {
+                slot[2048 + rr] = scales[r * nb + kb];
+                for (int e = 0; e < MXO_BLOCK; ++e) {
+                    const int mag = c[e] < 0 ? -c[e] : c[e];
+                    const uint8_t nib = (uint8_t)(((c[e] < 0) << 3) | mag);
+                    const int i = e / 8, within = e % 8;       /* word i of the row */
+                    uint8_t *byte = slot + 16 * rr + 4 * i + (within % 4);
+                    *byte |= (uint8_t)(within < 4 ? nib : (nib << 4));
+                }
+            } else {
+                slot[4096 + rr] = scales[r * nb + kb];
+                for (int e = 0; e < MXO_BLOCK; ++e) {
+                    const int mag = c[e] < 0 ? -c[e] : c[e];
+                    slot[32 * rr + e] = (uint8_t)(((c[e] < 0) << 7) | mag);
                 }
             }
         }

@@ -29,22 +29,23 @@ __host__ __device__ inline int slot_width(const Plan &p, int s) {
 
 __host__ __device__ inline int64_t align256(int64_t v) { return (v + 255) / 256 * 256; }
 
-// Packed weights: tile t (16 rows) is TB = 272*n4 + 528*n68 contiguous bytes;
-// a 4-bit slot is 256 code bytes + 16 scale bytes, a 6/8-bit slot 512 + 16.
+// Packed weights: group g (128 rows) is GB = 2176*n4 + 4224*n68 contiguous
+// bytes; a 4-bit slot is 128 x 16 code bytes + 128 scale bytes, a 6/8-bit
+// slot 128 x 32 + 128.
 struct WeightOffsets {
-    int64_t T, Np, TB, compact, planes, sf, total;
+    int64_t G, Np, GB, compact, planes, sf, total;
 };
 
 __host__ __device__ inline int64_t slot_offset(const Plan &p, int s) {
-    return s < p.n4 ? 272 * (int64_t)s : 272 * (int64_t)p.n4 + 528 * (int64_t)(s - p.n4);
+    return s < p.n4 ? 2176 * (int64_t)s : 2176 * (int64_t)p.n4 + 4224 * (int64_t)(s - p.n4);
 }
 
 __host__ __device__ inline WeightOffsets weight_offsets(const Plan &p, int64_t N, bool with_planes) {
     WeightOffsets w;
-    w.T = (N + 15) / 16;
-    w.Np = w.T * 16;
-    w.TB = 272 * (int64_t)p.n4 + 528 * (int64_t)p.n68;
-    w.compact = align256(w.T * w.TB);
+    w.G = (N + 127) / 128;
+    w.Np = w.G * 128;
+    w.GB = 2176 * (int64_t)p.n4 + 4224 * (int64_t)p.n68;
+    w.compact = align256(w.G * w.GB);
     w.planes = w.compact;
     w.sf = align256(w.planes + N * p.kp);
     w.total = with_planes ? align256(w.sf + (N + 127) / 128 * p.nst * 512) : w.compact;

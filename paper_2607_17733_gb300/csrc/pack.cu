@@ -3,9 +3,9 @@
 // Same MXINT rule as the activations (Appendix A.2: weights and activations
 // of every linear layer are quantized; Sec. 4.1: one width per 32-element
 // block).  One thread owns one (row, slot) block: it loads the 32 bf16 values
-// with four 128-bit loads and scatters the codes (sign-magnitude) into the
-// 16-row fragment tiles read by the decode kernel, the scale byte, and
-// optionally the e4m3
+// with four 128-bit loads and writes the row's sign-magnitude codes and scale
+// byte into its 128-row group (read by the decode kernel), and optionally the
+// e4m3
 // digit planes and scale tiles read by the tensor-core prefill kernel.  The
 // buffer is cleared first, so padding rows and slots read as zero.  This runs
 // once per layer and is not on the timed path.
@@ -54,35 +54,33 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
     // sign-magnitude codes: (sign << 3) | |m| for 4 bits, (sign << 7) | |m| for 6/8 bits
     auto sm4 = [](int v) { return (uint32_t)(((v < 0) << 3) | (v < 0 ? -v : v)); };
     auto sm8 = [](int v) { return (uint32_t)(((v < 0) << 7) | (v < 0 ? -v : v)); };
-    const int64_t t = n >> 4;
-    const int rr = (int)(n & 15), g = rr & 7, hh = rr >> 3;
-    uint8_t *slot = a.out + t * a.off.TB + slot_offset(p, s);
+    const int64_t grp = n >> 7;
+    const int rr = (int)(n & 127);
+    uint8_t *slot = a.out + grp * a.off.GB + slot_offset(p, s);
     if (b == 4) {
-        uint8_t *chunk = slot;
+        // row word i: byte j = element 8i+j (low nibble) | element 8i+4+j (high nibble)
+        uint32_t w[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            uint32_t word = 0;
+        for (int i = 0; i < 4; ++i) {
+            w[i] = 0;
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-                word |= ((sm4(m[4 * q + j]) << 4) | sm4(m[16 + 4 * q + j])) << (8 * j);
-            *reinterpret_cast<uint32_t *>(chunk + 8 * (4 * g + q) + 4 * hh) = word;
+            for (int j = 0; j < 4; ++j) w[i] |= (sm4(m[8 * i + j]) | (sm4(m[8 * i + 4 + j]) << 4)) << (8 * j);
         }
+        *reinterpret_cast<uint4 *>(slot + 16 * rr) = make_uint4(w[0], w[1], w[2], w[3]);
+        slot[2048 + rr] = (uint8_t)S;
     } else {
-        uint8_t *chunk = slot;
+        uint32_t w[8];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            uint32_t w0 = 0, w1 = 0;
+        for (int i = 0; i < 8; ++i) {
+            w[i] = 0;
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                w0 |= sm8(m[4 * q + j]) << (8 * j);
-                w1 |= sm8(m[16 + 4 * q + j]) << (8 * j);
-            }
-            uint8_t *lane = chunk + 16 * (4 * g + q);
-            *reinterpret_cast<uint32_t *>(lane + 4 * hh) = w0;
-            *reinterpret_cast<uint32_t *>(lane + 4 * (2 + hh)) = w1;
+            for (int j = 0; j < 4; ++j) w[i] |= sm8(m[4 * i + j]) << (8 * j);
         }
+        uint4 *dst = reinterpret_cast<uint4 *>(slot + 32 * rr);
+        dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+        dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+        slot[4096 + rr] = (uint8_t)S;
     }
-    slot[(b == 4 ? 256 : 512) + rr] = (uint8_t)S;
 
     if (a.with_planes) {
         uint8_t *prow = a.out + a.off.planes + n * p.kp;

@@ -54,8 +54,8 @@ def decode_act(bits, pcodes, pscales):
 
 def weight_compact(N, bits):
     sb, (n4, n6, n8) = slot_blocks(bits)
-    T = (N + 15) // 16
-    return align256(T * (272 * n4 + 528 * (n6 + n8)))
+    G = (N + 127) // 128
+    return align256(G * (2176 * n4 + 4224 * (n6 + n8)))
 
 
 def decode_weight(N, bits, buf):
@@ -64,33 +64,27 @@ def decode_weight(N, bits, buf):
     n68 = n6 + n8
     nb = len(bits)
     K = 32 * nb
-    T = (N + 15) // 16
-    TB = 272 * n4 + 528 * n68
-    codes = np.zeros((16 * T, K), np.int8)
-    scales = np.zeros((16 * T, nb), np.uint8)
-    lanes = np.arange(32)
-    g, q = lanes // 4, lanes % 4
+    G = (N + 127) // 128
+    GB = 2176 * n4 + 4224 * n68
+    codes = np.zeros((128 * G, K), np.int8)
+    scales = np.zeros((128 * G, nb), np.uint8)
+    # element e of a 4-bit row: word e//8, byte (e%8)%4, low nibble if e%8 < 4
+    e = np.arange(32)
+    byte_of = 4 * (e // 8) + (e % 8) % 4
+    high = (e % 8) >= 4
     for s, kb in enumerate(sb):
-        for t in range(T):
+        for grp in range(G):
+            rows = slice(128 * grp, 128 * grp + 128)
             if s < n4:
-                base = t * TB + 272 * s
-                ch = buf[base:base + 256].reshape(32, 2, 4)  # lane, h, j
-                for h in range(2):
-                    for j in range(4):
-                        rows = 16 * t + g + 8 * h
-                        byte = ch[:, h, j]
-                        codes[rows, 32 * kb + 4 * q + j] = signmag4(byte >> 4)
-                        codes[rows, 32 * kb + 16 + 4 * q + j] = signmag4(byte & 0xF)
-                scales[16 * t:16 * t + 16, kb] = buf[base + 256:base + 272]
+                base = grp * GB + 2176 * s
+                blk = buf[base:base + 2048].reshape(128, 16)
+                nib = np.where(high[None, :], blk[:, byte_of] >> 4, blk[:, byte_of] & 0xF)
+                codes[rows, 32 * kb:32 * kb + 32] = signmag4(nib)
+                scales[rows, kb] = buf[base + 2048:base + 2176]
             else:
-                base = t * TB + 272 * n4 + 528 * (s - n4)
-                ch = signmag8(buf[base:base + 512].reshape(32, 4, 4))  # lane, reg, j
-                for reg in range(4):
-                    h = reg % 2
-                    e0 = 16 if reg >= 2 else 0
-                    for j in range(4):
-                        codes[16 * t + g + 8 * h, 32 * kb + e0 + 4 * q + j] = ch[:, reg, j]
-                scales[16 * t:16 * t + 16, kb] = buf[base + 512:base + 528]
+                base = grp * GB + 2176 * n4 + 4224 * (s - n4)
+                codes[rows, 32 * kb:32 * kb + 32] = signmag8(buf[base:base + 4096].reshape(128, 32))
+                scales[rows, kb] = buf[base + 4096:base + 4224]
     return scales[:N], codes[:N]
 
 
