@@ -53,8 +53,10 @@ def parse():
                     help="decoder layers per step (default 32 for decode, 8 for prefill)")
     ap.add_argument("--workload", default="llama3-8b-decode", choices=["llama3-8b-decode", "llama3-8b-prefill"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--unfused", action="store_true",
-                    help="separate quantize and GEMM launches instead of the fused decode kernel")
+    ap.add_argument("--path", default="planes", choices=["planes", "fused", "codes"],
+                    help="decode activation path: quantize all projections to MMA planes, then the GEMMs "
+                         "(planes); mxs_linear_decode per projection, the GEMM a programmatic dependent of "
+                         "its quantizer (fused); quantize to packed codes, GEMM over the codes (codes)")
     ap.add_argument("--eager", action="store_true",
                     help="launch the step's kernels directly (no CUDA graph, no events): for ncu runs")
     return ap.parse_args()
@@ -318,12 +320,15 @@ def run_ours(args):
     # ---- algorithmic work per step
     step_bytes = sum(lin.weight_bytes + M * lin.K * 2 + M * lin.N * 4 for M, lin, _, _ in items)
     step_ops = sum(2 * M * lin.N * lin.K for M, lin, _, _ in items)
-    if args.unfused:  # the GEMM reads the packed codes the quantizer wrote
+    if args.path == "codes":  # the GEMM reads the packed codes the quantizer wrote
         gemm_bytes = sum(lin.weight_bytes + M * (mxs.act_row_bytes(lin.K, lin.bits) + lin.K // 32) + M * lin.N * 4
                          for M, lin, _, _ in items)
-    else:  # the fused kernel reads the bf16 activations itself
+    elif args.path == "planes":  # the GEMM reads the activations' MMA planes (digits + scale tiles)
+        gemm_bytes = sum(lin.weight_bytes + mxs.act_planes_bytes(M, lin.K, lin.bits) + M * lin.N * 4
+                         for M, lin, _, _ in items)
+    else:  # the timed segment is quantize + GEMM: bf16 activations in, y out
         gemm_bytes = step_bytes
-    launches_per_step = (2 if args.unfused else 1) * len(items)
+    launches_per_step = 2 * len(items)
 
     # ---- the step as one CUDA graph.  Inputs are independent synthetic draws, so
     # for each M the graph runs all activation quantizations, then all GEMMs;
@@ -336,16 +341,23 @@ def run_ours(args):
     def make_step(events=None):
         def fn():
             for gi, grp in enumerate(groups):
-                if args.unfused:
+                if args.path != "fused":
                     for M, lin, x, bufs in grp:
-                        lin.quantize(x, bufs)
+                        if args.path == "codes":
+                            lin.quantize(x, bufs)
+                        else:
+                            mxs.quantize_act(x, lin.bits, rounding=lin.rounding, planes=bufs["planes"],
+                                             want_codes=False, want_planes=True)
                 if events is not None:
                     events[gi][0].record()
                 for M, lin, x, bufs in grp:
-                    if args.unfused:
+                    if args.path == "codes":
                         lin.matmul(bufs)
+                    elif args.path == "planes":
+                        mxs.gemm_decode(None, None, lin.bits, lin.packed, lin.N, y=bufs["y"], planes=bufs["planes"],
+                                        M=M)
                     else:
-                        lin.fused(x, bufs["y"])
+                        lin.fused(x, bufs["y"], bufs["planes"])
                 if events is not None:
                     events[gi][1].record()
         return fn
@@ -416,7 +428,8 @@ def run_ours(args):
         gemm_ms = sum(s.elapsed_time(e) for evs in ev_sets for s, e in evs) / len(ev_sets)  # per step
         achieved = gemm_bytes / (gemm_ms * 1e-3) / 1e9
         traffic = profile_traffic("gemm_decode.cu", "gemm_decode_llama3_8b_decode.md")
-        roofline = {"kernel": "gemm_decode_kernel" + ("" if args.unfused else " (fused quantize)"),
+        roofline = {"kernel": "gemm_decode_kernel" + (" + quantize_act_kernel (PDL chain)" if args.path == "fused"
+                                                      else f" (from {args.path})"),
                     "bound": "hbm", "achieved": achieved,
                     "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": achieved / pk["hbm_gbs"],
                     "peak_source": pk["source"], "traffic": traffic,
@@ -453,7 +466,9 @@ def run_ours(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "int8+f32",
             "data": "synthetic (seeded; weights N(0,0.02), activations N(0,1) with 1% outlier columns x30)",
             "config": {"workload": "llama3-8b-decode", "M": list(DECODE_MS), "layers": L,
-                       "path": "quantize + GEMM" if args.unfused else "fused quantize-GEMM (one launch per projection)",
+                       "path": {"planes": "quantize to MMA planes, then GEMM over the planes (TMA)",
+                                "fused": "mxs_linear_decode: quantize + GEMM chained by programmatic dependent launch",
+                                "codes": "quantize to packed codes, GEMM over the codes"}[args.path],
                        "projections": [p[0] for p in I.LLAMA3_8B], "map_4_6_8": list(MAP),
                        "parallelism": f"replicas x{ws}", "l2": "inputs larger than L2 (packed weights "
                        f"{sum(lin.weight_bytes for p in layers for lin in p) / 1e9:.2f} GB per step)"},

@@ -141,9 +141,9 @@ MXS_API int mxs_pack_weight(const void *w_bf16, int64_t N, int64_t K, int64_t ld
  * operands.  act_bits must equal w_bits (the paper allocates one map per
  * linear layer and applies it to W and A); other pairs return
  * MXS_ERR_UNSUPPORTED.  `w_layout` is the layout W was packed with.
- * mxs_gemm picks the decode kernel for M <= 16 (needs codes/scales) and the
- * tensor-core prefill kernel otherwise (needs act_planes and a weight packed
- * with MXS_W_COMPACT_AND_PLANES).  workspace may be NULL when
+ * mxs_gemm picks the decode kernel for M <= 16 (over act_planes when given,
+ * else over codes/scales) and the tensor-core prefill kernel otherwise (needs
+ * act_planes and a weight packed with MXS_W_COMPACT_AND_PLANES).  workspace may be NULL when
  * mxs_gemm_workspace_bytes() is 0. */
 MXS_API int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const void *act_planes,
              const uint8_t *act_bits, const void *packed_w, int w_layout, const uint8_t *w_bits,
@@ -151,22 +151,30 @@ MXS_API int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const voi
              void *workspace, size_t ws_bytes, void *stream);
 
 /* Decode path only (M <= 16): weights streamed once from the compact layout by
- * bulk copies into a shared-memory ring; exact FP8 warp MMAs per block on
- * sign-magnitude digits, fp32 fold; when K is split over a thread-block
- * cluster the partial tiles are added in rank order.  Needs no workspace
- * (ws may be NULL).  Waits are bounded like the prefill kernel's. */
-MXS_API int mxs_gemm_decode(const void *act_codes, const uint8_t *act_scales, const uint8_t *bits,
-                    const void *packed_w, int64_t M, int64_t N, int64_t K,
+ * bulk copies into shared memory, converted there to exact e4m3 digits and
+ * multiplied on the block-scaled tensor-core MMA (tcgen05, fp32 accumulation
+ * in tensor memory); when K is split over a thread-block cluster the partial
+ * tiles are added in rank order.  The activations are given EITHER as packed
+ * codes + scales (act_planes NULL) OR as the MMA planes written by
+ * mxs_quantize_act (codes and scales NULL; faster: the operand is loaded by
+ * TMA instead of being rebuilt by every CTA).  Needs no workspace (ws may be
+ * NULL).  Waits inside the kernel are bounded like the prefill kernel's. */
+MXS_API int mxs_gemm_decode(const void *act_codes, const uint8_t *act_scales, const void *act_planes,
+                    const uint8_t *bits, const void *packed_w, int64_t M, int64_t N, int64_t K,
                     float *y, int64_t ld_y, void *workspace, size_t ws_bytes, void *stream);
 
-/* A1 fused into A4 (M <= 16): quantizes x (bf16 [M,K], row stride ld_x) with
- * `bits` and `rounding` inside the decode GEMM's prologue -- the same codes
- * mxs_quantize_act would write, never stored -- and returns y [M,N] fp32 =
- * x W^T like mxs_gemm_decode.  One launch per linear layer and token batch
- * (Appendix A.2: activations are quantized on the fly). */
+/* A1 + A4 for one linear layer at decode (M <= 16): quantizes x (bf16 [M,K],
+ * row stride ld_x elements) with `bits` and `rounding` into MMA planes in
+ * `workspace` (at least mxs_act_planes_bytes(M, K, bits) bytes, 16-byte
+ * aligned; the same planes mxs_quantize_act writes) and returns
+ * y [M,N] fp32 = x W^T like mxs_gemm_decode.  Two kernels on `stream`; the
+ * GEMM is launched as a programmatic dependent of the quantizer, so its
+ * weight stream starts while the activations are quantized (Appendix A.2:
+ * activations are quantized on the fly).  The workspace is scratch: it may be
+ * reused once the call's work on `stream` has finished. */
 MXS_API int mxs_linear_decode(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits,
                               int rounding, const void *packed_w, int64_t N, float *y, int64_t ld_y,
-                              void *stream);
+                              void *workspace, size_t ws_bytes, void *stream);
 
 /* Prefill path only (any M >= 1, efficient for M >= 128): the tensor-core
  * kernel over the MMA planes of the activations (mxs_quantize_act `planes`)

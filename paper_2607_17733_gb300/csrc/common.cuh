@@ -3,6 +3,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include "../../include/mxs.h"
@@ -106,13 +107,16 @@ int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rou
 int launch_pack_weight(const Plan &p, const void *w, int64_t N, int64_t ld, int rounding, bool planes,
                        void *packed, cudaStream_t st);
 int64_t decode_workspace_bytes(const Plan &p, int64_t M, int64_t N);
-int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, const void *packed,
-                       int64_t M, int64_t N, float *y, int64_t ld_y, void *ws, size_t ws_bytes,
-                       cudaStream_t st);
-int launch_linear_decode(const Plan &p, const void *x, int64_t ld_x, int rounding, const void *packed, int64_t M,
-                         int64_t N, float *y, int64_t ld_y, cudaStream_t st);
+// decode GEMM over packed codes + scales (act_planes NULL) or over the
+// activation MMA planes (codes/scales NULL); pdl: the launch may overlap the
+// tail of the previous kernel on the stream (programmatic dependent launch)
+int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, const void *act_planes,
+                       const void *packed, int64_t M, int64_t N, float *y, int64_t ld_y, bool pdl, cudaStream_t st);
 int decode_status(int *status, int reset);
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N,
                         float *y, int64_t ld_y, int starve, cudaStream_t st);
 int prefill_status(int *status, int reset, cudaStream_t st);
+// 2-D TMA map over an e4m3 plane matrix [rows, kp] (row stride kp bytes):
+// boxes of 128 bytes x box_rows rows, 128-byte swizzle, zero fill outside
+int make_plane_map(CUtensorMap *map, const void *base, int64_t rows, int64_t kp, int box_rows);
 }  // namespace mxs

@@ -304,32 +304,6 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
     }
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (!fn) {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    }
-    return fn;
-}
-
-int make_map(CUtensorMap *map, const void *base, int64_t rows, int64_t kp, int box_rows) {
-    auto fn = encode_fn();
-    if (!fn) return fail(MXS_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
-    cuuint64_t dims[2] = {(cuuint64_t)kp, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)kp};
-    cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
-    cuuint32_t estr[2] = {1, 1};
-    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return fail(MXS_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
-    return MXS_OK;
-}
-
 }  // namespace
 
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N, float *y,
@@ -339,9 +313,9 @@ int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packe
     const uint8_t *wb = static_cast<const uint8_t *>(packed_w);
     const WeightOffsets off = weight_offsets(p, N, true);
     CUtensorMap ta, tb;
-    int rc = make_map(&ta, ap, M, p.kp, kBM);
+    int rc = make_plane_map(&ta, ap, M, p.kp, kBM);
     if (rc) return rc;
-    rc = make_map(&tb, wb + off.planes, N, p.kp, kBN);
+    rc = make_plane_map(&tb, wb + off.planes, N, p.kp, kBN);
     if (rc) return rc;
     PrefillArgs a;
     a.sfa = ap + align256(M * p.kp);

@@ -6,6 +6,8 @@
 #include <cstdio>
 #include <cstring>
 
+#include <cudaTypedefs.h>
+
 #include "common.cuh"
 
 namespace mxs {
@@ -77,6 +79,33 @@ int check_device() {
     const bool ok = major == 10 && minor == 3;
     if (dev >= 0 && dev < 64) cached[dev] = ok ? 1 : 2;
     if (!ok) return fail(MXS_ERR_UNSUPPORTED, "device %d is sm_%d%d; libmxs is built for sm_103a only", dev, major, minor);
+    return MXS_OK;
+}
+
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    }
+    return fn;
+}
+
+int make_plane_map(CUtensorMap *map, const void *base, int64_t rows, int64_t kp, int box_rows) {
+    auto fn = encode_fn();
+    if (!fn) return fail(MXS_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+    cuuint64_t dims[2] = {(cuuint64_t)kp, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)kp};
+    cuuint32_t box[2] = {128u, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(MXS_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
     return MXS_OK;
 }
 
@@ -165,30 +194,33 @@ int mxs_pack_weight(const void *w, int64_t N, int64_t K, int64_t ld_w, const uin
                               static_cast<cudaStream_t>(stream));
 }
 
-int mxs_gemm_decode(const void *codes, const uint8_t *scales, const uint8_t *bits, const void *packed_w,
-                    int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, void *ws, size_t ws_bytes,
-                    void *stream) {
+int mxs_gemm_decode(const void *codes, const uint8_t *scales, const void *act_planes, const uint8_t *bits,
+                    const void *packed_w, int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, void *ws,
+                    size_t ws_bytes, void *stream) {
     Plan p;
     int rc = build_plan(bits, K, &p);
     if (rc) return rc;
     if (M < 0 || N < 0) return fail(MXS_ERR_SHAPE, "M=%lld N=%lld", (long long)M, (long long)N);
     if (M > 16) return fail(MXS_ERR_SHAPE, "decode path takes M <= 16 (M=%lld)", (long long)M);
-    if (!codes || !scales || !packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
+    if (!packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
+    if (act_planes ? (codes || scales) : (!codes || !scales))
+        return fail(MXS_ERR_INVALID_ARG, "give either act_planes or codes and scales");
     if (ld_y < N) return fail(MXS_ERR_INVALID_ARG, "ld_y=%lld < N", (long long)ld_y);
-    if (!aligned16(codes) || !aligned16(packed_w) || (reinterpret_cast<uintptr_t>(y) & 3))
-        return fail(MXS_ERR_ALIGN, "codes/packed_w must be 16-byte aligned, y 4-byte aligned");
+    if ((codes && !aligned16(codes)) || (act_planes && !aligned16(act_planes)) || !aligned16(packed_w) ||
+        (reinterpret_cast<uintptr_t>(y) & 3))
+        return fail(MXS_ERR_ALIGN, "codes/act_planes/packed_w must be 16-byte aligned, y 4-byte aligned");
     const int64_t need = decode_workspace_bytes(p, M, N);
     if ((int64_t)ws_bytes < need || (need > 0 && !ws))
         return fail(MXS_ERR_BUFFER, "workspace of %lld bytes needed, %zu given", (long long)need, ws_bytes);
-    if (ws && !aligned16(ws)) return fail(MXS_ERR_ALIGN, "workspace must be 16-byte aligned");
     if (M == 0 || N == 0) return MXS_OK;
     if ((rc = check_device())) return rc;
-    return launch_gemm_decode(p, codes, scales, packed_w, M, N, y, ld_y, ws, ws_bytes,
+    return launch_gemm_decode(p, codes, scales, act_planes, packed_w, M, N, y, ld_y, false,
                               static_cast<cudaStream_t>(stream));
 }
 
 int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits, int rounding,
-                      const void *packed_w, int64_t N, float *y, int64_t ld_y, void *stream) {
+                      const void *packed_w, int64_t N, float *y, int64_t ld_y, void *ws, size_t ws_bytes,
+                      void *stream) {
     Plan p;
     int rc = build_plan(bits, K, &p);
     if (rc) return rc;
@@ -198,11 +230,17 @@ int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const u
     if (!x || !packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
     if (ld_x < K || ld_x % 8 != 0) return fail(MXS_ERR_INVALID_ARG, "ld_x=%lld must be >= K and a multiple of 8", (long long)ld_x);
     if (ld_y < N) return fail(MXS_ERR_INVALID_ARG, "ld_y=%lld < N", (long long)ld_y);
-    if (!aligned16(x) || !aligned16(packed_w) || (reinterpret_cast<uintptr_t>(y) & 3))
-        return fail(MXS_ERR_ALIGN, "x/packed_w must be 16-byte aligned, y 4-byte aligned");
+    const int64_t need = align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);  // mxs_act_planes_bytes
+    if ((int64_t)ws_bytes < need || (need > 0 && !ws))
+        return fail(MXS_ERR_BUFFER, "workspace of %lld bytes needed, %zu given", (long long)need, ws_bytes);
+    if (!aligned16(x) || !aligned16(packed_w) || (ws && !aligned16(ws)) || (reinterpret_cast<uintptr_t>(y) & 3))
+        return fail(MXS_ERR_ALIGN, "x/packed_w/workspace must be 16-byte aligned, y 4-byte aligned");
     if (M == 0 || N == 0) return MXS_OK;
     if ((rc = check_device())) return rc;
-    return launch_linear_decode(p, x, ld_x, rounding, packed_w, M, N, y, ld_y, static_cast<cudaStream_t>(stream));
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    rc = launch_quantize(p, x, M, ld_x, rounding, nullptr, nullptr, ws, st);
+    if (rc) return rc;
+    return launch_gemm_decode(p, nullptr, nullptr, ws, packed_w, M, N, y, ld_y, true, st);
 }
 
 int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const void *act_planes, const uint8_t *act_bits,
@@ -216,8 +254,9 @@ int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const void *act_p
         return fail(MXS_ERR_UNSUPPORTED, "activation and weight maps differ; one map per layer is supported");
     if (w_layout != MXS_W_COMPACT && w_layout != MXS_W_COMPACT_AND_PLANES)
         return fail(MXS_ERR_INVALID_ARG, "w_layout=%d", w_layout);
-    if (M <= 16)
-        return mxs_gemm_decode(act_codes, act_scales, act_bits, packed_w, M, N, K, y, ld_y, ws, ws_bytes, stream);
+    if (M <= 16)  // over the planes when given, else over the packed codes
+        return mxs_gemm_decode(act_planes ? nullptr : act_codes, act_planes ? nullptr : act_scales, act_planes,
+                               act_bits, packed_w, M, N, K, y, ld_y, ws, ws_bytes, stream);
     if (w_layout != MXS_W_COMPACT_AND_PLANES)
         return fail(MXS_ERR_INVALID_ARG, "M > 16 needs a weight packed with MXS_W_COMPACT_AND_PLANES");
     return mxs_gemm_prefill(act_planes, act_bits, packed_w, M, N, K, y, ld_y, stream);

@@ -23,6 +23,9 @@ struct QuantArgs {
 
 __global__ void __launch_bounds__(256) quantize_act_kernel(const __grid_constant__ Plan p,
                                                            const __grid_constant__ QuantArgs a) {
+    // a decode GEMM launched after this kernel with programmatic dependent
+    // launch may start now; it waits for this grid's writes before reading them
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int64_t gid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int l = threadIdx.x & 3;
     const int64_t item = gid >> 2;

@@ -66,9 +66,9 @@ def lib() -> ctypes.CDLL:
         L.mxs_pack_weight.restype = I
         L.mxs_gemm.argtypes = [P, P, P, P, P, I, P, I64, I64, I64, P, I64, P, SZ, P]
         L.mxs_gemm.restype = I
-        L.mxs_gemm_decode.argtypes = [P, P, P, P, I64, I64, I64, P, I64, P, SZ, P]
+        L.mxs_gemm_decode.argtypes = [P, P, P, P, P, I64, I64, I64, P, I64, P, SZ, P]
         L.mxs_gemm_decode.restype = I
-        L.mxs_linear_decode.argtypes = [P, I64, I64, I64, P, I, P, I64, P, I64, P]
+        L.mxs_linear_decode.argtypes = [P, I64, I64, I64, P, I, P, I64, P, I64, P, SZ, P]
         L.mxs_linear_decode.restype = I
         L.mxs_gemm_prefill.argtypes = [P, P, P, I64, I64, I64, P, I64, P]
         L.mxs_gemm_prefill.restype = I
@@ -193,10 +193,14 @@ def gemm(codes, scales, planes, bits, packed_w, N: int, w_layout: int = W_COMPAC
     return y
 
 
-def gemm_decode(codes, scales, bits, packed_w, N: int, y=None, workspace=None, stream=None):
+def gemm_decode(codes, scales, bits, packed_w, N: int, y=None, workspace=None, stream=None, planes=None,
+                M: int | None = None):
+    """Decode kernel (M <= 16) over packed codes + scales, or over the MMA
+    planes of quantize_act (pass planes=..., M=... and codes = scales = None)."""
     import torch
     b = _Bits(bits)
-    M = codes.shape[0]
+    if M is None:
+        M = codes.shape[0]
     K = 32 * len(b)
     if y is None:
         y = torch.empty((M, N), dtype=torch.float32, device=packed_w.device)
@@ -204,20 +208,25 @@ def gemm_decode(codes, scales, bits, packed_w, N: int, y=None, workspace=None, s
     if workspace is None and ws_need > 0:
         workspace = torch.empty(ws_need, dtype=torch.uint8, device=packed_w.device)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    check(lib().mxs_gemm_decode(_ptr(codes), _ptr(scales), b.ptr, _ptr(packed_w), M, N, K, _ptr(y),
+    check(lib().mxs_gemm_decode(_ptr(codes), _ptr(scales), _ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y),
                                 y.stride(0), _ptr(workspace), ws_bytes, _stream(stream)))
     return y
 
 
-def linear_decode(x, bits, packed_w, N: int, rounding: int = RNE, y=None, stream=None):
-    """Fused activation quantization + decode GEMM (M <= 16): y [M, N] fp32."""
+def linear_decode(x, bits, packed_w, N: int, rounding: int = RNE, y=None, workspace=None, stream=None):
+    """Activation quantization + decode GEMM (M <= 16) in one call: y [M, N]
+    fp32.  workspace: uint8 of at least act_planes_bytes(M, K, bits) bytes
+    (allocated when None)."""
     import torch
     b = _Bits(bits)
     M, K = x.shape
     if y is None:
         y = torch.empty((M, N), dtype=torch.float32, device=packed_w.device)
+    if workspace is None:
+        workspace = torch.empty(max(act_planes_bytes(M, K, b.arr), 16), dtype=torch.uint8, device=packed_w.device)
+    ws_bytes = workspace.numel() * workspace.element_size()
     check(lib().mxs_linear_decode(_ptr(x), M, K, x.stride(0), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
-                                  y.stride(0), _stream(stream)))
+                                  y.stride(0), _ptr(workspace), ws_bytes, _stream(stream)))
     return y
 
 

@@ -38,6 +38,9 @@ class MxLinear:
             "scales": torch.empty((M, self.K // 32), dtype=torch.uint8, device=device),
             "y": torch.empty((M, self.N), dtype=torch.float32, device=device),
             "ws": None,
+            # MMA planes of the activations, written and read inside fused()
+            "planes": torch.empty(max(mxs.act_planes_bytes(M, self.K, self.bits), 16), dtype=torch.uint8,
+                                  device=device) if M <= 16 else None,
         }
 
     def quantize(self, x: torch.Tensor, bufs: dict):
@@ -47,14 +50,15 @@ class MxLinear:
         return mxs.gemm(bufs["codes"], bufs["scales"], None, self.bits, self.packed, self.N,
                         w_layout=self.layout, y=bufs["y"], workspace=bufs["ws"])
 
-    def fused(self, x: torch.Tensor, y: torch.Tensor) -> torch.Tensor:
-        """M <= 16: activation quantization inside the decode GEMM (one launch)."""
-        return mxs.linear_decode(x, self.bits, self.packed, self.N, rounding=self.rounding, y=y)
+    def fused(self, x: torch.Tensor, y: torch.Tensor, planes: torch.Tensor | None = None) -> torch.Tensor:
+        """M <= 16: quantize to MMA planes and run the decode GEMM in one call
+        (two kernels, the GEMM a programmatic dependent of the quantizer)."""
+        return mxs.linear_decode(x, self.bits, self.packed, self.N, rounding=self.rounding, y=y, workspace=planes)
 
     def __call__(self, x: torch.Tensor, bufs: dict | None = None) -> torch.Tensor:
         bufs = bufs or self.buffers(x.shape[0], x.device)
         if x.shape[0] <= 16:
-            return self.fused(x, bufs["y"])
+            return self.fused(x, bufs["y"], bufs["planes"])
         self.quantize(x, bufs)
         return self.matmul(bufs)
 

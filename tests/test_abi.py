@@ -98,10 +98,20 @@ def test_pack_and_gemm_validation(L):
     g = L.mxs_gemm
     assert g(FAKE, FAKE, None, b, FAKE, 0, other.ctypes.data, 4, 16, 128, FAKE, 16, None, 0, None) == 8
     d = L.mxs_gemm_decode
-    assert d(FAKE, FAKE, b, FAKE, 17, 16, 128, FAKE, 16, None, 0, None) == 2   # M > 16
-    assert d(FAKE, FAKE, b, FAKE, 4, 16, 128, FAKE, 8, None, 0, None) == 1     # ld_y < N
-    assert d(FAKE, FAKE, b, None, 4, 16, 128, FAKE, 16, None, 0, None) == 1
-    assert d(FAKE, FAKE, b, FAKE, 4, 16, 128, FAKE + 2, 16, None, 0, None) == 4
+    assert d(FAKE, FAKE, None, b, FAKE, 17, 16, 128, FAKE, 16, None, 0, None) == 2   # M > 16
+    assert d(FAKE, FAKE, None, b, FAKE, 4, 16, 128, FAKE, 8, None, 0, None) == 1     # ld_y < N
+    assert d(FAKE, FAKE, None, b, None, 4, 16, 128, FAKE, 16, None, 0, None) == 1
+    assert d(FAKE, FAKE, None, b, FAKE, 4, 16, 128, FAKE + 2, 16, None, 0, None) == 4
+    assert d(FAKE, FAKE, FAKE, b, FAKE, 4, 16, 128, FAKE, 16, None, 0, None) == 1    # codes and planes
+    assert d(None, None, None, b, FAKE, 4, 16, 128, FAKE, 16, None, 0, None) == 1    # neither
+    assert d(None, None, FAKE + 8, b, FAKE, 4, 16, 128, FAKE, 16, None, 0, None) == 4
+    ld = L.mxs_linear_decode
+    need = L.mxs_act_planes_bytes(4, 128, b)
+    assert need > 0
+    assert ld(FAKE, 4, 128, 128, b, 0, FAKE, 16, FAKE, 16, FAKE, need - 1, None) == 5  # workspace too small
+    assert ld(FAKE, 4, 128, 128, b, 0, FAKE, 16, FAKE, 16, None, need, None) == 5
+    assert ld(FAKE, 4, 128, 128, b, 0, FAKE, 16, FAKE, 16, FAKE + 4, need, None) == 4
+    assert ld(FAKE, 17, 128, 128, b, 0, FAKE, 16, FAKE, 16, FAKE, need, None) == 2
 
 
 def test_valid_call_without_gpu_reports_cuda_error(L):

@@ -23,6 +23,16 @@ def layer(torch, M, K, N, bits, g, w_sigma=0.02, outlier_frac=0.01, outlier_scal
     return xb, wb, codes, scales, packed
 
 
+def decode_from(torch, src, xb, bits, packed, N, codes=None, scales=None):
+    """The decode kernel over packed codes, or over the MMA planes of the same
+    activations (TMA-loaded token operand)."""
+    M = xb.shape[0]
+    if src == "codes":
+        return mxs.gemm(codes, scales, None, bits, packed, N)
+    _, _, planes = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits, want_codes=False, want_planes=True)
+    return mxs.gemm_decode(None, None, bits, packed, N, planes=planes, M=M)
+
+
 def oracle_full(xb, wb, bits):
     a_s, a_c = mxo.quantize_bf16(xb, bits)
     w_s, w_c = mxo.quantize_bf16(wb, bits)
@@ -35,9 +45,28 @@ def test_decode_small(torch, M, N, nb):
     g = I.rng(M, N, nb)
     bits = I.width_map(nb, 0.7, 0.2, 0.1, g)
     xb, wb, codes, scales, packed = layer(torch, M, 32 * nb, N, bits, g)
-    y = mxs.gemm(codes, scales, None, bits, packed, N)
+    y = mxs.gemm(codes, scales, None, bits, packed, N).cpu().numpy()
     ref, ab = oracle_full(xb, wb, bits)
-    U.check_gemm(y.cpu().numpy(), ref, ab)
+    U.check_gemm(y, ref, ab)
+    # the same products in the same order over the planes: the same bits
+    y_planes = decode_from(torch, "planes", xb, bits, packed, N).cpu().numpy()
+    assert np.array_equal(y_planes, y, equal_nan=True)
+
+
+@pytest.mark.parametrize("M", [1, 5, 16])
+@pytest.mark.parametrize("N,nb,p", [(130, 3, (1, 0, 0)), (129, 7, (0, 0.5, 0.5)), (640, 61, (0.7, 0.2, 0.1)),
+                                    (256, 333, (0.9, 0.05, 0.05))])
+def test_decode_from_planes_ragged(torch, M, N, nb, p):
+    """Ragged stage counts (n4 % 4, n68 % 2 != 0), ragged N, K split over
+    cluster ranks: the planes path against the oracle."""
+    g = I.rng(60, M, N, nb)
+    bits = I.width_map(nb, *p, g)
+    xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=30.0)
+    wb = I.normal_bf16((N, 32 * nb), 0.02, g)
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
+    y = decode_from(torch, "planes", xb, bits, packed, N).cpu().numpy()
+    ref, ab = oracle_full(xb, wb, bits)
+    U.check_gemm(y, ref, ab)
 
 
 @pytest.mark.parametrize("p", [(1, 0, 0), (0, 1, 0), (0, 0, 1), (0.5, 0.3, 0.2)])
@@ -82,16 +111,17 @@ def test_decode_nan_block(torch):
 LLAMA3 = {name: (K, N) for name, K, N in I.LLAMA3_8B}
 
 
+@pytest.mark.parametrize("src", ["codes", "planes"])
 @pytest.mark.parametrize("proj", ["q", "k", "o", "gate", "down"])
 @pytest.mark.parametrize("M", [1, 4, 16])
-def test_decode_llama3_8b_full_size(torch, proj, M):
+def test_decode_llama3_8b_full_size(torch, proj, M, src):
     """8B decode projections at full size; map 85/10/5, 1% outlier columns x30.
     Every output is checked for M=1/4, 2048 sampled columns for M=16."""
     K, N = LLAMA3[proj]
     g = I.rng(1, K, N, M)
     bits = I.width_map(K // 32, 0.85, 0.10, 0.05, g)
     xb, wb, codes, scales, packed = layer(torch, M, K, N, bits, g)
-    y = mxs.gemm(codes, scales, None, bits, packed, N).cpu().numpy()
+    y = decode_from(torch, src, xb, bits, packed, N, codes, scales).cpu().numpy()
     a_s, a_c = mxo.quantize_bf16(xb, bits)
     cols = np.arange(N) if M < 16 or N <= 2048 else np.sort(np.random.default_rng(0).choice(N, 2048, replace=False))
     w_s, w_c = mxo.quantize_bf16(wb[cols], bits)
@@ -109,6 +139,7 @@ def test_decode_sweep_70b_shape_sampled(torch, maps):
     bits = I.width_map(K // 32, *p, g, clustered=maps.endswith("clustered"))
     xb, wb, codes, scales, packed = layer(torch, M, K, N, bits, g, outlier_scale=50.0)
     y = mxs.gemm(codes, scales, None, bits, packed, N).cpu().numpy()
+    assert np.array_equal(decode_from(torch, "planes", xb, bits, packed, N).cpu().numpy(), y)
     cols = np.sort(np.random.default_rng(1).choice(N, 512, replace=False))
     a_s, a_c = mxo.quantize_bf16(xb, bits)
     w_s, w_c = mxo.quantize_bf16(wb[cols], bits)
@@ -138,6 +169,7 @@ def test_decode_wide_dynamic_range(torch, M, nb, p):
     codes, scales, _ = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits)
     packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
     y = mxs.gemm(codes, scales, None, bits, packed, N).cpu().numpy()
+    assert np.array_equal(decode_from(torch, "planes", xb, bits, packed, N).cpu().numpy(), y)
     ref, ab = oracle_full(xb, wb, bits)
     assert np.mean(ref.astype(np.float32).astype(np.float64) == ref) < 0.5  # rounding really happens
     err = U.check_gemm(y, ref, ab)
@@ -148,8 +180,9 @@ def test_decode_wide_dynamic_range(torch, M, nb, p):
 @pytest.mark.parametrize("N,nb,p", [(37, 5, (0.6, 0.2, 0.2)), (1000, 128, (0.85, 0.10, 0.05)),
                                     (64, 448, (0.8, 0.15, 0.05)), (300, 896, (0.5, 0.3, 0.2))])
 def test_fused_linear_decode(torch, M, N, nb, p):
-    """Quantization inside the GEMM prologue: same y as quantize + GEMM (bit for
-    bit) and within the bar of the oracle."""
+    """Quantize-to-planes + GEMM in one call (the GEMM a programmatic dependent
+    of the quantizer): same y as quantize + GEMM over the codes (bit for bit)
+    and within the bar of the oracle."""
     g = I.rng(50, M, N, nb)
     bits = I.width_map(nb, *p, g)
     xb, wb, codes, scales, packed = layer(torch, M, 32 * nb, N, bits, g)
