@@ -53,7 +53,7 @@ def parse():
                     help="decoder layers per step (default 32 for decode, 8 for prefill)")
     ap.add_argument("--workload", default="llama3-8b-decode", choices=["llama3-8b-decode", "llama3-8b-prefill"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--path", default="planes", choices=["planes", "fused", "codes"],
+    ap.add_argument("--path", default="fused", choices=["planes", "fused", "codes"],
                     help="decode activation path: quantize all projections to MMA planes, then the GEMMs "
                          "(planes); mxs_linear_decode per projection, the GEMM a programmatic dependent of "
                          "its quantizer (fused); quantize to packed codes, GEMM over the codes (codes)")

@@ -33,7 +33,12 @@
  *     surface at the caller's next synchronisation.
  *   - Outputs are overwritten in full, padding rows and slots included; only
  *     the alignment gaps between the sections of an activation planes buffer
- *     are left unwritten.
+ *     and the scale-tile bytes of its rows beyond M (which no GEMM reads) are
+ *     left unwritten.
+ *   - Kernels use programmatic dependent launch: mxs_quantize_act and
+ *     mxs_linear_decode may start before the preceding work on `stream` has
+ *     finished and wait for it before they touch their inputs and outputs.
+ *     The one exception is stated at mxs_linear_decode (its weights).
  *   - Only sm_103a devices are supported (MXS_ERR_UNSUPPORTED otherwise).
  *
  * Storage format (the "packed" layouts; byte offsets are exact):
@@ -63,7 +68,7 @@
  *       SF at align256(P + rows*Kp): per 128-row tile and 128-byte K' stage,
  *       512 B ordered [i<32][w<4][q<4] = S of row 128*tile+32w+i, slot 4*st+q
  *       (4-bit stages) or 2*(st-ceil(n4/4))+q for q<2 (6/8-bit stages); every
- *       other byte 0.
+ *       other byte 0 (for activations: every other byte of the rows < M).
  *     For weights P and SF follow the compact part inside the same buffer.
  */
 #ifndef MXS_H_
@@ -169,9 +174,13 @@ MXS_API int mxs_gemm_decode(const void *act_codes, const uint8_t *act_scales, co
  * aligned; the same planes mxs_quantize_act writes) and returns
  * y [M,N] fp32 = x W^T like mxs_gemm_decode.  Two kernels on `stream`; the
  * GEMM is launched as a programmatic dependent of the quantizer, so its
- * weight stream starts while the activations are quantized (Appendix A.2:
- * activations are quantized on the fly).  The workspace is scratch: it may be
- * reused once the call's work on `stream` has finished. */
+ * weight stream starts while the activations are quantized -- and, in a chain
+ * of such calls, while the previous layer finishes (Appendix A.2: activations
+ * are quantized on the fly).  Hence packed_w must not be written by work that
+ * is still in flight on `stream` when the call is made (weights are static;
+ * pack them, then synchronise, before the first use).  x, y and the workspace
+ * have the ordinary stream semantics; the workspace may be reused by the next
+ * call on the same stream. */
 MXS_API int mxs_linear_decode(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits,
                               int rounding, const void *packed_w, int64_t N, float *y, int64_t ld_y,
                               void *workspace, size_t ws_bytes, void *stream);

@@ -290,6 +290,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
     S.init(p, c0, c1);
     const int nchunks = (S.n + 1) / 2;  // a copy stage holds two MMA stages
 
+    // the next kernel on the stream may launch now (it waits for this grid
+    // before it touches what this grid writes)
+    if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (threadIdx.x == 0) {
         for (int i = 0; i < a.ring; ++i) {
             mbar_init(&full_c[i], 1);
@@ -480,6 +483,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                 bulk_load(sfb, a.tok_sf + (int64_t)sg0 * 512, (uint32_t)S.n * 512, tok_full);
             }
         } else {
+            // the codes may come from the kernel just before this one
+            asm volatile("griddepcontrol.wait;" ::: "memory");
             // zero the token planes and scale tiles of every stage, then fill them from the codes
             for (int i = et; i < S.n * (kTokBytes + 512) / 16; i += 128) {
                 const int off = i * 16;
@@ -593,8 +598,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                 float out[16];
 #pragma unroll
                 for (int t = 0; t < 16; ++t) out[t] = __uint_as_float(v[t]);
+                const bool more = a.GS > 1 && g + (int)gridDim.x < a.G;  // the ranks send another tile
                 if (a.GS > 1) {
-                    if (!warp_wait<true>(xfull, gi & 1, abort)) break;
+                    // the partial tiles arrived by bulk copy, completing on this CTA's barrier
+                    if (!warp_wait(xfull, gi & 1, abort)) break;
                     for (int k = 1; k < a.GS; ++k) {
                         const float4 *src = reinterpret_cast<const float4 *>(xbuf + ((k - 1) * 128 + r) * 16);
 #pragma unroll
@@ -606,17 +613,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                             out[4 * i + 3] += u.w;
                         }
                     }
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(xread);
-                    bool freed = true;
-                    if (et == 0) {
-                        freed = mbar_wait(xread, gi & 1, abort);  // every thread has read the tiles
-                        if (freed) {
-                            if (g + (int)gridDim.x < a.G) mbar_expect_tx(xfull, (uint32_t)(a.GS - 1) * kXBytes);
-                            for (int k = 1; k < a.GS; ++k) mbar_arrive_remote(xempty, (uint32_t)k);
-                        }
+                    if (more) {
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(xread);
                     }
-                    if (!__shfl_sync(0xffffffffu, freed, 0)) break;  // whole warp
                 }
                 if (n < a.N) {
 #pragma unroll
@@ -625,6 +625,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                             float *dst = a.y + (int64_t)t * a.ld_y + n;
                             *dst = a.accumulate ? *dst + out[t] : out[t];  // a later K pass, same thread
                         }
+                }
+                if (more) {
+                    // every thread has read the tiles: re-arm, and let the ranks send the next ones
+                    bool freed = true;
+                    if (et == 0) {
+                        freed = mbar_wait(xread, gi & 1, abort);
+                        if (freed) {
+                            mbar_expect_tx(xfull, (uint32_t)(a.GS - 1) * kXBytes);
+                            for (int k = 1; k < a.GS; ++k) mbar_arrive_remote(xempty, (uint32_t)k);
+                        }
+                    }
+                    if (!__shfl_sync(0xffffffffu, freed, 0)) break;  // whole warp
                 }
             }
         }

@@ -15,7 +15,7 @@ namespace {
 
 struct QuantArgs {
     const uint16_t *x;
-    int64_t M, ld, rows;  // rows = M, or M rounded up to 128 when planes are written
+    int64_t M, ld;
     int64_t V;            // work slots per row (with plane padding when planes are written)
     int rhaz;
     uint8_t *codes, *scales, *planes, *sf;
@@ -23,15 +23,18 @@ struct QuantArgs {
 
 __global__ void __launch_bounds__(256) quantize_act_kernel(const __grid_constant__ Plan p,
                                                            const __grid_constant__ QuantArgs a) {
-    // a decode GEMM launched after this kernel with programmatic dependent
-    // launch may start now; it waits for this grid's writes before reading them
+    // Programmatic dependent launch, both ways: a decode GEMM launched after
+    // this kernel may start now (it waits for this grid before reading the
+    // planes), and this grid waits for the kernel before it (which may write
+    // x or still read the output buffers) before touching memory.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int64_t gid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int l = threadIdx.x & 3;
     const int64_t item = gid >> 2;
     const int64_t row = item / a.V;
     const int vs = (int)(item - row * a.V);
-    const bool in_grid = row < a.rows;
+    const bool in_grid = row < a.M;
 
     // virtual slot -> real slot (or padding) and its plane / scale-tile position
     int s = -1, st = 0, q = 0;
@@ -145,14 +148,21 @@ int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rou
     a.scales = scales;
     a.planes = static_cast<uint8_t *>(planes);
     a.sf = planes ? a.planes + align256(M * p.kp) : nullptr;
-    a.rows = planes ? (M + 127) / 128 * 128 : M;
     a.V = planes ? 4 * (int64_t)p.st4 + 2 * (int64_t)((p.n68 + 1) / 2) : p.nb;
-    const int64_t threads = a.rows * a.V * 4;
+    const int64_t threads = M * a.V * 4;
     if (threads == 0) return MXS_OK;
     const int64_t blocks = (threads + 255) / 256;
     if (blocks > 0x7FFFFFFF) return fail(MXS_ERR_SHAPE, "quantize: problem too large");
-    quantize_act_kernel<<<(unsigned)blocks, 256, 0, st>>>(p, a);
-    return cuda_fail(cudaGetLastError(), "quantize_act_kernel launch");
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks, 1, 1);
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // the kernel waits before any access
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cuda_fail(cudaLaunchKernelEx(&cfg, quantize_act_kernel, p, a), "quantize_act_kernel launch");
 }
 
 }  // namespace mxs

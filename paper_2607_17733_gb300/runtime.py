@@ -24,6 +24,7 @@ class MxLinear:
         self.rounding = rounding
         self.layout = mxs.W_COMPACT_AND_PLANES if with_planes else mxs.W_COMPACT
         self.packed = mxs.pack_weight(w, self.bits, layout=self.layout, rounding=rounding)
+        torch.cuda.current_stream().synchronize()  # static from here on (fused() streams it early)
         n4 = int(np.sum(self.bits == 4))
         n68 = self.bits.size - n4
         # bytes a GEMM must read of this weight: codes + one scale byte per block

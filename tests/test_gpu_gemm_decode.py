@@ -20,6 +20,7 @@ def layer(torch, M, K, N, bits, g, w_sigma=0.02, outlier_frac=0.01, outlier_scal
     wb = I.normal_bf16((N, K), w_sigma, g)
     codes, scales, _ = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits)
     packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
+    torch.cuda.synchronize()  # weights are static: packed before the first linear_decode
     return xb, wb, codes, scales, packed
 
 
@@ -203,6 +204,7 @@ def test_fused_linear_decode_rhaz_and_stride(torch):
     wide[:, :K] = xb
     x = U.to_dev_bf16(torch, wide)[:, :K]
     packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits, rounding=mxs.RHAZ)
+    torch.cuda.synchronize()
     y = mxs.linear_decode(x, bits, packed, N, rounding=mxs.RHAZ).cpu().numpy()
     a_s, a_c = mxo.quantize_bf16(xb, bits, mxo.RHAZ)
     w_s, w_c = mxo.quantize_bf16(wb, bits, mxo.RHAZ)
