@@ -6,12 +6,12 @@
 // a shared power-of-two scale) with the per-block widths of Sec. 4.1.
 //
 // Decode reads every weight byte once, so the kernel keeps the weights in
-// their compact form (4-bit nibbles, 6/8-bit bytes) all the way into shared
-// memory and does all arithmetic on the tensor core:
+// their compact form (4-bit nibbles, 6/8-bit bytes) until they are in
+// registers, and does all arithmetic on the tensor core:
 //   * the block-scaled FP8 MMA (tcgen05.mma kind::mxf8f6f4, scale_vec::1X)
-//     with the weights as the 128-row A operand and the <= 16 tokens as the
-//     N = 16 B operand; per-block scales are applied by the hardware and the
-//     sum over K stays in an fp32 tensor-memory accumulator;
+//     with 128 weight rows as the A operand and the <= 16 tokens as the N = 16
+//     B operand; per-block scales are applied by the hardware and the sum over
+//     K stays in fp32 tensor-memory accumulators;
 //   * a weight code of magnitude <= 15 is fed as the e4m3 byte
 //     (sign << 7) | |m|, whose value is |m| * 2^-9 (subnormals and the first
 //     binade); 6/8-bit codes split as |m| = 16h + l into two such digits
@@ -22,25 +22,26 @@
 //   * the token operand is the activations' MMA-plane form (the layout the
 //     prefill GEMM reads: e4m3 values m/4, or a high and a low digit, under
 //     the block's own scale byte).  It is either loaded by TMA from planes
-//     written by mxs_quantize_act -- the launch may then overlap the
-//     quantizer's tail (programmatic dependent launch) -- or built in the
-//     prologue from packed codes;
-//   * warp 0 streams each 128-row weight group's K range into a ring of
-//     shared-memory stages with cp.async.bulk (two MMA stages, about 17 KB,
-//     per copy: the copy count, not the byte count, limits bulk copies);
-//   * warps 6-13 (two per scheduler) convert a stage into e4m3 digit planes in
-//     the 128-byte swizzled K-major layout the MMA reads and write the weight
-//     scale tile; one thread per (row, half stage), a few integer operations
-//     per eight codes;
-//   * warp 1 owns tensor memory and issues tcgen05.cp (scales) and the MMAs;
-//     the token scale tiles go to tensor memory once per CTA;
-//   * warps 2-5 drain the accumulator (tcgen05.ld) and store y;
-//   * K is split over the CTAs of a thread-block cluster when N alone cannot
-//     occupy the GPU or the token operand would not fit; the other ranks hand
-//     their partial accumulator tiles to rank 0 with one bulk copy each
-//     through distributed shared memory, and rank 0 adds them in rank order.
-//     A K range too large for one cluster's shared memory runs as several
-//     passes, each adding into y.
+//     written by mxs_quantize_act -- the launch may then overlap the kernel
+//     before it (programmatic dependent launch) -- or built in the prologue
+//     from packed codes.
+// Work: a CTA owns 128-row weight groups and (in a cluster) a K range of them,
+// cut into MMA stages of 128 K'-bytes (four 4-bit slots or two 6/8-bit
+// slots).  Up to ten worker warps own whole stages, round robin: a worker
+// loads its stage's codes straight from HBM into registers (coalesced 16-byte
+// loads, the next stage in flight while it converts the current one), writes
+// the e4m3 digits into its own 128-byte-swizzled plane buffer and the weight
+// scale tile, and issues the stage's MMAs into its own accumulator.  Workers
+// never wait for one another; the epilogue warps add the workers' partial
+// accumulators in worker order (a fixed order: results are deterministic).
+// Other warps: warp 0 owns tensor memory and loads the token operand; warps
+// 1-4 run the epilogue (and build the token operand from codes).
+// K is split over the CTAs of a thread-block cluster when N alone cannot
+// occupy the GPU.  The ranks then reduce-scatter through distributed shared
+// memory: rank k receives rows [k*R, (k+1)*R) (R = 128/cluster size) of every
+// other rank's partial tile by bulk copy, adds the partials in rank order and
+// stores those rows.  A K range whose token operand does not fit shared
+// memory runs as several passes, each adding into y.
 // Every mbarrier wait is bounded; on expiry the kernel records
 // MXS_ERR_TIMEOUT, stops, drains what it issued and frees tensor memory.
 // Weight scale bytes above 245 (|w| >= 2^118) saturate at 254 after the digit
@@ -59,15 +60,18 @@ __device__ int g_decode_status;  // sticky MXS_ERR_TIMEOUT, read by mxs_device_s
 
 namespace {
 
-constexpr int kThreads = 448;  // 14 warps
-constexpr int kConv = 4;        // converted weight-plane stages
+constexpr int kMaxWorkers = 10;                                 // worker warps per CTA, chosen per launch
+constexpr int kWorkerWarp0 = 5;                                 // warps 5..
+constexpr int kMaxThreads = (kWorkerWarp0 + kMaxWorkers) * 32;  // 480
 constexpr int kPlaneBytes = 128 * 128;  // 128 rows x 128 bytes of K' (SW128)
 constexpr int kTokBytes = 16 * 128;     // 16 token rows x 128 bytes of K'
-constexpr int kAccCols = 32;            // two 16-column accumulators
-constexpr int kSfaCol = kAccCols;       // kConv x 4 columns of weight scales
-constexpr int kSfbCol = kSfaCol + 4 * kConv;  // 4 columns per MMA stage of token scales
-constexpr int kXBytes = 128 * 16 * 4;   // one fp32 partial tile
-constexpr int kMinSmem = 116 * 1024;    // keeps one CTA per SM (tensor memory is allocated per CTA)
+constexpr int kAccCols = 16;            // one accumulator: 16 token columns
+constexpr int kSfaCol = 2 * kMaxWorkers * kAccCols;  // 320: 4 columns of weight scales per worker
+constexpr int kSfbCol = kSfaCol + 4 * kMaxWorkers;   // 360: 4 columns per MMA stage of token scales
+constexpr int kTmemCols = 512;
+constexpr int kMaxStages = (kTmemCols - kSfbCol) / 4;  // 38
+constexpr int kXBytes = 128 * 16 * 4;  // one fp32 partial tile
+constexpr int kMinSmem = 116 * 1024;   // one CTA per SM (each allocates all of tensor memory)
 constexpr long long kWaitCycles = 4000000000ll;  // ~2 s at the maximum SM clock
 
 struct DecodeArgs {
@@ -77,14 +81,13 @@ struct DecodeArgs {
     const uint8_t *w;       // packed weight buffer
     float *y;
     int64_t ld_y;
-    int M, N, G;           // tokens, output features, 128-row groups
-    int GS;                // CTAs per cluster along K
-    int bound[9];          // rank r streams slots [bound[r], bound[r+1]) (stage-aligned)
-    int ring, ring_bytes;  // copy stages, bytes per copy stage
-    int max_mst;           // most MMA stages any rank holds (token operand carve)
-    int tmem_cols;
-    int accumulate;        // add into y (a later K pass) instead of storing
-    int64_t GB;            // bytes of one 128-row weight group
+    int M, N, G;      // tokens, output features, 128-row groups
+    int GS;           // CTAs per cluster along K
+    int bound[9];     // rank r owns slots [bound[r], bound[r+1]) (stage-aligned)
+    int max_mst;      // most MMA stages any rank holds (token operand carve)
+    int workers;      // worker warps (blockDim = (5 + workers) warps)
+    int accumulate;   // add into y (a later K pass) instead of storing
+    int64_t GB;       // bytes of one 128-row weight group
 };
 
 // ------------------------------------------------------------------ PTX helpers
@@ -179,9 +182,24 @@ __device__ __forceinline__ void bulk_to_rank(uint32_t dst_cluster, const void *s
         "r"(su32(src)), "r"(bytes), "r"(bar_cluster)
         : "memory");
 }
+// streaming loads of weight codes: read once, not kept in L1
+__device__ __forceinline__ uint4 ld_stream16(const uint8_t *p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+__device__ __forceinline__ uint32_t ld_stream1(const uint8_t *p) {
+    uint16_t v;
+    asm volatile("ld.global.nc.L1::no_allocate.u8 %0, [%1];" : "=h"(v) : "l"(p));
+    return v;
+}
 // generic-proxy shared-memory writes -> visible to the tensor core / bulk copies
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire;" ::: "memory"); }
 
 // UMMA shared-memory descriptors (as in the prefill kernel): 128B-swizzled
 // K-major operand tiles (8-row atoms of 1024 B) and 32 x 16 B scale tiles.
@@ -259,25 +277,118 @@ struct Stages {  // MMA stages of a CTA's K range [c0, c1): 4-bit ones (4 slots)
     }
 };
 
-__global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_constant__ Plan p,
-                                                                  const __grid_constant__ DecodeArgs a,
-                                                                  const __grid_constant__ CUtensorMap tok_map) {
+// One half of a worker's stage in registers: lane l holds rows l + 32i
+// (i < 4).  A 4-bit half is slots 2h, 2h+1 (v[4k+i] = slot 2h+k, row i); a
+// 6/8-bit half is slot h (v[2i], v[2i+1] = the two 16-byte words of row i).
+// Either way the half fills 16-byte chunks 4h..4h+3 of each row and
+// scale-tile bytes 2h, 2h+1.
+struct Half {
+    uint4 v[8];
+    uint32_t s[8];  // scale bytes (4-bit: [4k+i] = slot 2h+k, row i; 6/8-bit: [i] = row i)
+};
+
+// Load half `h` of stage `st` of the weight group at `wg` (lane l: rows l + 32i).
+__device__ __forceinline__ void load_half(const Plan &p, const Stages &S, const uint8_t *wg, int st, int h, int l,
+                                          Half &x) {
+    int lo, hi;
+    S.range(st, lo, hi);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        x.v[i] = make_uint4(0, 0, 0, 0);
+        x.s[i] = 0;
+    }
+    if (st < S.st4) {
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int q = 2 * h + k;
+            if (lo + q < hi) {  // a partial last stage has fewer slots
+                const uint8_t *slot = wg + slot_offset(p, lo + q);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    x.v[4 * k + i] = ld_stream16(slot + 16 * (l + 32 * i));
+                    x.s[4 * k + i] = ld_stream1(slot + 2048 + l + 32 * i);
+                }
+            }
+        }
+    } else if (lo + h < hi) {
+        const uint8_t *slot = wg + slot_offset(p, lo + h);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            x.v[2 * i] = ld_stream16(slot + 32 * (l + 32 * i));
+            x.v[2 * i + 1] = ld_stream16(slot + 32 * (l + 32 * i) + 16);
+            x.s[i] = ld_stream1(slot + 4096 + l + 32 * i);
+        }
+    }
+}
+
+// Convert a loaded half into digit-plane chunks 4h..4h+3 of rows l + 32i and
+// return the row's scale-tile bytes 2h, 2h+1 (bits 16i..16i+15 for row i).
+__device__ __forceinline__ uint64_t store_half(const Plan &p, const Stages &S, int st, int h, int l, const Half &x,
+                                               uint8_t *pl) {
+    int lo, hi;
+    S.range(st, lo, hi);
+    uint64_t sf = 0;
+    if (st < S.st4) {
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int q = 2 * h + k;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = l + 32 * i;
+                const uint4 v = x.v[4 * k + i];
+                // word j: bytes hold elements 8j..8j+3 (low nibbles), 8j+4..8j+7 (high nibbles)
+                *reinterpret_cast<uint4 *>(pl + sw128(r, 2 * q)) =
+                    make_uint4(lo_nib(v.x), hi_nib(v.x), lo_nib(v.y), hi_nib(v.y));
+                *reinterpret_cast<uint4 *>(pl + sw128(r, 2 * q + 1)) =
+                    make_uint4(lo_nib(v.z), hi_nib(v.z), lo_nib(v.w), hi_nib(v.w));
+                // absent slots hold zero codes under scale byte 0 (a zero term)
+                sf |= (uint64_t)(lo + q < hi ? shifted(x.s[4 * k + i], 7) : 0u) << (16 * i + 8 * k);
+            }
+        }
+    } else {
+        const bool six = lo + h < hi && slot_width(p, lo + h) == 6;
+        const uint32_t sh_hi = six ? 9 : 7, sh_lo = six ? 5 : 3;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int r = l + 32 * i;
+            const uint4 v0 = x.v[2 * i], v1 = x.v[2 * i + 1];
+            *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * h)) =
+                make_uint4(hi_digit(v0.x), hi_digit(v0.y), hi_digit(v0.z), hi_digit(v0.w));
+            *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * h + 1)) =
+                make_uint4(hi_digit(v1.x), hi_digit(v1.y), hi_digit(v1.z), hi_digit(v1.w));
+            *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * h + 2)) =
+                make_uint4(lo_digit(v0.x), lo_digit(v0.y), lo_digit(v0.z), lo_digit(v0.w));
+            *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * h + 3)) =
+                make_uint4(lo_digit(v1.x), lo_digit(v1.y), lo_digit(v1.z), lo_digit(v1.w));
+            const uint32_t b2 = lo + h < hi ? (shifted(x.s[i], sh_hi) | (shifted(x.s[i], sh_lo) << 8)) : 0u;
+            sf |= (uint64_t)b2 << (16 * i);
+        }
+    }
+    return sf;
+}
+
+__global__ void __launch_bounds__(kMaxThreads, 1) gemm_decode_kernel(const __grid_constant__ Plan p,
+                                                                     const __grid_constant__ DecodeArgs a,
+                                                                     const __grid_constant__ CUtensorMap tok_map) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t sbase = su32(smem_raw);
     uint8_t *smem = smem_raw + (((sbase + 1023) & ~1023u) - sbase);  // 1024-aligned for the swizzled tiles
-    uint8_t *planes = smem;                                   // kConv x 16 KB
-    uint8_t *tok = planes + kConv * kPlaneBytes;              // max_mst x 2 KB
-    uint8_t *sfa = tok + (size_t)a.max_mst * kTokBytes;       // kConv x 512
-    uint8_t *sfb = sfa + kConv * 512;                         // max_mst x 512
-    uint8_t *ring = sfb + (size_t)a.max_mst * 512;            // ring x ring_bytes
-    float *xout = reinterpret_cast<float *>(ring + (size_t)a.ring * a.ring_bytes);  // [128][16] (GS > 1)
-    float *xbuf = xout + (a.GS > 1 ? 128 * 16 : 0);                                 // [GS-1][128][16] (rank 0)
-    uint64_t *bars = reinterpret_cast<uint64_t *>(xbuf + (size_t)(a.GS - 1) * 128 * 16);
-    uint64_t *full_c = bars, *empty_c = full_c + a.ring;
-    uint64_t *conv_full = empty_c + a.ring, *conv_empty = conv_full + kConv;
-    uint64_t *acc_full = conv_empty + kConv, *acc_empty = acc_full + 2;
-    uint64_t *tok_full = acc_empty + 2, *xfull = tok_full + 1, *xempty = xfull + 1;
-    uint64_t *xstage = xempty + 1, *xread = xstage + 1;
+    const int W = a.workers;
+    uint8_t *planes = smem;                              // W x 16 KB
+    uint8_t *tok = planes + W * kPlaneBytes;             // max_mst x 2 KB
+    uint8_t *sfa = tok + (size_t)a.max_mst * kTokBytes;  // W x 512
+    uint8_t *sfb = sfa + W * 512;                        // max_mst x 512
+    // cluster reduce-scatter: rank k adds up rows [k*R, (k+1)*R) of the GS partial
+    // tiles (R = 128/GS) and stores them; xout is this rank's whole partial tile,
+    // xbuf the slices the other ranks send here (slot of sender j: j, or j-1 past k)
+    const int R = 128 / a.GS;
+    float *xout = reinterpret_cast<float *>(sfb + (size_t)a.max_mst * 512);  // [128][16] (GS > 1)
+    float *xbuf = xout + (a.GS > 1 ? 128 * 16 : 0);                          // [GS-1][R][16]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(xbuf + (size_t)(a.GS - 1) * R * 16);
+    uint64_t *plane_free = bars;  // [W] tcgen05.commit
+    uint64_t *acc_full = plane_free + W, *acc_empty = acc_full + 2;
+    uint64_t *tok_full = acc_empty + 2, *tok_ready = tok_full + 1;
+    uint64_t *xfull = tok_ready + 1, *xempty = xfull + 1, *xstage = xempty + 1, *xread = xstage + 1;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(xread + 1);
     int *abort_flag = reinterpret_cast<int *>(tmem_slot + 1);
     volatile int *abort = abort_flag;
@@ -288,201 +399,154 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
     const bool from_planes = a.tok_sf != nullptr;
     Stages S;
     S.init(p, c0, c1);
-    const int nchunks = (S.n + 1) / 2;  // a copy stage holds two MMA stages
+    const int nw = min(W, S.n);  // workers with a stage in every group
+    const uint32_t xslice = (uint32_t)(R * 16 * 4);
+
+    // Workers put their first stage's loads in flight before anything else:
+    // the weights are static (see mxs_linear_decode), so they need no wait.
+    Half A, B;
+    if (warp >= kWorkerWarp0 && warp - kWorkerWarp0 < nw && (int)blockIdx.x < a.G) {
+        const uint8_t *wg = a.w + (int64_t)blockIdx.x * a.GB;
+        load_half(p, S, wg, warp - kWorkerWarp0, 0, lane, A);
+        load_half(p, S, wg, warp - kWorkerWarp0, 1, lane, B);
+    }
 
     // the next kernel on the stream may launch now (it waits for this grid
     // before it touches what this grid writes)
     if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (threadIdx.x == 0) {
-        for (int i = 0; i < a.ring; ++i) {
-            mbar_init(&full_c[i], 1);
-            mbar_init(&empty_c[i], 8);  // the eight converter warps
-        }
-        for (int i = 0; i < kConv; ++i) {
-            mbar_init(&conv_full[i], 8);
-            mbar_init(&conv_empty[i], 1);  // tcgen05.commit
-        }
+        for (int i = 0; i < W; ++i) mbar_init(&plane_free[i], 1);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&acc_full[i], 1);
+            mbar_init(&acc_full[i], nw);  // each active worker commits once per group
             mbar_init(&acc_empty[i], 4);  // the four epilogue warps
         }
         mbar_init(tok_full, from_planes ? 1 : 4);
-        mbar_init(xfull, 1);   // rank 0: armed per tile with the bytes of GS-1 partial tiles
-        mbar_init(xempty, 1);  // rank > 0: rank 0 has consumed this rank's previous tile (copy done)
-        mbar_init(xstage, 4);  // rank > 0: the four epilogue warps have staged the tile
-        mbar_init(xread, 4);   // rank 0: the four epilogue warps have read the partial tiles
+        mbar_init(tok_ready, 1);              // tcgen05.commit once the token scales are in tensor memory
+        mbar_init(xfull, 1);                  // armed per tile with the bytes of GS-1 slices
+        mbar_init(xempty, max(1, a.GS - 1));  // every receiver took this rank's previous slices (copies done)
+        mbar_init(xstage, 4);                 // the four epilogue warps have staged the partial tile
+        mbar_init(xread, 4);                  // the four epilogue warps are done with xout and xbuf
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        // rank 0 arms the first phase of its receive barrier: (GS-1) partial tiles
-        if (a.GS > 1 && rank == 0) mbar_expect_tx(xfull, (uint32_t)(a.GS - 1) * kXBytes);
+        if (a.GS > 1) mbar_expect_tx(xfull, (uint32_t)(a.GS - 1) * xslice);  // the first tile's slices
     }
-    if (warp == 1) {
+    if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)),
-                     "r"(a.tmem_cols)
+                     "r"(kTmemCols)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
     fence_before();
     __syncthreads();
     fence_after();
-    if (a.GS > 1) cg::this_cluster().sync();  // partners' barriers exist before any remote access
+    // Partners' barriers must exist before any remote access: every thread
+    // arrives now; the epilogue warps (the only ones with remote traffic) wait
+    // before their first remote operation, the others just before the teardown.
+    if (a.GS > 1) cluster_arrive();
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0) {
-        // ------------------------------------------------------------ weight producer
+        // ------------------------------------------------------------ token operand -> smem, scales -> TMEM
         if (lane == 0) {
-            uint32_t qc = 0;
-            bool stop = false;
-            for (int g = blockIdx.x; g < a.G && !stop; g += gridDim.x) {
-                const uint8_t *wg = a.w + (int64_t)g * a.GB;
-                for (int k = 0; k < nchunks; ++k, ++qc) {
-                    const int s = (int)(qc % a.ring);
-                    if (!mbar_wait(&empty_c[s], ((qc / a.ring) & 1) ^ 1, abort)) { stop = true; break; }
-                    int lo, hi, lo2, hi2;
-                    S.range(2 * k, lo, hi);
-                    if (2 * k + 1 < S.n) S.range(2 * k + 1, lo2, hi2); else hi2 = hi;
-                    const int64_t off = slot_offset(p, lo);
-                    const uint32_t bytes = (uint32_t)(slot_offset(p, hi2) - off);
-                    mbar_expect_tx(&full_c[s], bytes);
-                    bulk_load(ring + (size_t)s * a.ring_bytes, wg + off, bytes, &full_c[s]);
-                }
-            }
-            const uint32_t first = qc > (uint32_t)a.ring ? qc - a.ring : 0;
-            for (uint32_t k = first; k < qc; ++k) drain_wait(&full_c[k % a.ring], (k / a.ring) & 1);
-        }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            bool ok = mbar_wait(tok_full, 0, abort);
-            if (ok) {
-                fence_after();
-                const uint64_t dsfb = desc_sf(su32(sfb));
-                for (int st = 0; st < S.n; ++st) tmem_cp_sf(tmem + kSfbCol + 4 * st, dsfb + 32 * st);
-            }
-            const uint64_t dA = desc_sw128(su32(planes)), dB = desc_sw128(su32(tok)), dsfa = desc_sf(su32(sfa));
-            uint32_t qs = 0;
-            int gi = 0, last = -1;
-            for (int g = blockIdx.x; g < a.G && ok; g += gridDim.x, ++gi) {
-                const int b = gi & 1;
-                if (!mbar_wait(&acc_empty[b], ((gi >> 1) & 1) ^ 1, abort)) break;
-                fence_after();
-                const uint32_t acc = tmem + 16 * b;
-                for (int st = 0; st < S.n; ++st, ++qs) {
-                    const int pc = (int)(qs % kConv);
-                    if (!mbar_wait(&conv_full[pc], (qs / kConv) & 1, abort)) { ok = false; break; }
-                    fence_after();
-                    const uint32_t sfa_t = tmem + kSfaCol + 4 * pc, sfb_t = tmem + kSfbCol + 4 * st;
-                    tmem_cp_sf(sfa_t, dsfa + 32 * pc);
-                    const uint64_t da = dA + (uint64_t)(pc * (kPlaneBytes >> 4));
-                    const uint64_t db = dB + (uint64_t)(st * (kTokBytes >> 4));
-                    const uint32_t first = st > 0 ? 1u : 0u;
-                    if (st < S.st4) {
-                        // slot q: weight digits at K' bytes 32q.., token values at 32q..
-                        mma_mx(acc, da, db, idesc(0, 0), sfa_t, sfb_t, first);
-                        mma_mx(acc, da + 2, db + 2, idesc(1, 1), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, da + 4, db + 4, idesc(2, 2), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, da + 6, db + 6, idesc(3, 3), sfa_t, sfb_t, 1u);
-                    } else {
-                        // slot j: weight digit pa (high, low) at 64j + 32pa under scale 2j + pa;
-                        // token digit pb at 64j + 32pb under the slot's scale byte j
-                        mma_mx(acc, da, db, idesc(0, 0), sfa_t, sfb_t, first);
-                        mma_mx(acc, da, db + 2, idesc(0, 0), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, da + 2, db, idesc(1, 0), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, da + 2, db + 2, idesc(1, 0), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, da + 4, db + 4, idesc(2, 1), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, da + 4, db + 6, idesc(2, 1), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, da + 6, db + 4, idesc(3, 1), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, da + 6, db + 6, idesc(3, 1), sfa_t, sfb_t, 1u);
-                    }
-                    mma_commit(&conv_empty[pc]);  // frees the plane stage once these MMAs have read it
-                    last = (int)qs;
-                }
-                if (!ok) break;
-                mma_commit(&acc_full[b]);
-            }
-            if (last >= 0) drain_wait(&conv_empty[last % kConv], ((uint32_t)last / kConv) & 1);
-        }
-    } else if (warp >= 6) {
-        // ------------------------------------------------------------ converters: thread = (row, half stage)
-        const int cth = threadIdx.x - 192;  // 0..255
-        const int r = cth & 127, h = cth >> 7;
-        uint8_t *sfa_cell = sfa + (r & 31) * 16 + (r >> 5) * 4 + 2 * h;
-        uint32_t qc = 0, qs = 0;
-        bool stop = false;
-        for (int g = blockIdx.x; g < a.G && !stop; g += gridDim.x) {
-            for (int k = 0; k < nchunks && !stop; ++k, ++qc) {
-                const int s = (int)(qc % a.ring);
-                if (!warp_wait(&full_c[s], (qc / a.ring) & 1, abort)) { stop = true; break; }
-                int clo, chi;
-                S.range(2 * k, clo, chi);
-                const uint8_t *chunk = ring + (size_t)s * a.ring_bytes - slot_offset(p, clo);  // + slot_offset(slot)
-                for (int st = 2 * k; st < min(2 * k + 2, S.n); ++st, ++qs) {
-                    const int pc = (int)(qs % kConv);
-                    if (!warp_wait(&conv_empty[pc], ((qs / kConv) & 1) ^ 1, abort)) { stop = true; break; }
-                    int lo, hi;
-                    S.range(st, lo, hi);
-                    uint8_t *pl = planes + pc * kPlaneBytes;
-                    uint32_t sf2 = 0;
-                    if (st < S.st4) {
-#pragma unroll
-                        for (int i = 0; i < 2; ++i) {
-                            const int q = 2 * h + i;
-                            uint4 o0 = make_uint4(0, 0, 0, 0), o1 = o0;
-                            if (lo + q < hi) {
-                                const uint8_t *slot = chunk + slot_offset(p, lo + q);
-                                const uint4 v = *reinterpret_cast<const uint4 *>(slot + 16 * r);
-                                // word i: bytes hold elements 8i..8i+3 (low nibbles), 8i+4..8i+7 (high nibbles)
-                                o0 = make_uint4(lo_nib(v.x), hi_nib(v.x), lo_nib(v.y), hi_nib(v.y));
-                                o1 = make_uint4(lo_nib(v.z), hi_nib(v.z), lo_nib(v.w), hi_nib(v.w));
-                                sf2 |= shifted(slot[2048 + r], 7) << (8 * i);
-                            }
-                            *reinterpret_cast<uint4 *>(pl + sw128(r, 2 * q)) = o0;
-                            *reinterpret_cast<uint4 *>(pl + sw128(r, 2 * q + 1)) = o1;
-                        }
-                    } else {
-                        const int j = h;
-                        uint4 h0 = make_uint4(0, 0, 0, 0), h1 = h0, l0 = h0, l1 = h0;
-                        if (lo + j < hi) {
-                            const uint8_t *slot = chunk + slot_offset(p, lo + j);
-                            const uint4 v0 = *reinterpret_cast<const uint4 *>(slot + 32 * r);
-                            const uint4 v1 = *reinterpret_cast<const uint4 *>(slot + 32 * r + 16);
-                            h0 = make_uint4(hi_digit(v0.x), hi_digit(v0.y), hi_digit(v0.z), hi_digit(v0.w));
-                            h1 = make_uint4(hi_digit(v1.x), hi_digit(v1.y), hi_digit(v1.z), hi_digit(v1.w));
-                            l0 = make_uint4(lo_digit(v0.x), lo_digit(v0.y), lo_digit(v0.z), lo_digit(v0.w));
-                            l1 = make_uint4(lo_digit(v1.x), lo_digit(v1.y), lo_digit(v1.z), lo_digit(v1.w));
-                            const uint32_t Sw = slot[4096 + r];
-                            const bool six = slot_width(p, lo + j) == 6;
-                            sf2 = shifted(Sw, six ? 9 : 7) | (shifted(Sw, six ? 5 : 3) << 8);
-                        }
-                        *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * j)) = h0;
-                        *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * j + 1)) = h1;
-                        *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * j + 2)) = l0;
-                        *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * j + 3)) = l1;
-                    }
-                    // scale tile: row r at lane r%32, column r/32, byte = sf id (this half: 2h, 2h+1)
-                    *reinterpret_cast<uint16_t *>(sfa_cell + pc * 512) = (uint16_t)sf2;
-                    fence_async_smem();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&conv_full[pc]);
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&empty_c[s]);
-            }
-        }
-    } else {
-        // ------------------------------------------------------------ warps 2-5: token operand, then epilogue
-        const int et = threadIdx.x - 64;  // 0..127
-        if (from_planes) {
-            if (et == 0) {
+            if (from_planes) {
                 // the planes may come from the kernel just before this one (programmatic
                 // dependent launch): wait for it before the first read
                 asm volatile("griddepcontrol.wait;" ::: "memory");
                 const int sg0 = c0 < p.n4 ? c0 / 4 : p.st4 + (c0 - p.n4) / 2;
                 mbar_expect_tx(tok_full, (uint32_t)S.n * (kTokBytes + 512));
-                for (int st = 0; st < S.n; ++st) tma_load_2d(tok + st * kTokBytes, &tok_map, tok_full, 128 * (sg0 + st), 0);
+                for (int st = 0; st < S.n; ++st)
+                    tma_load_2d(tok + st * kTokBytes, &tok_map, tok_full, 128 * (sg0 + st), 0);
                 bulk_load(sfb, a.tok_sf + (int64_t)sg0 * 512, (uint32_t)S.n * 512, tok_full);
             }
-        } else {
+            if (mbar_wait(tok_full, 0, abort)) {
+                fence_after();
+                const uint64_t dsfb = desc_sf(su32(sfb));
+                for (int st = 0; st < S.n; ++st) tmem_cp_sf(tmem + kSfbCol + 4 * st, dsfb + 32 * st);
+                mma_commit(tok_ready);
+                drain_wait(tok_ready, 0);
+            }
+        }
+    } else if (warp >= kWorkerWarp0) {
+        // ------------------------------------------------------------ workers
+        const int w = warp - kWorkerWarp0;
+        if (w < nw) {
+            uint8_t *pl = planes + w * kPlaneBytes;
+            uint8_t *sfa_cell = sfa + w * 512 + 16 * lane;  // rows lane + 32i: bytes 4i..4i+3
+            const uint64_t dA = desc_sw128(su32(pl)), dB = desc_sw128(su32(tok));
+            const uint64_t dsfa = desc_sf(su32(sfa + w * 512));
+            const uint32_t sfa_t = tmem + kSfaCol + 4 * w;
+            bool ok = warp_wait(tok_ready, 0, abort);
+            if (ok) fence_after();
+            uint32_t qw = 0;  // stages this worker has issued (plane_free phases)
+            int g = blockIdx.x, st = w, gi = 0;
+            bool first_in_group = true;
+            while (ok && g < a.G) {
+                const int b = gi & 1;
+                if (first_in_group) ok = warp_wait(&acc_empty[b], ((gi >> 1) & 1) ^ 1, abort);
+                // the plane buffer is free once this worker's previous MMAs have read it
+                if (ok && qw > 0) ok = warp_wait(&plane_free[w], (qw - 1) & 1, abort);
+                if (!ok) break;
+                // next stage of this worker: st + W, else its first stage of the next group
+                int g2 = g, st2 = st + W;
+                if (st2 >= S.n) {
+                    g2 = g + gridDim.x;
+                    st2 = w;
+                }
+                const uint8_t *wg2 = a.w + (int64_t)(g2 < a.G ? g2 : g) * a.GB;
+                const uint64_t sf0 = store_half(p, S, st, 0, lane, A, pl);
+                if (g2 < a.G) load_half(p, S, wg2, st2, 0, lane, A);
+                const uint64_t sf1 = store_half(p, S, st, 1, lane, B, pl);
+                if (g2 < a.G) load_half(p, S, wg2, st2, 1, lane, B);
+                // scale tile: the lane's 16 bytes are rows lane + 32i, 4 bytes each
+                // (sf ids 0, 1 from half 0 and 2, 3 from half 1)
+                uint32_t cell[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    cell[i] = (uint32_t)((sf0 >> (16 * i)) & 0xFFFF) | ((uint32_t)((sf1 >> (16 * i)) & 0xFFFF) << 16);
+                *reinterpret_cast<uint4 *>(sfa_cell) = make_uint4(cell[0], cell[1], cell[2], cell[3]);
+                fence_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    fence_after();
+                    tmem_cp_sf(sfa_t, dsfa);
+                    const uint32_t acc = tmem + kAccCols * (kMaxWorkers * b + w);
+                    const uint32_t sfb_t = tmem + kSfbCol + 4 * st;
+                    const uint64_t db = dB + (uint64_t)(st * (kTokBytes >> 4));
+                    const uint32_t accum = first_in_group ? 0u : 1u;
+                    if (st < S.st4) {
+                        // slot q: weight digits at K' bytes 32q.., token values at 32q..
+                        mma_mx(acc, dA, db, idesc(0, 0), sfa_t, sfb_t, accum);
+                        mma_mx(acc, dA + 2, db + 2, idesc(1, 1), sfa_t, sfb_t, 1u);
+                        mma_mx(acc, dA + 4, db + 4, idesc(2, 2), sfa_t, sfb_t, 1u);
+                        mma_mx(acc, dA + 6, db + 6, idesc(3, 3), sfa_t, sfb_t, 1u);
+                    } else {
+                        // slot j: weight digit pa (high, low) at 64j + 32pa under scale 2j + pa;
+                        // token digit pb at 64j + 32pb under the slot's scale byte j
+                        mma_mx(acc, dA, db, idesc(0, 0), sfa_t, sfb_t, accum);
+                        mma_mx(acc, dA, db + 2, idesc(0, 0), sfa_t, sfb_t, 1u);
+                        mma_mx(acc, dA + 2, db, idesc(1, 0), sfa_t, sfb_t, 1u);
+                        mma_mx(acc, dA + 2, db + 2, idesc(1, 0), sfa_t, sfb_t, 1u);
+                        mma_mx(acc, dA + 4, db + 4, idesc(2, 1), sfa_t, sfb_t, 1u);
+                        mma_mx(acc, dA + 4, db + 6, idesc(2, 1), sfa_t, sfb_t, 1u);
+                        mma_mx(acc, dA + 6, db + 4, idesc(3, 1), sfa_t, sfb_t, 1u);
+                        mma_mx(acc, dA + 6, db + 6, idesc(3, 1), sfa_t, sfb_t, 1u);
+                    }
+                    mma_commit(&plane_free[w]);  // planes + scale tile free once these MMAs have read them
+                    if (g2 != g) mma_commit(&acc_full[b]);  // this worker's share of the group is issued
+                }
+                __syncwarp();
+                ++qw;
+                first_in_group = g2 != g;
+                if (g2 != g) ++gi;
+                g = g2;
+                st = st2;
+            }
+            if (lane == 0 && qw > 0) drain_wait(&plane_free[w], (qw - 1) & 1);
+        }
+    } else {
+        // ------------------------------------------------------------ warps 1-4: token operand (codes), epilogue
+        const int et = threadIdx.x - 32;  // 0..127
+        if (!from_planes) {
             // the codes may come from the kernel just before this one
             asm volatile("griddepcontrol.wait;" ::: "memory");
             // zero the token planes and scale tiles of every stage, then fill them from the codes
@@ -561,7 +625,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
             if (lane == 0) mbar_arrive(tok_full);
         }
 
-        // epilogue: accumulator row (= weight row) 32*quad + lane, columns = tokens
+        // epilogue: accumulator row (= weight row) 32*quad + lane, columns = tokens;
+        // the workers' partial sums are added in worker order
+        if (a.GS > 1) cluster_wait();
         const int quad = warp & 3;
         const int r = 32 * quad + lane;
         int gi = 0;
@@ -569,55 +635,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
             const int b = gi & 1;
             if (!warp_wait(&acc_full[b], (gi >> 1) & 1, abort)) break;
             fence_after();
-            uint32_t v[16];
-            tmem_ld16(tmem + ((uint32_t)(32 * quad) << 16) + 16 * b, v);
+            float out[16];
+            for (int w = 0; w < nw; ++w) {
+                uint32_t v[16];
+                tmem_ld16(tmem + ((uint32_t)(32 * quad) << 16) + kAccCols * (kMaxWorkers * b + w), v);
+#pragma unroll
+                for (int t = 0; t < 16; ++t) out[t] = w == 0 ? __uint_as_float(v[t]) : out[t] + __uint_as_float(v[t]);
+            }
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&acc_empty[b]);
-            const int n = 128 * g + r;
-            if (a.GS > 1 && rank > 0) {
-                // stage the partial tile once rank 0 has taken the previous one (its
-                // arrival also means that copy has finished reading the staging
-                // buffer), then one thread copies it to rank 0's slot
-                if (!warp_wait<true>(xempty, (gi & 1) ^ 1, abort)) break;
-                float4 *dst = reinterpret_cast<float4 *>(xout + r * 16);
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
-                                         __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
-                fence_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(xstage);
-                bool sent = true;
-                if (et == 0) {
-                    sent = mbar_wait(xstage, gi & 1, abort);  // all four warps staged
-                    if (sent) bulk_to_rank(map_rank(xbuf + (rank - 1) * 128 * 16, 0), xout, kXBytes, map_rank(xfull, 0));
-                }
-                if (!__shfl_sync(0xffffffffu, sent, 0)) break;  // whole warp
-            } else {
-                float out[16];
-#pragma unroll
-                for (int t = 0; t < 16; ++t) out[t] = __uint_as_float(v[t]);
-                const bool more = a.GS > 1 && g + (int)gridDim.x < a.G;  // the ranks send another tile
-                if (a.GS > 1) {
-                    // the partial tiles arrived by bulk copy, completing on this CTA's barrier
-                    if (!warp_wait(xfull, gi & 1, abort)) break;
-                    for (int k = 1; k < a.GS; ++k) {
-                        const float4 *src = reinterpret_cast<const float4 *>(xbuf + ((k - 1) * 128 + r) * 16);
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            const float4 u = src[i];
-                            out[4 * i] += u.x;
-                            out[4 * i + 1] += u.y;
-                            out[4 * i + 2] += u.z;
-                            out[4 * i + 3] += u.w;
-                        }
-                    }
-                    if (more) {
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(xread);
-                    }
-                }
+            const bool more = g + (int)gridDim.x < a.G;  // another group follows
+            if (a.GS == 1) {
+                const int n = 128 * g + r;
                 if (n < a.N) {
 #pragma unroll
                     for (int t = 0; t < 16; ++t)
@@ -626,30 +656,87 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                             *dst = a.accumulate ? *dst + out[t] : out[t];  // a later K pass, same thread
                         }
                 }
-                if (more) {
-                    // every thread has read the tiles: re-arm, and let the ranks send the next ones
-                    bool freed = true;
-                    if (et == 0) {
-                        freed = mbar_wait(xread, gi & 1, abort);
-                        if (freed) {
-                            mbar_expect_tx(xfull, (uint32_t)(a.GS - 1) * kXBytes);
-                            for (int k = 1; k < a.GS; ++k) mbar_arrive_remote(xempty, (uint32_t)k);
-                        }
+                continue;
+            }
+            // stage the partial tile once this CTA is done with the previous one and
+            // every receiver took the previous slices (which also means those copies
+            // have finished reading xout)
+            if (!warp_wait(xread, (gi & 1) ^ 1, abort)) break;
+            if (!warp_wait<true>(xempty, (gi & 1) ^ 1, abort)) break;
+            float4 *dst = reinterpret_cast<float4 *>(xout + r * 16);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) dst[i] = make_float4(out[4 * i], out[4 * i + 1], out[4 * i + 2], out[4 * i + 3]);
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(xstage);
+            bool sent = true;
+            if (et == 0) {
+                sent = mbar_wait(xstage, gi & 1, abort);  // all four warps staged
+                if (sent)
+                    for (int k = 0; k < a.GS; ++k) {
+                        if (k == (int)rank) continue;
+                        const int slot = (int)rank < k ? (int)rank : (int)rank - 1;  // this rank's slot at k
+                        bulk_to_rank(map_rank(xbuf + slot * R * 16, (uint32_t)k), xout + k * R * 16, xslice,
+                                     map_rank(xfull, (uint32_t)k));
                     }
-                    if (!__shfl_sync(0xffffffffu, freed, 0)) break;  // whole warp
+            }
+            if (!__shfl_sync(0xffffffffu, sent, 0)) break;  // whole warp
+            // the other ranks' slices of this rank's rows arrived by bulk copy
+            if (!warp_wait(xfull, gi & 1, abort)) break;
+            const int lr = r - (int)rank * R;  // row within this rank's slice
+            if (lr >= 0 && lr < R) {
+                float sum[16];
+                for (int j = 0; j < a.GS; ++j) {  // rank order
+                    const float *src = j == (int)rank ? xout + r * 16 : xbuf + ((j < (int)rank ? j : j - 1) * R + lr) * 16;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float4 u = reinterpret_cast<const float4 *>(src)[i];
+                        sum[4 * i] = j == 0 ? u.x : sum[4 * i] + u.x;
+                        sum[4 * i + 1] = j == 0 ? u.y : sum[4 * i + 1] + u.y;
+                        sum[4 * i + 2] = j == 0 ? u.z : sum[4 * i + 2] + u.z;
+                        sum[4 * i + 3] = j == 0 ? u.w : sum[4 * i + 3] + u.w;
+                    }
                 }
+                const int n = 128 * g + r;
+                if (n < a.N) {
+#pragma unroll
+                    for (int t = 0; t < 16; ++t)
+                        if (t < a.M) {
+                            float *yd = a.y + (int64_t)t * a.ld_y + n;
+                            *yd = a.accumulate ? *yd + sum[t] : sum[t];  // a later K pass, same thread
+                        }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(xread);
+            if (more) {
+                // re-arm the receive barrier, then tell every sender its slot here is free
+                bool freed = true;
+                if (et == 0) {
+                    freed = mbar_wait(xread, gi & 1, abort);
+                    if (freed) {
+                        mbar_expect_tx(xfull, (uint32_t)(a.GS - 1) * xslice);
+                        for (int k = 0; k < a.GS; ++k)
+                            if (k != (int)rank) mbar_arrive_remote(xempty, (uint32_t)k);
+                    }
+                }
+                if (!__shfl_sync(0xffffffffu, freed, 0)) break;  // whole warp
             }
         }
     }
 
+    // No CTA leaves while a partner may still copy into or out of its memory:
+    // every thread arrives once its own cluster traffic is done and waits only
+    // before the CTA's exit.
+    if (a.GS > 1 && !(warp >= 1 && warp < kWorkerWarp0)) cluster_wait();  // (the set-up phase)
+    if (a.GS > 1) cluster_arrive();
     fence_before();
     __syncthreads();
-    if (a.GS > 1) cg::this_cluster().sync();  // no CTA leaves while a partner may still touch its memory
-    if (warp == 1) {
+    if (a.GS > 1) cluster_wait();
+    if (warp == 0) {
         __syncwarp();
         fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(a.tmem_cols)
-                     : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
     }
 }
 
@@ -660,9 +747,10 @@ int stage_lo(const Plan &p, int sg) {
 }
 
 struct DecodeShape {
-    int GS, ring, ring_bytes, max_mst, grid, tmem_cols;
+    int GS, max_mst, grid, workers;
     int bound[9];  // slots
     size_t smem;
+    bool ok;
 };
 
 // Stage boundaries splitting stages [g0, g1) into `parts` ranges of about
@@ -681,47 +769,44 @@ bool split_stages(const Plan &p, int g0, int g1, int parts, int *gb) {
     return true;
 }
 
+size_t smem_bytes(int GS, int max_mst, int workers) {
+    // partial tile + (GS-1) received slices of 128/GS rows
+    const size_t xbytes = GS > 1 ? (size_t)kXBytes + (size_t)(GS - 1) * (kXBytes / GS) : 0;
+    return 1024 + (size_t)workers * (kPlaneBytes + 512) + (size_t)max_mst * (kTokBytes + 512) + xbytes + 512;
+}
+
 DecodeShape shape_for(const Plan &p, int GS, int64_t G, int sms, int g0, int g1) {
     DecodeShape sh = {};
     sh.GS = GS;
     int gb[9];
     if (!split_stages(p, g0, g1, GS, gb)) return sh;
-    int max_copy = 0;
     for (int r = 0; r <= GS; ++r) sh.bound[r] = stage_lo(p, gb[r]);
-    for (int r = 0; r < GS; ++r) {
-        sh.max_mst = std::max(sh.max_mst, gb[r + 1] - gb[r]);
-        for (int k = gb[r]; k < gb[r + 1]; k += 2) {
-            const int e = std::min(k + 2, gb[r + 1]);
-            max_copy = std::max(max_copy, (int)(slot_offset(p, stage_lo(p, e)) - slot_offset(p, stage_lo(p, k))));
-        }
-    }
-    const int cols = kSfbCol + 4 * sh.max_mst;
-    if (cols > 512) return sh;
-    sh.tmem_cols = 64;
-    while (sh.tmem_cols < cols) sh.tmem_cols *= 2;
-    sh.ring_bytes = (max_copy + 127) / 128 * 128;
-    const size_t fixed = 1024 + (size_t)kConv * (kPlaneBytes + 512) + (size_t)sh.max_mst * (kTokBytes + 512) +
-                         (GS > 1 ? (size_t)GS * kXBytes : 0) + 512;
-    const size_t budget = 225 * 1024;
-    sh.ring = fixed + 2 * (size_t)sh.ring_bytes <= budget
-                  ? (int)std::min<size_t>(8, (budget - fixed) / std::max(1, sh.ring_bytes))
-                  : 0;
-    sh.smem = std::max<size_t>(kMinSmem, fixed + (size_t)sh.ring * sh.ring_bytes);
+    for (int r = 0; r < GS; ++r) sh.max_mst = std::max(sh.max_mst, gb[r + 1] - gb[r]);
+    // as many workers as fit, up to one per stage
+    sh.workers = std::min(kMaxWorkers, sh.max_mst);
+    while (sh.workers > 1 && smem_bytes(GS, sh.max_mst, sh.workers) > 225 * 1024) --sh.workers;
+    sh.smem = std::max<size_t>(kMinSmem, smem_bytes(GS, sh.max_mst, sh.workers));
+    sh.ok = sh.max_mst <= kMaxStages && sh.smem <= 225 * 1024 && sh.workers >= std::min(4, sh.max_mst);
     sh.grid = (int)std::min<int64_t>(G, std::max(1, sms / GS));
     return sh;
 }
 
-// Choose the K split: the fewest rounds of 128-row groups per CTA, weighted by
-// the K share each CTA streams, among plans that fit shared memory with at
-// least two copy stages; ties go to the smaller split.
+// Choose the K split.  A CTA's time is about (groups it owns) x (stages a
+// worker owns per group + a fixed cost per group), in units of one worker
+// stage (~2.5 us, the latency of its loads).  In a cluster every group after
+// the first also waits for the previous group's cross-rank exchange, which
+// measured at 8-13 us on GB300 (q/gate/down projections of an 8B model, each
+// cluster size forced in turn), so clusters pay off only when their CTAs own
+// one group each.  Ties go to the smaller cluster.
 DecodeShape pick_shape(const Plan &p, int64_t G, int sms, int g0, int g1) {
     DecodeShape best = {};
     double best_cost = 1e30;
     for (int GS = 1; GS <= 8 && GS <= g1 - g0; GS *= 2) {
         const DecodeShape sh = shape_for(p, GS, G, sms, g0, g1);
-        if (sh.ring < 2) continue;
+        if (!sh.ok) continue;
         const double rounds = (double)((G + sh.grid - 1) / sh.grid);
-        const double cost = rounds / GS * (1.0 + 0.02 * GS);  // small charge for the cross-CTA reduction
+        const double cost = rounds * ((sh.max_mst + sh.workers - 1) / sh.workers + 1.0) +
+                            (GS > 1 ? 0.3 + 8.0 * (rounds - 1.0) : 0.0);
         if (cost < best_cost - 1e-9) {
             best_cost = cost;
             best = sh;
@@ -777,24 +862,22 @@ int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, 
         bool ok = true;
         for (int k = 0; k < passes && ok; ++k) {
             plan[k] = pick_shape(p, a.G, sm_count(), win[k], win[k + 1]);
-            ok = plan[k].ring >= 2;
+            ok = plan[k].ok;
         }
         if (!ok) continue;
         for (int k = 0; k < passes; ++k) {
             const DecodeShape &sh = plan[k];
             a.GS = sh.GS;
             for (int i = 0; i < 9; ++i) a.bound[i] = i <= sh.GS ? sh.bound[i] : sh.bound[sh.GS];
-            a.ring = sh.ring;
-            a.ring_bytes = sh.ring_bytes;
             a.max_mst = sh.max_mst;
-            a.tmem_cols = sh.tmem_cols;
+            a.workers = sh.workers;
             a.accumulate = k > 0;
             cudaError_t e =
                 cudaFuncSetAttribute(gemm_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh.smem);
             if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(decode smem)");
             cudaLaunchConfig_t cfg = {};
             cfg.gridDim = dim3((unsigned)sh.grid, (unsigned)sh.GS, 1);
-            cfg.blockDim = dim3(kThreads, 1, 1);
+            cfg.blockDim = dim3((unsigned)((kWorkerWarp0 + sh.workers) * 32), 1, 1);
             cfg.dynamicSmemBytes = sh.smem;
             cfg.stream = st;
             cudaLaunchAttribute attr[2];
