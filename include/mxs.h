@@ -185,6 +185,27 @@ MXS_API int mxs_linear_decode(const void *x_bf16, int64_t M, int64_t K, int64_t 
                               int rounding, const void *packed_w, int64_t N, float *y, int64_t ld_y,
                               void *workspace, size_t ws_bytes, void *stream);
 
+/* mxs_linear_decode for callers that cannot allocate device memory (an
+ * allocator-free runtime that owns all device memory, a plug-in whose host
+ * forbids allocation on its hot path, a real-time loop that must not block in
+ * the allocator).  The paper has no counterpart.  Same arguments, results
+ * and launches as mxs_linear_decode, but the activation planes live in a
+ * fixed 2 MiB array inside the library (a __device__ variable every GPU that
+ * loads the library holds until exit) instead of a caller workspace; the call
+ * allocates nothing.  Sizes whose planes exceed 2 MiB
+ * (mxs_act_planes_bytes(M, K, bits) > 2 MiB; M <= 16 fits for K <= 49152
+ * with any map) return MXS_ERR_BUFFER.  The first call on each device looks
+ * up the array's device address (cudaGetSymbolAddress, current device):
+ * make that first call before any stream capture.  All calls share the one
+ * array and leave their planes in it: calls ordered on one stream are safe
+ * (each waits for the one before it as mxs_linear_decode does), calls that
+ * overlap on the GPU (other streams, other host threads) race and give wrong
+ * results.  Nothing in the array has to start at zero: every byte the GEMM
+ * reads is written by the same call's quantizer. */
+MXS_API int mxs_linear_decode_noalloc(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits,
+                                      int rounding, const void *packed_w, int64_t N, float *y, int64_t ld_y,
+                                      void *stream);
+
 /* Prefill path only (any M >= 1, efficient for M >= 128): the tensor-core
  * kernel over the MMA planes of the activations (mxs_quantize_act `planes`)
  * and of the weights (packed with MXS_W_COMPACT_AND_PLANES).  Sec. 6: the

@@ -25,7 +25,8 @@ LIB_PATH = os.path.join(_HERE, "libmxs.so")
 EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_bytes",
            "mxs_act_planes_bytes", "mxs_weight_bytes", "mxs_gemm_workspace_bytes",
            "mxs_quantize_act", "mxs_pack_weight", "mxs_gemm", "mxs_gemm_decode",
-           "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode"]
+           "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode",
+           "mxs_linear_decode_noalloc"]
 
 _lock = threading.Lock()
 _lib = None
@@ -70,6 +71,8 @@ def lib() -> ctypes.CDLL:
         L.mxs_gemm_decode.restype = I
         L.mxs_linear_decode.argtypes = [P, I64, I64, I64, P, I, P, I64, P, I64, P, SZ, P]
         L.mxs_linear_decode.restype = I
+        L.mxs_linear_decode_noalloc.argtypes = [P, I64, I64, I64, P, I, P, I64, P, I64, P]
+        L.mxs_linear_decode_noalloc.restype = I
         L.mxs_gemm_prefill.argtypes = [P, P, P, I64, I64, I64, P, I64, P]
         L.mxs_gemm_prefill.restype = I
         L.mxs_test_prefill_starve.argtypes = [P, P, P, I64, I64, I64, P, I64, I, P]
@@ -227,6 +230,19 @@ def linear_decode(x, bits, packed_w, N: int, rounding: int = RNE, y=None, worksp
     ws_bytes = workspace.numel() * workspace.element_size()
     check(lib().mxs_linear_decode(_ptr(x), M, K, x.stride(0), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
                                   y.stride(0), _ptr(workspace), ws_bytes, _stream(stream)))
+    return y
+
+
+def linear_decode_noalloc(x, bits, packed_w, N: int, rounding: int = RNE, y=None, stream=None):
+    """linear_decode without a workspace: the planes go to the library's own
+    2 MiB device array (for callers that cannot allocate; see the header)."""
+    import torch
+    b = _Bits(bits)
+    M, K = x.shape
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float32, device=packed_w.device)
+    check(lib().mxs_linear_decode_noalloc(_ptr(x), M, K, x.stride(0), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
+                                          y.stride(0), _stream(stream)))
     return y
 
 

@@ -121,3 +121,15 @@ def test_valid_call_without_gpu_reports_cuda_error(L):
     bits = np.full(4, 4, np.uint8)
     rc = L.mxs_quantize_act(FAKE, 4, 128, 128, bits.ctypes.data, 0, FAKE, FAKE, None, None)
     assert rc == 6 and "cudaGetDevice" in mxs.last_error()
+
+
+def test_noalloc_rejects_sizes_beyond_its_scratch(L):
+    """mxs_linear_decode_noalloc keeps the planes in a fixed 2 MiB array: a
+    16-token K=65536 all-8-bit layer needs more and is refused before any
+    device call (so no GPU is needed here)."""
+    bits = np.full(2048, 8, np.uint8)
+    assert L.mxs_act_planes_bytes(16, 65536, bits.ctypes.data) > 2 << 20
+    rc = L.mxs_linear_decode_noalloc(FAKE, 16, 65536, 65536, bits.ctypes.data, 0, FAKE, 16, FAKE, 16, None)
+    assert rc == 5 and "built-in scratch" in mxs.last_error()
+    small = np.full(4, 4, np.uint8)
+    assert L.mxs_linear_decode_noalloc(FAKE, 17, 128, 128, small.ctypes.data, 0, FAKE, 16, FAKE, 16, None) == 2
