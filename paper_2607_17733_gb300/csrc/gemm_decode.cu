@@ -5,13 +5,14 @@
 // two blocks' mantissas): the MXINT product of Sec. 2 (fixed-point MACs under
 // a shared power-of-two scale) with the per-block widths of Sec. 4.1.
 //
-// Decode reads every weight byte once, so the kernel keeps the weights in
-// their compact form (4-bit nibbles, 6/8-bit bytes) until they are in
-// registers, and does all arithmetic on the tensor core:
+// Decode reads every weight byte once, so the kernel streams the weights in
+// their compact form (4-bit nibbles, 6/8-bit bytes) and does all arithmetic on
+// the tensor core:
 //   * the block-scaled FP8 MMA (tcgen05.mma kind::mxf8f6f4, scale_vec::1X)
-//     with 128 weight rows as the A operand and the <= 16 tokens as the N = 16
-//     B operand; per-block scales are applied by the hardware and the sum over
-//     K stays in fp32 tensor-memory accumulators;
+//     with 128 weight rows as the A operand -- in tensor memory -- and the
+//     <= 16 tokens as the N = 16 B operand in shared memory; per-block scales
+//     are applied by the hardware and the sum over K stays in fp32
+//     tensor-memory accumulators;
 //   * a weight code of magnitude <= 15 is fed as the e4m3 byte
 //     (sign << 7) | |m|, whose value is |m| * 2^-9 (subnormals and the first
 //     binade); 6/8-bit codes split as |m| = 16h + l into two such digits
@@ -27,23 +28,26 @@
 //     from packed codes.
 // Work: a CTA owns 128-row weight groups and (in a cluster) a K range of them,
 // cut into MMA stages of 128 K'-bytes (four 4-bit slots or two 6/8-bit
-// slots).  Up to ten worker warps own whole stages, round robin: a worker
-// loads its stage's codes straight from HBM into registers (coalesced 16-byte
-// loads, the next stage in flight while it converts the current one), writes
-// the e4m3 digits into its own 128-byte-swizzled plane buffer and the weight
-// scale tile, and issues the stage's MMAs into its own accumulator.  Workers
-// never wait for one another; the epilogue warps add the workers' partial
-// accumulators in worker order (a fixed order: results are deterministic).
-// Other warps: warp 0 owns tensor memory and loads the token operand; warps
-// 1-4 run the epilogue (and build the token operand from codes).
+// slots); two stages make one copy chunk.  One thread streams the chunks into
+// a shared-memory ring with cp.async.bulk (about 17 KB per copy, up to eight
+// in flight: the ring, not registers, holds the bytes in flight).  Four quads
+// of four worker warps take the chunks round robin; each warp converts its 32
+// rows (its tensor-memory lane quarter) of a stage and writes the e4m3 digits
+// straight into the quad's A tile in tensor memory (tcgen05.st), the quad
+// meets at a hardware named barrier, and one thread issues the stage's MMAs
+// into the quad's accumulator.  Quads never wait for one another; the
+// epilogue warps add the quads' partial accumulators in quad order (a fixed
+// order: results are deterministic).  Warps 1-4 also load the token operand.
 // K is split over the CTAs of a thread-block cluster when N alone cannot
 // occupy the GPU.  The ranks then reduce-scatter through distributed shared
 // memory: rank k receives rows [k*R, (k+1)*R) (R = 128/cluster size) of every
 // other rank's partial tile by bulk copy, adds the partials in rank order and
 // stores those rows.  A K range whose token operand does not fit shared
 // memory runs as several passes, each adding into y.
-// Every mbarrier wait is bounded; on expiry the kernel records
-// MXS_ERR_TIMEOUT, stops, drains what it issued and frees tensor memory.
+// Every wait is bounded; on expiry the kernel records MXS_ERR_TIMEOUT, stops,
+// drains what it issued and frees tensor memory.  The quads' named barrier
+// carries an AND of the four warps' status, so a warp that gave up stops its
+// quad at the next stage instead of leaving the others at the barrier.
 // Weight scale bytes above 245 (|w| >= 2^118) saturate at 254 after the digit
 // shift.
 #include <algorithm>
@@ -60,18 +64,19 @@ __device__ int g_decode_status;  // sticky MXS_ERR_TIMEOUT, read by mxs_device_s
 
 namespace {
 
-constexpr int kMaxWorkers = 10;                                 // worker warps per CTA, chosen per launch
-constexpr int kWorkerWarp0 = 5;                                 // warps 5..
-constexpr int kMaxThreads = (kWorkerWarp0 + kMaxWorkers) * 32;  // 480
-constexpr int kPlaneBytes = 128 * 128;  // 128 rows x 128 bytes of K' (SW128)
-constexpr int kTokBytes = 16 * 128;     // 16 token rows x 128 bytes of K'
-constexpr int kAccCols = 16;            // one accumulator: 16 token columns
-constexpr int kSfaCol = 2 * kMaxWorkers * kAccCols;  // 320: 4 columns of weight scales per worker
-constexpr int kSfbCol = kSfaCol + 4 * kMaxWorkers;   // 360: 4 columns per MMA stage of token scales
-constexpr int kTmemCols = 512;
-constexpr int kMaxStages = (kTmemCols - kSfbCol) / 4;  // 38
+constexpr int kQuads = 4;                                 // worker quads (4 warps each)
+constexpr int kWorkerWarp0 = 5;                           // warps 5..20
+constexpr int kThreads = (kWorkerWarp0 + 4 * kQuads) * 32;  // 672
+constexpr int kTokBytes = 16 * 128;                       // 16 token rows x 128 bytes of K'
+constexpr int kAccCols = 16;                              // one accumulator: 16 token columns
+// tensor-memory columns: quad j's A tiles at kACol + 32 (2j + buf), its
+// accumulators at kAccCol + 16 (2j + b), its weight / token scale columns at
+// kSfaCol / kSfbCol + 4 (2j + buf)
+constexpr int kACol = 0, kAccCol = 256, kSfaCol = 384, kSfbCol = 416, kTmemCols = 512;
 constexpr int kXBytes = 128 * 16 * 4;  // one fp32 partial tile
 constexpr int kMinSmem = 116 * 1024;   // one CTA per SM (each allocates all of tensor memory)
+constexpr int kQuadBar0 = 8;           // named barriers 8..11: one per quad
+constexpr int kCodesBar = 12;          // named barrier of the token prologue (codes mode)
 constexpr long long kWaitCycles = 4000000000ll;  // ~2 s at the maximum SM clock
 
 struct DecodeArgs {
@@ -81,13 +86,14 @@ struct DecodeArgs {
     const uint8_t *w;       // packed weight buffer
     float *y;
     int64_t ld_y;
-    int M, N, G;      // tokens, output features, 128-row groups
-    int GS;           // CTAs per cluster along K
-    int bound[9];     // rank r owns slots [bound[r], bound[r+1]) (stage-aligned)
-    int max_mst;      // most MMA stages any rank holds (token operand carve)
-    int workers;      // worker warps (blockDim = (5 + workers) warps)
-    int accumulate;   // add into y (a later K pass) instead of storing
-    int64_t GB;       // bytes of one 128-row weight group
+    int M, N, G;           // tokens, output features, 128-row groups
+    int GS;                // CTAs per cluster along K
+    int bound[9];          // rank r owns slots [bound[r], bound[r+1]) (stage-aligned)
+    int max_mst;           // most MMA stages any rank holds (token operand carve)
+    int ring, slot_bytes;  // copy chunks in flight, bytes per ring slot (a multiple of 1024)
+    int w_off;             // weights' offset in a slot: after the streamed token tiles (planes mode), else 0
+    int accumulate;        // add into y (a later K pass) instead of storing
+    int64_t GB;            // bytes of one 128-row weight group
 };
 
 // ------------------------------------------------------------------ PTX helpers
@@ -182,22 +188,19 @@ __device__ __forceinline__ void bulk_to_rank(uint32_t dst_cluster, const void *s
         "r"(su32(src)), "r"(bytes), "r"(bar_cluster)
         : "memory");
 }
-// streaming loads of weight codes: read once, not kept in L1
-__device__ __forceinline__ uint4 ld_stream16(const uint8_t *p) {
-    uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
-    return v;
-}
-__device__ __forceinline__ uint32_t ld_stream1(const uint8_t *p) {
-    uint16_t v;
-    asm volatile("ld.global.nc.L1::no_allocate.u8 %0, [%1];" : "=h"(v) : "l"(p));
-    return v;
-}
 // generic-proxy shared-memory writes -> visible to the tensor core / bulk copies
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+// named barrier over n threads (whole warps) that also ANDs a flag across them
+__device__ __forceinline__ bool bar_and(int id, int n, bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n bar.red.and.pred po, %2, %3, pi;\n selp.u32 %0, 1, 0, po;\n}"
+        : "=r"(r)
+        : "r"((uint32_t)v), "r"(id), "r"(n)
+        : "memory");
+    return r != 0;
+}
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release;" ::: "memory"); }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire;" ::: "memory"); }
 
@@ -217,12 +220,25 @@ constexpr uint32_t kIdesc = ((uint32_t)(16 >> 3) << 17) | (1u << 23) | ((uint32_
 __device__ __forceinline__ constexpr uint32_t idesc(int sfa_id, int sfb_id) {
     return kIdesc | ((uint32_t)sfb_id << 4) | ((uint32_t)sfa_id << 29);
 }
-__device__ __forceinline__ void mma_mx(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t sfa, uint32_t sfb,
-                                       uint32_t accum) {
+// the same with the A operand in tensor memory (K-major: row i in lane i, four
+// 8-bit elements per 32-bit column)
+__device__ __forceinline__ void mma_mx_t(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t id, uint32_t sfa,
+                                         uint32_t sfb, uint32_t accum) {
     asm volatile(
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%5], [%6], p;\n}" ::"r"(d),
-        "l"(a), "l"(b), "r"(id), "r"(accum), "r"(sfa), "r"(sfb)
+        " tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], [%1], %2, %3, [%5], [%6], p;\n}" ::"r"(d),
+        "r"(a_tmem), "l"(b), "r"(id), "r"(accum), "r"(sfa), "r"(sfb)
+        : "memory");
+}
+// 32 consecutive 32-bit columns of this thread's lane
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+        "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]), "r"(v[17]), "r"(v[18]),
+        "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]),
+        "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
         : "memory");
 }
 __device__ __forceinline__ void tmem_cp_sf(uint32_t taddr, uint64_t desc) {
@@ -277,118 +293,29 @@ struct Stages {  // MMA stages of a CTA's K range [c0, c1): 4-bit ones (4 slots)
     }
 };
 
-// One half of a worker's stage in registers: lane l holds rows l + 32i
-// (i < 4).  A 4-bit half is slots 2h, 2h+1 (v[4k+i] = slot 2h+k, row i); a
-// 6/8-bit half is slot h (v[2i], v[2i+1] = the two 16-byte words of row i).
-// Either way the half fills 16-byte chunks 4h..4h+3 of each row and
-// scale-tile bytes 2h, 2h+1.
-struct Half {
-    uint4 v[8];
-    uint32_t s[8];  // scale bytes (4-bit: [4k+i] = slot 2h+k, row i; 6/8-bit: [i] = row i)
-};
-
-// Load half `h` of stage `st` of the weight group at `wg` (lane l: rows l + 32i).
-__device__ __forceinline__ void load_half(const Plan &p, const Stages &S, const uint8_t *wg, int st, int h, int l,
-                                          Half &x) {
-    int lo, hi;
-    S.range(st, lo, hi);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        x.v[i] = make_uint4(0, 0, 0, 0);
-        x.s[i] = 0;
-    }
-    if (st < S.st4) {
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            const int q = 2 * h + k;
-            if (lo + q < hi) {  // a partial last stage has fewer slots
-                const uint8_t *slot = wg + slot_offset(p, lo + q);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    x.v[4 * k + i] = ld_stream16(slot + 16 * (l + 32 * i));
-                    x.s[4 * k + i] = ld_stream1(slot + 2048 + l + 32 * i);
-                }
-            }
-        }
-    } else if (lo + h < hi) {
-        const uint8_t *slot = wg + slot_offset(p, lo + h);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            x.v[2 * i] = ld_stream16(slot + 32 * (l + 32 * i));
-            x.v[2 * i + 1] = ld_stream16(slot + 32 * (l + 32 * i) + 16);
-            x.s[i] = ld_stream1(slot + 4096 + l + 32 * i);
-        }
-    }
-}
-
-// Convert a loaded half into digit-plane chunks 4h..4h+3 of rows l + 32i and
-// return the row's scale-tile bytes 2h, 2h+1 (bits 16i..16i+15 for row i).
-__device__ __forceinline__ uint64_t store_half(const Plan &p, const Stages &S, int st, int h, int l, const Half &x,
-                                               uint8_t *pl) {
-    int lo, hi;
-    S.range(st, lo, hi);
-    uint64_t sf = 0;
-    if (st < S.st4) {
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            const int q = 2 * h + k;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int r = l + 32 * i;
-                const uint4 v = x.v[4 * k + i];
-                // word j: bytes hold elements 8j..8j+3 (low nibbles), 8j+4..8j+7 (high nibbles)
-                *reinterpret_cast<uint4 *>(pl + sw128(r, 2 * q)) =
-                    make_uint4(lo_nib(v.x), hi_nib(v.x), lo_nib(v.y), hi_nib(v.y));
-                *reinterpret_cast<uint4 *>(pl + sw128(r, 2 * q + 1)) =
-                    make_uint4(lo_nib(v.z), hi_nib(v.z), lo_nib(v.w), hi_nib(v.w));
-                // absent slots hold zero codes under scale byte 0 (a zero term)
-                sf |= (uint64_t)(lo + q < hi ? shifted(x.s[4 * k + i], 7) : 0u) << (16 * i + 8 * k);
-            }
-        }
-    } else {
-        const bool six = lo + h < hi && slot_width(p, lo + h) == 6;
-        const uint32_t sh_hi = six ? 9 : 7, sh_lo = six ? 5 : 3;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int r = l + 32 * i;
-            const uint4 v0 = x.v[2 * i], v1 = x.v[2 * i + 1];
-            *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * h)) =
-                make_uint4(hi_digit(v0.x), hi_digit(v0.y), hi_digit(v0.z), hi_digit(v0.w));
-            *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * h + 1)) =
-                make_uint4(hi_digit(v1.x), hi_digit(v1.y), hi_digit(v1.z), hi_digit(v1.w));
-            *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * h + 2)) =
-                make_uint4(lo_digit(v0.x), lo_digit(v0.y), lo_digit(v0.z), lo_digit(v0.w));
-            *reinterpret_cast<uint4 *>(pl + sw128(r, 4 * h + 3)) =
-                make_uint4(lo_digit(v1.x), lo_digit(v1.y), lo_digit(v1.z), lo_digit(v1.w));
-            const uint32_t b2 = lo + h < hi ? (shifted(x.s[i], sh_hi) | (shifted(x.s[i], sh_lo) << 8)) : 0u;
-            sf |= (uint64_t)b2 << (16 * i);
-        }
-    }
-    return sf;
-}
-
-__global__ void __launch_bounds__(kMaxThreads, 1) gemm_decode_kernel(const __grid_constant__ Plan p,
-                                                                     const __grid_constant__ DecodeArgs a,
-                                                                     const __grid_constant__ CUtensorMap tok_map) {
+__global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_constant__ Plan p,
+                                                                  const __grid_constant__ DecodeArgs a,
+                                                                  const __grid_constant__ CUtensorMap tok_map) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t sbase = su32(smem_raw);
     uint8_t *smem = smem_raw + (((sbase + 1023) & ~1023u) - sbase);  // 1024-aligned for the swizzled tiles
-    const int W = a.workers;
-    uint8_t *planes = smem;                              // W x 16 KB
-    uint8_t *tok = planes + W * kPlaneBytes;             // max_mst x 2 KB
-    uint8_t *sfa = tok + (size_t)a.max_mst * kTokBytes;  // W x 512
-    uint8_t *sfb = sfa + W * 512;                        // max_mst x 512
+    // ring slot: [two token tiles (planes mode)][their two scale tiles][compact weight chunk]
+    uint8_t *ring = smem;                                        // ring x slot_bytes
+    uint8_t *tok = ring + (size_t)a.ring * a.slot_bytes;         // codes mode: max_mst x 2 KB resident token planes
+    uint8_t *sfb = tok + (size_t)a.max_mst * kTokBytes;          // codes mode: max_mst x 512 token scale tiles
+    uint8_t *sfa = sfb + (size_t)a.max_mst * 512;                // kQuads x 2 x 512 weight scale tiles
     // cluster reduce-scatter: rank k adds up rows [k*R, (k+1)*R) of the GS partial
     // tiles (R = 128/GS) and stores them; xout is this rank's whole partial tile,
     // xbuf the slices the other ranks send here (slot of sender j: j, or j-1 past k)
     const int R = 128 / a.GS;
-    float *xout = reinterpret_cast<float *>(sfb + (size_t)a.max_mst * 512);  // [128][16] (GS > 1)
-    float *xbuf = xout + (a.GS > 1 ? 128 * 16 : 0);                          // [GS-1][R][16]
+    float *xout = reinterpret_cast<float *>(sfa + kQuads * 2 * 512);  // [128][16] (GS > 1)
+    float *xbuf = xout + (a.GS > 1 ? 128 * 16 : 0);                                 // [GS-1][R][16]
     uint64_t *bars = reinterpret_cast<uint64_t *>(xbuf + (size_t)(a.GS - 1) * R * 16);
-    uint64_t *plane_free = bars;  // [W] tcgen05.commit
-    uint64_t *acc_full = plane_free + W, *acc_empty = acc_full + 2;
-    uint64_t *tok_full = acc_empty + 2, *tok_ready = tok_full + 1;
-    uint64_t *xfull = tok_ready + 1, *xempty = xfull + 1, *xstage = xempty + 1, *xread = xstage + 1;
+    uint64_t *full_c = bars, *empty_c = full_c + a.ring;
+    uint64_t *a_free = empty_c + a.ring;  // [kQuads][2] tcgen05.commit
+    uint64_t *acc_full = a_free + 2 * kQuads, *acc_empty = acc_full + 2;
+    uint64_t *tok_full = acc_empty + 2;
+    uint64_t *xfull = tok_full + 1, *xempty = xfull + 1, *xstage = xempty + 1, *xread = xstage + 1;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(xread + 1);
     int *abort_flag = reinterpret_cast<int *>(tmem_slot + 1);
     volatile int *abort = abort_flag;
@@ -399,29 +326,54 @@ __global__ void __launch_bounds__(kMaxThreads, 1) gemm_decode_kernel(const __gri
     const bool from_planes = a.tok_sf != nullptr;
     Stages S;
     S.init(p, c0, c1);
-    const int nw = min(W, S.n);  // workers with a stage in every group
+    const int nchunks = (S.n + 1) / 2;          // a copy chunk holds two MMA stages
+    const int nq = min(kQuads, nchunks);        // quads with a chunk in every group
+    const int ngroups = (int)blockIdx.x < a.G ? (a.G - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+    const int total = ngroups * nchunks;        // chunks this CTA streams
     const uint32_t xslice = (uint32_t)(R * 16 * 4);
+    const int sg0 = c0 < p.n4 ? c0 / 4 : p.st4 + (c0 - p.n4) / 2;  // the rank's first stage in the planes
 
-    // Workers put their first stage's loads in flight before anything else:
-    // the weights are static (see mxs_linear_decode), so they need no wait.
-    Half A, B;
-    if (warp >= kWorkerWarp0 && warp - kWorkerWarp0 < nw && (int)blockIdx.x < a.G) {
-        const uint8_t *wg = a.w + (int64_t)blockIdx.x * a.GB;
-        load_half(p, S, wg, warp - kWorkerWarp0, 0, lane, A);
-        load_half(p, S, wg, warp - kWorkerWarp0, 1, lane, B);
-    }
+    // chunk qc (in streaming order): group blockIdx.x + (qc / nchunks) * gridDim.x,
+    // stages 2k, 2k+1 with k = qc % nchunks; it goes to ring slot qc % ring and is
+    // converted by quad qc % kQuads (ring is a multiple of kQuads, so each slot
+    // has one consumer, which takes its slots in order)
+    auto issue = [&](int qc) {
+        const int gi = qc / nchunks, k = qc - gi * nchunks;
+        const int s = qc % a.ring;
+        int lo, hi, lo2, hi2;
+        S.range(2 * k, lo, hi);
+        if (2 * k + 1 < S.n) S.range(2 * k + 1, lo2, hi2); else hi2 = hi;
+        const int64_t off = slot_offset(p, lo);
+        const uint32_t bytes = (uint32_t)(slot_offset(p, hi2) - off);
+        const uint8_t *wg = a.w + (int64_t)((int)blockIdx.x + gi * (int)gridDim.x) * a.GB;
+        const int nst = min(2, S.n - 2 * k);
+        // planes mode: the chunk's token tiles complete on the same barrier (issue_tok)
+        mbar_expect_tx(&full_c[s], bytes + (from_planes ? (uint32_t)nst * (kTokBytes + 512) : 0u));
+        bulk_load(ring + (size_t)s * a.slot_bytes + a.w_off, wg + off, bytes, &full_c[s]);
+    };
+    // planes mode: the token operand of chunk qc's stages, by TMA from the planes
+    auto issue_tok = [&](int qc) {
+        const int k = qc % nchunks, s = qc % a.ring;
+        const int nst = min(2, S.n - 2 * k);
+        uint8_t *slot = ring + (size_t)s * a.slot_bytes;
+        for (int i = 0; i < nst; ++i) tma_load_2d(slot + i * kTokBytes, &tok_map, &full_c[s], 128 * (sg0 + 2 * k + i), 0);
+        bulk_load(slot + 2 * kTokBytes, a.tok_sf + (int64_t)(sg0 + 2 * k) * 512, (uint32_t)nst * 512, &full_c[s]);
+    };
 
     // the next kernel on the stream may launch now (it waits for this grid
     // before it touches what this grid writes)
     if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (threadIdx.x == 0) {
-        for (int i = 0; i < W; ++i) mbar_init(&plane_free[i], 1);
+        for (int i = 0; i < a.ring; ++i) {
+            mbar_init(&full_c[i], 1);
+            mbar_init(&empty_c[i], 1);  // tcgen05.commit after the chunk's MMAs (they read its token tiles)
+        }
+        for (int i = 0; i < 2 * kQuads; ++i) mbar_init(&a_free[i], 1);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&acc_full[i], nw);  // each active worker commits once per group
+            mbar_init(&acc_full[i], nq);  // each quad with a chunk in the group commits once
             mbar_init(&acc_empty[i], 4);  // the four epilogue warps
         }
         mbar_init(tok_full, from_planes ? 1 : 4);
-        mbar_init(tok_ready, 1);              // tcgen05.commit once the token scales are in tensor memory
         mbar_init(xfull, 1);                  // armed per tile with the bytes of GS-1 slices
         mbar_init(xempty, max(1, a.GS - 1));  // every receiver took this rank's previous slices (copies done)
         mbar_init(xstage, 4);                 // the four epilogue warps have staged the partial tile
@@ -429,8 +381,11 @@ __global__ void __launch_bounds__(kMaxThreads, 1) gemm_decode_kernel(const __gri
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         if (a.GS > 1) mbar_expect_tx(xfull, (uint32_t)(a.GS - 1) * xslice);  // the first tile's slices
+        // the weights are static (see mxs_linear_decode): fill the ring right away
+        for (int qc = 0; qc < min(a.ring, total); ++qc) issue(qc);
     }
     if (warp == 0) {
+        __syncwarp();
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)),
                      "r"(kTmemCols)
                      : "memory");
@@ -446,106 +401,176 @@ __global__ void __launch_bounds__(kMaxThreads, 1) gemm_decode_kernel(const __gri
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 0) {
-        // ------------------------------------------------------------ token operand -> smem, scales -> TMEM
+        // ------------------------------------------------------------ producer: the rest of the chunks
         if (lane == 0) {
             if (from_planes) {
                 // the planes may come from the kernel just before this one (programmatic
-                // dependent launch): wait for it before the first read
+                // dependent launch): wait for it before the first token load
                 asm volatile("griddepcontrol.wait;" ::: "memory");
-                const int sg0 = c0 < p.n4 ? c0 / 4 : p.st4 + (c0 - p.n4) / 2;
-                mbar_expect_tx(tok_full, (uint32_t)S.n * (kTokBytes + 512));
-                for (int st = 0; st < S.n; ++st)
-                    tma_load_2d(tok + st * kTokBytes, &tok_map, tok_full, 128 * (sg0 + st), 0);
-                bulk_load(sfb, a.tok_sf + (int64_t)sg0 * 512, (uint32_t)S.n * 512, tok_full);
+                for (int qc = 0; qc < min(a.ring, total); ++qc) issue_tok(qc);
             }
-            if (mbar_wait(tok_full, 0, abort)) {
-                fence_after();
-                const uint64_t dsfb = desc_sf(su32(sfb));
-                for (int st = 0; st < S.n; ++st) tmem_cp_sf(tmem + kSfbCol + 4 * st, dsfb + 32 * st);
-                mma_commit(tok_ready);
-                drain_wait(tok_ready, 0);
+            for (int qc = a.ring; qc < total; ++qc) {
+                const int s = qc % a.ring;
+                if (!mbar_wait(&empty_c[s], ((qc / a.ring) & 1) ^ 1, abort)) break;
+                issue(qc);
+                if (from_planes) issue_tok(qc);
             }
+            const int first = total > a.ring ? total - a.ring : 0;
+            for (int qc = first; qc < total; ++qc) drain_wait(&full_c[qc % a.ring], (qc / a.ring) & 1);
         }
     } else if (warp >= kWorkerWarp0) {
-        // ------------------------------------------------------------ workers
-        const int w = warp - kWorkerWarp0;
-        if (w < nw) {
-            uint8_t *pl = planes + w * kPlaneBytes;
-            uint8_t *sfa_cell = sfa + w * 512 + 16 * lane;  // rows lane + 32i: bytes 4i..4i+3
-            const uint64_t dA = desc_sw128(su32(pl)), dB = desc_sw128(su32(tok));
-            const uint64_t dsfa = desc_sf(su32(sfa + w * 512));
-            const uint32_t sfa_t = tmem + kSfaCol + 4 * w;
-            bool ok = warp_wait(tok_ready, 0, abort);
-            if (ok) fence_after();
-            uint32_t qw = 0;  // stages this worker has issued (plane_free phases)
-            int g = blockIdx.x, st = w, gi = 0;
-            bool first_in_group = true;
-            while (ok && g < a.G) {
-                const int b = gi & 1;
-                if (first_in_group) ok = warp_wait(&acc_empty[b], ((gi >> 1) & 1) ^ 1, abort);
-                // the plane buffer is free once this worker's previous MMAs have read it
-                if (ok && qw > 0) ok = warp_wait(&plane_free[w], (qw - 1) & 1, abort);
-                if (!ok) break;
-                // next stage of this worker: st + W, else its first stage of the next group
-                int g2 = g, st2 = st + W;
-                if (st2 >= S.n) {
-                    g2 = g + gridDim.x;
-                    st2 = w;
-                }
-                const uint8_t *wg2 = a.w + (int64_t)(g2 < a.G ? g2 : g) * a.GB;
-                const uint64_t sf0 = store_half(p, S, st, 0, lane, A, pl);
-                if (g2 < a.G) load_half(p, S, wg2, st2, 0, lane, A);
-                const uint64_t sf1 = store_half(p, S, st, 1, lane, B, pl);
-                if (g2 < a.G) load_half(p, S, wg2, st2, 1, lane, B);
-                // scale tile: the lane's 16 bytes are rows lane + 32i, 4 bytes each
-                // (sf ids 0, 1 from half 0 and 2, 3 from half 1)
-                uint32_t cell[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    cell[i] = (uint32_t)((sf0 >> (16 * i)) & 0xFFFF) | ((uint32_t)((sf1 >> (16 * i)) & 0xFFFF) << 16);
-                *reinterpret_cast<uint4 *>(sfa_cell) = make_uint4(cell[0], cell[1], cell[2], cell[3]);
-                fence_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    fence_after();
-                    tmem_cp_sf(sfa_t, dsfa);
-                    const uint32_t acc = tmem + kAccCols * (kMaxWorkers * b + w);
-                    const uint32_t sfb_t = tmem + kSfbCol + 4 * st;
-                    const uint64_t db = dB + (uint64_t)(st * (kTokBytes >> 4));
-                    const uint32_t accum = first_in_group ? 0u : 1u;
+        // ------------------------------------------------------------ worker quads
+        const int wq = warp - kWorkerWarp0;
+        const int j = wq >> 2;                           // quad
+        const int qtr = warp & 3;                        // this warp's tensor-memory lane quarter
+        const int r = 32 * qtr + lane;                   // weight row (within the group) of this thread
+        const bool leader = (wq & 3) == 0 && lane == 0;  // issues the quad's tcgen05 work
+        const uint32_t a_lane = (uint32_t)(32 * qtr) << 16;
+        uint8_t *sfa_q = sfa + j * 1024;                 // two 512-byte tiles
+        const uint64_t dB = desc_sw128(su32(tok)), dsfa = desc_sf(su32(sfa_q)), dsfb = desc_sf(su32(sfb));
+        bool ok = true, tok_seen = false, stop = false;
+        uint32_t qw = 0;  // stages this quad has issued (a_free phases)
+        for (int qc = j; qc < total && !stop; qc += kQuads) {
+            const int gi = qc / nchunks, k = qc - gi * nchunks, b = gi & 1;
+            const int s = qc % a.ring;
+            if (ok) ok = warp_wait(&full_c[s], (qc / a.ring) & 1, abort);
+            int clo, chi;
+            S.range(2 * k, clo, chi);
+            uint8_t *slot_base = ring + (size_t)s * a.slot_bytes;
+            const uint8_t *chunk = slot_base + a.w_off - slot_offset(p, clo);  // + slot_offset(slot)
+            const bool first_chunk = k < kQuads;           // the quad's first chunk of the group
+            const bool last_chunk = k + kQuads >= nchunks;  // ... and its last
+            const int st_end = min(2 * k + 2, S.n);
+            for (int st = 2 * k; st < st_end; ++st, ++qw) {
+                const int buf = qw & 1;
+                // the A tile and scale tile of this buffer are free once the MMAs of two stages ago ran
+                if (ok && qw >= 2) ok = warp_wait(&a_free[2 * j + buf], ((qw >> 1) - 1) & 1, abort);
+                if (ok) {
+                    int lo, hi;
+                    S.range(st, lo, hi);
+                    uint32_t d[32], sfw = 0;
                     if (st < S.st4) {
-                        // slot q: weight digits at K' bytes 32q.., token values at 32q..
-                        mma_mx(acc, dA, db, idesc(0, 0), sfa_t, sfb_t, accum);
-                        mma_mx(acc, dA + 2, db + 2, idesc(1, 1), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, dA + 4, db + 4, idesc(2, 2), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, dA + 6, db + 6, idesc(3, 3), sfa_t, sfb_t, 1u);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            uint4 v = make_uint4(0, 0, 0, 0);
+                            uint32_t sc = 0;
+                            if (lo + q < hi) {
+                                const uint8_t *slot = chunk + slot_offset(p, lo + q);
+                                v = *reinterpret_cast<const uint4 *>(slot + 16 * r);
+                                sc = shifted(slot[2048 + r], 7);
+                            }
+                            // word i: bytes hold elements 8i..8i+3 (low nibbles), 8i+4..8i+7 (high nibbles)
+                            d[8 * q + 0] = lo_nib(v.x);
+                            d[8 * q + 1] = hi_nib(v.x);
+                            d[8 * q + 2] = lo_nib(v.y);
+                            d[8 * q + 3] = hi_nib(v.y);
+                            d[8 * q + 4] = lo_nib(v.z);
+                            d[8 * q + 5] = hi_nib(v.z);
+                            d[8 * q + 6] = lo_nib(v.w);
+                            d[8 * q + 7] = hi_nib(v.w);
+                            sfw |= sc << (8 * q);
+                        }
                     } else {
-                        // slot j: weight digit pa (high, low) at 64j + 32pa under scale 2j + pa;
-                        // token digit pb at 64j + 32pb under the slot's scale byte j
-                        mma_mx(acc, dA, db, idesc(0, 0), sfa_t, sfb_t, accum);
-                        mma_mx(acc, dA, db + 2, idesc(0, 0), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, dA + 2, db, idesc(1, 0), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, dA + 2, db + 2, idesc(1, 0), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, dA + 4, db + 4, idesc(2, 1), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, dA + 4, db + 6, idesc(2, 1), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, dA + 6, db + 4, idesc(3, 1), sfa_t, sfb_t, 1u);
-                        mma_mx(acc, dA + 6, db + 6, idesc(3, 1), sfa_t, sfb_t, 1u);
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
+                            uint32_t b2 = 0;
+                            if (lo + h < hi) {
+                                const uint8_t *slot = chunk + slot_offset(p, lo + h);
+                                v0 = *reinterpret_cast<const uint4 *>(slot + 32 * r);
+                                v1 = *reinterpret_cast<const uint4 *>(slot + 32 * r + 16);
+                                const uint32_t Sw = slot[4096 + r];
+                                const bool six = slot_width(p, lo + h) == 6;
+                                b2 = shifted(Sw, six ? 9 : 7) | (shifted(Sw, six ? 5 : 3) << 8);
+                            }
+                            // high digits at K' bytes 64h.., low digits at 64h+32..
+                            d[16 * h + 0] = hi_digit(v0.x);
+                            d[16 * h + 1] = hi_digit(v0.y);
+                            d[16 * h + 2] = hi_digit(v0.z);
+                            d[16 * h + 3] = hi_digit(v0.w);
+                            d[16 * h + 4] = hi_digit(v1.x);
+                            d[16 * h + 5] = hi_digit(v1.y);
+                            d[16 * h + 6] = hi_digit(v1.z);
+                            d[16 * h + 7] = hi_digit(v1.w);
+                            d[16 * h + 8] = lo_digit(v0.x);
+                            d[16 * h + 9] = lo_digit(v0.y);
+                            d[16 * h + 10] = lo_digit(v0.z);
+                            d[16 * h + 11] = lo_digit(v0.w);
+                            d[16 * h + 12] = lo_digit(v1.x);
+                            d[16 * h + 13] = lo_digit(v1.y);
+                            d[16 * h + 14] = lo_digit(v1.z);
+                            d[16 * h + 15] = lo_digit(v1.w);
+                            sfw |= b2 << (16 * h);
+                        }
                     }
-                    mma_commit(&plane_free[w]);  // planes + scale tile free once these MMAs have read them
-                    if (g2 != g) mma_commit(&acc_full[b]);  // this worker's share of the group is issued
+                    // the row's 128 K' bytes into its lane of the quad's A tile (32 columns)
+                    tmem_st32(tmem + a_lane + kACol + 32 * (2 * j + buf), d);
+                    // scale tile: row r = 32 qtr + lane at lane `lane`, column qtr; byte = sf id
+                    *reinterpret_cast<uint32_t *>(sfa_q + buf * 512 + lane * 16 + qtr * 4) = sfw;
+                    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                    fence_async_smem();
+                    fence_before();
                 }
-                __syncwarp();
-                ++qw;
-                first_in_group = g2 != g;
-                if (g2 != g) ++gi;
-                g = g2;
-                st = st2;
+                // the quad's four warps have written the stage (or one of them gave up:
+                // then all four stop here)
+                if (!bar_and(kQuadBar0 + j, 128, ok)) {
+                    stop = true;
+                    break;
+                }
+                if (leader) {
+                    bool go = true;
+                    if (!tok_seen && !from_planes) {
+                        go = mbar_wait(tok_full, 0, abort);  // the token operand is in shared memory
+                        tok_seen = true;
+                    }
+                    const bool first = first_chunk && st == 2 * k;
+                    if (go && first) go = mbar_wait(&acc_empty[b], ((gi >> 1) & 1) ^ 1, abort);
+                    if (go) {
+                        fence_after();
+                        const uint32_t sfa_t = tmem + kSfaCol + 4 * (2 * j + buf);
+                        const uint32_t sfb_t = tmem + kSfbCol + 4 * (2 * j + buf);
+                        tmem_cp_sf(sfa_t, dsfa + 32 * buf);
+                        // token scales: the chunk's tile (planes mode) or the resident one
+                        tmem_cp_sf(sfb_t, from_planes ? desc_sf(su32(slot_base + 2 * kTokBytes)) + 32 * (st - 2 * k)
+                                                      : dsfb + 32 * st);
+                        const uint32_t acc = tmem + kAccCol + kAccCols * (2 * j + b);
+                        const uint32_t aT = tmem + kACol + 32 * (2 * j + buf);
+                        const uint64_t db = from_planes ? desc_sw128(su32(slot_base)) + (uint64_t)((st - 2 * k) * (kTokBytes >> 4))
+                                                        : dB + (uint64_t)(st * (kTokBytes >> 4));
+                        const uint32_t accum = first ? 0u : 1u;
+                        if (st < S.st4) {
+                            // slot q: weight digits at columns 8q.. (K' bytes 32q..), token values at 32q..
+                            mma_mx_t(acc, aT, db, idesc(0, 0), sfa_t, sfb_t, accum);
+                            mma_mx_t(acc, aT + 8, db + 2, idesc(1, 1), sfa_t, sfb_t, 1u);
+                            mma_mx_t(acc, aT + 16, db + 4, idesc(2, 2), sfa_t, sfb_t, 1u);
+                            mma_mx_t(acc, aT + 24, db + 6, idesc(3, 3), sfa_t, sfb_t, 1u);
+                        } else {
+                            // slot h: weight digit pa (high, low) at K' bytes 64h + 32pa under scale
+                            // 2h + pa; token digit pb at 64h + 32pb under the slot's scale byte h
+                            mma_mx_t(acc, aT, db, idesc(0, 0), sfa_t, sfb_t, accum);
+                            mma_mx_t(acc, aT, db + 2, idesc(0, 0), sfa_t, sfb_t, 1u);
+                            mma_mx_t(acc, aT + 8, db, idesc(1, 0), sfa_t, sfb_t, 1u);
+                            mma_mx_t(acc, aT + 8, db + 2, idesc(1, 0), sfa_t, sfb_t, 1u);
+                            mma_mx_t(acc, aT + 16, db + 4, idesc(2, 1), sfa_t, sfb_t, 1u);
+                            mma_mx_t(acc, aT + 16, db + 6, idesc(2, 1), sfa_t, sfb_t, 1u);
+                            mma_mx_t(acc, aT + 24, db + 4, idesc(3, 1), sfa_t, sfb_t, 1u);
+                            mma_mx_t(acc, aT + 24, db + 6, idesc(3, 1), sfa_t, sfb_t, 1u);
+                        }
+                        mma_commit(&a_free[2 * j + buf]);  // A tile + scale tiles free once read
+                        if (st == st_end - 1) mma_commit(&empty_c[s]);  // the slot is free once these MMAs ran
+                        if (last_chunk && st == st_end - 1) mma_commit(&acc_full[b]);  // the quad's share is issued
+                    } else {
+                        ok = false;  // the quad's next barrier stops it
+                    }
+                }
             }
-            if (lane == 0 && qw > 0) drain_wait(&plane_free[w], (qw - 1) & 1);
+            if (stop) break;
         }
+        if (leader && qw > 0) drain_wait(&a_free[2 * j + ((qw - 1) & 1)], ((qw - 1) >> 1) & 1);
     } else {
-        // ------------------------------------------------------------ warps 1-4: token operand (codes), epilogue
+        // ------------------------------------------------------------ warps 1-4: token operand, epilogue
         const int et = threadIdx.x - 32;  // 0..127
+        // codes mode: build the resident token operand (planes mode streams it with the chunks)
         if (!from_planes) {
             // the codes may come from the kernel just before this one
             asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -555,7 +580,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1) gemm_decode_kernel(const __gri
                 uint8_t *dst = off < S.n * kTokBytes ? tok + off : sfb + (off - S.n * kTokBytes);
                 *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
             }
-            named_sync(1, 128);
+            named_sync(kCodesBar, 128);
             for (int it = et; it < (c1 - c0) * a.M; it += 128) {
                 const int s = c0 + it / a.M, t = it % a.M;
                 const int b = slot_width(p, s);
@@ -625,22 +650,26 @@ __global__ void __launch_bounds__(kMaxThreads, 1) gemm_decode_kernel(const __gri
             if (lane == 0) mbar_arrive(tok_full);
         }
 
-        // epilogue: accumulator row (= weight row) 32*quad + lane, columns = tokens;
-        // the workers' partial sums are added in worker order
+        // epilogue: accumulator row (= weight row) 32*qtr + lane, columns = tokens;
+        // the quads' partial sums are added in quad order
         if (a.GS > 1) cluster_wait();
-        const int quad = warp & 3;
-        const int r = 32 * quad + lane;
+        const int qtr = warp & 3;
+        const int r = 32 * qtr + lane;
         int gi = 0;
         for (int g = blockIdx.x; g < a.G; g += gridDim.x, ++gi) {
             const int b = gi & 1;
             if (!warp_wait(&acc_full[b], (gi >> 1) & 1, abort)) break;
             fence_after();
             float out[16];
-            for (int w = 0; w < nw; ++w) {
+            bool first = true;
+            for (int jq = 0; jq < kQuads; ++jq) {
+                // quads holding a chunk of this group: (gi * nchunks + k) % kQuads for k < nq
+                if (((jq - gi * nchunks) % kQuads + kQuads) % kQuads >= nq) continue;
                 uint32_t v[16];
-                tmem_ld16(tmem + ((uint32_t)(32 * quad) << 16) + kAccCols * (kMaxWorkers * b + w), v);
+                tmem_ld16(tmem + ((uint32_t)(32 * qtr) << 16) + kAccCol + kAccCols * (2 * jq + b), v);
 #pragma unroll
-                for (int t = 0; t < 16; ++t) out[t] = w == 0 ? __uint_as_float(v[t]) : out[t] + __uint_as_float(v[t]);
+                for (int t = 0; t < 16; ++t) out[t] = first ? __uint_as_float(v[t]) : out[t] + __uint_as_float(v[t]);
+                first = false;
             }
             fence_before();
             __syncwarp();
@@ -747,7 +776,7 @@ int stage_lo(const Plan &p, int sg) {
 }
 
 struct DecodeShape {
-    int GS, max_mst, grid, workers;
+    int GS, max_mst, most, grid, ring, slot_bytes, w_off;  // most: stages of the largest rank range
     int bound[9];  // slots
     size_t smem;
     bool ok;
@@ -769,44 +798,57 @@ bool split_stages(const Plan &p, int g0, int g1, int parts, int *gb) {
     return true;
 }
 
-size_t smem_bytes(int GS, int max_mst, int workers) {
-    // partial tile + (GS-1) received slices of 128/GS rows
-    const size_t xbytes = GS > 1 ? (size_t)kXBytes + (size_t)(GS - 1) * (kXBytes / GS) : 0;
-    return 1024 + (size_t)workers * (kPlaneBytes + 512) + (size_t)max_mst * (kTokBytes + 512) + xbytes + 512;
-}
-
-DecodeShape shape_for(const Plan &p, int GS, int64_t G, int sms, int g0, int g1) {
+DecodeShape shape_for(const Plan &p, int GS, int64_t G, int sms, int g0, int g1, bool stream_tok) {
     DecodeShape sh = {};
     sh.GS = GS;
     int gb[9];
     if (!split_stages(p, g0, g1, GS, gb)) return sh;
+    int max_copy = 0;
     for (int r = 0; r <= GS; ++r) sh.bound[r] = stage_lo(p, gb[r]);
-    for (int r = 0; r < GS; ++r) sh.max_mst = std::max(sh.max_mst, gb[r + 1] - gb[r]);
-    // as many workers as fit, up to one per stage
-    sh.workers = std::min(kMaxWorkers, sh.max_mst);
-    while (sh.workers > 1 && smem_bytes(GS, sh.max_mst, sh.workers) > 225 * 1024) --sh.workers;
-    sh.smem = std::max<size_t>(kMinSmem, smem_bytes(GS, sh.max_mst, sh.workers));
-    sh.ok = sh.max_mst <= kMaxStages && sh.smem <= 225 * 1024 && sh.workers >= std::min(4, sh.max_mst);
+    for (int r = 0; r < GS; ++r) {
+        sh.max_mst = std::max(sh.max_mst, gb[r + 1] - gb[r]);
+        for (int k = gb[r]; k < gb[r + 1]; k += 2) {  // chunks of two stages
+            const int e = std::min(k + 2, gb[r + 1]);
+            max_copy = std::max(max_copy, (int)(slot_offset(p, stage_lo(p, e)) - slot_offset(p, stage_lo(p, k))));
+        }
+    }
+    // planes mode streams two token tiles and their scale tiles with every chunk;
+    // codes mode keeps the rank's whole token operand resident
+    sh.w_off = stream_tok ? 2 * (kTokBytes + 512) : 0;
+    sh.slot_bytes = (sh.w_off + max_copy + 1023) / 1024 * 1024;
+    const int resident = stream_tok ? 0 : sh.max_mst;
+    // partial tile + (GS-1) received slices of 128/GS rows
+    const size_t xbytes = GS > 1 ? (size_t)kXBytes + (size_t)(GS - 1) * (kXBytes / GS) : 0;
+    const size_t fixed = 1024 + (size_t)resident * (kTokBytes + 512) + (size_t)kQuads * 1024 + xbytes + 512;
+    // The ring holds 8 or 4 chunks: a multiple of kQuads, so that slot s is
+    // only ever used by quad s % kQuads, which consumes its slots strictly in
+    // order.  A slot shared by quads could be polled for its next phase while
+    // its previous chunk is still in flight, and a parity wait would then
+    // pass early.
+    const size_t budget = 225 * 1024;
+    sh.ring = fixed + 8 * (size_t)sh.slot_bytes <= budget ? 8 : (fixed + 4 * (size_t)sh.slot_bytes <= budget ? 4 : 0);
+    sh.smem = std::max<size_t>(kMinSmem, fixed + (size_t)sh.ring * sh.slot_bytes + 16 * (size_t)sh.ring);
+    sh.most = sh.max_mst;
+    if (stream_tok) sh.max_mst = 0;  // no resident token operand
+    sh.ok = sh.ring >= kQuads && sh.smem <= 225 * 1024 + 1024;
     sh.grid = (int)std::min<int64_t>(G, std::max(1, sms / GS));
     return sh;
 }
 
-// Choose the K split.  A CTA's time is about (groups it owns) x (stages a
-// worker owns per group + a fixed cost per group), in units of one worker
-// stage (~2.5 us, the latency of its loads).  In a cluster every group after
-// the first also waits for the previous group's cross-rank exchange, which
-// measured at 8-13 us on GB300 (q/gate/down projections of an 8B model, each
-// cluster size forced in turn), so clusters pay off only when their CTAs own
-// one group each.  Ties go to the smaller cluster.
-DecodeShape pick_shape(const Plan &p, int64_t G, int sms, int g0, int g1) {
+// Choose the K split.  A CTA's time is about (groups it owns) x (copy chunks
+// a quad converts per group + a fixed cost per group).  In a cluster every
+// group after the first also waits for the previous group's cross-rank
+// exchange, which measured at 8-13 us on GB300, so clusters pay off only when
+// their CTAs own one group each.  Ties go to the smaller cluster.
+DecodeShape pick_shape(const Plan &p, int64_t G, int sms, int g0, int g1, bool stream_tok) {
     DecodeShape best = {};
     double best_cost = 1e30;
     for (int GS = 1; GS <= 8 && GS <= g1 - g0; GS *= 2) {
-        const DecodeShape sh = shape_for(p, GS, G, sms, g0, g1);
+        const DecodeShape sh = shape_for(p, GS, G, sms, g0, g1, stream_tok);
         if (!sh.ok) continue;
         const double rounds = (double)((G + sh.grid - 1) / sh.grid);
-        const double cost = rounds * ((sh.max_mst + sh.workers - 1) / sh.workers + 1.0) +
-                            (GS > 1 ? 0.3 + 8.0 * (rounds - 1.0) : 0.0);
+        const int nchunks = (sh.most + 1) / 2;
+        const double cost = rounds * ((nchunks + kQuads - 1) / kQuads + 1.0) + (GS > 1 ? 0.3 + 8.0 * (rounds - 1.0) : 0.0);
         if (cost < best_cost - 1e-9) {
             best_cost = cost;
             best = sh;
@@ -861,7 +903,7 @@ int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, 
         DecodeShape plan[16];
         bool ok = true;
         for (int k = 0; k < passes && ok; ++k) {
-            plan[k] = pick_shape(p, a.G, sm_count(), win[k], win[k + 1]);
+            plan[k] = pick_shape(p, a.G, sm_count(), win[k], win[k + 1], act_planes != nullptr);
             ok = plan[k].ok;
         }
         if (!ok) continue;
@@ -870,14 +912,16 @@ int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, 
             a.GS = sh.GS;
             for (int i = 0; i < 9; ++i) a.bound[i] = i <= sh.GS ? sh.bound[i] : sh.bound[sh.GS];
             a.max_mst = sh.max_mst;
-            a.workers = sh.workers;
+            a.ring = sh.ring;
+            a.slot_bytes = sh.slot_bytes;
+            a.w_off = sh.w_off;
             a.accumulate = k > 0;
             cudaError_t e =
                 cudaFuncSetAttribute(gemm_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh.smem);
             if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(decode smem)");
             cudaLaunchConfig_t cfg = {};
             cfg.gridDim = dim3((unsigned)sh.grid, (unsigned)sh.GS, 1);
-            cfg.blockDim = dim3((unsigned)((kWorkerWarp0 + sh.workers) * 32), 1, 1);
+            cfg.blockDim = dim3(kThreads, 1, 1);
             cfg.dynamicSmemBytes = sh.smem;
             cfg.stream = st;
             cudaLaunchAttribute attr[2];
