@@ -64,9 +64,10 @@ __device__ int g_decode_status;  // sticky MXS_ERR_TIMEOUT, read by mxs_device_s
 
 namespace {
 
-constexpr int kQuads = 4;                                 // worker quads (4 warps each)
-constexpr int kWorkerWarp0 = 5;                           // warps 5..20
-constexpr int kThreads = (kWorkerWarp0 + 4 * kQuads) * 32;  // 672
+constexpr int kQuads = 4;                                         // worker quads
+constexpr int kQuadWarps = 5;                                     // four converters + one MMA issuer
+constexpr int kWorkerWarp0 = 5;                                   // warps 5..24
+constexpr int kThreads = (kWorkerWarp0 + kQuadWarps * kQuads) * 32;  // 800
 constexpr int kTokBytes = 16 * 128;                       // 16 token rows x 128 bytes of K'
 constexpr int kAccCols = 16;                              // one accumulator: 16 token columns
 // tensor-memory columns: quad j's A tiles at kACol + 32 (2j + buf), its
@@ -269,8 +270,12 @@ __device__ __forceinline__ uint32_t hi_nib(uint32_t w) { return ((w >> 4) & 0x07
 // high (|m| >> 4) and low (|m| & 15) digit of four sign-magnitude 8-bit codes
 __device__ __forceinline__ uint32_t hi_digit(uint32_t x) { return ((x >> 4) & 0x07070707u) | (x & 0x80808080u); }
 __device__ __forceinline__ uint32_t lo_digit(uint32_t x) { return x & 0x8F8F8F8Fu; }
-// scale byte carrying the digit's fixed-point weight; 255 (NaN) stays
-__device__ __forceinline__ uint32_t shifted(uint32_t S, uint32_t sh) { return S == 255 ? 255u : min(S + sh, 254u); }
+// four scale bytes carrying their digits' fixed-point weights (shift per byte
+// in `add`), saturating at 254; 255 (NaN) stays
+__device__ __forceinline__ uint32_t shifted4(uint32_t S4, uint32_t add) {
+    const uint32_t t = __vminu4(__vaddus4(S4, add), 0xFEFEFEFEu);
+    return t | __vcmpeq4(S4, 0xFFFFFFFFu);
+}
 
 struct Stages {  // MMA stages of a CTA's K range [c0, c1): 4-bit ones (4 slots), then 6/8-bit ones (2 slots)
     int a4, e4, a8, e8, st4, n;
@@ -420,153 +425,169 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         }
     } else if (warp >= kWorkerWarp0) {
         // ------------------------------------------------------------ worker quads
+        // quad j = warps 5+5j .. 9+5j: four converters (one per tensor-memory lane
+        // quarter) and one MMA issuer; all five meet at the quad's barrier once per stage
         const int wq = warp - kWorkerWarp0;
-        const int j = wq >> 2;                           // quad
-        const int qtr = warp & 3;                        // this warp's tensor-memory lane quarter
-        const int r = 32 * qtr + lane;                   // weight row (within the group) of this thread
-        const bool leader = (wq & 3) == 0 && lane == 0;  // issues the quad's tcgen05 work
+        const int j = wq / kQuadWarps, role = wq % kQuadWarps;  // role 4: the issuer
+        const int qtr = warp & 3;                                // a converter's lane quarter
+        const int r = 32 * qtr + lane;                           // its weight row within the group
         const uint32_t a_lane = (uint32_t)(32 * qtr) << 16;
-        uint8_t *sfa_q = sfa + j * 1024;                 // two 512-byte tiles
+        uint8_t *sfa_q = sfa + j * 1024;  // two 512-byte tiles
         const uint64_t dB = desc_sw128(su32(tok)), dsfa = desc_sf(su32(sfa_q)), dsfb = desc_sf(su32(sfb));
         bool ok = true, tok_seen = false, stop = false;
         uint32_t qw = 0;  // stages this quad has issued (a_free phases)
         for (int qc = j; qc < total && !stop; qc += kQuads) {
             const int gi = qc / nchunks, k = qc - gi * nchunks, b = gi & 1;
             const int s = qc % a.ring;
-            if (ok) ok = warp_wait(&full_c[s], (qc / a.ring) & 1, abort);
+            if (ok && role < 4) ok = warp_wait(&full_c[s], (qc / a.ring) & 1, abort);
+            uint8_t *slot_base = ring + (size_t)s * a.slot_bytes;
             int clo, chi;
             S.range(2 * k, clo, chi);
-            uint8_t *slot_base = ring + (size_t)s * a.slot_bytes;
             const uint8_t *chunk = slot_base + a.w_off - slot_offset(p, clo);  // + slot_offset(slot)
             const bool first_chunk = k < kQuads;           // the quad's first chunk of the group
             const bool last_chunk = k + kQuads >= nchunks;  // ... and its last
             const int st_end = min(2 * k + 2, S.n);
             for (int st = 2 * k; st < st_end; ++st, ++qw) {
                 const int buf = qw & 1;
-                // the A tile and scale tile of this buffer are free once the MMAs of two stages ago ran
-                if (ok && qw >= 2) ok = warp_wait(&a_free[2 * j + buf], ((qw >> 1) - 1) & 1, abort);
-                if (ok) {
-                    int lo, hi;
-                    S.range(st, lo, hi);
-                    uint32_t d[32], sfw = 0;
-                    if (st < S.st4) {
+                if (role < 4) {
+                    // the A tile and scale tile of this buffer are free once the MMAs of two stages ago ran
+                    if (ok && qw >= 2) ok = warp_wait(&a_free[2 * j + buf], ((qw >> 1) - 1) & 1, abort);
+                    if (ok) {
+                        int lo, hi;
+                        S.range(st, lo, hi);
+                        const int nsl = hi - lo;                      // slots present in the stage
+                        const uint8_t *s0 = chunk + slot_offset(p, lo);  // its first slot
+                        uint32_t d[32], sfw;
+                        if (st < S.st4) {
+                            // all loads first: four 16-byte code words and four scale bytes of row r
+                            uint4 v[4];
+                            uint32_t sb = 0;
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            uint4 v = make_uint4(0, 0, 0, 0);
-                            uint32_t sc = 0;
-                            if (lo + q < hi) {
-                                const uint8_t *slot = chunk + slot_offset(p, lo + q);
-                                v = *reinterpret_cast<const uint4 *>(slot + 16 * r);
-                                sc = shifted(slot[2048 + r], 7);
+                            for (int q = 0; q < 4; ++q) {
+                                v[q] = make_uint4(0, 0, 0, 0);
+                                if (q < nsl) {
+                                    v[q] = *reinterpret_cast<const uint4 *>(s0 + 2176 * q + 16 * r);
+                                    sb |= (uint32_t)s0[2176 * q + 2048 + r] << (8 * q);
+                                }
                             }
-                            // word i: bytes hold elements 8i..8i+3 (low nibbles), 8i+4..8i+7 (high nibbles)
-                            d[8 * q + 0] = lo_nib(v.x);
-                            d[8 * q + 1] = hi_nib(v.x);
-                            d[8 * q + 2] = lo_nib(v.y);
-                            d[8 * q + 3] = hi_nib(v.y);
-                            d[8 * q + 4] = lo_nib(v.z);
-                            d[8 * q + 5] = hi_nib(v.z);
-                            d[8 * q + 6] = lo_nib(v.w);
-                            d[8 * q + 7] = hi_nib(v.w);
-                            sfw |= sc << (8 * q);
-                        }
-                    } else {
 #pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
-                            uint32_t b2 = 0;
-                            if (lo + h < hi) {
-                                const uint8_t *slot = chunk + slot_offset(p, lo + h);
-                                v0 = *reinterpret_cast<const uint4 *>(slot + 32 * r);
-                                v1 = *reinterpret_cast<const uint4 *>(slot + 32 * r + 16);
-                                const uint32_t Sw = slot[4096 + r];
-                                const bool six = slot_width(p, lo + h) == 6;
-                                b2 = shifted(Sw, six ? 9 : 7) | (shifted(Sw, six ? 5 : 3) << 8);
+                            for (int q = 0; q < 4; ++q) {
+                                // word i: bytes hold elements 8i..8i+3 (low nibbles), 8i+4..8i+7 (high nibbles)
+                                d[8 * q + 0] = lo_nib(v[q].x);
+                                d[8 * q + 1] = hi_nib(v[q].x);
+                                d[8 * q + 2] = lo_nib(v[q].y);
+                                d[8 * q + 3] = hi_nib(v[q].y);
+                                d[8 * q + 4] = lo_nib(v[q].z);
+                                d[8 * q + 5] = hi_nib(v[q].z);
+                                d[8 * q + 6] = lo_nib(v[q].w);
+                                d[8 * q + 7] = hi_nib(v[q].w);
                             }
-                            // high digits at K' bytes 64h.., low digits at 64h+32..
-                            d[16 * h + 0] = hi_digit(v0.x);
-                            d[16 * h + 1] = hi_digit(v0.y);
-                            d[16 * h + 2] = hi_digit(v0.z);
-                            d[16 * h + 3] = hi_digit(v0.w);
-                            d[16 * h + 4] = hi_digit(v1.x);
-                            d[16 * h + 5] = hi_digit(v1.y);
-                            d[16 * h + 6] = hi_digit(v1.z);
-                            d[16 * h + 7] = hi_digit(v1.w);
-                            d[16 * h + 8] = lo_digit(v0.x);
-                            d[16 * h + 9] = lo_digit(v0.y);
-                            d[16 * h + 10] = lo_digit(v0.z);
-                            d[16 * h + 11] = lo_digit(v0.w);
-                            d[16 * h + 12] = lo_digit(v1.x);
-                            d[16 * h + 13] = lo_digit(v1.y);
-                            d[16 * h + 14] = lo_digit(v1.z);
-                            d[16 * h + 15] = lo_digit(v1.w);
-                            sfw |= b2 << (16 * h);
+                            sfw = shifted4(sb, 0x07070707u);
+                        } else {
+                            uint4 v0[2], v1[2];
+                            uint32_t sb = 0, add = 0;
+#pragma unroll
+                            for (int h = 0; h < 2; ++h) {
+                                v0[h] = v1[h] = make_uint4(0, 0, 0, 0);
+                                if (h < nsl) {
+                                    v0[h] = *reinterpret_cast<const uint4 *>(s0 + 4224 * h + 32 * r);
+                                    v1[h] = *reinterpret_cast<const uint4 *>(s0 + 4224 * h + 32 * r + 16);
+                                    sb |= (uint32_t)s0[4224 * h + 4096 + r] * (0x0101u << (16 * h));
+                                    // byte 2h: the high digit's shift, byte 2h+1: the low digit's
+                                    add |= (slot_width(p, lo + h) == 6 ? 0x0509u : 0x0307u) << (16 * h);
+                                }
+                            }
+#pragma unroll
+                            for (int h = 0; h < 2; ++h) {
+                                // high digits at K' bytes 64h.., low digits at 64h+32..
+                                d[16 * h + 0] = hi_digit(v0[h].x);
+                                d[16 * h + 1] = hi_digit(v0[h].y);
+                                d[16 * h + 2] = hi_digit(v0[h].z);
+                                d[16 * h + 3] = hi_digit(v0[h].w);
+                                d[16 * h + 4] = hi_digit(v1[h].x);
+                                d[16 * h + 5] = hi_digit(v1[h].y);
+                                d[16 * h + 6] = hi_digit(v1[h].z);
+                                d[16 * h + 7] = hi_digit(v1[h].w);
+                                d[16 * h + 8] = lo_digit(v0[h].x);
+                                d[16 * h + 9] = lo_digit(v0[h].y);
+                                d[16 * h + 10] = lo_digit(v0[h].z);
+                                d[16 * h + 11] = lo_digit(v0[h].w);
+                                d[16 * h + 12] = lo_digit(v1[h].x);
+                                d[16 * h + 13] = lo_digit(v1[h].y);
+                                d[16 * h + 14] = lo_digit(v1[h].z);
+                                d[16 * h + 15] = lo_digit(v1[h].w);
+                            }
+                            sfw = shifted4(sb, add);
                         }
+                        // absent slots: zero digits (their scale bytes do not matter)
+                        // the row's 128 K' bytes into its lane of the quad's A tile (32 columns)
+                        tmem_st32(tmem + a_lane + kACol + 32 * (2 * j + buf), d);
+                        // scale tile: row r = 32 qtr + lane at lane `lane`, column qtr; byte = sf id
+                        *reinterpret_cast<uint32_t *>(sfa_q + buf * 512 + lane * 16 + qtr * 4) = sfw;
+                        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                        fence_async_smem();
+                        fence_before();
                     }
-                    // the row's 128 K' bytes into its lane of the quad's A tile (32 columns)
-                    tmem_st32(tmem + a_lane + kACol + 32 * (2 * j + buf), d);
-                    // scale tile: row r = 32 qtr + lane at lane `lane`, column qtr; byte = sf id
-                    *reinterpret_cast<uint32_t *>(sfa_q + buf * 512 + lane * 16 + qtr * 4) = sfw;
-                    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-                    fence_async_smem();
-                    fence_before();
                 }
-                // the quad's four warps have written the stage (or one of them gave up:
-                // then all four stop here)
-                if (!bar_and(kQuadBar0 + j, 128, ok)) {
+                // the quad's converters have written the stage (or a warp gave up: then
+                // all five stop here)
+                if (!bar_and(kQuadBar0 + j, kQuadWarps * 32, ok)) {
                     stop = true;
                     break;
                 }
-                if (leader) {
-                    bool go = true;
-                    if (!tok_seen && !from_planes) {
-                        go = mbar_wait(tok_full, 0, abort);  // the token operand is in shared memory
-                        tok_seen = true;
-                    }
-                    const bool first = first_chunk && st == 2 * k;
-                    if (go && first) go = mbar_wait(&acc_empty[b], ((gi >> 1) & 1) ^ 1, abort);
-                    if (go) {
-                        fence_after();
-                        const uint32_t sfa_t = tmem + kSfaCol + 4 * (2 * j + buf);
-                        const uint32_t sfb_t = tmem + kSfbCol + 4 * (2 * j + buf);
-                        tmem_cp_sf(sfa_t, dsfa + 32 * buf);
-                        // token scales: the chunk's tile (planes mode) or the resident one
-                        tmem_cp_sf(sfb_t, from_planes ? desc_sf(su32(slot_base + 2 * kTokBytes)) + 32 * (st - 2 * k)
-                                                      : dsfb + 32 * st);
-                        const uint32_t acc = tmem + kAccCol + kAccCols * (2 * j + b);
-                        const uint32_t aT = tmem + kACol + 32 * (2 * j + buf);
-                        const uint64_t db = from_planes ? desc_sw128(su32(slot_base)) + (uint64_t)((st - 2 * k) * (kTokBytes >> 4))
-                                                        : dB + (uint64_t)(st * (kTokBytes >> 4));
-                        const uint32_t accum = first ? 0u : 1u;
-                        if (st < S.st4) {
-                            // slot q: weight digits at columns 8q.. (K' bytes 32q..), token values at 32q..
-                            mma_mx_t(acc, aT, db, idesc(0, 0), sfa_t, sfb_t, accum);
-                            mma_mx_t(acc, aT + 8, db + 2, idesc(1, 1), sfa_t, sfb_t, 1u);
-                            mma_mx_t(acc, aT + 16, db + 4, idesc(2, 2), sfa_t, sfb_t, 1u);
-                            mma_mx_t(acc, aT + 24, db + 6, idesc(3, 3), sfa_t, sfb_t, 1u);
-                        } else {
-                            // slot h: weight digit pa (high, low) at K' bytes 64h + 32pa under scale
-                            // 2h + pa; token digit pb at 64h + 32pb under the slot's scale byte h
-                            mma_mx_t(acc, aT, db, idesc(0, 0), sfa_t, sfb_t, accum);
-                            mma_mx_t(acc, aT, db + 2, idesc(0, 0), sfa_t, sfb_t, 1u);
-                            mma_mx_t(acc, aT + 8, db, idesc(1, 0), sfa_t, sfb_t, 1u);
-                            mma_mx_t(acc, aT + 8, db + 2, idesc(1, 0), sfa_t, sfb_t, 1u);
-                            mma_mx_t(acc, aT + 16, db + 4, idesc(2, 1), sfa_t, sfb_t, 1u);
-                            mma_mx_t(acc, aT + 16, db + 6, idesc(2, 1), sfa_t, sfb_t, 1u);
-                            mma_mx_t(acc, aT + 24, db + 4, idesc(3, 1), sfa_t, sfb_t, 1u);
-                            mma_mx_t(acc, aT + 24, db + 6, idesc(3, 1), sfa_t, sfb_t, 1u);
+                if (role == 4) {
+                    if (lane == 0) {
+                        bool go = true;
+                        if (!tok_seen && !from_planes) {
+                            go = mbar_wait(tok_full, 0, abort);  // the resident token operand is built
+                            tok_seen = true;
                         }
-                        mma_commit(&a_free[2 * j + buf]);  // A tile + scale tiles free once read
-                        if (st == st_end - 1) mma_commit(&empty_c[s]);  // the slot is free once these MMAs ran
-                        if (last_chunk && st == st_end - 1) mma_commit(&acc_full[b]);  // the quad's share is issued
-                    } else {
-                        ok = false;  // the quad's next barrier stops it
+                        const bool first = first_chunk && st == 2 * k;
+                        if (go && first) go = mbar_wait(&acc_empty[b], ((gi >> 1) & 1) ^ 1, abort);
+                        if (go) {
+                            fence_after();
+                            const uint32_t sfa_t = tmem + kSfaCol + 4 * (2 * j + buf);
+                            const uint32_t sfb_t = tmem + kSfbCol + 4 * (2 * j + buf);
+                            tmem_cp_sf(sfa_t, dsfa + 32 * buf);
+                            // token scales: the chunk's tile (planes mode) or the resident one
+                            tmem_cp_sf(sfb_t, from_planes ? desc_sf(su32(slot_base + 2 * kTokBytes)) + 32 * (st - 2 * k)
+                                                          : dsfb + 32 * st);
+                            const uint32_t acc = tmem + kAccCol + kAccCols * (2 * j + b);
+                            const uint32_t aT = tmem + kACol + 32 * (2 * j + buf);
+                            const uint64_t db = from_planes
+                                                    ? desc_sw128(su32(slot_base)) + (uint64_t)((st - 2 * k) * (kTokBytes >> 4))
+                                                    : dB + (uint64_t)(st * (kTokBytes >> 4));
+                            const uint32_t accum = first ? 0u : 1u;
+                            if (st < S.st4) {
+                                // slot q: weight digits at columns 8q.. (K' bytes 32q..), token values at 32q..
+                                mma_mx_t(acc, aT, db, idesc(0, 0), sfa_t, sfb_t, accum);
+                                mma_mx_t(acc, aT + 8, db + 2, idesc(1, 1), sfa_t, sfb_t, 1u);
+                                mma_mx_t(acc, aT + 16, db + 4, idesc(2, 2), sfa_t, sfb_t, 1u);
+                                mma_mx_t(acc, aT + 24, db + 6, idesc(3, 3), sfa_t, sfb_t, 1u);
+                            } else {
+                                // slot h: weight digit pa (high, low) at K' bytes 64h + 32pa under scale
+                                // 2h + pa; token digit pb at 64h + 32pb under the slot's scale byte h
+                                mma_mx_t(acc, aT, db, idesc(0, 0), sfa_t, sfb_t, accum);
+                                mma_mx_t(acc, aT, db + 2, idesc(0, 0), sfa_t, sfb_t, 1u);
+                                mma_mx_t(acc, aT + 8, db, idesc(1, 0), sfa_t, sfb_t, 1u);
+                                mma_mx_t(acc, aT + 8, db + 2, idesc(1, 0), sfa_t, sfb_t, 1u);
+                                mma_mx_t(acc, aT + 16, db + 4, idesc(2, 1), sfa_t, sfb_t, 1u);
+                                mma_mx_t(acc, aT + 16, db + 6, idesc(2, 1), sfa_t, sfb_t, 1u);
+                                mma_mx_t(acc, aT + 24, db + 4, idesc(3, 1), sfa_t, sfb_t, 1u);
+                                mma_mx_t(acc, aT + 24, db + 6, idesc(3, 1), sfa_t, sfb_t, 1u);
+                            }
+                            mma_commit(&a_free[2 * j + buf]);  // A tile + scale tiles free once read
+                            if (st == st_end - 1) mma_commit(&empty_c[s]);  // the slot is free once these MMAs ran
+                            if (last_chunk && st == st_end - 1) mma_commit(&acc_full[b]);  // the quad's share is issued
+                        } else {
+                            ok = false;  // the quad's next barrier stops it
+                        }
                     }
+                    ok = __shfl_sync(0xffffffffu, ok, 0);
                 }
             }
-            if (stop) break;
         }
-        if (leader && qw > 0) drain_wait(&a_free[2 * j + ((qw - 1) & 1)], ((qw - 1) >> 1) & 1);
+        if (role == 4 && lane == 0 && qw > 0) drain_wait(&a_free[2 * j + ((qw - 1) & 1)], ((qw - 1) >> 1) & 1);
     } else {
         // ------------------------------------------------------------ warps 1-4: token operand, epilogue
         const int et = threadIdx.x - 32;  // 0..127
