@@ -202,7 +202,10 @@ __device__ __forceinline__ bool bar_and(int id, int n, bool v) {
         : "memory");
     return r != 0;
 }
-__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release;" ::: "memory"); }
+// relaxed: the barrier inits are published by fence.mbarrier_init.release.cluster,
+// and the teardown only needs every rank's arrival (each receive barrier already
+// proves that the copies into it have landed)
+__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory"); }
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire;" ::: "memory"); }
 
 // UMMA shared-memory descriptors (as in the prefill kernel): 128B-swizzled
@@ -386,10 +389,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         if (a.GS > 1) mbar_expect_tx(xfull, (uint32_t)(a.GS - 1) * xslice);  // the first tile's slices
-        // the weights are static (see mxs_linear_decode): fill the ring right away
-        for (int qc = 0; qc < min(a.ring, total); ++qc) issue(qc);
     }
     if (warp == 0) {
+        __syncwarp();
+        // the weights are static (see mxs_linear_decode): fill the ring right away,
+        // one chunk per lane
+        if (lane < min(a.ring, total)) issue(lane);
         __syncwarp();
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)),
                      "r"(kTmemCols)
@@ -407,13 +412,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer: the rest of the chunks
+        if (from_planes) {
+            // the planes may come from the kernel just before this one (programmatic
+            // dependent launch): wait for it before the first token load
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            if (lane < min(a.ring, total)) issue_tok(lane);  // the first chunks' tokens, one per lane
+        }
         if (lane == 0) {
-            if (from_planes) {
-                // the planes may come from the kernel just before this one (programmatic
-                // dependent launch): wait for it before the first token load
-                asm volatile("griddepcontrol.wait;" ::: "memory");
-                for (int qc = 0; qc < min(a.ring, total); ++qc) issue_tok(qc);
-            }
             for (int qc = a.ring; qc < total; ++qc) {
                 const int s = qc % a.ring;
                 if (!mbar_wait(&empty_c[s], ((qc / a.ring) & 1) ^ 1, abort)) break;
