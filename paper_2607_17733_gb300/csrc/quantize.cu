@@ -2,25 +2,32 @@
 //
 // Sec. 4.1 (one mantissa width per 32-element block, widths 4/6/8) and
 // Appendix A.2 (activations of every linear layer are quantized at run time).
-// Two lanes own one 32-element block: each lane issues its two 128-bit loads
-// (16 bf16) together, the block maximum is combined with one xor-shuffle, and
-// every lane writes its half of the packed codes (8 B of nibbles or 16 B of
-// int8), of the e4m3 MMA planes (16 B per digit plane) and of the scale bytes.
-// The grid is two-dimensional -- y walks the rows, x the work slots of a row
-// -- and the work is enumerated in slot (grouped) order, so the writes of a
-// warp are contiguous and the reads are 64-byte runs of one source row.
+// One lane owns one 32-element block: it issues its four 128-bit loads
+// together, finds the block maximum with packed bf16 max instructions, and
+// writes its block's packed codes (16 B of nibbles or 32 B of int8), its e4m3
+// MMA planes (32 B per digit plane) and its scale byte.  The work is
+// enumerated in slot (grouped) order, so a warp writes 32 consecutive slots
+// of one row and the lanes of one K' stage combine their scale bytes into
+// one 32-bit word of the scale tile.  The grid is rows x slots.
 //
 // Arithmetic.  With E the block's shared exponent (S - 127), an element's
-// mantissa is m = clamp(round(y), +-Q_b) where y = x * 2^(b-2-E).  y is a
-// power-of-two scaling of a bf16 value, so it is exact, and a fused
-// multiply-add with C = 1.5 * 2^23 rounds it: fma(x, 2^(b-2-E), C) rounds the
-// exact x * 2^(b-2-E) + C once with unit spacing, to nearest even, so its
-// result is C + RNE(y) (|y| < 2^(b-1) is far inside the +-2^22 where this
-// holds) and its low bits are m in two's complement.  Ties away from zero
-// instead floor |y| + 1/2 with a round-toward-zero addition of 2^23 (|y| +
-// 1/2 is exact wherever its floor is not 0).  The MMA digits come from the
-// same word: lo = m mod 2^sh is read from its low bits, hi = (m - lo) / 2^sh
-// by exact float arithmetic, and both are converted to e4m3 exactly.
+// mantissa is m = clamp(round(y), +-Q_b) where y = x * 2^(b-2-E).
+//  * The clamp is applied to x, two elements per instruction: the bound
+//    Q_b * 2^(E+2-b) is a bf16 value (Q_b has at most 7 significant bits),
+//    so clamped elements scale to exactly +-Q_b and the others are unchanged.
+//  * y is a power-of-two scaling of a bf16 value, so it is exact, and a fused
+//    multiply-add with C = 1.5 * 2^23 rounds it: fma(x, 2^(b-2-E), C) rounds
+//    the exact x * 2^(b-2-E) + C once with unit spacing, to nearest even, so
+//    its result is C + RNE(y) (|y| <= Q_b is far inside the +-2^22 where
+//    this holds) and its low bits are m in two's complement.  Ties away from
+//    zero instead floor |y| + 1/2 with a round-toward-zero addition of 2^23
+//    (|y| + 1/2 is exact wherever its floor is not 0).
+//  * The MMA digits come from the same word: lo = m mod 2^sh is read from its
+//    low bits, hi = (m - lo) / 2^sh by exact float arithmetic, and both are
+//    converted to e4m3 exactly.
+// Blocks whose maximum is below 2^-119 (S < 8) take a slower path: 2^(b-2-E)
+// is then not a normal float, so x is first scaled by 2^8 (exact) and the
+// clamp is done in float.
 #include <algorithm>
 
 #include "common.cuh"
@@ -44,8 +51,33 @@ struct QuantArgs {
 __device__ __forceinline__ uint32_t low_bytes(uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
     return __byte_perm(__byte_perm(a, b, 0x0040), __byte_perm(c, d, 0x0040), 0x5410);
 }
+// max of |a|, |b| per bf16 half, NaN-propagating (the sign bits of the result are not used)
+__device__ __forceinline__ uint32_t bf2_max_abs(uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("max.NaN.xorsign.abs.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
+}
+// two fused multiply-adds (each rounded once, to nearest even) in one instruction
+__device__ __forceinline__ void fma2(float &d0, float &d1, float a0, float a1, float b0, float b1, float c0, float c1) {
+    asm("{\n .reg .b64 a, b, c, d;\n mov.b64 a, {%2, %3};\n mov.b64 b, {%4, %5};\n mov.b64 c, {%6, %7};\n"
+        " fma.rn.f32x2 d, a, b, c;\n mov.b64 {%0, %1}, d;\n}"
+        : "=f"(d0), "=f"(d1)
+        : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+}
+__device__ __forceinline__ void sub2(float &d0, float &d1, float a0, float a1, float b0, float b1) {
+    asm("{\n .reg .b64 a, b, d;\n mov.b64 a, {%2, %3};\n mov.b64 b, {%4, %5};\n"
+        " sub.rn.f32x2 d, a, b;\n mov.b64 {%0, %1}, d;\n}"
+        : "=f"(d0), "=f"(d1)
+        : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+__device__ __forceinline__ uint32_t bf2_clamp(uint32_t w, uint32_t hi, uint32_t lo) {
+    uint32_t r;
+    asm("min.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(w), "r"(hi));
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(r), "r"(lo));
+    return r;
+}
 
-template <bool kRhaz>
+template <bool kCodes, bool kPlanes, bool kRhaz>
 __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_constant__ Plan p,
                                                                    const __grid_constant__ QuantArgs a) {
     // Programmatic dependent launch, both ways: a decode GEMM launched after
@@ -54,14 +86,13 @@ __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_
     // x or still read the output buffers) before touching memory.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    const int lane_in_row = blockIdx.x * blockDim.x + threadIdx.x;
-    const int l = lane_in_row & 1;
-    const int vs = lane_in_row >> 1;
-    const bool in_row = vs < a.V;
 
-    // virtual slot -> real slot (or padding) and its plane / scale-tile position
-    int s = -1, st = 0, q = 0, poff = 0;
-    if (a.planes) {
+    // work slot vs -> real slot (or plane padding), its plane offset and its
+    // scale byte (K' stage st, byte q of the stage's scale word)
+    const int vs = blockIdx.x * blockDim.x + threadIdx.x;
+    if ((vs & ~31) >= a.V) return;  // a warp with no slot of the row (uniform: blockDim.x is a multiple of 32)
+    int s, st = 0, q = 0, poff = 0;
+    if (kPlanes) {
         if (vs < 4 * p.st4) {
             s = vs < p.n4 ? vs : -1;
             st = vs >> 2;
@@ -77,123 +108,171 @@ __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_
     } else {
         s = vs;
     }
+    const bool in_row = vs < a.V;
     const bool live = in_row && s >= 0;
     // padding slots are written as zero digits: one plane in the 4-bit
     // region, two in the 6/8-bit region
     const int b = s >= 0 ? slot_width(p, s) : (vs < 4 * p.st4 ? 4 : 8);
     const float Q = (float)((1 << (b - 1)) - 1);
     const int kb = live ? p.slot_block[s] : 0;
+    // the lane that writes its K' stage's scale word: the first of 4 (4-bit) or 2 (6/8-bit)
+    const bool sf_writer = q == 0;
+    const bool stage4 = st < p.st4;
 
     // a warp lies in one row (blockDim.x is a multiple of 32), so the row
-    // loop is warp-uniform and every lane reaches the shuffle
+    // loop is warp-uniform and every lane reaches the shuffles
     for (int64_t row = (int64_t)blockIdx.y * blockDim.y + threadIdx.y; row < a.M;
          row += (int64_t)gridDim.y * blockDim.y) {
-        uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
+        uint32_t w[16];
         if (live) {
-            const uint4 *src = reinterpret_cast<const uint4 *>(a.x + row * a.ld + kBlock * kb + 16 * l);
-            v0 = __ldg(src);
-            v1 = __ldg(src + 1);
-        }
-        uint32_t w[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-        uint32_t mx = 0;
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.x + row * a.ld + kBlock * kb);
+            const uint4 v0 = __ldg(src), v1 = __ldg(src + 1), v2 = __ldg(src + 2), v3 = __ldg(src + 3);
+            w[0] = v0.x, w[1] = v0.y, w[2] = v0.z, w[3] = v0.w, w[4] = v1.x, w[5] = v1.y, w[6] = v1.z, w[7] = v1.w;
+            w[8] = v2.x, w[9] = v2.y, w[10] = v2.z, w[11] = v2.w, w[12] = v3.x, w[13] = v3.y, w[14] = v3.z,
+            w[15] = v3.w;
+        } else {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) mx = __vmaxu2(mx, w[i] & 0x7FFF7FFFu);
-        mx = max(mx & 0xFFFFu, mx >> 16);
-        mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+            for (int i = 0; i < 16; ++i) w[i] = 0;
+        }
+        uint32_t mx = bf2_max_abs(w[0], w[1]);
+#pragma unroll
+        for (int i = 2; i < 16; ++i) mx = bf2_max_abs(mx, w[i]);
+        mx = max(mx & 0x7FFFu, (mx >> 16) & 0x7FFFu);
         const int S = (int)(mx >> 7);  // E8M0 scale: the exponent field of the block maximum
 
-        if (S == 255) {  // an Inf or NaN in the block: every code is 0
-#pragma unroll
-            for (int i = 0; i < 8; ++i) w[i] = 0;
-        }
-        float xf[16];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            xf[2 * i] = __uint_as_float(w[i] << 16);
-            xf[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-        }
-        int k = 125 + b - S;  // b - 2 - E
-        if (S < 8) {  // 2^k would not be a normal float: move 8 powers of two into x (exact)
-#pragma unroll
-            for (int j = 0; j < 16; ++j) xf[j] *= 256.0f;
-            k -= 8;
-        }
+        // k = b - 2 - E.  Blocks below 2^-119 scale x by 2^8 first (k - 8);
+        // empty blocks (all zero, padding) use k = 0, which codes them as 0.
+        const bool tiny = S < 8 && mx != 0;
+        const int k = mx == 0 ? 0 : (tiny ? 117 + b - S : 125 + b - S);
         const float f = __int_as_float((k + 127) << 23);
-
-        float tf[16];  // C + m
+        // the clamp bound Q * 2^-k (bf16-exact), for x and for 2^8 x; an Inf
+        // or NaN in the block (S = 255) clamps every element to 0
+        const float T = Q * __int_as_float((127 - k) << 23);
+        if (!tiny) {
+            const uint32_t t = S == 255 ? 0u : __float_as_uint(T) >> 16;
+            const uint32_t hi = t | (t << 16), lo = hi | 0x80008000u;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            if (kRhaz) {
-                float r = __fadd_rz(fmaf(fabsf(xf[j]), f, 0.5f), kTwo23);  // 2^23 + floor(|y| + 1/2)
-                r = fminf(r, kTwo23 + Q) - kTwo23;
-                r = __uint_as_float(__float_as_uint(r) | (__float_as_uint(xf[j]) & 0x80000000u));
-                tf[j] = kMagic + r;
-            } else {
-                tf[j] = fminf(fmaxf(fmaf(xf[j], f, kMagic), kMagic - Q), kMagic + Q);
+            for (int i = 0; i < 16; ++i) w[i] = bf2_clamp(w[i], hi, lo);
+        }
+
+        uint4 pl[4];  // 4-bit: plane halves in pl[0..1]; 6/8-bit: hi halves pl[0..1], lo halves pl[2..3]
+        uint4 cd[2];  // codes: 4-bit in cd[0]; 8-bit halves in cd[0..1]
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            float xf[16];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                xf[2 * i] = __uint_as_float(w[8 * h + i] << 16);
+                xf[2 * i + 1] = __uint_as_float(w[8 * h + i] & 0xFFFF0000u);
+            }
+            if (tiny) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) xf[j] = fminf(fmaxf(xf[j] * 256.0f, -T), T);
+            }
+            float tf[16];  // C + m
+#pragma unroll
+            for (int j = 0; j < 16; j += 2) {
+                if (kRhaz) {
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        float r = __fadd_rz(fmaf(fabsf(xf[j + e]), f, 0.5f), kTwo23) - kTwo23;  // floor(|y| + 1/2)
+                        r = __uint_as_float(__float_as_uint(r) | (__float_as_uint(xf[j + e]) & 0x80000000u));
+                        tf[j + e] = kMagic + r;
+                    }
+                } else {
+                    fma2(tf[j], tf[j + 1], xf[j], xf[j + 1], f, f, kMagic, kMagic);
+                }
+            }
+            uint32_t tb[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) tb[j] = __float_as_uint(tf[j]);
+
+            if (kCodes) {
+                if (b == 4) {
+                    uint32_t c[2];
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const uint32_t ev = low_bytes(tb[8 * e], tb[8 * e + 2], tb[8 * e + 4], tb[8 * e + 6]);
+                        const uint32_t od = low_bytes(tb[8 * e + 1], tb[8 * e + 3], tb[8 * e + 5], tb[8 * e + 7]);
+                        c[e] = (ev & 0x0F0F0F0Fu) | ((od << 4) & 0xF0F0F0F0u);
+                    }
+                    if (h == 0) cd[0].x = c[0], cd[0].y = c[1];
+                    else cd[0].z = c[0], cd[0].w = c[1];
+                } else {
+                    cd[h] = make_uint4(low_bytes(tb[0], tb[1], tb[2], tb[3]), low_bytes(tb[4], tb[5], tb[6], tb[7]),
+                                       low_bytes(tb[8], tb[9], tb[10], tb[11]),
+                                       low_bytes(tb[12], tb[13], tb[14], tb[15]));
+                }
+            }
+            if (kPlanes) {
+                if (b == 4) {  // one plane of m / 4
+                    uint32_t c[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        float v0, v1;
+                        fma2(v0, v1, tf[2 * i], tf[2 * i + 1], 0.25f, 0.25f, -0.25f * kMagic, -0.25f * kMagic);
+                        c[i] = e4m3x2(v0, v1);
+                    }
+                    pl[h] = make_uint4(c[0] | (c[1] << 16), c[2] | (c[3] << 16), c[4] | (c[5] << 16),
+                                       c[6] | (c[7] << 16));
+                } else {  // m = 2^sh * hi + lo: planes hi * 2^sh * fl and lo * fl
+                    const uint32_t mask = b == 6 ? 7u : 15u;
+                    const float fl = b == 6 ? 0.0625f : 0.015625f;
+                    uint32_t ch[8], cl[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int j = 2 * i;
+                        const float L0 = __uint_as_float((tb[j] & mask) | 0x4B000000u);  // 2^23 + lo
+                        const float L1 = __uint_as_float((tb[j + 1] & mask) | 0x4B000000u);
+                        float hs0, hs1, ls0, ls1, d0, d1;
+                        fma2(ls0, ls1, L0, L1, fl, fl, -fl * kTwo23, -fl * kTwo23);
+                        sub2(d0, d1, tf[j], tf[j + 1], L0, L1);  // 2^22 + (m - lo), exact
+                        fma2(hs0, hs1, d0, d1, fl, fl, -fl * kTwo22, -fl * kTwo22);
+                        ch[i] = e4m3x2(hs0, hs1);
+                        cl[i] = e4m3x2(ls0, ls1);
+                    }
+                    pl[h] = make_uint4(ch[0] | (ch[1] << 16), ch[2] | (ch[3] << 16), ch[4] | (ch[5] << 16),
+                                       ch[6] | (ch[7] << 16));
+                    pl[2 + h] = make_uint4(cl[0] | (cl[1] << 16), cl[2] | (cl[3] << 16), cl[4] | (cl[5] << 16),
+                                           cl[6] | (cl[7] << 16));
+                }
             }
         }
-        uint32_t tb[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) tb[j] = __float_as_uint(tf[j]);
 
-        if (live && a.codes) {
+        if (kCodes && live) {
             uint8_t *rowp = a.codes + row * p.row_bytes;
             if (b == 4) {
-                uint32_t c[2];
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const uint32_t ev = low_bytes(tb[8 * h], tb[8 * h + 2], tb[8 * h + 4], tb[8 * h + 6]);
-                    const uint32_t od = low_bytes(tb[8 * h + 1], tb[8 * h + 3], tb[8 * h + 5], tb[8 * h + 7]);
-                    c[h] = (ev & 0x0F0F0F0Fu) | ((od << 4) & 0xF0F0F0F0u);
-                }
-                *reinterpret_cast<uint2 *>(rowp + 16 * (int64_t)s + 8 * l) = make_uint2(c[0], c[1]);
+                *reinterpret_cast<uint4 *>(rowp + 16 * (int64_t)s) = cd[0];
             } else {
-                uint4 c;
-                c.x = low_bytes(tb[0], tb[1], tb[2], tb[3]);
-                c.y = low_bytes(tb[4], tb[5], tb[6], tb[7]);
-                c.z = low_bytes(tb[8], tb[9], tb[10], tb[11]);
-                c.w = low_bytes(tb[12], tb[13], tb[14], tb[15]);
-                *reinterpret_cast<uint4 *>(rowp + 16 * (int64_t)p.n4 + 32 * (int64_t)(s - p.n4) + 16 * l) = c;
+                uint4 *dst = reinterpret_cast<uint4 *>(rowp + 16 * (int64_t)p.n4 + 32 * (int64_t)(s - p.n4));
+                dst[0] = cd[0];
+                dst[1] = cd[1];
             }
-            if (l == 0) a.scales[row * p.nb + s] = (uint8_t)S;
+            a.scales[row * p.nb + s] = (uint8_t)S;
         }
-
-        if (in_row && a.planes) {
-            uint8_t *pr = a.planes + row * p.kp + poff + 16 * l;
-            if (b == 4) {  // one plane of m / 4
-                uint32_t c[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    c[i] = e4m3x2(fmaf(tf[2 * i], 0.25f, -0.25f * kMagic), fmaf(tf[2 * i + 1], 0.25f, -0.25f * kMagic));
-                *reinterpret_cast<uint4 *>(pr) =
-                    make_uint4(c[0] | (c[1] << 16), c[2] | (c[3] << 16), c[4] | (c[5] << 16), c[6] | (c[7] << 16));
-            } else {  // m = 2^sh * hi + lo: planes hi * 2^sh * fl and lo * fl
-                const uint32_t mask = b == 6 ? 7u : 15u;
-                const float fl = b == 6 ? 0.0625f : 0.015625f;
-                float hs[16], ls[16];
-#pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    const float L = __uint_as_float((tb[j] & mask) | 0x4B000000u);  // 2^23 + lo
-                    ls[j] = fmaf(L, fl, -fl * kTwo23);
-                    hs[j] = fmaf(tf[j] - L, fl, -fl * kTwo22);  // tf - L = 2^22 + (m - lo), exact
+        if (kPlanes) {
+            // the scale word of a K' stage row: bytes q = 0..3 (4-bit) or
+            // 0..1 then two zero bytes (6/8-bit), from the stage's lanes
+            const uint32_t sb = live ? (uint32_t)S : 0u;
+            const uint32_t s1 = __shfl_down_sync(0xffffffffu, sb, 1);
+            const uint32_t s2 = __shfl_down_sync(0xffffffffu, sb, 2);
+            const uint32_t s3 = __shfl_down_sync(0xffffffffu, sb, 3);
+            if (in_row) {
+                uint4 *pr = reinterpret_cast<uint4 *>(a.planes + row * p.kp + poff);
+                pr[0] = pl[0];
+                pr[1] = pl[1];
+                if (b != 4) {
+                    pr[2] = pl[2];
+                    pr[3] = pl[3];
                 }
-                uint32_t ch[8], cl[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    ch[i] = e4m3x2(hs[2 * i], hs[2 * i + 1]);
-                    cl[i] = e4m3x2(ls[2 * i], ls[2 * i + 1]);
+                if (sf_writer) {
+                    const int64_t tile = row >> 7;
+                    const int r = (int)(row & 127);
+                    const uint32_t word = stage4 ? sb | (s1 << 8) | (s2 << 16) | (s3 << 24) : sb | (s1 << 8);
+                    *reinterpret_cast<uint32_t *>(a.sf + ((tile * p.nst + st) * 32 + (r & 31)) * 16 + 4 * (r >> 5)) =
+                        word;
                 }
-                *reinterpret_cast<uint4 *>(pr) =
-                    make_uint4(ch[0] | (ch[1] << 16), ch[2] | (ch[3] << 16), ch[4] | (ch[5] << 16), ch[6] | (ch[7] << 16));
-                *reinterpret_cast<uint4 *>(pr + 32) =
-                    make_uint4(cl[0] | (cl[1] << 16), cl[2] | (cl[3] << 16), cl[4] | (cl[5] << 16), cl[6] | (cl[7] << 16));
             }
-            // scale tile byte; 6/8-bit stages also clear their unused bytes 2 and 3
-            const int64_t tile = row >> 7;
-            const int r = (int)(row & 127);
-            uint8_t *cell = a.sf + ((tile * p.nst + st) * 32 + (r & 31)) * 16 + 4 * (r >> 5);
-            if (l == 0) cell[q] = s >= 0 ? (uint8_t)S : 0;
-            if (l == 1 && st >= p.st4) cell[q + 2] = 0;
         }
     }
 }
@@ -212,16 +291,15 @@ int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rou
     a.sf = planes ? a.planes + align256(M * p.kp) : nullptr;
     a.V = planes ? 4 * p.st4 + 2 * ((p.n68 + 1) / 2) : p.nb;
     if (M == 0 || a.V == 0) return MXS_OK;
-    // a row's 2V lanes: one CTA of whole warps for short rows (several rows
+    // a row's V lanes: one CTA of whole warps for short rows (several rows
     // to a CTA), else the fewest CTAs of at most 256 threads, evenly filled
-    const int T = 2 * a.V;
     int nx = 1, tx, ry = 1;
-    if (T <= kCtaThreads) {
-        tx = (T + 31) / 32 * 32;
+    if (a.V <= kCtaThreads) {
+        tx = (a.V + 31) / 32 * 32;
         ry = kCtaThreads / tx;
     } else {
-        nx = (T + kCtaThreads - 1) / kCtaThreads;
-        tx = ((T + nx - 1) / nx + 31) / 32 * 32;
+        nx = (a.V + kCtaThreads - 1) / kCtaThreads;
+        tx = ((a.V + nx - 1) / nx + 31) / 32 * 32;
     }
     const int64_t gy = std::min<int64_t>((M + ry - 1) / ry, 65535);
     cudaLaunchConfig_t cfg = {};
@@ -233,8 +311,13 @@ int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rou
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = rounding == MXS_RHAZ ? cudaLaunchKernelEx(&cfg, quantize_act_kernel<true>, p, a)
-                                               : cudaLaunchKernelEx(&cfg, quantize_act_kernel<false>, p, a);
+    using Kernel = void (*)(Plan, QuantArgs);
+    static const Kernel kernels[3][2] = {
+        {quantize_act_kernel<true, false, false>, quantize_act_kernel<true, false, true>},
+        {quantize_act_kernel<false, true, false>, quantize_act_kernel<false, true, true>},
+        {quantize_act_kernel<true, true, false>, quantize_act_kernel<true, true, true>}};
+    const int which = !planes ? 0 : (!codes ? 1 : 2);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kernels[which][rounding == MXS_RHAZ], p, a);
     return cuda_fail(e, "quantize_act_kernel launch");
 }
 

@@ -116,6 +116,22 @@ def test_prefill_shapes_full_size(torch, M, K):
     compare(torch, xb, bits)
 
 
+@pytest.mark.parametrize("M,K", [(1219, 4096), (601, 8192), (153, 17408), (157, 28672), (4871, 1024)])
+@pytest.mark.parametrize("rounding", [mxs.RNE, mxs.RHAZ])
+def test_many_rows_with_special_blocks(torch, M, K, rounding):
+    """Many rows (several CTAs per row and rows per grid column, ragged last
+    scale tile) with Inf/NaN, all-zero, subnormal and tie blocks planted among
+    ordinary ones; odd M also reads strided source rows."""
+    g = I.rng(7, K, M)
+    bits = I.width_map(K // 32, 0.7, 0.2, 0.1, g)
+    xb = I.activations_bf16(M, bits, g, 0.01, student_t=True)
+    xb[1] = 0
+    xb[2, :] = I.f32_to_bf16_bits((np.ldexp(np.float32(1), -133) * (np.arange(K) % 5)).astype(np.float32))
+    xb[M - 1, 7], xb[M - 1, 300] = 0x7F80, 0xFFC1
+    xb[M // 2] = I.f32_to_bf16_bits(np.tile((np.arange(32) - 16 + 0.5).astype(np.float32) * 0.25, K // 32))
+    compare(torch, xb, bits, rounding, ld=K + 64 if M % 2 else None)
+
+
 # ---------------------------------------------------------------- weights
 @pytest.mark.parametrize("N,nb,p", [(16, 4, (0.5, 0.25, 0.25)), (37, 11, (0.6, 0.2, 0.2)),
                                     (200, 128, (0.8, 0.15, 0.05)), (1, 3, (0, 0, 1)), (300, 7, (1, 0, 0))])
