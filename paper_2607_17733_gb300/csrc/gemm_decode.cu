@@ -135,6 +135,17 @@ __device__ __forceinline__ bool poll(uint64_t *bar, uint32_t parity) {
             : "memory");
     return ok != 0;
 }
+// non-blocking test of a phase (try_wait may suspend the thread for a while
+// when the phase is not complete: wrong for a loop that serves two barriers)
+__device__ __forceinline__ bool test_phase(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(su32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
 template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
     if (poll<kCluster>(bar, parity)) return true;
@@ -280,6 +291,23 @@ __device__ __forceinline__ uint32_t shifted4(uint32_t S4, uint32_t add) {
     return t | __vcmpeq4(S4, 0xFFFFFFFFu);
 }
 
+// y[t][n] for the M tokens.  The two cases are separate loops so that the
+// plain store never waits for a read of y (a select between "y + v" and "v"
+// would let the compiler load y for every store); a later K pass adds into
+// the y that the same thread stored in the pass before.
+__device__ __forceinline__ void store_y(const DecodeArgs &a, int n, const float (&v)[16]) {
+    float *col = a.y + n;
+    if (a.accumulate) {
+#pragma unroll
+        for (int t = 0; t < 16; ++t)
+            if (t < a.M) col[(int64_t)t * a.ld_y] += v[t];
+    } else {
+#pragma unroll
+        for (int t = 0; t < 16; ++t)
+            if (t < a.M) col[(int64_t)t * a.ld_y] = v[t];
+    }
+}
+
 struct Stages {  // MMA stages of a CTA's K range [c0, c1): 4-bit ones (4 slots), then 6/8-bit ones (2 slots)
     int a4, e4, a8, e8, st4, n;
     __device__ void init(const Plan &p, int c0, int c1) {
@@ -319,9 +347,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
     float *xout = reinterpret_cast<float *>(sfa + kQuads * 2 * 512);  // [128][16] (GS > 1)
     float *xbuf = xout + (a.GS > 1 ? 128 * 16 : 0);                                 // [GS-1][R][16]
     uint64_t *bars = reinterpret_cast<uint64_t *>(xbuf + (size_t)(a.GS - 1) * R * 16);
-    uint64_t *full_c = bars, *empty_c = full_c + a.ring;
-    uint64_t *a_free = empty_c + a.ring;  // [kQuads][2] tcgen05.commit
-    uint64_t *acc_full = a_free + 2 * kQuads, *acc_empty = acc_full + 2;
+    // a ring slot's weight bytes (full_c / empty_c: the converters have loaded
+    // them) and its token tiles (full_t / empty_t: the MMAs have read them) are
+    // filled and released separately, so the next weights stream in while the
+    // MMAs of the chunk before are still pending
+    uint64_t *full_c = bars, *empty_c = full_c + a.ring, *full_t = empty_c + a.ring, *empty_t = full_t + a.ring;
+    uint64_t *a_free = empty_t + a.ring;  // [kQuads][2] tcgen05.commit
+    uint64_t *a_full = a_free + 2 * kQuads;  // [kQuads][2] the four converter warps
+    uint64_t *acc_full = a_full + 2 * kQuads, *acc_empty = acc_full + 2;
     uint64_t *tok_full = acc_empty + 2;
     uint64_t *xfull = tok_full + 1, *xempty = xfull + 1, *xstage = xempty + 1, *xread = xstage + 1;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(xread + 1);
@@ -354,9 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         const int64_t off = slot_offset(p, lo);
         const uint32_t bytes = (uint32_t)(slot_offset(p, hi2) - off);
         const uint8_t *wg = a.w + (int64_t)((int)blockIdx.x + gi * (int)gridDim.x) * a.GB;
-        const int nst = min(2, S.n - 2 * k);
-        // planes mode: the chunk's token tiles complete on the same barrier (issue_tok)
-        mbar_expect_tx(&full_c[s], bytes + (from_planes ? (uint32_t)nst * (kTokBytes + 512) : 0u));
+        mbar_expect_tx(&full_c[s], bytes);
         bulk_load(ring + (size_t)s * a.slot_bytes + a.w_off, wg + off, bytes, &full_c[s]);
     };
     // planes mode: the token operand of chunk qc's stages, by TMA from the planes
@@ -364,8 +395,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         const int k = qc % nchunks, s = qc % a.ring;
         const int nst = min(2, S.n - 2 * k);
         uint8_t *slot = ring + (size_t)s * a.slot_bytes;
-        for (int i = 0; i < nst; ++i) tma_load_2d(slot + i * kTokBytes, &tok_map, &full_c[s], 128 * (sg0 + 2 * k + i), 0);
-        bulk_load(slot + 2 * kTokBytes, a.tok_sf + (int64_t)(sg0 + 2 * k) * 512, (uint32_t)nst * 512, &full_c[s]);
+        mbar_expect_tx(&full_t[s], (uint32_t)nst * (kTokBytes + 512));
+        for (int i = 0; i < nst; ++i) tma_load_2d(slot + i * kTokBytes, &tok_map, &full_t[s], 128 * (sg0 + 2 * k + i), 0);
+        bulk_load(slot + 2 * kTokBytes, a.tok_sf + (int64_t)(sg0 + 2 * k) * 512, (uint32_t)nst * 512, &full_t[s]);
     };
 
     // the next kernel on the stream may launch now (it waits for this grid
@@ -374,9 +406,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
     if (threadIdx.x == 0) {
         for (int i = 0; i < a.ring; ++i) {
             mbar_init(&full_c[i], 1);
-            mbar_init(&empty_c[i], 1);  // tcgen05.commit after the chunk's MMAs (they read its token tiles)
+            mbar_init(&empty_c[i], 4);  // the quad's four converter warps have loaded the chunk
+            mbar_init(&full_t[i], 1);
+            mbar_init(&empty_t[i], 1);  // tcgen05.commit after the chunk's MMAs
         }
-        for (int i = 0; i < 2 * kQuads; ++i) mbar_init(&a_free[i], 1);
+        for (int i = 0; i < 2 * kQuads; ++i) {
+            mbar_init(&a_free[i], 1);
+            mbar_init(&a_full[i], 4);
+        }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&acc_full[i], nq);  // each quad with a chunk in the group commits once
             mbar_init(&acc_empty[i], 4);  // the four epilogue warps
@@ -418,16 +455,45 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
             asm volatile("griddepcontrol.wait;" ::: "memory");
             if (lane < min(a.ring, total)) issue_tok(lane);  // the first chunks' tokens, one per lane
         }
-        if (lane == 0) {
-            for (int qc = a.ring; qc < total; ++qc) {
-                const int s = qc % a.ring;
-                if (!mbar_wait(&empty_c[s], ((qc / a.ring) & 1) ^ 1, abort)) break;
-                issue(qc);
-                if (from_planes) issue_tok(qc);
+        // Refills.  Bulk copies issued by one thread are served one after
+        // another (about 0.3 us each on GB300, whatever their size), so each
+        // quad's chunks get their own issuing lane: lane j (< 4) sends the
+        // weights of chunks qc = j mod 4 once the quad's converters have loaded
+        // chunk qc - ring, lane 4 + j their token tiles once the MMAs of chunk
+        // qc - ring have run.  The lanes poll in step without blocking; a stall
+        // of kWaitCycles with no lane moving gives up.
+        const int role = lane < 4 ? 0 : (lane < 8 && from_planes ? 1 : 2);  // 0 weights, 1 tokens, 2 idle
+        int nx = a.ring + (lane & 3);  // the next chunk this lane refills
+        if (role == 2) nx = total;
+        long long t0 = clock64();
+        while (__any_sync(0xffffffffu, nx < total)) {
+            bool moved = false;
+            if (nx < total) {
+                const uint32_t par = ((nx / a.ring) & 1) ^ 1;
+                if (role == 0 ? test_phase(&empty_c[nx % a.ring], par) : test_phase(&empty_t[nx % a.ring], par)) {
+                    if (role == 0) issue(nx); else issue_tok(nx);
+                    nx += kQuads;
+                    moved = true;
+                }
             }
-            const int first = total > a.ring ? total - a.ring : 0;
-            for (int qc = first; qc < total; ++qc) drain_wait(&full_c[qc % a.ring], (qc / a.ring) & 1);
+            if (__any_sync(0xffffffffu, moved)) {
+                t0 = clock64();
+            } else if (*abort) {
+                break;
+            } else if (clock64() - t0 > kWaitCycles) {
+                if (lane == 0) {
+                    *abort = 1;
+                    atomicExch(&g_decode_status, MXS_ERR_TIMEOUT);
+                }
+                break;
+            }
         }
+        // copies still in flight land in shared memory before the CTA exits:
+        // each lane waits for the latest chunk of each of its slots (its
+        // residue's last ring / kQuads chunks that exist)
+        if (role != 2)
+            for (int qc = nx - kQuads, n = 0; qc >= 0 && n < a.ring / kQuads; qc -= kQuads, ++n)
+                if (qc < total) drain_wait(role == 0 ? &full_c[qc % a.ring] : &full_t[qc % a.ring], (qc / a.ring) & 1);
     } else if (warp >= kWorkerWarp0) {
         // ------------------------------------------------------------ worker quads
         // quad j = warps 5+5j .. 9+5j: four converters (one per tensor-memory lane
@@ -524,6 +590,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                             }
                             sfw = shifted4(sb, add);
                         }
+                        if (st == st_end - 1) {
+                            // the chunk's last stage is in registers: its weight bytes are free
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&empty_c[s]);
+                        }
                         // absent slots: zero digits (their scale bytes do not matter)
                         // the row's 128 K' bytes into its lane of the quad's A tile (32 columns)
                         tmem_st32(tmem + a_lane + kACol + 32 * (2 * j + buf), d);
@@ -534,16 +605,22 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                         fence_before();
                     }
                 }
-                // the quad's converters have written the stage (or a warp gave up: then
-                // all five stop here)
-                if (!bar_and(kQuadBar0 + j, kQuadWarps * 32, ok)) {
-                    stop = true;
-                    break;
-                }
-                if (role == 4) {
+                if (role < 4) {
+                    // this warp's 32 rows of the stage are in tensor memory: tell the
+                    // issuer, and go on to the next stage without waiting for it
+                    __syncwarp();
+                    if (ok && lane == 0) mbar_arrive(&a_full[2 * j + buf]);
+                    if (!ok) {
+                        stop = true;
+                        break;
+                    }
+                } else {
                     if (lane == 0) {
-                        bool go = true;
-                        if (!tok_seen && !from_planes) {
+                        // the four converter warps have written the stage
+                        bool go = mbar_wait(&a_full[2 * j + buf], (qw >> 1) & 1, abort);
+                        // planes mode: the chunk's token tiles have landed
+                        if (go && from_planes && st == 2 * k) go = mbar_wait(&full_t[s], (qc / a.ring) & 1, abort);
+                        if (go && !tok_seen && !from_planes) {
                             go = mbar_wait(tok_full, 0, abort);  // the resident token operand is built
                             tok_seen = true;
                         }
@@ -582,13 +659,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                                 mma_mx_t(acc, aT + 24, db + 6, idesc(3, 1), sfa_t, sfb_t, 1u);
                             }
                             mma_commit(&a_free[2 * j + buf]);  // A tile + scale tiles free once read
-                            if (st == st_end - 1) mma_commit(&empty_c[s]);  // the slot is free once these MMAs ran
+                            if (from_planes && st == st_end - 1) mma_commit(&empty_t[s]);  // token tiles free once read
                             if (last_chunk && st == st_end - 1) mma_commit(&acc_full[b]);  // the quad's share is issued
                         } else {
-                            ok = false;  // the quad's next barrier stops it
+                            ok = false;
                         }
                     }
                     ok = __shfl_sync(0xffffffffu, ok, 0);
+                    if (!ok) {
+                        stop = true;
+                        break;
+                    }
                 }
             }
         }
@@ -703,14 +784,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
             const bool more = g + (int)gridDim.x < a.G;  // another group follows
             if (a.GS == 1) {
                 const int n = 128 * g + r;
-                if (n < a.N) {
-#pragma unroll
-                    for (int t = 0; t < 16; ++t)
-                        if (t < a.M) {
-                            float *dst = a.y + (int64_t)t * a.ld_y + n;
-                            *dst = a.accumulate ? *dst + out[t] : out[t];  // a later K pass, same thread
-                        }
-                }
+                if (n < a.N) store_y(a, n, out);
                 continue;
             }
             // stage the partial tile once this CTA is done with the previous one and
@@ -753,14 +827,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                     }
                 }
                 const int n = 128 * g + r;
-                if (n < a.N) {
-#pragma unroll
-                    for (int t = 0; t < 16; ++t)
-                        if (t < a.M) {
-                            float *yd = a.y + (int64_t)t * a.ld_y + n;
-                            *yd = a.accumulate ? *yd + sum[t] : sum[t];  // a later K pass, same thread
-                        }
-                }
+                if (n < a.N) store_y(a, n, sum);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(xread);
@@ -853,7 +920,7 @@ DecodeShape shape_for(const Plan &p, int GS, int64_t G, int sms, int g0, int g1,
     // pass early.
     const size_t budget = 225 * 1024;
     sh.ring = fixed + 8 * (size_t)sh.slot_bytes <= budget ? 8 : (fixed + 4 * (size_t)sh.slot_bytes <= budget ? 4 : 0);
-    sh.smem = std::max<size_t>(kMinSmem, fixed + (size_t)sh.ring * sh.slot_bytes + 16 * (size_t)sh.ring);
+    sh.smem = std::max<size_t>(kMinSmem, fixed + (size_t)sh.ring * sh.slot_bytes + 32 * (size_t)sh.ring);
     sh.most = sh.max_mst;
     if (stream_tok) sh.max_mst = 0;  // no resident token operand
     sh.ok = sh.ring >= kQuads && sh.smem <= 225 * 1024 + 1024;
