@@ -24,7 +24,8 @@ struct Plan {
     uint16_t slot_block[kMaxNb];
 };
 
-__host__ __device__ inline int slot_width(const Plan &p, int s) {
+template <class P>
+__host__ __device__ inline int slot_width(const P &p, int s) {
     return s < p.n4 ? 4 : (s < p.n4 + p.n6 ? 6 : 8);
 }
 
@@ -37,7 +38,8 @@ struct WeightOffsets {
     int64_t G, Np, GB, compact, planes, sf, total;
 };
 
-__host__ __device__ inline int64_t slot_offset(const Plan &p, int s) {
+template <class P>
+__host__ __device__ inline int64_t slot_offset(const P &p, int s) {
     return s < p.n4 ? 2176 * (int64_t)s : 2176 * (int64_t)p.n4 + 4224 * (int64_t)(s - p.n4);
 }
 

@@ -308,9 +308,23 @@ __device__ __forceinline__ void store_y(const DecodeArgs &a, int n, const float 
     }
 }
 
+// The counts of the grouping plan that the kernel reads.  The kernel's
+// parameters hold these and the launch arguments side by side (a few hundred
+// bytes): the first reads of a launch miss the constant cache, and the whole
+// plan with its slot table would spread them over 4 KB.
+struct PlanCounts {
+    int nb, n4, n6, n8, n68;
+    int st4, nst;
+    int64_t row_bytes, kp;
+};
+struct DecodeParams {
+    PlanCounts p;
+    DecodeArgs a;
+};
+
 struct Stages {  // MMA stages of a CTA's K range [c0, c1): 4-bit ones (4 slots), then 6/8-bit ones (2 slots)
     int a4, e4, a8, e8, st4, n;
-    __device__ void init(const Plan &p, int c0, int c1) {
+    __device__ void init(const PlanCounts &p, int c0, int c1) {
         a4 = min(c0, p.n4);
         e4 = min(c1, p.n4);
         a8 = max(c0, p.n4);
@@ -329,9 +343,10 @@ struct Stages {  // MMA stages of a CTA's K range [c0, c1): 4-bit ones (4 slots)
     }
 };
 
-__global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_constant__ Plan p,
-                                                                  const __grid_constant__ DecodeArgs a,
+__global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_constant__ DecodeParams dp,
                                                                   const __grid_constant__ CUtensorMap tok_map) {
+    const PlanCounts &p = dp.p;
+    const DecodeArgs &a = dp.a;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t sbase = su32(smem_raw);
     uint8_t *smem = smem_raw + (((sbase + 1023) & ~1023u) - sbase);  // 1024-aligned for the swizzled tiles
@@ -1031,7 +1046,11 @@ int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, 
             }
             cfg.attrs = attr;
             cfg.numAttrs = na;
-            e = cudaLaunchKernelEx(&cfg, gemm_decode_kernel, p, a, map);
+            DecodeParams dp;
+            dp.p.nb = p.nb, dp.p.n4 = p.n4, dp.p.n6 = p.n6, dp.p.n8 = p.n8, dp.p.n68 = p.n68;
+            dp.p.st4 = p.st4, dp.p.nst = p.nst, dp.p.row_bytes = p.row_bytes, dp.p.kp = p.kp;
+            dp.a = a;
+            e = cudaLaunchKernelEx(&cfg, gemm_decode_kernel, dp, map);
             if (e != cudaSuccess) return cuda_fail(e, "gemm_decode_kernel launch");
         }
         return MXS_OK;
