@@ -233,6 +233,57 @@ MXS_API int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits,
                                     int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, int stage,
                                     void *stream);
 
+/* ---------------------------------------------------------------- offline allocation
+ * Calibration that produces the width maps (Alg. 1, Alg. 3, Theorem 1).  Not
+ * on the inference path; run once per model over calibration activations.
+ *
+ * mxs_column_sensitivity -- Alg. 1 (Sec. 3.1): the column sensitivity of a
+ * linear layer is the diagonal of H = X^T X summed over the calibration
+ * samples, s[j] = sum_k X[k][j]^2.  One call adds one batch:
+ *   x        device, bf16 [T, K] row-major with row stride ld_x elements
+ *            (ld_x >= K, a multiple of 8; x 16-byte aligned); T >= 0 rows
+ *   K        a positive multiple of 32 (the layer's input dimension)
+ *   s        device, fp64 [K], 8-byte aligned: s[j] = (accumulate ? s[j] : 0)
+ *            + sum of x[k][j]^2 over the T rows
+ * Deterministic: the result depends on x, T and K only.  Each square of a bf16
+ * is exact; runs of 8 rows are added in fp32 (relative error <= 2^-21 of the
+ * run) unless a run leaves [2^-100, 2^100), in which case it is added in fp64;
+ * the runs are added in fp64.  NaN or Inf in a column makes its s NaN or Inf.
+ * Asynchronous on `stream`; allocates nothing.  Errors: MXS_ERR_SHAPE (T < 0,
+ * K), MXS_ERR_INVALID_ARG (NULL, ld_x), MXS_ERR_ALIGN, MXS_ERR_CUDA. */
+MXS_API int mxs_column_sensitivity(const void *x_bf16, int64_t T, int64_t K, int64_t ld_x, double *s, int accumulate,
+                                   void *stream);
+
+/* mxs_allocation_r -- Theorem 1 (Appendix A): the control parameter R that
+ * makes the triplet allocation average B bits per column over n layers (32
+ * columns per layer at 8 bits, R * S_i * (d_i - 32) at 6, the rest at 4),
+ * before any flooring:
+ *   R = ((B - 4) * sum_i d_i - 4 * 32 * n) / sum_i 2 * S_i * (d_i - 32).
+ * Host only (all arguments host memory): d_in[n] positive multiples of 32,
+ * s_layer[n] the layer sensitivities of Alg. 2 in [0, 1] (an input here).
+ * Errors: MXS_ERR_SHAPE (n, d_in), MXS_ERR_INVALID_ARG (NULL, S outside
+ * [0, 1], no layer with S > 0 and d > 32, or B below the 8-bit floor: R < 0). */
+MXS_API int mxs_allocation_r(int64_t n, const int64_t *d_in, const double *s_layer, double B, double *R);
+
+/* mxs_allocate_layer -- Alg. 3 for one layer with K = d_in columns:
+ *   s      device, fp64 [K] column sensitivities (mxs_column_sensitivity);
+ *          NaN keys give an unspecified order
+ *   perm   device, int32 [K] out: perm[p] = the original column at position p
+ *          of the descending order of s (equal values by column index)
+ *   bits   host, uint8 [K/32] out, written before the call returns: the width
+ *          of each 32-column block of that order -- block 0: 8 bits (the 32
+ *          most sensitive columns), then floor(N6 / 32) blocks of 6 bits (the
+ *          6-bit columns in whole blocks, Sec. 4.1), the rest 4 bits
+ *   n6     host out (may be NULL): N6 = floor(R * s_layer * (K - 32)) clamped
+ *          to [0, K - 32]
+ * K a multiple of 32 in [32, MXS_MAX_K]; R >= 0; s_layer in [0, 1].  The order
+ * is computed on the GPU, asynchronously on `stream` (O(K^2) comparisons).
+ * Applying the order (permuting the layer's weight columns and, upstream, its
+ * input channels) is the caller's.  Errors: MXS_ERR_SHAPE, MXS_ERR_INVALID_ARG,
+ * MXS_ERR_ALIGN (s 8-byte, perm 4-byte aligned), MXS_ERR_CUDA. */
+MXS_API int mxs_allocate_layer(const double *s, int64_t K, double R, double s_layer, int32_t *perm, uint8_t *bits,
+                               int64_t *n6, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

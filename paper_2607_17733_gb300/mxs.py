@@ -26,7 +26,7 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_act_planes_bytes", "mxs_weight_bytes", "mxs_gemm_workspace_bytes",
            "mxs_quantize_act", "mxs_pack_weight", "mxs_gemm", "mxs_gemm_decode",
            "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode",
-           "mxs_linear_decode_noalloc"]
+           "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer"]
 
 _lock = threading.Lock()
 _lib = None
@@ -79,6 +79,13 @@ def lib() -> ctypes.CDLL:
         L.mxs_test_prefill_starve.restype = I
         L.mxs_device_status.argtypes = [ctypes.POINTER(ctypes.c_int), I, P]
         L.mxs_device_status.restype = I
+        D = ctypes.c_double
+        L.mxs_column_sensitivity.argtypes = [P, I64, I64, I64, P, I, P]
+        L.mxs_column_sensitivity.restype = I
+        L.mxs_allocation_r.argtypes = [I64, P, P, D, ctypes.POINTER(D)]
+        L.mxs_allocation_r.restype = I
+        L.mxs_allocate_layer.argtypes = [P, I64, D, D, P, P, ctypes.POINTER(I64), P]
+        L.mxs_allocate_layer.restype = I
         _lib = L
         return L
 
@@ -275,3 +282,39 @@ def device_status(reset: bool = False, stream=None) -> int:
     st = ctypes.c_int(0)
     check(lib().mxs_device_status(ctypes.byref(st), int(reset), _stream(stream)))
     return st.value
+
+
+# ---------------------------------------------------------------- offline allocation
+def column_sensitivity(x, s=None, accumulate: bool = False, stream=None):
+    """Alg. 1: s[j] (fp64, device) = (accumulate ? s[j] : 0) + sum over the rows of x[:, j]^2
+    for a bf16 x [T, K] on the GPU (mxs_column_sensitivity)."""
+    import torch
+    T, K = x.shape
+    if s is None:
+        s = torch.zeros(K, dtype=torch.float64, device=x.device)
+    check(lib().mxs_column_sensitivity(_ptr(x), T, K, x.stride(0), _ptr(s), int(bool(accumulate)), _stream(stream)))
+    return s
+
+
+def allocation_r(d_in, s_layer, B: float) -> float:
+    """Theorem 1: the control parameter R for an average of B bits (host only)."""
+    d = np.ascontiguousarray(np.asarray(d_in, dtype=np.int64))
+    sl = np.ascontiguousarray(np.asarray(s_layer, dtype=np.float64))
+    if d.size != sl.size:
+        raise ValueError("d_in and s_layer differ in length")
+    r = ctypes.c_double()
+    check(lib().mxs_allocation_r(d.size, d.ctypes.data, sl.ctypes.data, float(B), ctypes.byref(r)))
+    return r.value
+
+
+def allocate_layer(s, R: float, s_layer: float, perm=None, stream=None):
+    """Alg. 3 for one layer: (perm [K] int32 on the device, bits [K/32] uint8 on the host, N6)."""
+    import torch
+    K = s.numel()
+    if perm is None:
+        perm = torch.empty(K, dtype=torch.int32, device=s.device)
+    bits = np.zeros(max(K // 32, 1), dtype=np.uint8)
+    n6 = ctypes.c_int64()
+    check(lib().mxs_allocate_layer(_ptr(s), K, float(R), float(s_layer), _ptr(perm), bits.ctypes.data,
+                                   ctypes.byref(n6), _stream(stream)))
+    return perm, bits, n6.value

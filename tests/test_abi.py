@@ -133,3 +133,38 @@ def test_noalloc_rejects_sizes_beyond_its_scratch(L):
     assert rc == 5 and "built-in scratch" in mxs.last_error()
     small = np.full(4, 4, np.uint8)
     assert L.mxs_linear_decode_noalloc(FAKE, 17, 128, 128, small.ctypes.data, 0, FAKE, 16, FAKE, 16, None) == 2
+
+
+def test_allocation_r_runs_on_the_host(L):
+    """Theorem 1's R needs no device: the library against the oracle's closed form."""
+    from oracle import alloc as A
+    d = [4096, 4096, 14336, 1024, 28672]
+    s = [1.0, 0.3, 0.7, 0.05, 0.5]
+    for B in (4.1, 4.5, 5.75):
+        assert abs(mxs.allocation_r(d, s, B) - A.allocation_r(d, s, B)) <= 1e-12 * max(1.0, A.allocation_r(d, s, B))
+
+
+def test_allocation_validation(L):
+    r = ctypes.c_double()
+    d = np.array([4096, 100], np.int64)
+    sl = np.array([0.5, 0.5])
+    assert L.mxs_allocation_r(2, d.ctypes.data, sl.ctypes.data, 4.5, ctypes.byref(r)) == 2
+    d = np.array([4096, 4096], np.int64)
+    sl = np.array([0.5, 1.5])
+    assert L.mxs_allocation_r(2, d.ctypes.data, sl.ctypes.data, 4.5, ctypes.byref(r)) == 1
+    sl = np.array([0.0, 0.0])
+    assert L.mxs_allocation_r(2, d.ctypes.data, sl.ctypes.data, 4.5, ctypes.byref(r)) == 1
+    sl = np.array([0.5, 0.5])
+    assert L.mxs_allocation_r(2, d.ctypes.data, sl.ctypes.data, 4.0, ctypes.byref(r)) == 1
+    assert L.mxs_allocation_r(0, d.ctypes.data, sl.ctypes.data, 4.5, ctypes.byref(r)) == 2
+    # device calls: rejected before any CUDA call
+    fake = ctypes.c_void_p(1 << 20)
+    bits = np.zeros(8, np.uint8)
+    n6 = ctypes.c_int64()
+    assert L.mxs_column_sensitivity(fake, 4, 100, 104, fake, 0, None) == 2
+    assert L.mxs_column_sensitivity(fake, -1, 64, 64, fake, 0, None) == 2
+    assert L.mxs_column_sensitivity(fake, 4, 64, 60, fake, 0, None) == 1
+    assert L.mxs_column_sensitivity(ctypes.c_void_p((1 << 20) + 8), 4, 64, 64, fake, 0, None) == 4
+    assert L.mxs_allocate_layer(fake, 100, 0.5, 0.5, fake, bits.ctypes.data, ctypes.byref(n6), None) == 2
+    assert L.mxs_allocate_layer(fake, 256, -1.0, 0.5, fake, bits.ctypes.data, ctypes.byref(n6), None) == 1
+    assert L.mxs_allocate_layer(fake, 1 << 20, 0.5, 0.5, fake, bits.ctypes.data, ctypes.byref(n6), None) == 2
