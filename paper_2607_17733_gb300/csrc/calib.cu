@@ -8,12 +8,12 @@
 // a cluster split the rows of one strip and add their partial sums in rank
 // order through distributed shared memory, so the result does not depend on
 // timing and no workspace is needed.  A lane loads 16 B (8 columns) of a row;
-// 32 lanes x 8 rows per step keep 32 KB of loads in flight per CTA.  The square
-// of a bf16 value is exact in fp32 unless it under- or overflows, so each lane
-// adds 8 rows of squares per column in fp32 (at most 8 roundings, relative
-// error <= 2^-21) and adds that partial to an fp64 sum; a partial outside
-// [2^-100, 2^100) is recomputed in fp64 from the same 8 values, so tiny and
-// huge activations keep their exact squares.
+// 32 lanes x 16 rows per step keep 64 KB of loads in flight per CTA.  The
+// square of a bf16 value is exact in fp32 unless it under- or overflows, so
+// each lane adds 16 rows of squares per column in fp32 (at most 16 roundings,
+// relative error <= 2^-20) and adds that partial to an fp64 sum; a partial
+// outside [2^-100, 2^100) is read again and added in fp64, so tiny and huge
+// activations keep their exact squares.
 //
 // Column order (Alg. 3): the position of column i is the number of columns
 // with a larger sensitivity, or an equal one and a smaller index (a stable
@@ -30,7 +30,7 @@ namespace {
 constexpr int kStrip = 64;   // columns per CTA
 constexpr int kRanks = 8;    // CTAs per cluster: row ranges of one strip
 constexpr int kCalThreads = 256;
-constexpr int kSteps = 8;    // rows per lane between fp64 additions (8 x 32 rows per step)
+constexpr int kSteps = 16;   // rows per lane between fp64 additions (16 x 32 rows per step)
 
 __device__ __forceinline__ uint32_t map_rank(const void *p, uint32_t rank) {
     uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(p)), r;
@@ -86,14 +86,14 @@ __global__ void __cluster_dims__(1, kRanks, 1) __launch_bounds__(kCalThreads, 2)
         for (int e = 0; e < 8; ++e) {
             if (p[e] >= 0x1p-100f && p[e] < 0x1p100f) {
                 acc[e] += (double)p[e];
-            } else {  // an under- or overflowing square (or only zeros): exact in fp64
+            } else {  // an under- or overflowing square (or only zeros): read the run again, in fp64
                 double q = 0.0;
-#pragma unroll
                 for (int u = 0; u < kSteps; ++u) {
-                    const int h = e >> 1;
-                    const uint32_t w = h == 0 ? v[u].x : (h == 1 ? v[u].y : (h == 2 ? v[u].z : v[u].w));
-                    const double d = (double)__uint_as_float((e & 1) ? (w & 0xFFFF0000u) : (w << 16));
-                    q = fma(d, d, q);
+                    const int64_t rr = row + 32 * u;
+                    if (has && rr < r1) {
+                        const double d = (double)__uint_as_float((uint32_t)__ldg(x + rr * ld + col + e) << 16);
+                        q = fma(d, d, q);
+                    }
                 }
                 acc[e] += q;
             }
