@@ -233,6 +233,25 @@ MXS_API int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits,
                                     int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, int stage,
                                     void *stream);
 
+/* mxs_quantize_act_permuted / mxs_pack_weight_permuted -- the layer's
+ * columns in the order of the allocation (Alg. 3 returns column lists, and the
+ * 32 most sensitive columns form one 8-bit block only once they are placed
+ * together, Sec. 4.1): mxs_quantize_act and mxs_pack_weight of x[:, perm] and
+ * w[:, perm], i.e. position p of the quantized row holds source column
+ * perm[p].  perm: device int32 [K], 16-byte aligned, a permutation of
+ * 0..K-1 (mxs_allocate_layer writes one); values outside [0, K) give
+ * unspecified results (they are clamped, never read outside the row).  The
+ * GEMMs then run unchanged on the outputs: y = x W^T does not depend on the
+ * order of the K terms.  Other arguments, layouts and errors as in
+ * mxs_quantize_act / mxs_pack_weight (plus MXS_ERR_INVALID_ARG for a NULL
+ * perm, MXS_ERR_ALIGN for an unaligned one).  The gather reads 2 bytes per
+ * element (the rows are read through the L1/L2 caches). */
+MXS_API int mxs_quantize_act_permuted(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x, const int32_t *perm,
+                                      const uint8_t *act_bits, int rounding, void *codes, uint8_t *scales,
+                                      void *planes_or_null, void *stream);
+MXS_API int mxs_pack_weight_permuted(const void *w_bf16, int64_t N, int64_t K, int64_t ld_w, const int32_t *perm,
+                                     const uint8_t *w_bits, int rounding, int layout, void *packed, void *stream);
+
 /* ---------------------------------------------------------------- offline allocation
  * Calibration that produces the width maps (Alg. 1, Alg. 3, Theorem 1).  Not
  * on the inference path; run once per model over calibration activations.

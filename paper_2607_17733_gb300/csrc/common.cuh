@@ -104,10 +104,14 @@ int check_device();
 int cuda_fail(cudaError_t e, const char *what);
 
 // kernel launchers (one translation unit each)
+int quantize_act_impl(const void *x, int64_t M, int64_t K, int64_t ld_x, const int32_t *perm, const uint8_t *bits,
+                      int rounding, void *codes, uint8_t *scales, void *planes, void *stream);
+int pack_weight_impl(const void *w, int64_t N, int64_t K, int64_t ld_w, const int32_t *perm, const uint8_t *bits,
+                     int rounding, int layout, void *packed, void *stream);
 int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rounding, void *codes,
-                    uint8_t *scales, void *planes, cudaStream_t st);
+                    uint8_t *scales, void *planes, cudaStream_t st, const int32_t *perm = nullptr);
 int launch_pack_weight(const Plan &p, const void *w, int64_t N, int64_t ld, int rounding, bool planes,
-                       void *packed, cudaStream_t st);
+                       void *packed, cudaStream_t st, const int32_t *perm = nullptr);
 int64_t decode_workspace_bytes(const Plan &p, int64_t M, int64_t N);
 // decode GEMM over packed codes + scales (act_planes NULL) or over the
 // activation MMA planes (codes/scales NULL); pdl: the launch may overlap the

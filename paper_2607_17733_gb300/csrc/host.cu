@@ -158,8 +158,37 @@ int64_t mxs_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K, const uint8_t 
     return M <= 16 ? decode_workspace_bytes(p, M, N) : 0;
 }
 
+int mxs_quantize_act_permuted(const void *x, int64_t M, int64_t K, int64_t ld_x, const int32_t *perm,
+                              const uint8_t *bits, int rounding, void *codes, uint8_t *scales, void *planes,
+                              void *stream) {
+    if (!perm) return fail(MXS_ERR_INVALID_ARG, "perm is NULL");
+    if (!aligned16(perm)) return fail(MXS_ERR_ALIGN, "perm must be 16-byte aligned");
+    return quantize_act_impl(x, M, K, ld_x, perm, bits, rounding, codes, scales, planes, stream);
+}
+
 int mxs_quantize_act(const void *x, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits, int rounding,
                      void *codes, uint8_t *scales, void *planes, void *stream) {
+    return quantize_act_impl(x, M, K, ld_x, nullptr, bits, rounding, codes, scales, planes, stream);
+}
+
+int mxs_pack_weight_permuted(const void *w, int64_t N, int64_t K, int64_t ld_w, const int32_t *perm,
+                             const uint8_t *bits, int rounding, int layout, void *packed, void *stream) {
+    if (!perm) return fail(MXS_ERR_INVALID_ARG, "perm is NULL");
+    if (!aligned16(perm)) return fail(MXS_ERR_ALIGN, "perm must be 16-byte aligned");
+    return pack_weight_impl(w, N, K, ld_w, perm, bits, rounding, layout, packed, stream);
+}
+
+int mxs_pack_weight(const void *w, int64_t N, int64_t K, int64_t ld_w, const uint8_t *bits, int rounding,
+                    int layout, void *packed, void *stream) {
+    return pack_weight_impl(w, N, K, ld_w, nullptr, bits, rounding, layout, packed, stream);
+}
+
+}  // extern "C"
+
+namespace mxs {
+
+int quantize_act_impl(const void *x, int64_t M, int64_t K, int64_t ld_x, const int32_t *perm, const uint8_t *bits,
+                      int rounding, void *codes, uint8_t *scales, void *planes, void *stream) {
     Plan p;
     int rc = build_plan(bits, K, &p);
     if (rc) return rc;
@@ -173,11 +202,11 @@ int mxs_quantize_act(const void *x, int64_t M, int64_t K, int64_t ld_x, const ui
         return fail(MXS_ERR_ALIGN, "x, codes and planes must be 16-byte aligned");
     if (M == 0) return MXS_OK;
     if ((rc = check_device())) return rc;
-    return launch_quantize(p, x, M, ld_x, rounding, codes, scales, planes, static_cast<cudaStream_t>(stream));
+    return launch_quantize(p, x, M, ld_x, rounding, codes, scales, planes, static_cast<cudaStream_t>(stream), perm);
 }
 
-int mxs_pack_weight(const void *w, int64_t N, int64_t K, int64_t ld_w, const uint8_t *bits, int rounding,
-                    int layout, void *packed, void *stream) {
+int pack_weight_impl(const void *w, int64_t N, int64_t K, int64_t ld_w, const int32_t *perm, const uint8_t *bits,
+                     int rounding, int layout, void *packed, void *stream) {
     Plan p;
     int rc = build_plan(bits, K, &p);
     if (rc) return rc;
@@ -191,8 +220,12 @@ int mxs_pack_weight(const void *w, int64_t N, int64_t K, int64_t ld_w, const uin
     if (N == 0) return MXS_OK;
     if ((rc = check_device())) return rc;
     return launch_pack_weight(p, w, N, ld_w, rounding, layout == MXS_W_COMPACT_AND_PLANES, packed,
-                              static_cast<cudaStream_t>(stream));
+                              static_cast<cudaStream_t>(stream), perm);
 }
+
+}  // namespace mxs
+
+extern "C" {
 
 int mxs_gemm_decode(const void *codes, const uint8_t *scales, const void *act_planes, const uint8_t *bits,
                     const void *packed_w, int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, void *ws,

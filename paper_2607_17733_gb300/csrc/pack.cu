@@ -20,6 +20,7 @@ struct PackArgs {
     int rhaz, with_planes;
     uint8_t *out;
     WeightOffsets off;
+    const int32_t *perm;  // column order (Alg. 3): block kb holds columns perm[32 kb ..], or nullptr
 };
 
 __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant__ Plan p,
@@ -32,16 +33,23 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
     const int b = slot_width(p, s);
 
     uint32_t h[32];
-    const uint4 *src = reinterpret_cast<const uint4 *>(a.w + n * a.ld + kBlock * kb);
     uint32_t mag = 0;
+    if (a.perm) {  // the block's 32 columns gathered in the allocation's order
+        const int32_t *pc = a.perm + kBlock * kb;
+        const uint32_t kmax = (uint32_t)(kBlock * p.nb - 1);  // an invalid order reads wrong columns, never outside the row
 #pragma unroll
-    for (int v = 0; v < 4; ++v) {
-        const uint4 u = __ldg(src + v);
-        const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+        for (int i = 0; i < 32; ++i) h[i] = __ldg(a.w + n * a.ld + min((uint32_t)__ldg(pc + i), kmax));
+    } else {
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.w + n * a.ld + kBlock * kb);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            h[8 * v + 2 * i] = w4[i] & 0xFFFF;
-            h[8 * v + 2 * i + 1] = w4[i] >> 16;
+        for (int v = 0; v < 4; ++v) {
+            const uint4 u = __ldg(src + v);
+            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                h[8 * v + 2 * i] = w4[i] & 0xFFFF;
+                h[8 * v + 2 * i + 1] = w4[i] >> 16;
+            }
         }
     }
 #pragma unroll
@@ -124,8 +132,9 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
 }  // namespace
 
 int launch_pack_weight(const Plan &p, const void *w, int64_t N, int64_t ld, int rounding, bool planes,
-                       void *packed, cudaStream_t st) {
+                       void *packed, cudaStream_t st, const int32_t *perm) {
     PackArgs a;
+    a.perm = perm;
     a.w = static_cast<const uint16_t *>(w);
     a.N = N;
     a.ld = ld;

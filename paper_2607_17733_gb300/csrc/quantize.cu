@@ -45,6 +45,7 @@ struct QuantArgs {
     int64_t M, ld;
     int V;  // work slots per row (with plane padding when planes are written)
     uint8_t *codes, *scales, *planes, *sf;
+    const int32_t *perm;  // column order (Alg. 3): block kb holds columns perm[32 kb ..], or nullptr
 };
 
 // low bytes of four words, in order
@@ -77,7 +78,7 @@ __device__ __forceinline__ uint32_t bf2_clamp(uint32_t w, uint32_t hi, uint32_t 
     return r;
 }
 
-template <bool kCodes, bool kPlanes, bool kRhaz>
+template <bool kCodes, bool kPlanes, bool kRhaz, bool kPerm>
 __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_constant__ Plan p,
                                                                    const __grid_constant__ QuantArgs a) {
     // Programmatic dependent launch, both ways: a decode GEMM launched after
@@ -124,7 +125,18 @@ __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_
     for (int64_t row = (int64_t)blockIdx.y * blockDim.y + threadIdx.y; row < a.M;
          row += (int64_t)gridDim.y * blockDim.y) {
         uint32_t w[16];
-        if (live) {
+        if (kPerm && live) {  // the block's 32 columns gathered in the allocation's order
+            const int4 *pc = reinterpret_cast<const int4 *>(a.perm + kBlock * kb);
+            const uint16_t *xr = a.x + row * a.ld;
+            const uint32_t kmax = (uint32_t)(kBlock * p.nb - 1);  // an invalid order reads wrong columns, never outside the row
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int4 c = __ldg(pc + i);
+                w[2 * i] = (uint32_t)__ldg(xr + min((uint32_t)c.x, kmax)) | ((uint32_t)__ldg(xr + min((uint32_t)c.y, kmax)) << 16);
+                w[2 * i + 1] =
+                    (uint32_t)__ldg(xr + min((uint32_t)c.z, kmax)) | ((uint32_t)__ldg(xr + min((uint32_t)c.w, kmax)) << 16);
+            }
+        } else if (live) {
             const uint4 *src = reinterpret_cast<const uint4 *>(a.x + row * a.ld + kBlock * kb);
             const uint4 v0 = __ldg(src), v1 = __ldg(src + 1), v2 = __ldg(src + 2), v3 = __ldg(src + 3);
             w[0] = v0.x, w[1] = v0.y, w[2] = v0.z, w[3] = v0.w, w[4] = v1.x, w[5] = v1.y, w[6] = v1.z, w[7] = v1.w;
@@ -280,8 +292,9 @@ __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_
 }  // namespace
 
 int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rounding, void *codes,
-                    uint8_t *scales, void *planes, cudaStream_t st) {
+                    uint8_t *scales, void *planes, cudaStream_t st, const int32_t *perm) {
     QuantArgs a;
+    a.perm = perm;
     a.x = static_cast<const uint16_t *>(x);
     a.M = M;
     a.ld = ld;
@@ -312,12 +325,15 @@ int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rou
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     using Kernel = void (*)(Plan, QuantArgs);
-    static const Kernel kernels[3][2] = {
-        {quantize_act_kernel<true, false, false>, quantize_act_kernel<true, false, true>},
-        {quantize_act_kernel<false, true, false>, quantize_act_kernel<false, true, true>},
-        {quantize_act_kernel<true, true, false>, quantize_act_kernel<true, true, true>}};
+    static const Kernel kernels[2][3][2] = {
+        {{quantize_act_kernel<true, false, false, false>, quantize_act_kernel<true, false, true, false>},
+         {quantize_act_kernel<false, true, false, false>, quantize_act_kernel<false, true, true, false>},
+         {quantize_act_kernel<true, true, false, false>, quantize_act_kernel<true, true, true, false>}},
+        {{quantize_act_kernel<true, false, false, true>, quantize_act_kernel<true, false, true, true>},
+         {quantize_act_kernel<false, true, false, true>, quantize_act_kernel<false, true, true, true>},
+         {quantize_act_kernel<true, true, false, true>, quantize_act_kernel<true, true, true, true>}}};
     const int which = !planes ? 0 : (!codes ? 1 : 2);
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, kernels[which][rounding == MXS_RHAZ], p, a);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kernels[perm != nullptr][which][rounding == MXS_RHAZ], p, a);
     return cuda_fail(e, "quantize_act_kernel launch");
 }
 

@@ -26,7 +26,8 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_act_planes_bytes", "mxs_weight_bytes", "mxs_gemm_workspace_bytes",
            "mxs_quantize_act", "mxs_pack_weight", "mxs_gemm", "mxs_gemm_decode",
            "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode",
-           "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer"]
+           "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer",
+           "mxs_quantize_act_permuted", "mxs_pack_weight_permuted"]
 
 _lock = threading.Lock()
 _lib = None
@@ -65,6 +66,10 @@ def lib() -> ctypes.CDLL:
         L.mxs_quantize_act.restype = I
         L.mxs_pack_weight.argtypes = [P, I64, I64, I64, P, I, I, P, P]
         L.mxs_pack_weight.restype = I
+        L.mxs_quantize_act_permuted.argtypes = [P, I64, I64, I64, P, P, I, P, P, P, P]
+        L.mxs_quantize_act_permuted.restype = I
+        L.mxs_pack_weight_permuted.argtypes = [P, I64, I64, I64, P, P, I, I, P, P]
+        L.mxs_pack_weight_permuted.restype = I
         L.mxs_gemm.argtypes = [P, P, P, P, P, I, P, I64, I64, I64, P, I64, P, SZ, P]
         L.mxs_gemm.restype = I
         L.mxs_gemm_decode.argtypes = [P, P, P, P, P, I64, I64, I64, P, I64, P, SZ, P]
@@ -116,6 +121,12 @@ class _Bits:
         return self.arr.size
 
 
+def _ld(t) -> int:
+    """Row stride in elements of a 2-D tensor; a single row has no meaningful
+    stride (torch may report anything), so its row length is used."""
+    return int(t.shape[1]) if t.shape[0] <= 1 else int(t.stride(0))
+
+
 def _ptr(t) -> int | None:
     return None if t is None else t.data_ptr()
 
@@ -155,9 +166,10 @@ def gemm_workspace_bytes(M: int, N: int, K: int, bits) -> int:
 
 # ------------------------------------------------------------------ calls
 def quantize_act(x, bits, rounding: int = RNE, codes=None, scales=None, planes=None,
-                 want_codes: bool = True, want_planes: bool = False, stream=None):
+                 want_codes: bool = True, want_planes: bool = False, stream=None, perm=None):
     """x: bf16 [M, K] CUDA tensor (row stride may exceed K).  Returns
-    (codes uint8 [M, row_bytes] | None, scales uint8 [M, K/32] | None, planes uint8 | None)."""
+    (codes uint8 [M, row_bytes] | None, scales uint8 [M, K/32] | None, planes uint8 | None).
+    perm (int32 [K] CUDA tensor): quantize x[:, perm] (mxs_quantize_act_permuted)."""
     import torch
     M, K = x.shape
     b = _Bits(bits)
@@ -166,20 +178,28 @@ def quantize_act(x, bits, rounding: int = RNE, codes=None, scales=None, planes=N
         scales = torch.empty((M, K // 32), dtype=torch.uint8, device=x.device)
     if want_planes and planes is None:
         planes = torch.empty(act_planes_bytes(M, K, b.arr), dtype=torch.uint8, device=x.device)
-    check(lib().mxs_quantize_act(_ptr(x), M, K, x.stride(0), b.ptr, rounding, _ptr(codes), _ptr(scales),
-                                 _ptr(planes), _stream(stream)))
+    if perm is not None:
+        check(lib().mxs_quantize_act_permuted(_ptr(x), M, K, _ld(x), _ptr(perm), b.ptr, rounding, _ptr(codes),
+                                              _ptr(scales), _ptr(planes), _stream(stream)))
+    else:
+        check(lib().mxs_quantize_act(_ptr(x), M, K, _ld(x), b.ptr, rounding, _ptr(codes), _ptr(scales),
+                                     _ptr(planes), _stream(stream)))
     return codes, scales, planes
 
 
-def pack_weight(w, bits, layout: int = W_COMPACT, rounding: int = RNE, out=None, stream=None):
-    """w: bf16 [N, K] CUDA tensor -> packed uint8 buffer."""
+def pack_weight(w, bits, layout: int = W_COMPACT, rounding: int = RNE, out=None, stream=None, perm=None):
+    """w: bf16 [N, K] CUDA tensor -> packed uint8 buffer (of w[:, perm] when perm is given)."""
     import torch
     N, K = w.shape
     b = _Bits(bits)
     if out is None:
         out = torch.empty(weight_bytes(N, K, b.arr, layout), dtype=torch.uint8, device=w.device)
-    check(lib().mxs_pack_weight(_ptr(w), N, K, w.stride(0), b.ptr, rounding, layout, _ptr(out),
-                                _stream(stream)))
+    if perm is not None:
+        check(lib().mxs_pack_weight_permuted(_ptr(w), N, K, _ld(w), _ptr(perm), b.ptr, rounding, layout,
+                                             _ptr(out), _stream(stream)))
+    else:
+        check(lib().mxs_pack_weight(_ptr(w), N, K, _ld(w), b.ptr, rounding, layout, _ptr(out),
+                                    _stream(stream)))
     return out
 
 
@@ -199,7 +219,7 @@ def gemm(codes, scales, planes, bits, packed_w, N: int, w_layout: int = W_COMPAC
         workspace = torch.empty(ws_need, dtype=torch.uint8, device=dev)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     check(lib().mxs_gemm(_ptr(codes), _ptr(scales), _ptr(planes), b.ptr, _ptr(packed_w), w_layout, b.ptr,
-                         M, N, K, _ptr(y), y.stride(0), _ptr(workspace), ws_bytes, _stream(stream)))
+                         M, N, K, _ptr(y), _ld(y), _ptr(workspace), ws_bytes, _stream(stream)))
     return y
 
 
@@ -219,7 +239,7 @@ def gemm_decode(codes, scales, bits, packed_w, N: int, y=None, workspace=None, s
         workspace = torch.empty(ws_need, dtype=torch.uint8, device=packed_w.device)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     check(lib().mxs_gemm_decode(_ptr(codes), _ptr(scales), _ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y),
-                                y.stride(0), _ptr(workspace), ws_bytes, _stream(stream)))
+                                _ld(y), _ptr(workspace), ws_bytes, _stream(stream)))
     return y
 
 
@@ -235,8 +255,8 @@ def linear_decode(x, bits, packed_w, N: int, rounding: int = RNE, y=None, worksp
     if workspace is None:
         workspace = torch.empty(max(act_planes_bytes(M, K, b.arr), 16), dtype=torch.uint8, device=packed_w.device)
     ws_bytes = workspace.numel() * workspace.element_size()
-    check(lib().mxs_linear_decode(_ptr(x), M, K, x.stride(0), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
-                                  y.stride(0), _ptr(workspace), ws_bytes, _stream(stream)))
+    check(lib().mxs_linear_decode(_ptr(x), M, K, _ld(x), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
+                                  _ld(y), _ptr(workspace), ws_bytes, _stream(stream)))
     return y
 
 
@@ -248,8 +268,8 @@ def linear_decode_noalloc(x, bits, packed_w, N: int, rounding: int = RNE, y=None
     M, K = x.shape
     if y is None:
         y = torch.empty((M, N), dtype=torch.float32, device=packed_w.device)
-    check(lib().mxs_linear_decode_noalloc(_ptr(x), M, K, x.stride(0), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
-                                          y.stride(0), _stream(stream)))
+    check(lib().mxs_linear_decode_noalloc(_ptr(x), M, K, _ld(x), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
+                                          _ld(y), _stream(stream)))
     return y
 
 
@@ -261,7 +281,7 @@ def gemm_prefill(planes, bits, packed_w, M: int, N: int, y=None, stream=None):
     K = 32 * len(b)
     if y is None:
         y = torch.empty((M, N), dtype=torch.float32, device=packed_w.device)
-    check(lib().mxs_gemm_prefill(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), y.stride(0),
+    check(lib().mxs_gemm_prefill(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), _ld(y),
                                  _stream(stream)))
     return y
 
@@ -273,7 +293,7 @@ def test_prefill_starve(planes, bits, packed_w, M: int, N: int, stage: int, y=No
     K = 32 * len(b)
     if y is None:
         y = torch.zeros((M, N), dtype=torch.float32, device=packed_w.device)
-    check(lib().mxs_test_prefill_starve(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), y.stride(0),
+    check(lib().mxs_test_prefill_starve(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), _ld(y),
                                         int(stage), _stream(stream)))
     return y
 
@@ -292,7 +312,7 @@ def column_sensitivity(x, s=None, accumulate: bool = False, stream=None):
     T, K = x.shape
     if s is None:
         s = torch.zeros(K, dtype=torch.float64, device=x.device)
-    check(lib().mxs_column_sensitivity(_ptr(x), T, K, x.stride(0), _ptr(s), int(bool(accumulate)), _stream(stream)))
+    check(lib().mxs_column_sensitivity(_ptr(x), T, K, _ld(x), _ptr(s), int(bool(accumulate)), _stream(stream)))
     return s
 
 

@@ -3,14 +3,20 @@
 the block widths exactly, and an end-to-end allocation checked for validity
 against the oracle's sensitivities.
 
-Tolerance of the column sums: a lane adds 8 rows of exact squares in fp32
-(at most 8 roundings of a sum of positive terms: relative error <= 8 * 2^-24
-= 2^-21) and adds the runs in fp64, so every column is within 2^-21 (+ fp64
-noise) of the exact sum; the tests use 1e-6."""
+Tolerance of the column sums: a lane adds 16 rows of exact squares in fp32
+(at most 16 roundings of a sum of positive terms: relative error <= 16 *
+2^-24 = 2^-20 ~ 9.5e-7) and adds the runs in fp64, so every column is within
+2^-20 (+ fp64 noise) of the exact sum; the tests use 1e-6.
+
+The permuted quantizer and packer (the allocation's column order applied on
+the inference path) are compared byte for byte with the oracle's
+quantization of x[:, perm] and w[:, perm], and one layer runs end to end:
+calibration sums, allocation, permuted packing and quantization, GEMM."""
 import numpy as np
 import pytest
 
 from oracle import alloc as A
+from oracle import mxo
 from paper_2607_17733_gb300 import inputs as I
 from paper_2607_17733_gb300 import mxs
 import gpu_util as U
@@ -144,3 +150,97 @@ def test_end_to_end_allocation_is_valid(torch):
             assert set(perm[:32]) == set(A.column_order(ref)[:32])
         maps.append(bits)
     assert A.average_width(maps, d_in) <= 4.5 + 1e-12
+
+
+# ---------------------------------------------------------------- the allocation on the inference path
+
+def _random_perm(torch, K, seed):
+    g = np.random.default_rng(seed)
+    p = g.permutation(K).astype(np.int32)
+    return p, torch.from_numpy(p).cuda()
+
+
+@pytest.mark.parametrize("M,nb,p", [(1, 4, (0.5, 0.25, 0.25)), (7, 37, (0.7, 0.2, 0.1)), (129, 128, (0.8, 0.15, 0.05))])
+@pytest.mark.parametrize("rounding", [mxs.RNE, mxs.RHAZ])
+def test_permuted_quantize_matches_oracle_of_permuted_x(torch, M, nb, p, rounding):
+    """mxs_quantize_act_permuted(x, perm) is byte for byte the quantization of x[:, perm]."""
+    g = I.rng(21, M, nb)
+    bits = I.width_map(nb, *p, g)
+    K = 32 * nb
+    xb = calib_activations(M, K, seed=nb)
+    perm, perm_d = _random_perm(torch, K, seed=M)
+    codes, scales, planes = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits, rounding=rounding, want_planes=True,
+                                             perm=perm_d)
+    torch.cuda.synchronize()
+    a_s, a_c = mxo.quantize_bf16(np.ascontiguousarray(xb[:, perm]), bits, rounding)
+    pc, ps = mxo.pack_act(bits, a_s, a_c)
+    assert np.array_equal(codes.cpu().numpy(), pc) and np.array_equal(scales.cpu().numpy(), ps)
+    pl, sf = mxo.planes(bits, a_s, a_c)
+    kp = pl.shape[1]
+    got = planes.cpu().numpy()
+    assert np.array_equal(got[:M * kp].reshape(M, kp), pl)
+    # scale tiles [tile][stage][i<32][w<4][q<4] = row 128*tile + 32w + i; rows >= M are not written
+    off = (M * kp + 255) // 256 * 256
+    tiles = got[off:off + sf.size].reshape(-1, kp // 128, 32, 4, 4)
+    rows = 128 * np.arange(tiles.shape[0])[:, None, None, None, None] + 32 * np.arange(4)[None, None, None, :, None] \
+        + np.arange(32)[None, None, :, None, None]
+    valid = np.broadcast_to(rows < M, tiles.shape)
+    assert np.array_equal(tiles[valid], sf.reshape(tiles.shape)[valid])
+
+
+@pytest.mark.parametrize("N,nb", [(200, 40), (37, 5)])
+@pytest.mark.parametrize("layout", [mxs.W_COMPACT, mxs.W_COMPACT_AND_PLANES])
+def test_permuted_pack_matches_oracle_of_permuted_w(torch, N, nb, layout):
+    g = I.rng(22, N, nb)
+    bits = I.width_map(nb, 0.6, 0.25, 0.15, g)
+    K = 32 * nb
+    wb = I.normal_bf16((N, K), 0.02, g)
+    perm, perm_d = _random_perm(torch, K, seed=N)
+    got = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits, layout=layout, perm=perm_d)
+    torch.cuda.synchronize()
+    w_s, w_c = mxo.quantize_bf16(np.ascontiguousarray(wb[:, perm]), bits)
+    want = mxo.pack_weight(bits, w_s, w_c, with_planes=layout == mxs.W_COMPACT_AND_PLANES)
+    assert np.array_equal(got.cpu().numpy()[:want.size], want)
+
+
+@pytest.mark.parametrize("M", [1, 16, 256])
+def test_mxsens_layer_end_to_end(torch, M):
+    """The method on one layer: calibration sums (Alg. 1), the allocation (Alg.
+    3, Theorem 1's R at B = 4.5 for this layer alone) giving the column order
+    and block widths, weights packed and activations quantized in that order,
+    and the GEMM (decode for M <= 16, tensor-core prefill above) -- against the
+    oracle computing the same allocation from its own sums and the exact GEMM
+    of the permuted, quantized operands.  The allocation is taken from the GPU
+    and checked valid against the oracle's sums (near-ties may order
+    differently within the sum tolerance); the GEMM is then compared for that
+    allocation."""
+    K, N = 4096, 1024
+    calib = calib_activations(2048, K, seed=77)
+    s = gpu_sensitivity(torch, calib)
+    R = mxs.allocation_r([K], [1.0], 4.5)
+    perm_d, bits, n6 = mxs.allocate_layer(s, R, 1.0)
+    torch.cuda.synchronize()
+    perm = perm_d.cpu().numpy()
+    ref = A.column_sensitivity(calib)
+    ordered = ref[perm]
+    assert np.all(ordered[1:] <= ordered[:-1] * (1 + 2 * REL))
+    _, want_bits, want_n6 = A.allocate_layer(ref, A.allocation_r([K], [1.0], 4.5), 1.0)
+    assert np.array_equal(bits, want_bits) and n6 == want_n6
+
+    g = I.rng(23, M)
+    x = g.standard_normal((M, K)).astype(np.float32)
+    x[:, np.argsort(-ref)[:16]] *= 50.0  # the calibration's outlier channels stay outliers
+    xb = I.f32_to_bf16_bits(x)
+    wb = I.normal_bf16((N, K), 0.02, g)
+    layout = mxs.W_COMPACT if M <= 16 else mxs.W_COMPACT_AND_PLANES
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits, layout=layout, perm=perm_d)
+    _, _, planes = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits, want_codes=False, want_planes=True, perm=perm_d)
+    torch.cuda.synchronize()
+    if M <= 16:
+        y = mxs.gemm_decode(None, None, bits, packed, N, planes=planes, M=M)
+    else:
+        y = mxs.gemm_prefill(planes, bits, packed, M, N)
+    a_s, a_c = mxo.quantize_bf16(np.ascontiguousarray(xb[:, perm]), bits)
+    w_s, w_c = mxo.quantize_bf16(np.ascontiguousarray(wb[:, perm]), bits)
+    yr, abssum = mxo.gemm(bits, a_c, a_s, w_c, w_s)
+    U.check_gemm(y.cpu().numpy(), yr, abssum)
