@@ -252,6 +252,37 @@ MXS_API int mxs_quantize_act_permuted(const void *x_bf16, int64_t M, int64_t K, 
 MXS_API int mxs_pack_weight_permuted(const void *w_bf16, int64_t N, int64_t K, int64_t ld_w, const int32_t *perm,
                                      const uint8_t *w_bits, int rounding, int layout, void *packed, void *stream);
 
+/* ---------------------------------------------------------------- KV cache
+ * The paper quantizes the KV cache too, with a 4-8 bit configuration
+ * (Appendix A.2).  A cache is two code buffers in the activation layout of
+ * mxs_quantize_act: row t holds token t's K (or V) values of all KV heads,
+ * H_kv * D of them, quantized along the row with that cache's width map
+ * (codes [T_max, mxs_act_row_bytes(H_kv * D, bits)], scales [T_max, H_kv*D/32]).
+ * Appending token t is one mxs_quantize_act call of M = 1 row into row t.
+ *
+ * mxs_attention_decode -- one decode step of one sequence over the cached
+ * tokens 0..T-1: for query head h (reading KV head h / (H / H_kv)),
+ *   out[h] = sum_t softmax_t(scale * <q[h], k_t>) * v_t
+ * with k_t, v_t the MXINT element values of the cache (code * 2^(S-127-(b-2))).
+ *   q        device, bf16 [H, D], row-major
+ *   k_*, v_* device code rows and scales as above (code buffers 16-byte
+ *            aligned); k_bits, v_bits host width maps of H_kv * D / 32 entries
+ *   out      device, fp32 [H, D]
+ *   workspace device, mxs_attention_decode_workspace_bytes(T, H, D) bytes,
+ *            16-byte aligned (per-chunk partial sums; overwritten)
+ * D is 64 or 128, H a multiple of H_kv with H / H_kv <= 8, H_kv * D <= 8192,
+ * 1 <= T.  The products and sums are fp32 (the element values are exact in
+ * fp32); chunks of 128 tokens are combined in order, so the result is
+ * deterministic.  A cache block with scale 255 (NaN/Inf when written) makes
+ * the heads that read it NaN.  Asynchronous on `stream`; allocates nothing.
+ * Errors: MXS_ERR_UNSUPPORTED (D), MXS_ERR_SHAPE, MXS_ERR_BITS,
+ * MXS_ERR_INVALID_ARG, MXS_ERR_ALIGN, MXS_ERR_BUFFER, MXS_ERR_CUDA. */
+MXS_API int64_t mxs_attention_decode_workspace_bytes(int64_t T, int64_t H, int64_t D);
+MXS_API int mxs_attention_decode(const void *q_bf16, int64_t H, int64_t H_kv, int64_t D, const void *k_codes,
+                                 const uint8_t *k_scales, const uint8_t *k_bits, const void *v_codes,
+                                 const uint8_t *v_scales, const uint8_t *v_bits, int64_t T, float scale, float *out,
+                                 void *workspace, size_t ws_bytes, void *stream);
+
 /* ---------------------------------------------------------------- offline allocation
  * Calibration that produces the width maps (Alg. 1, Alg. 3, Theorem 1).  Not
  * on the inference path; run once per model over calibration activations.

@@ -27,7 +27,8 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_quantize_act", "mxs_pack_weight", "mxs_gemm", "mxs_gemm_decode",
            "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode",
            "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer",
-           "mxs_quantize_act_permuted", "mxs_pack_weight_permuted"]
+           "mxs_quantize_act_permuted", "mxs_pack_weight_permuted", "mxs_attention_decode_workspace_bytes",
+           "mxs_attention_decode"]
 
 _lock = threading.Lock()
 _lib = None
@@ -91,6 +92,10 @@ def lib() -> ctypes.CDLL:
         L.mxs_allocation_r.restype = I
         L.mxs_allocate_layer.argtypes = [P, I64, D, D, P, P, ctypes.POINTER(I64), P]
         L.mxs_allocate_layer.restype = I
+        L.mxs_attention_decode_workspace_bytes.argtypes = [I64, I64, I64]
+        L.mxs_attention_decode_workspace_bytes.restype = I64
+        L.mxs_attention_decode.argtypes = [P, I64, I64, I64, P, P, P, P, P, P, I64, ctypes.c_float, P, P, SZ, P]
+        L.mxs_attention_decode.restype = I
         _lib = L
         return L
 
@@ -338,3 +343,22 @@ def allocate_layer(s, R: float, s_layer: float, perm=None, stream=None):
     check(lib().mxs_allocate_layer(_ptr(s), K, float(R), float(s_layer), _ptr(perm), bits.ctypes.data,
                                    ctypes.byref(n6), _stream(stream)))
     return perm, bits, n6.value
+
+
+# ---------------------------------------------------------------- KV cache
+def attention_decode(q, H_kv: int, k_codes, k_scales, k_bits, v_codes, v_scales, v_bits, T: int, scale: float,
+                     out=None, workspace=None, stream=None):
+    """One decode step over an MXINT KV cache (mxs_attention_decode).  q: bf16 [H, D];
+    the caches as written by quantize_act (codes [T_max, row bytes], scales [T_max, nb])."""
+    import torch
+    H, D = q.shape
+    kb, vb = _Bits(k_bits), _Bits(v_bits)
+    if out is None:
+        out = torch.empty((H, D), dtype=torch.float32, device=q.device)
+    need = _size(lib().mxs_attention_decode_workspace_bytes(T, H, D))
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=q.device)
+    check(lib().mxs_attention_decode(_ptr(q), H, H_kv, D, _ptr(k_codes), _ptr(k_scales), kb.ptr, _ptr(v_codes),
+                                     _ptr(v_scales), vb.ptr, T, float(scale), _ptr(out), _ptr(workspace),
+                                     workspace.numel() * workspace.element_size(), _stream(stream)))
+    return out
