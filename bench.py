@@ -20,6 +20,7 @@ on a bounded sample of the same workload, on the host cores.
 from __future__ import annotations
 
 import argparse
+import math
 import json
 import os
 import statistics
@@ -52,7 +53,8 @@ def parse():
     ap.add_argument("--layers", type=int, default=None,
                     help="decoder layers per step (default 32 for decode, 8 for prefill)")
     ap.add_argument("--workload", default="llama3-8b-decode",
-                    choices=["llama3-8b-decode", "llama3-8b-prefill", "llama3-8b-calibration"])
+                    choices=["llama3-8b-decode", "llama3-8b-prefill", "llama3-8b-calibration",
+                             "llama3-8b-decode-attention"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="fused", choices=["planes", "fused", "codes"],
                     help="decode activation path: quantize all projections to MMA planes, then the GEMMs "
@@ -725,6 +727,151 @@ def run_calibration(args):
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": len(xs) * args.steps, "clocks": clocks}), flush=True)
 
 
+ATTN_T, ATTN_H, ATTN_HKV, ATTN_D = 4096, 32, 8, 128
+
+
+def run_attention(args):
+    """Decode attention over an MXINT KV cache (the paper's KV quantization,
+    4-8 bit configuration): one step = one decode token of one sequence through
+    the attention of `layers` LLaMA-3-8B-shaped layers (default 32) with
+    4096 cached tokens (32 query heads, 8 KV heads of 128 dims).  Each layer's
+    K and V caches are quantized rows of 1024 values with one 8-bit block
+    (the most sensitive 32 columns) and 31 4-bit blocks.  Metric: GB/s of
+    cache bytes read (codes + scales; HBM-bound), the step captured in a CUDA
+    graph."""
+    import torch
+
+    ws, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_17733_gb300 import build as B
+    from paper_2607_17733_gb300 import mxs
+    if not os.path.exists(mxs.LIB_PATH):
+        B.build()
+    mxs.lib()
+    L = args.layers or 32
+    T, H, Hkv, D = ATTN_T, ATTN_H, ATTN_HKV, ATTN_D
+    K = Hkv * D
+    gen = torch.Generator(device=dev)
+    layers = []
+    for l in range(L):
+        g = I.rng(SEED, rank, 9, l)
+        kb = np.full(K // 32, 4, np.uint8)
+        kb[g.integers(K // 32)] = 8
+        vb = np.full(K // 32, 4, np.uint8)
+        vb[g.integers(K // 32)] = 8
+        gen.manual_seed(SEED * 19 + rank * 10_007 + l)
+        kx = torch.randn((T, K), generator=gen, device=dev, dtype=torch.float32)
+        kx[:, torch.randperm(K, generator=gen, device=dev)[: K // 100]] *= 20.0
+        vx = torch.randn((T, K), generator=gen, device=dev, dtype=torch.float32)
+        kc, ks, _ = mxs.quantize_act(kx.to(torch.bfloat16), kb)
+        vc, vs, _ = mxs.quantize_act(vx.to(torch.bfloat16), vb)
+        del kx, vx
+        q = torch.randn((H, D), generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
+        out = torch.empty((H, D), dtype=torch.float32, device=dev)
+        wsb = torch.empty(mxs.lib().mxs_attention_decode_workspace_bytes(T, H, D), dtype=torch.uint8, device=dev)
+        layers.append((q, kc, ks, kb, vc, vs, vb, out, wsb))
+    torch.cuda.synchronize()
+    step_bytes = sum(t.numel() for (_, kc, ks, _, vc, vs, _, _, _) in layers for t in (kc, ks, vc, vs)) \
+        + sum(q.numel() * 2 + o.numel() * 4 for (q, *_rest, o, _w) in layers)
+    scale = 1.0 / math.sqrt(D)
+
+    def fn():
+        for q, kc, ks, kb, vc, vs, vb, out, wsb in layers:
+            mxs.attention_decode(q, Hkv, kc, ks, kb, vc, vs, vb, T, scale, out=out, workspace=wsb)
+
+    if args.eager:
+        for _ in range(args.warmup + args.steps):
+            fn()
+        torch.cuda.synchronize()
+        if rank == 0:
+            print(json.dumps({"eager_steps": args.steps, "launches_per_step": 2 * L}), flush=True)
+        return
+    st = torch.cuda.Stream(device=dev)
+    st.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(st):
+        fn()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=st):
+        fn()
+    for _ in range(max(args.warmup, 3)):
+        graph.replay()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(None)
+    barrier(ws)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.1)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(args.steps):
+        graph.replay()
+    t1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = allreduce_max(t0.elapsed_time(t1) / args.steps, ws)
+    value = ws * step_bytes / (ms * 1e-3) / 1e9
+    pk = peaks()
+
+    # end to end: the step's queries from pinned host memory, the outputs back
+    q_host = [q.cpu().pin_memory() for (q, *_r) in layers]
+    o_host = [torch.empty((H, D), dtype=torch.float32).pin_memory() for _ in layers]
+    barrier(ws)
+    torch.cuda.synchronize()
+    e2e_steps = max(1, min(args.steps, 20))
+    t0.record()
+    for _ in range(e2e_steps):
+        for (q, kc, ks, kb, vc, vs, vb, out, wsb), qh, oh in zip(layers, q_host, o_host):
+            q.copy_(qh, non_blocking=True)
+            mxs.attention_decode(q, Hkv, kc, ks, kb, vc, vs, vb, T, scale, out=out, workspace=wsb)
+            oh.copy_(out, non_blocking=True)
+    t1.record()
+    torch.cuda.synchronize()
+    e2e_ms = allreduce_max(t0.elapsed_time(t1) / e2e_steps, ws)
+    e2e = {"value": ws * step_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s", "h2d_bytes_per_step": L * H * D * 2,
+           "d2h_bytes_per_step": L * H * D * 4, "ms_per_step": e2e_ms}
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        from oracle import attention as AT
+        from oracle import mxo
+        q, kc, ks, kb, vc, vs, vb, _, _ = layers[0]
+        kx = torch.randn((T, K), generator=gen.manual_seed(SEED * 19 + rank * 10_007), device=dev).to(torch.bfloat16)
+        kbits = kx.cpu().view(torch.int16).numpy().view(np.uint16)
+        vbits = torch.randn((T, K), device=dev).to(torch.bfloat16).cpu().view(torch.int16).numpy().view(np.uint16)
+        qv = q.float().cpu().numpy().astype(np.float64)
+        kd = AT.dequantized_cache(kbits, kb)
+        vd = AT.dequantized_cache(vbits, vb)
+        lb = sum(t.numel() for t in (kc, ks, vc, vs))
+        nbytes, t_start, passes = 0, time.perf_counter(), 0
+        while True:
+            AT.attention(qv, kd, vd, Hkv, scale)
+            nbytes += lb
+            passes += 1
+            if time.perf_counter() - t_start >= 10.0:
+                break
+        dt = time.perf_counter() - t_start
+        cpu = {"value": nbytes / dt / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+               "sample": f"one layer's attention over 4096 dequantized cached tokens, {passes} pass(es) "
+                         "(cache dequantized once, not timed): numpy fp64", "seconds": dt}
+    if rank == 0:
+        print(json.dumps({
+            "metric": "mxint_kv_attention_gbps", "value": value, "unit": "GB/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "MXINT codes in, f32 math",
+            "data": "synthetic (seeded; keys N(0,1) with 1% of channels x20, values N(0,1))",
+            "config": {"workload": "llama3-8b-decode-attention", "context_tokens": T, "layers": L,
+                       "heads": H, "kv_heads": Hkv, "head_dim": D, "kv_map": "1 x 8-bit + 31 x 4-bit blocks",
+                       "l2": f"inputs larger than L2 ({step_bytes / 1e9:.3f} GB of cache per step)"},
+            "roofline": {"kernel": "attention_chunk_kernel + attention_combine_kernel", "bound": "hbm",
+                         "achieved": step_bytes / (ms * 1e-3) / 1e9, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                         "frac": step_bytes / (ms * 1e-3) / 1e9 / pk["hbm_gbs"], "peak_source": pk["source"],
+                         "traffic": None},
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": 2 * L * args.steps, "clocks": clocks}), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -733,6 +880,8 @@ def main():
         run_prefill(args)
     elif args.workload == "llama3-8b-calibration":
         run_calibration(args)
+    elif args.workload == "llama3-8b-decode-attention":
+        run_attention(args)
     else:
         if args.layers is None:
             args.layers = 32
