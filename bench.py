@@ -56,10 +56,12 @@ def parse():
                     choices=["llama3-8b-decode", "llama3-8b-prefill", "llama3-8b-calibration",
                              "llama3-8b-decode-attention"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--path", default="fused", choices=["planes", "fused", "codes"],
+    ap.add_argument("--path", default="fused", choices=["planes", "fused", "codes", "grouped"],
                     help="decode activation path: quantize all projections to MMA planes, then the GEMMs "
                          "(planes); mxs_linear_decode per projection, the GEMM a programmatic dependent of "
-                         "its quantizer (fused); quantize to packed codes, GEMM over the codes (codes)")
+                         "its quantizer (fused); quantize to packed codes, GEMM over the codes (codes); as fused, "
+                         "but the projections that share an input in a decoder layer (q/k/v, gate/up) in one "
+                         "grouped GEMM launch (grouped)")
     ap.add_argument("--eager", action="store_true",
                     help="launch the step's kernels directly (no CUDA graph, no events): for ncu runs")
     return ap.parse_args()
@@ -332,6 +334,9 @@ def run_ours(args):
     else:  # the timed segment is quantize + GEMM: bf16 activations in, y out
         gemm_bytes = step_bytes
     launches_per_step = 2 * len(items)
+    STAGES = [[0, 1, 2], [3], [4, 5], [6]]  # q k v | o | gate up | down: the projections of a stage share an input
+    if args.path == "grouped":
+        launches_per_step = len(items) + len(items) // 7 * len(STAGES)
 
     # ---- the step as one CUDA graph.  Inputs are independent synthetic draws, so
     # for each M the graph runs all activation quantizations, then all GEMMs;
@@ -344,7 +349,7 @@ def run_ours(args):
     def make_step(events=None):
         def fn():
             for gi, grp in enumerate(groups):
-                if args.path != "fused":
+                if args.path not in ("fused", "grouped"):
                     for M, lin, x, bufs in grp:
                         if args.path == "codes":
                             lin.quantize(x, bufs)
@@ -353,7 +358,17 @@ def run_ours(args):
                                              want_codes=False, want_planes=True)
                 if events is not None:
                     events[gi][0].record()
-                for M, lin, x, bufs in grp:
+                if args.path == "grouped":
+                    for base in range(0, len(grp), 7):
+                        for stage in STAGES:
+                            its = [grp[base + i] for i in stage]
+                            if len(its) == 1:
+                                M, lin, x, bufs = its[0]
+                                lin.fused(x, bufs["y"], bufs["planes"])
+                            else:
+                                mxs.linear_decode_group([(x, lin.bits, lin.packed, lin.N, bufs["y"], bufs["planes"])
+                                                         for M, lin, x, bufs in its])
+                for M, lin, x, bufs in (grp if args.path != "grouped" else []):
                     if args.path == "codes":
                         lin.matmul(bufs)
                     elif args.path == "planes":
@@ -471,6 +486,8 @@ def run_ours(args):
             "config": {"workload": "llama3-8b-decode", "M": list(DECODE_MS), "layers": L,
                        "path": {"planes": "quantize to MMA planes, then GEMM over the planes (TMA)",
                                 "fused": "mxs_linear_decode: quantize + GEMM chained by programmatic dependent launch",
+                                "grouped": "mxs_linear_decode_group for q/k/v and gate/up (one GEMM launch per "
+                                           "group, the quantizers chained before it), mxs_linear_decode for o, down",
                                 "codes": "quantize to packed codes, GEMM over the codes"}[args.path],
                        "projections": [p[0] for p in I.LLAMA3_8B], "map_4_6_8": list(MAP),
                        "parallelism": f"replicas x{ws}", "l2": "inputs larger than L2 (packed weights "

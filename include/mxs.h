@@ -252,6 +252,33 @@ MXS_API int mxs_quantize_act_permuted(const void *x_bf16, int64_t M, int64_t K, 
 MXS_API int mxs_pack_weight_permuted(const void *w_bf16, int64_t N, int64_t K, int64_t ld_w, const int32_t *perm,
                                      const uint8_t *w_bits, int rounding, int layout, void *packed, void *stream);
 
+/* mxs_linear_decode_group -- up to three decode layers in one launch: the
+ * projections of a decoder layer that share an input (q, k and v; gate and
+ * up) each run exactly as mxs_linear_decode (own activations, width map,
+ * weights, output and planes workspace), but their GEMMs are one kernel
+ * launch: the set-up, the wait for the activations and the teardown are paid
+ * once, and the CTAs are shared out among the problems by their weight bytes.
+ * The activations of every problem are quantized first (one quantizer launch
+ * each, chained by programmatic dependent launch), then the grouped GEMM.
+ * Same operands, layouts and contract as mxs_linear_decode (weights static;
+ * 1 <= count <= 3; M <= 16, the same for every problem); every problem needs
+ * its own workspace (mxs_act_planes_bytes(M, K, bits) bytes).  The K split of
+ * a problem may differ from its single launch, so results agree with
+ * mxs_linear_decode to fp32 rounding, not bit for bit.  Errors as
+ * mxs_linear_decode, per problem (the message names it). */
+typedef struct mxs_decode_problem {
+    const void *x;         /* device, bf16 [M, K], row stride ld_x */
+    int64_t K, ld_x;
+    const uint8_t *bits;   /* host, K/32 widths */
+    const void *packed_w;  /* device, compact layout (mxs_pack_weight) */
+    int64_t N;
+    float *y;              /* device, fp32 [M, N], row stride ld_y */
+    int64_t ld_y;
+    void *workspace;       /* device, the activation planes of this problem */
+    size_t ws_bytes;
+} mxs_decode_problem;
+MXS_API int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t M, int rounding, void *stream);
+
 /* ---------------------------------------------------------------- KV cache
  * The paper quantizes the KV cache too, with a 4-8 bit configuration
  * (Appendix A.2).  A cache is two code buffers in the activation layout of

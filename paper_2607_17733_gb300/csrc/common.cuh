@@ -118,6 +118,11 @@ int64_t decode_workspace_bytes(const Plan &p, int64_t M, int64_t N);
 // tail of the previous kernel on the stream (programmatic dependent launch)
 int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, const void *act_planes,
                        const void *packed, int64_t M, int64_t N, float *y, int64_t ld_y, bool pdl, cudaStream_t st);
+// up to three decode GEMMs (planes mode) in one launch; returns -1, with no
+// error recorded, when no cluster size fits every problem
+int launch_gemm_decode_group(const Plan *const *plans, const void *const *act_planes, const void *const *packed,
+                             const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, bool pdl,
+                             cudaStream_t st);
 int decode_status(int *status, int reset);
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N,
                         float *y, int64_t ld_y, int starve, cudaStream_t st);

@@ -317,9 +317,18 @@ struct PlanCounts {
     int st4, nst;
     int64_t row_bytes, kp;
 };
-struct DecodeParams {
+// A launch holds up to kMaxProblems independent GEMMs (the projections of a
+// decoder layer that share an input): problem i owns the CTAs
+// [cta0, cta0 + ncta) along x, and a cluster (along y) never spans two.
+constexpr int kMaxProblems = 3;
+struct DecodeProblem {
     PlanCounts p;
     DecodeArgs a;
+    int cta0, ncta;
+};
+struct DecodeParams {
+    DecodeProblem prob[kMaxProblems];
+    int nprob;
 };
 
 struct Stages {  // MMA stages of a CTA's K range [c0, c1): 4-bit ones (4 slots), then 6/8-bit ones (2 slots)
@@ -344,9 +353,16 @@ struct Stages {  // MMA stages of a CTA's K range [c0, c1): 4-bit ones (4 slots)
 };
 
 __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_constant__ DecodeParams dp,
-                                                                  const __grid_constant__ CUtensorMap tok_map) {
-    const PlanCounts &p = dp.p;
-    const DecodeArgs &a = dp.a;
+                                                                  const __grid_constant__ CUtensorMap map0,
+                                                                  const __grid_constant__ CUtensorMap map1,
+                                                                  const __grid_constant__ CUtensorMap map2) {
+    // the problem this CTA serves, and its CTA index and count within it
+    int pi = 0;
+    while (pi + 1 < dp.nprob && (int)blockIdx.x >= dp.prob[pi + 1].cta0) ++pi;
+    const PlanCounts &p = dp.prob[pi].p;
+    const DecodeArgs &a = dp.prob[pi].a;
+    const int bx = (int)blockIdx.x - dp.prob[pi].cta0, gx = dp.prob[pi].ncta;
+    const CUtensorMap *tok_map = pi == 0 ? &map0 : (pi == 1 ? &map1 : &map2);
     extern __shared__ uint8_t smem_raw[];
     const uint32_t sbase = su32(smem_raw);
     uint8_t *smem = smem_raw + (((sbase + 1023) & ~1023u) - sbase);  // 1024-aligned for the swizzled tiles
@@ -384,12 +400,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
     S.init(p, c0, c1);
     const int nchunks = (S.n + 1) / 2;          // a copy chunk holds two MMA stages
     const int nq = min(kQuads, nchunks);        // quads with a chunk in every group
-    const int ngroups = (int)blockIdx.x < a.G ? (a.G - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+    const int ngroups = bx < a.G ? (a.G - 1 - bx) / gx + 1 : 0;
     const int total = ngroups * nchunks;        // chunks this CTA streams
     const uint32_t xslice = (uint32_t)(R * 16 * 4);
     const int sg0 = c0 < p.n4 ? c0 / 4 : p.st4 + (c0 - p.n4) / 2;  // the rank's first stage in the planes
 
-    // chunk qc (in streaming order): group blockIdx.x + (qc / nchunks) * gridDim.x,
+    // chunk qc (in streaming order): group bx + (qc / nchunks) * gx,
     // stages 2k, 2k+1 with k = qc % nchunks; it goes to ring slot qc % ring and is
     // converted by quad qc % kQuads (ring is a multiple of kQuads, so each slot
     // has one consumer, which takes its slots in order)
@@ -401,7 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         if (2 * k + 1 < S.n) S.range(2 * k + 1, lo2, hi2); else hi2 = hi;
         const int64_t off = slot_offset(p, lo);
         const uint32_t bytes = (uint32_t)(slot_offset(p, hi2) - off);
-        const uint8_t *wg = a.w + (int64_t)((int)blockIdx.x + gi * (int)gridDim.x) * a.GB;
+        const uint8_t *wg = a.w + (int64_t)(bx + gi * gx) * a.GB;
         mbar_expect_tx(&full_c[s], bytes);
         bulk_load(ring + (size_t)s * a.slot_bytes + a.w_off, wg + off, bytes, &full_c[s]);
     };
@@ -411,7 +427,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         const int nst = min(2, S.n - 2 * k);
         uint8_t *slot = ring + (size_t)s * a.slot_bytes;
         mbar_expect_tx(&full_t[s], (uint32_t)nst * (kTokBytes + 512));
-        for (int i = 0; i < nst; ++i) tma_load_2d(slot + i * kTokBytes, &tok_map, &full_t[s], 128 * (sg0 + 2 * k + i), 0);
+        for (int i = 0; i < nst; ++i) tma_load_2d(slot + i * kTokBytes, tok_map, &full_t[s], 128 * (sg0 + 2 * k + i), 0);
         bulk_load(slot + 2 * kTokBytes, a.tok_sf + (int64_t)(sg0 + 2 * k) * 512, (uint32_t)nst * 512, &full_t[s]);
     };
 
@@ -778,7 +794,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         const int qtr = warp & 3;
         const int r = 32 * qtr + lane;
         int gi = 0;
-        for (int g = blockIdx.x; g < a.G; g += gridDim.x, ++gi) {
+        for (int g = bx; g < a.G; g += gx, ++gi) {
             const int b = gi & 1;
             if (!warp_wait(&acc_full[b], (gi >> 1) & 1, abort)) break;
             fence_after();
@@ -796,7 +812,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&acc_empty[b]);
-            const bool more = g + (int)gridDim.x < a.G;  // another group follows
+            const bool more = g + gx < a.G;  // another group follows
             if (a.GS == 1) {
                 const int n = 128 * g + r;
                 if (n < a.N) store_y(a, n, out);
@@ -978,9 +994,129 @@ int sm_count() {
     return cached;
 }
 
+PlanCounts counts_of(const Plan &p) {
+    PlanCounts c;
+    c.nb = p.nb, c.n4 = p.n4, c.n6 = p.n6, c.n8 = p.n8, c.n68 = p.n68;
+    c.st4 = p.st4, c.nst = p.nst, c.row_bytes = p.row_bytes, c.kp = p.kp;
+    return c;
+}
+
+// chunk rounds of a problem with `ncta` CTAs (the decode cost model: a CTA's
+// groups one after another, four quads per group, the cluster exchange per
+// extra group)
+double problem_cost(const DecodeShape &sh, int64_t G, int ncta) {
+    const double rounds = (double)((G + ncta - 1) / ncta);
+    const int nchunks = (sh.most + 1) / 2;
+    return rounds * ((nchunks + kQuads - 1) / kQuads + 1.0) + (sh.GS > 1 ? 0.3 + 8.0 * (rounds - 1.0) : 0.0);
+}
+
 }  // namespace
 
 int64_t decode_workspace_bytes(const Plan &, int64_t, int64_t) { return 0; }
+
+int launch_gemm_decode_group(const Plan *const *plans, const void *const *act_planes, const void *const *packed,
+                             const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, bool pdl,
+                             cudaStream_t st) {
+    if (count < 1 || count > kMaxProblems) return fail(MXS_ERR_INVALID_ARG, "count=%d (1..%d)", count, kMaxProblems);
+    const int sms = sm_count();
+    int64_t G[kMaxProblems];
+    for (int i = 0; i < count; ++i) {
+        if (N[i] > (int64_t)0x7FFFFFF0) return fail(MXS_ERR_SHAPE, "N too large");
+        G[i] = weight_offsets(*plans[i], N[i], false).G;
+    }
+    // one cluster size for the launch; CTAs handed one at a time to the
+    // problem whose share currently costs most
+    double best_cost = 1e30;
+    DecodeShape best_sh[kMaxProblems];
+    int best_n[kMaxProblems] = {};
+    for (int GS = 1; GS <= 8; GS *= 2) {
+        DecodeShape sh[kMaxProblems];
+        bool ok = sms / GS >= count;
+        for (int i = 0; i < count && ok; ++i) {
+            ok = GS <= plans[i]->nst;
+            if (ok) sh[i] = shape_for(*plans[i], GS, G[i], sms, 0, plans[i]->nst, true);
+            ok = ok && sh[i].ok;
+        }
+        if (!ok) continue;
+        int n[kMaxProblems], used = count;
+        for (int i = 0; i < count; ++i) n[i] = 1;
+        while (used < sms / GS) {
+            int worst = -1;
+            double wc = -1.0;
+            for (int i = 0; i < count; ++i)
+                if (n[i] < G[i] && problem_cost(sh[i], G[i], n[i]) > wc) wc = problem_cost(sh[i], G[i], n[i]), worst = i;
+            if (worst < 0) break;
+            ++n[worst];
+            ++used;
+        }
+        double cost = 0.0;
+        for (int i = 0; i < count; ++i) cost = std::max(cost, problem_cost(sh[i], G[i], n[i]));
+        if (cost < best_cost - 1e-9) {
+            best_cost = cost;
+            for (int i = 0; i < count; ++i) best_sh[i] = sh[i], best_n[i] = n[i];
+        }
+    }
+    if (best_cost >= 1e29) return -1;  // no common plan: the caller launches the problems one by one
+    DecodeParams dp = {};
+    dp.nprob = count;
+    CUtensorMap maps[kMaxProblems];
+    size_t smem = 0;
+    int cta = 0;
+    for (int i = 0; i < count; ++i) {
+        const Plan &p = *plans[i];
+        const DecodeShape &sh = best_sh[i];
+        DecodeArgs a = {};
+        a.w = static_cast<const uint8_t *>(packed[i]);
+        a.y = y[i];
+        a.ld_y = ld_y[i];
+        a.M = (int)M;
+        a.N = (int)N[i];
+        a.G = (int)G[i];
+        a.GB = weight_offsets(p, N[i], false).GB;
+        std::memset(&maps[i], 0, sizeof(CUtensorMap));
+        const int rc = make_plane_map(&maps[i], act_planes[i], M, p.kp, 16);
+        if (rc) return rc;
+        a.tok_sf = static_cast<const uint8_t *>(act_planes[i]) + align256(M * p.kp);
+        a.GS = sh.GS;
+        for (int r = 0; r < 9; ++r) a.bound[r] = r <= sh.GS ? sh.bound[r] : sh.bound[sh.GS];
+        a.max_mst = sh.max_mst;
+        a.ring = sh.ring;
+        a.slot_bytes = sh.slot_bytes;
+        a.w_off = sh.w_off;
+        a.accumulate = 0;
+        dp.prob[i].p = counts_of(p);
+        dp.prob[i].a = a;
+        dp.prob[i].cta0 = cta;
+        dp.prob[i].ncta = best_n[i];
+        cta += best_n[i];
+        smem = std::max(smem, sh.smem);
+    }
+    for (int i = count; i < kMaxProblems; ++i) maps[i] = maps[0];
+    const int GS = best_sh[0].GS;
+    cudaError_t e = cudaFuncSetAttribute(gemm_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(decode smem)");
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)cta, (unsigned)GS, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    int na = 0;
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = 1;
+    attr[na].val.clusterDim.y = (unsigned)GS;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+    if (pdl) {
+        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = na;
+    e = cudaLaunchKernelEx(&cfg, gemm_decode_kernel, dp, maps[0], maps[1], maps[2]);
+    return cuda_fail(e, "gemm_decode_kernel launch");
+}
 
 int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, const void *act_planes,
                        const void *packed, int64_t M, int64_t N, float *y, int64_t ld_y, bool pdl, cudaStream_t st) {
@@ -1046,11 +1182,13 @@ int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, 
             }
             cfg.attrs = attr;
             cfg.numAttrs = na;
-            DecodeParams dp;
-            dp.p.nb = p.nb, dp.p.n4 = p.n4, dp.p.n6 = p.n6, dp.p.n8 = p.n8, dp.p.n68 = p.n68;
-            dp.p.st4 = p.st4, dp.p.nst = p.nst, dp.p.row_bytes = p.row_bytes, dp.p.kp = p.kp;
-            dp.a = a;
-            e = cudaLaunchKernelEx(&cfg, gemm_decode_kernel, dp, map);
+            DecodeParams dp = {};
+            dp.nprob = 1;
+            dp.prob[0].p = counts_of(p);
+            dp.prob[0].a = a;
+            dp.prob[0].cta0 = 0;
+            dp.prob[0].ncta = sh.grid;
+            e = cudaLaunchKernelEx(&cfg, gemm_decode_kernel, dp, map, map, map);
             if (e != cudaSuccess) return cuda_fail(e, "gemm_decode_kernel launch");
         }
         return MXS_OK;

@@ -251,6 +251,71 @@ int mxs_gemm_decode(const void *codes, const uint8_t *scales, const void *act_pl
                               static_cast<cudaStream_t>(stream));
 }
 
+int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t M, int rounding, void *stream) {
+    if (!probs || count < 1 || count > 3) return fail(MXS_ERR_INVALID_ARG, "count=%d (1..3 problems)", count);
+    if (M < 0) return fail(MXS_ERR_SHAPE, "M=%lld", (long long)M);
+    if (M > 16) return fail(MXS_ERR_SHAPE, "the fused decode path takes M <= 16 (M=%lld)", (long long)M);
+    if (rounding != MXS_RNE && rounding != MXS_RHAZ) return fail(MXS_ERR_INVALID_ARG, "rounding=%d", rounding);
+    Plan plans[3];
+    const Plan *pp[3];
+    const void *planes[3], *packed[3];
+    int64_t N[3], ld_y[3];
+    float *y[3];
+    bool empty = M == 0;
+    for (int i = 0; i < count; ++i) {
+        const mxs_decode_problem &q = probs[i];
+        int rc = build_plan(q.bits, q.K, &plans[i]);
+        if (rc) return rc;
+        const Plan &p = plans[i];
+        if (q.N < 0) return fail(MXS_ERR_SHAPE, "problem %d: N=%lld", i, (long long)q.N);
+        if (!q.x || !q.packed_w || !q.y) return fail(MXS_ERR_INVALID_ARG, "problem %d: NULL operand", i);
+        if (q.ld_x < q.K || q.ld_x % 8 != 0)
+            return fail(MXS_ERR_INVALID_ARG, "problem %d: ld_x=%lld must be >= K and a multiple of 8", i, (long long)q.ld_x);
+        if (q.ld_y < q.N) return fail(MXS_ERR_INVALID_ARG, "problem %d: ld_y=%lld < N", i, (long long)q.ld_y);
+        const int64_t need = align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);  // mxs_act_planes_bytes
+        if ((int64_t)q.ws_bytes < need || (need > 0 && !q.workspace))
+            return fail(MXS_ERR_BUFFER, "problem %d: workspace of %lld bytes needed, %zu given", i, (long long)need,
+                        q.ws_bytes);
+        if (!aligned16(q.x) || !aligned16(q.packed_w) || (q.workspace && !aligned16(q.workspace)) ||
+            (reinterpret_cast<uintptr_t>(q.y) & 3))
+            return fail(MXS_ERR_ALIGN, "problem %d: x/packed_w/workspace must be 16-byte aligned, y 4-byte aligned", i);
+        for (int j = 0; j < i; ++j)
+            if (probs[j].workspace == q.workspace)
+                return fail(MXS_ERR_INVALID_ARG, "problems %d and %d share a workspace", j, i);
+        empty = empty || q.N == 0;
+        pp[i] = &plans[i];
+        planes[i] = q.workspace;
+        packed[i] = q.packed_w;
+        N[i] = q.N;
+        y[i] = q.y;
+        ld_y[i] = q.ld_y;
+    }
+    if (empty) {  // nothing to compute for an empty problem: run the others one by one
+        for (int i = 0; i < count; ++i) {
+            const mxs_decode_problem &q = probs[i];
+            const int rc = mxs_linear_decode(q.x, M, q.K, q.ld_x, q.bits, rounding, q.packed_w, q.N, q.y, q.ld_y,
+                                             q.workspace, q.ws_bytes, stream);
+            if (rc) return rc;
+        }
+        return MXS_OK;
+    }
+    int rc = check_device();
+    if (rc) return rc;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    for (int i = 0; i < count; ++i) {
+        rc = launch_quantize(plans[i], probs[i].x, M, probs[i].ld_x, rounding, nullptr, nullptr, probs[i].workspace, st);
+        if (rc) return rc;
+    }
+    rc = launch_gemm_decode_group(pp, planes, packed, N, y, ld_y, count, M, true, st);
+    for (int i = 0; rc < 0 && i < count; ++i) {  // no grouped plan: one launch per problem
+        const int r = launch_gemm_decode(plans[i], nullptr, nullptr, planes[i], packed[i], M, N[i], y[i], ld_y[i],
+                                         true, st);
+        if (r) return r;
+        if (i == count - 1) rc = MXS_OK;
+    }
+    return rc;
+}
+
 int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits, int rounding,
                       const void *packed_w, int64_t N, float *y, int64_t ld_y, void *ws, size_t ws_bytes,
                       void *stream) {

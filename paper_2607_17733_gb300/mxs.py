@@ -28,7 +28,7 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode",
            "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer",
            "mxs_quantize_act_permuted", "mxs_pack_weight_permuted", "mxs_attention_decode_workspace_bytes",
-           "mxs_attention_decode"]
+           "mxs_attention_decode", "mxs_linear_decode_group"]
 
 _lock = threading.Lock()
 _lib = None
@@ -92,6 +92,8 @@ def lib() -> ctypes.CDLL:
         L.mxs_allocation_r.restype = I
         L.mxs_allocate_layer.argtypes = [P, I64, D, D, P, P, ctypes.POINTER(I64), P]
         L.mxs_allocate_layer.restype = I
+        L.mxs_linear_decode_group.argtypes = [P, I, I64, I, P]
+        L.mxs_linear_decode_group.restype = I
         L.mxs_attention_decode_workspace_bytes.argtypes = [I64, I64, I64]
         L.mxs_attention_decode_workspace_bytes.restype = I64
         L.mxs_attention_decode.argtypes = [P, I64, I64, I64, P, P, P, P, P, P, I64, ctypes.c_float, P, P, SZ, P]
@@ -263,6 +265,29 @@ def linear_decode(x, bits, packed_w, N: int, rounding: int = RNE, y=None, worksp
     check(lib().mxs_linear_decode(_ptr(x), M, K, _ld(x), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
                                   _ld(y), _ptr(workspace), ws_bytes, _stream(stream)))
     return y
+
+
+class DecodeProblem(ctypes.Structure):
+    """ctypes mirror of mxs_decode_problem (include/mxs.h)."""
+    _fields_ = [("x", ctypes.c_void_p), ("K", ctypes.c_int64), ("ld_x", ctypes.c_int64), ("bits", ctypes.c_void_p),
+                ("packed_w", ctypes.c_void_p), ("N", ctypes.c_int64), ("y", ctypes.c_void_p), ("ld_y", ctypes.c_int64),
+                ("workspace", ctypes.c_void_p), ("ws_bytes", ctypes.c_size_t)]
+
+
+def linear_decode_group(problems, rounding: int = RNE, stream=None):
+    """Up to three decode layers in one grouped launch (mxs_linear_decode_group).
+    problems: sequence of (x [M, K] bf16, bits, packed_w, N, y [M, N] fp32, workspace uint8)."""
+    arr = (DecodeProblem * len(problems))()
+    keep = []
+    M = problems[0][0].shape[0]
+    for i, (x, bits, packed_w, N, y, ws) in enumerate(problems):
+        b = _Bits(bits)
+        keep.append(b)
+        if x.shape[0] != M:
+            raise ValueError("every problem of a group has the same M")
+        arr[i] = DecodeProblem(_ptr(x), x.shape[1], _ld(x), b.ptr, _ptr(packed_w), N, _ptr(y), _ld(y), _ptr(ws),
+                               ws.numel() * ws.element_size())
+    check(lib().mxs_linear_decode_group(ctypes.addressof(arr), len(problems), M, rounding, _stream(stream)))
 
 
 def linear_decode_noalloc(x, bits, packed_w, N: int, rounding: int = RNE, y=None, stream=None):

@@ -168,3 +168,39 @@ def test_allocation_validation(L):
     assert L.mxs_allocate_layer(fake, 100, 0.5, 0.5, fake, bits.ctypes.data, ctypes.byref(n6), None) == 2
     assert L.mxs_allocate_layer(fake, 256, -1.0, 0.5, fake, bits.ctypes.data, ctypes.byref(n6), None) == 1
     assert L.mxs_allocate_layer(fake, 1 << 20, 0.5, 0.5, fake, bits.ctypes.data, ctypes.byref(n6), None) == 2
+
+
+def test_decode_group_validation(L):
+    """mxs_linear_decode_group checks every problem before any device call."""
+    bits = np.full(4, 4, np.uint8)
+    b = bits.ctypes.data
+    need = L.mxs_act_planes_bytes(4, 128, b)
+
+    def prob(**kw):
+        f = dict(x=FAKE, K=128, ld_x=128, bits=b, packed_w=FAKE, N=16, y=FAKE, ld_y=16, workspace=FAKE,
+                 ws_bytes=need)
+        f.update(kw)
+        return mxs.DecodeProblem(**f)
+
+    def call(probs, M=4, rounding=0, count=None):
+        arr = (mxs.DecodeProblem * max(1, len(probs)))(*probs)
+        return L.mxs_linear_decode_group(ctypes.addressof(arr), len(probs) if count is None else count, M,
+                                         rounding, None)
+
+    ws2 = FAKE + (1 << 16)
+    bad = np.full(4, 5, np.uint8)
+    assert call([prob()], count=0) == 1
+    assert call([prob(), prob(workspace=ws2), prob(workspace=ws2 * 2)], count=4) == 1
+    assert call([prob()], M=17) == 2
+    assert call([prob()], M=-1) == 2
+    assert call([prob()], rounding=3) == 1
+    assert call([prob(), prob(K=100)]) == 2
+    assert call([prob(), prob(workspace=ws2, bits=bad.ctypes.data)]) == 3
+    assert call([prob(), prob(workspace=ws2, ld_y=8)]) == 1
+    assert call([prob(), prob(workspace=ws2, ld_x=132)]) == 1
+    assert call([prob(), prob(workspace=ws2, y=None)]) == 1
+    assert call([prob(), prob(workspace=ws2, ws_bytes=need - 1)]) == 5
+    assert call([prob(), prob(workspace=ws2 + 8)]) == 4
+    assert call([prob(), prob(workspace=ws2, packed_w=FAKE + 4)]) == 4
+    assert call([prob(), prob()]) == 1 and "share a workspace" in mxs.last_error()
+    assert call([prob(N=-1)]) == 2

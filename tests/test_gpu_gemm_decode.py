@@ -210,3 +210,32 @@ def test_fused_linear_decode_rhaz_and_stride(torch):
     w_s, w_c = mxo.quantize_bf16(wb, bits, mxo.RHAZ)
     ref, ab = mxo.gemm(bits, a_c, a_s, w_c, w_s)
     U.check_gemm(y, ref, ab)
+
+
+@pytest.mark.parametrize("M", [1, 5, 16])
+@pytest.mark.parametrize("shapes", [[(4096, 4096), (4096, 1024), (4096, 1024)], [(4096, 14336), (4096, 14336)],
+                                    [(512, 200), (1024, 37)], [(14336, 4096)]])
+def test_linear_decode_group(torch, M, shapes):
+    """Projections that share an input in one grouped launch (q/k/v, gate/up shapes and
+    ragged ones): every problem against the oracle, and against its own single launch
+    within the GEMM bound (the K split may differ)."""
+    probs, refs = [], []
+    for i, (K, N) in enumerate(shapes):
+        g = I.rng(61, M, K, N, i)
+        bits = I.width_map(K // 32, 0.8, 0.15, 0.05, g)
+        xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=30.0)
+        wb = I.normal_bf16((N, K), 0.02, g)
+        packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
+        x = U.to_dev_bf16(torch, xb)
+        y = torch.full((M, N), float("nan"), device="cuda")
+        ws = torch.empty(mxs.act_planes_bytes(M, K, bits), dtype=torch.uint8, device="cuda")
+        probs.append((x, bits, packed, N, y, ws))
+        refs.append(oracle_full(xb, wb, bits))
+    torch.cuda.synchronize()  # weights are static before the first decode call
+    mxs.linear_decode_group(probs)
+    torch.cuda.synchronize()
+    for (x, bits, packed, N, y, ws), (ref, ab) in zip(probs, refs):
+        got = y.cpu().numpy()
+        U.check_gemm(got, ref, ab)
+        single = mxs.linear_decode(x, bits, packed, N).cpu().numpy()
+        U.check_gemm(got, single.astype(np.float64), ab)
