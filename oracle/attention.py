@@ -15,6 +15,11 @@ h // (H / H_kv) (grouped-query attention).  For each query head:
 Readings: the scores, the softmax and the weighted sum are taken in real
 arithmetic on the dequantized cache (the paper keeps Softmax in FP16 and
 does not say how the products are formed); a block with S = 255 gives NaN.
+
+A decode batch (attention_batch) is B independent sequences: sequence b
+owns cache rows [b * T_cap, b * T_cap + T_b) and its own query; rows past
+its length are not read.  A sequence of length 0 attends to nothing and its
+output reads as zero (the paper does not define it).
 """
 from __future__ import annotations
 
@@ -44,4 +49,19 @@ def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, n_kv_heads: int, scal
         m = np.max(s) if T else 0.0
         p = np.exp(s - m)
         out[h] = (p @ vh) / np.sum(p)
+    return out
+
+
+def attention_batch(q: np.ndarray, k: np.ndarray, v: np.ndarray, lengths, T_cap: int, n_kv_heads: int,
+                    scale: float) -> np.ndarray:
+    """q [B, H, D]; k, v [B * T_cap, H_kv * D] fp64; lengths[b] tokens of
+    sequence b -> out [B, H, D] fp64 (see the module text)."""
+    q = np.asarray(q, np.float64)
+    B, H, D = q.shape
+    out = np.zeros((B, H, D))
+    for b in range(B):
+        T = int(lengths[b])
+        if T > 0:
+            rows = slice(b * T_cap, b * T_cap + T)
+            out[b] = attention(q[b], k[rows], v[rows], n_kv_heads, scale)
     return out

@@ -78,3 +78,28 @@ def test_cache_values_are_the_mxint_values():
             b = int(bits[kb])
             for i in range(32):
                 assert c[r, 32 * kb + i] == math.ldexp(int(codes[r, 32 * kb + i]), int(s[r, kb]) - 127 - (b - 2))
+
+
+def test_batch_reads_each_sequence_up_to_its_length():
+    """Sequence b sees rows [b*T_cap, b*T_cap + T_b) only: rows past its
+    length (set to NaN here) change nothing, an empty sequence is zero, and
+    each output equals the one-sequence call on its own rows."""
+    g = np.random.default_rng(6)
+    B, T_cap, H, H_kv, D = 4, 11, 4, 2, 16
+    lengths = [11, 0, 1, 6]
+    q = g.standard_normal((B, H, D))
+    k = g.standard_normal((B * T_cap, H_kv * D))
+    v = g.standard_normal((B * T_cap, H_kv * D))
+    for b, T in enumerate(lengths):
+        k[b * T_cap + T:(b + 1) * T_cap] = np.nan
+        v[b * T_cap + T:(b + 1) * T_cap] = np.nan
+    out = AT.attention_batch(q, k, v, lengths, T_cap, H_kv, 0.25)
+    assert np.all(np.isfinite(out))
+    assert np.all(out[1] == 0.0)
+    # one token: softmax of one score is 1, so the output is that token's value
+    for h in range(H):
+        c = (h // (H // H_kv)) * D
+        assert np.array_equal(out[2, h], v[2 * T_cap, c:c + D])
+    for b in (0, 3):
+        rows = slice(b * T_cap, b * T_cap + lengths[b])
+        assert np.array_equal(out[b], AT.attention(q[b], k[rows], v[rows], H_kv, 0.25))
