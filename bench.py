@@ -746,17 +746,19 @@ def run_calibration(args):
 
 
 ATTN_T, ATTN_H, ATTN_HKV, ATTN_D = 4096, 32, 8, 128
+ATTN_BATCHES = (1, 4, 16)
 
 
 def run_attention(args):
     """Decode attention over an MXINT KV cache (the paper's KV quantization,
-    4-8 bit configuration): one step = one decode token of one sequence through
-    the attention of `layers` LLaMA-3-8B-shaped layers (default 32) with
-    4096 cached tokens (32 query heads, 8 KV heads of 128 dims).  Each layer's
-    K and V caches are quantized rows of 1024 values with one 8-bit block
-    (the most sensitive 32 columns) and 31 4-bit blocks.  Metric: GB/s of
-    cache bytes read (codes + scales; HBM-bound), the step captured in a CUDA
-    graph."""
+    4-8 bit configuration): one step = one decode token of each sequence of a
+    batch, for batches of 1, 4 and 16 sequences of 4096 cached tokens, through
+    the attention of `layers` LLaMA-3-8B-shaped layers (default 32; 32 query
+    heads, 8 KV heads of 128 dims), one mxs_attention_decode_batch launch per
+    layer and batch.  Each layer's K and V caches are quantized rows of 1024
+    values with one 8-bit block (the most sensitive 32 columns) and 31 4-bit
+    blocks.  Metric: GB/s of cache bytes read (codes + scales; HBM-bound), the
+    step captured in a CUDA graph."""
     import torch
 
     ws, rank, local = dist_setup()
@@ -771,39 +773,45 @@ def run_attention(args):
     T, H, Hkv, D = ATTN_T, ATTN_H, ATTN_HKV, ATTN_D
     K = Hkv * D
     gen = torch.Generator(device=dev)
-    layers = []
-    for l in range(L):
-        g = I.rng(SEED, rank, 9, l)
-        kb = np.full(K // 32, 4, np.uint8)
-        kb[g.integers(K // 32)] = 8
-        vb = np.full(K // 32, 4, np.uint8)
-        vb[g.integers(K // 32)] = 8
-        gen.manual_seed(SEED * 19 + rank * 10_007 + l)
-        kx = torch.randn((T, K), generator=gen, device=dev, dtype=torch.float32)
-        kx[:, torch.randperm(K, generator=gen, device=dev)[: K // 100]] *= 20.0
-        vx = torch.randn((T, K), generator=gen, device=dev, dtype=torch.float32)
-        kc, ks, _ = mxs.quantize_act(kx.to(torch.bfloat16), kb)
-        vc, vs, _ = mxs.quantize_act(vx.to(torch.bfloat16), vb)
-        del kx, vx
-        q = torch.randn((H, D), generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
-        out = torch.empty((H, D), dtype=torch.float32, device=dev)
-        wsb = torch.empty(mxs.lib().mxs_attention_decode_workspace_bytes(T, H, D), dtype=torch.uint8, device=dev)
-        layers.append((q, kc, ks, kb, vc, vs, vb, out, wsb))
+    items = []  # (batch, q, kc, ks, kbits, vc, vs, vbits, out, workspace)
+    for nb in ATTN_BATCHES:
+        for l in range(L):
+            g = I.rng(SEED, rank, 9, nb, l)
+            kb = np.full(K // 32, 4, np.uint8)
+            kb[g.integers(K // 32)] = 8
+            vb = np.full(K // 32, 4, np.uint8)
+            vb[g.integers(K // 32)] = 8
+            gen.manual_seed(SEED * 19 + rank * 10_007 + nb * 101 + l)
+            kx = torch.randn((nb * T, K), generator=gen, device=dev, dtype=torch.float32)
+            kx[:, torch.randperm(K, generator=gen, device=dev)[: K // 100]] *= 20.0
+            kc, ks, _ = mxs.quantize_act(kx.to(torch.bfloat16), kb)
+            del kx
+            vx = torch.randn((nb * T, K), generator=gen, device=dev, dtype=torch.float32)
+            vc, vs, _ = mxs.quantize_act(vx.to(torch.bfloat16), vb)
+            del vx
+            q = torch.randn((nb, H, D), generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
+            out = torch.empty((nb, H, D), dtype=torch.float32, device=dev)
+            wsb = torch.zeros(mxs.attention_batch_workspace_bytes(nb, T, H, D), dtype=torch.uint8, device=dev)
+            items.append((nb, q, kc, ks, kb, vc, vs, vb, out, wsb))
     torch.cuda.synchronize()
-    step_bytes = sum(t.numel() for (_, kc, ks, _, vc, vs, _, _, _) in layers for t in (kc, ks, vc, vs)) \
-        + sum(q.numel() * 2 + o.numel() * 4 for (q, *_rest, o, _w) in layers)
+    cache_bytes = sum(t.numel() for it in items for t in (it[2], it[3], it[5], it[6]))
+    step_bytes = cache_bytes + sum(it[1].numel() * 2 + it[8].numel() * 4 for it in items)
     scale = 1.0 / math.sqrt(D)
 
+    def run(it):
+        nb, q, kc, ks, kb, vc, vs, vb, out, wsb = it
+        mxs.attention_decode_batch(q, Hkv, kc, ks, kb, vc, vs, vb, T, scale, out=out, workspace=wsb)
+
     def fn():
-        for q, kc, ks, kb, vc, vs, vb, out, wsb in layers:
-            mxs.attention_decode(q, Hkv, kc, ks, kb, vc, vs, vb, T, scale, out=out, workspace=wsb)
+        for it in items:
+            run(it)
 
     if args.eager:
         for _ in range(args.warmup + args.steps):
             fn()
         torch.cuda.synchronize()
         if rank == 0:
-            print(json.dumps({"eager_steps": args.steps, "launches_per_step": 2 * L}), flush=True)
+            print(json.dumps({"eager_steps": args.steps, "launches_per_step": len(items)}), flush=True)
         return
     st = torch.cuda.Stream(device=dev)
     st.wait_stream(torch.cuda.current_stream())
@@ -832,37 +840,59 @@ def run_attention(args):
     ms = allreduce_max(t0.elapsed_time(t1) / args.steps, ws)
     value = ws * step_bytes / (ms * 1e-3) / 1e9
     pk = peaks()
+    # per batch size: the same graph-free launches timed alone (device time)
+    per_batch = {}
+    for nb in ATTN_BATCHES:
+        sub = [it for it in items if it[0] == nb]
+        gb = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(st):
+            for it in sub:
+                run(it)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(gb, stream=st):
+            for it in sub:
+                run(it)
+        for _ in range(3):
+            gb.replay()
+        torch.cuda.synchronize()
+        t0.record()
+        for _ in range(args.steps):
+            gb.replay()
+        t1.record()
+        torch.cuda.synchronize()
+        mb = t0.elapsed_time(t1) / args.steps
+        byt = sum(t.numel() for it in sub for t in (it[2], it[3], it[5], it[6]))
+        per_batch[str(nb)] = {"us_per_layer": mb * 1e3 / L, "cache_gbps": byt / (mb * 1e-3) / 1e9}
 
     # end to end: the step's queries from pinned host memory, the outputs back
-    q_host = [q.cpu().pin_memory() for (q, *_r) in layers]
-    o_host = [torch.empty((H, D), dtype=torch.float32).pin_memory() for _ in layers]
+    q_host = [it[1].cpu().pin_memory() for it in items]
+    o_host = [torch.empty(tuple(it[8].shape), dtype=torch.float32).pin_memory() for it in items]
     barrier(ws)
     torch.cuda.synchronize()
     e2e_steps = max(1, min(args.steps, 20))
     t0.record()
     for _ in range(e2e_steps):
-        for (q, kc, ks, kb, vc, vs, vb, out, wsb), qh, oh in zip(layers, q_host, o_host):
-            q.copy_(qh, non_blocking=True)
-            mxs.attention_decode(q, Hkv, kc, ks, kb, vc, vs, vb, T, scale, out=out, workspace=wsb)
-            oh.copy_(out, non_blocking=True)
+        for it, qh, oh in zip(items, q_host, o_host):
+            it[1].copy_(qh, non_blocking=True)
+            run(it)
+            oh.copy_(it[8], non_blocking=True)
     t1.record()
     torch.cuda.synchronize()
     e2e_ms = allreduce_max(t0.elapsed_time(t1) / e2e_steps, ws)
-    e2e = {"value": ws * step_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s", "h2d_bytes_per_step": L * H * D * 2,
-           "d2h_bytes_per_step": L * H * D * 4, "ms_per_step": e2e_ms}
+    e2e = {"value": ws * step_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
+           "h2d_bytes_per_step": sum(it[1].numel() * 2 for it in items),
+           "d2h_bytes_per_step": sum(it[8].numel() * 4 for it in items), "ms_per_step": e2e_ms}
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         from oracle import attention as AT
-        from oracle import mxo
-        q, kc, ks, kb, vc, vs, vb, _, _ = layers[0]
-        kx = torch.randn((T, K), generator=gen.manual_seed(SEED * 19 + rank * 10_007), device=dev).to(torch.bfloat16)
-        kbits = kx.cpu().view(torch.int16).numpy().view(np.uint16)
+        nb, q, kc, ks, kb, vc, vs, vb, _, _ = items[0]
+        kbits = torch.randn((T, K), device=dev).to(torch.bfloat16).cpu().view(torch.int16).numpy().view(np.uint16)
         vbits = torch.randn((T, K), device=dev).to(torch.bfloat16).cpu().view(torch.int16).numpy().view(np.uint16)
-        qv = q.float().cpu().numpy().astype(np.float64)
+        qv = q[0].float().cpu().numpy().astype(np.float64)
         kd = AT.dequantized_cache(kbits, kb)
         vd = AT.dequantized_cache(vbits, vb)
-        lb = sum(t.numel() for t in (kc, ks, vc, vs))
+        lb = sum(t.numel() for t in (kc, ks, vc, vs)) // nb
         nbytes, t_start, passes = 0, time.perf_counter(), 0
         while True:
             AT.attention(qv, kd, vd, Hkv, scale)
@@ -872,22 +902,24 @@ def run_attention(args):
                 break
         dt = time.perf_counter() - t_start
         cpu = {"value": nbytes / dt / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
-               "sample": f"one layer's attention over 4096 dequantized cached tokens, {passes} pass(es) "
-                         "(cache dequantized once, not timed): numpy fp64", "seconds": dt}
+               "sample": f"one sequence's attention in one layer over 4096 dequantized cached tokens, {passes} "
+                         "pass(es) (cache dequantized once, not timed): numpy fp64", "seconds": dt}
     if rank == 0:
         print(json.dumps({
             "metric": "mxint_kv_attention_gbps", "value": value, "unit": "GB/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "MXINT codes in, f32 math",
+            "scaling": "weak", "vs_baseline": None, "dtype": "MXINT codes in, bf16 MMA (exact elements), f32 sums",
             "data": "synthetic (seeded; keys N(0,1) with 1% of channels x20, values N(0,1))",
-            "config": {"workload": "llama3-8b-decode-attention", "context_tokens": T, "layers": L,
-                       "heads": H, "kv_heads": Hkv, "head_dim": D, "kv_map": "1 x 8-bit + 31 x 4-bit blocks",
-                       "l2": f"inputs larger than L2 ({step_bytes / 1e9:.3f} GB of cache per step)"},
-            "roofline": {"kernel": "attention_chunk_kernel + attention_combine_kernel", "bound": "hbm",
+            "config": {"workload": "llama3-8b-decode-attention", "context_tokens": T, "batches": list(ATTN_BATCHES),
+                       "layers": L, "heads": H, "kv_heads": Hkv, "head_dim": D,
+                       "kv_map": "1 x 8-bit + 31 x 4-bit blocks",
+                       "l2": f"inputs larger than L2 ({cache_bytes / 1e9:.3f} GB of cache per step)"},
+            "per_batch": per_batch,
+            "roofline": {"kernel": "attention_decode_kernel", "bound": "hbm",
                          "achieved": step_bytes / (ms * 1e-3) / 1e9, "peak": pk["hbm_gbs"], "unit": "GB/s",
                          "frac": step_bytes / (ms * 1e-3) / 1e9 / pk["hbm_gbs"], "peak_source": pk["source"],
-                         "traffic": None},
-            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": 2 * L * args.steps, "clocks": clocks}), flush=True)
+                         "traffic": profile_traffic("attention.cu", "attention_decode_llama3_8b_kv4096.md")},
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": len(items) * args.steps, "clocks": clocks}), flush=True)
 
 
 def main():

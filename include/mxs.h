@@ -287,28 +287,50 @@ MXS_API int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, 
  * (codes [T_max, mxs_act_row_bytes(H_kv * D, bits)], scales [T_max, H_kv*D/32]).
  * Appending token t is one mxs_quantize_act call of M = 1 row into row t.
  *
- * mxs_attention_decode -- one decode step of one sequence over the cached
- * tokens 0..T-1: for query head h (reading KV head h / (H / H_kv)),
- *   out[h] = sum_t softmax_t(scale * <q[h], k_t>) * v_t
+ * mxs_attention_decode_batch -- one decode step of B sequences: sequence b
+ * owns cache rows [b * T_cap, b * T_cap + T_b) and has one query token; for
+ * its query head h (reading KV head h / (H / H_kv)),
+ *   out[b][h] = sum_t softmax_t(scale * <q[b][h], k_t>) * v_t,   t < T_b,
  * with k_t, v_t the MXINT element values of the cache (code * 2^(S-127-(b-2))).
- *   q        device, bf16 [H, D], row-major
- *   k_*, v_* device code rows and scales as above (code buffers 16-byte
- *            aligned); k_bits, v_bits host width maps of H_kv * D / 32 entries
- *   out      device, fp32 [H, D]
- *   workspace device, mxs_attention_decode_workspace_bytes(T, H, D) bytes,
- *            16-byte aligned (per-chunk partial sums; overwritten)
+ *   q        device, bf16 [B, H, D], row-major
+ *   k_*, v_* device code rows and scales as above, B * T_cap rows each (code
+ *            buffers 16-byte aligned); k_bits, v_bits host width maps of
+ *            H_kv * D / 32 entries
+ *   lengths  device int32 [B] (4-byte aligned): T_b, clamped to [0, T_cap];
+ *            NULL means every sequence has T_cap tokens.  A sequence of
+ *            length 0 gets zeros.
+ *   out      device, fp32 [B, H, D], 16-byte aligned
+ *   workspace device, mxs_attention_decode_batch_workspace_bytes(B, T_cap, H, D)
+ *            bytes, 16-byte aligned.  Its first bytes hold arrival counters
+ *            that must be zero when the call starts and are zero again when
+ *            its kernel ends: zero the workspace once after allocating it
+ *            (and again before using it with other sizes).  The rest holds
+ *            per-split partial sums, overwritten.
  * D is 64 or 128, H a multiple of H_kv with H / H_kv <= 8, H_kv * D <= 8192,
- * 1 <= T.  The products and sums are fp32 (the element values are exact in
- * fp32); chunks of 128 tokens are combined in order, so the result is
- * deterministic.  A cache block with scale 255 (NaN/Inf when written) makes
- * the heads that read it NaN.  Asynchronous on `stream`; allocates nothing.
- * Errors: MXS_ERR_UNSUPPORTED (D), MXS_ERR_SHAPE, MXS_ERR_BITS,
- * MXS_ERR_INVALID_ARG, MXS_ERR_ALIGN, MXS_ERR_BUFFER, MXS_ERR_CUDA. */
+ * 1 <= B <= 65535, 1 <= T_cap < 2^31.  Scores and weighted sums run on the
+ * tensor cores in bf16 with fp32 accumulation: the cache elements are exact in
+ * bf16, so every score product is exact; the softmax weights enter as a sum
+ * of two bf16 terms (relative error <= 2^-18).  Splits of a sequence and the
+ * warps within a split are combined in a fixed order: deterministic for given
+ * sizes on a given GPU.  A cache block with scale 255 (NaN/Inf when written)
+ * makes the heads that read it NaN.  Asynchronous on `stream`; allocates
+ * nothing.  Errors: MXS_ERR_UNSUPPORTED (D), MXS_ERR_SHAPE, MXS_ERR_BITS,
+ * MXS_ERR_INVALID_ARG, MXS_ERR_ALIGN, MXS_ERR_BUFFER, MXS_ERR_CUDA.
+ *
+ * mxs_attention_decode -- the same for one sequence of T tokens (B = 1,
+ * T_cap = T, no lengths); q bf16 [H, D], out fp32 [H, D], workspace of
+ * mxs_attention_decode_workspace_bytes(T, H, D) bytes with the same rule. */
 MXS_API int64_t mxs_attention_decode_workspace_bytes(int64_t T, int64_t H, int64_t D);
 MXS_API int mxs_attention_decode(const void *q_bf16, int64_t H, int64_t H_kv, int64_t D, const void *k_codes,
                                  const uint8_t *k_scales, const uint8_t *k_bits, const void *v_codes,
                                  const uint8_t *v_scales, const uint8_t *v_bits, int64_t T, float scale, float *out,
                                  void *workspace, size_t ws_bytes, void *stream);
+MXS_API int64_t mxs_attention_decode_batch_workspace_bytes(int64_t B, int64_t T_cap, int64_t H, int64_t D);
+MXS_API int mxs_attention_decode_batch(const void *q_bf16, int64_t B, int64_t H, int64_t H_kv, int64_t D,
+                                       const void *k_codes, const uint8_t *k_scales, const uint8_t *k_bits,
+                                       const void *v_codes, const uint8_t *v_scales, const uint8_t *v_bits,
+                                       const int32_t *lengths, int64_t T_cap, float scale, float *out,
+                                       void *workspace, size_t ws_bytes, void *stream);
 
 /* ---------------------------------------------------------------- offline allocation
  * Calibration that produces the width maps (Alg. 1, Alg. 3, Theorem 1).  Not

@@ -28,7 +28,8 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode",
            "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer",
            "mxs_quantize_act_permuted", "mxs_pack_weight_permuted", "mxs_attention_decode_workspace_bytes",
-           "mxs_attention_decode", "mxs_linear_decode_group"]
+           "mxs_attention_decode", "mxs_linear_decode_group",
+           "mxs_attention_decode_batch_workspace_bytes", "mxs_attention_decode_batch"]
 
 _lock = threading.Lock()
 _lib = None
@@ -98,6 +99,11 @@ def lib() -> ctypes.CDLL:
         L.mxs_attention_decode_workspace_bytes.restype = I64
         L.mxs_attention_decode.argtypes = [P, I64, I64, I64, P, P, P, P, P, P, I64, ctypes.c_float, P, P, SZ, P]
         L.mxs_attention_decode.restype = I
+        L.mxs_attention_decode_batch_workspace_bytes.argtypes = [I64, I64, I64, I64]
+        L.mxs_attention_decode_batch_workspace_bytes.restype = I64
+        L.mxs_attention_decode_batch.argtypes = [P, I64, I64, I64, I64, P, P, P, P, P, P, P, I64, ctypes.c_float, P, P,
+                                                 SZ, P]
+        L.mxs_attention_decode_batch.restype = I
         _lib = L
         return L
 
@@ -381,9 +387,35 @@ def attention_decode(q, H_kv: int, k_codes, k_scales, k_bits, v_codes, v_scales,
     if out is None:
         out = torch.empty((H, D), dtype=torch.float32, device=q.device)
     need = _size(lib().mxs_attention_decode_workspace_bytes(T, H, D))
-    if workspace is None:
-        workspace = torch.empty(need, dtype=torch.uint8, device=q.device)
+    if workspace is None:  # its counters must start at zero; the call leaves them zero
+        workspace = torch.zeros(need, dtype=torch.uint8, device=q.device)
     check(lib().mxs_attention_decode(_ptr(q), H, H_kv, D, _ptr(k_codes), _ptr(k_scales), kb.ptr, _ptr(v_codes),
                                      _ptr(v_scales), vb.ptr, T, float(scale), _ptr(out), _ptr(workspace),
                                      workspace.numel() * workspace.element_size(), _stream(stream)))
     return out
+
+
+def attention_decode_batch(q, H_kv: int, k_codes, k_scales, k_bits, v_codes, v_scales, v_bits, T_cap: int,
+                           scale: float, lengths=None, out=None, workspace=None, stream=None):
+    """One decode step of B sequences over an MXINT KV cache
+    (mxs_attention_decode_batch).  q: bf16 [B, H, D]; sequence b owns cache rows
+    [b * T_cap, b * T_cap + lengths[b]); lengths: device int32 [B] or None
+    (every sequence T_cap tokens).  workspace: zero-initialised uint8 of
+    attention_batch_workspace_bytes(...) bytes (allocated zeroed when None)."""
+    import torch
+    B, H, D = q.shape
+    kb, vb = _Bits(k_bits), _Bits(v_bits)
+    if out is None:
+        out = torch.empty((B, H, D), dtype=torch.float32, device=q.device)
+    if workspace is None:
+        workspace = torch.zeros(attention_batch_workspace_bytes(B, T_cap, H, D), dtype=torch.uint8, device=q.device)
+    check(lib().mxs_attention_decode_batch(_ptr(q), B, H, H_kv, D, _ptr(k_codes), _ptr(k_scales), kb.ptr,
+                                           _ptr(v_codes), _ptr(v_scales), vb.ptr,
+                                           None if lengths is None else _ptr(lengths), T_cap, float(scale),
+                                           _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                           _stream(stream)))
+    return out
+
+
+def attention_batch_workspace_bytes(B: int, T_cap: int, H: int, D: int) -> int:
+    return _size(lib().mxs_attention_decode_batch_workspace_bytes(B, T_cap, H, D))
