@@ -206,8 +206,9 @@ __global__ void __launch_bounds__(kThreads, 3) attention_decode_kernel(const __g
     const int ntile = (t1 - t0 + kTile - 1) / kTile;
     const int64_t row0 = (int64_t)b * a.T_cap;
 
-    // ---- producer role: thread tid stages token tid/2 of each tile, K (even tid) or V (odd)
-    const int ptok = tid >> 1, pv = tid & 1;
+    // ---- each warp stages its own 16 tokens of every tile (and only reads
+    // those): lane l copies token l/2 of the warp's slice, K (even l) or V (odd)
+    const int ptok = 16 * warp + (lane >> 1), pv = lane & 1;
     const uint8_t *const pcode = pv ? a.vc : a.kc;
     const uint8_t *const pscale = pv ? a.vs : a.ks;
     const int64_t prow = pv ? a.v_row : a.k_row;
@@ -281,6 +282,7 @@ __global__ void __launch_bounds__(kThreads, 3) attention_decode_kernel(const __g
     // ---- ring prologue: tiles 0 .. kStages-2.  The scale bytes travel through
     // registers: loaded when their tile's copies are issued, stored to shared
     // memory in the iteration before the tile is used (two iterations later).
+    // No barrier across warps: each warp waits for its own copies only.
     static_assert(kStages == 4, "the scale pipeline below holds two tiles");
     uint32_t pend1 = 0x7F7F7F7Fu, pend2 = 0x7F7F7F7Fu;  // scales of tiles tile+1, tile+2
     {
@@ -296,8 +298,8 @@ __global__ void __launch_bounds__(kThreads, 3) attention_decode_kernel(const __g
 
     for (int tile = 0; tile < ntile; ++tile) {
         cp_async_wait<kStages - 2>();
-        __syncthreads();  // this tile's copies and scales are in place; tile - 1's buffer is free
-        if (tile + 1 < ntile) put_scales(tile + 1, pend1);  // read after the next barrier
+        __syncwarp();  // the warp's copies and scales of this tile are in place; its tile - 1 rows are free
+        if (tile + 1 < ntile) put_scales(tile + 1, pend1);  // read after the next __syncwarp
         pend1 = pend2;
         if (tile + kStages - 1 < ntile) issue(tile + kStages - 1, pend2);
         cp_async_commit();
