@@ -35,6 +35,7 @@ namespace {
 
 constexpr int kBM = 128, kBN = 256, kBK = 128;  // tile rows (A), tile rows (W), K' bytes per stage
 constexpr int kStages = 4;
+constexpr int kBandM = 16;  // row tiles per band of the tile order
 constexpr int kABytes = kBM * kBK, kBBytes = kBN * kBK;  // 16 KB, 32 KB
 constexpr int kSfaBytes = 512, kSfbBytes = 1024;
 constexpr int kTmemCols = 512;
@@ -55,7 +56,7 @@ struct Smem {
     uint8_t b[kStages][kBBytes];
     uint8_t sfa[kStages][kSfaBytes];
     uint8_t sfb[kStages][kSfbBytes];
-    uint64_t full[kStages], empty[kStages], acc_full;
+    uint64_t full[kStages], empty[kStages], acc_full, acc_empty;
     uint32_t tmem_base;
     int abort;
 };
@@ -65,6 +66,9 @@ __device__ __forceinline__ uint32_t su32(const void *p) { return (uint32_t)__cvt
 
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(bar)) : "memory");
 }
 __device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes) : "memory");
@@ -165,7 +169,19 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
     Smem &sm = *reinterpret_cast<Smem *>(smem_raw + (((base + 1023) & ~1023u) - base));
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.y * kBM, n0 = blockIdx.x * kBN;
+    // Persistent: CTA c takes tiles c, c + gridDim.x, ... of the tile order:
+    // bands of kBandM row tiles, the band's row tiles fastest, so that the CTAs
+    // running at a time share few weight tiles (each read from DRAM about once
+    // per band) and the band's activation tiles stay in L2.  The producer runs
+    // ahead into the next tile while the epilogue drains the accumulator.
+    const int mt = (a.M + kBM - 1) / kBM, nt = (a.N + kBN - 1) / kBN, tiles = mt * nt;
+    auto tile_origin = [&](int id, int &m0, int &n0) {
+        const int band = id / (kBandM * nt);
+        const int first = band * kBandM, gm = min(kBandM, mt - first);
+        const int in = id - band * kBandM * nt;
+        m0 = (first + in % gm) * kBM;
+        n0 = (in / gm) * kBN;
+    };
     const int nst = a.nst;
 
     if (threadIdx.x == 0) {
@@ -174,6 +190,7 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
             mbar_init(&sm.empty[s], 1);
         }
         mbar_init(&sm.acc_full, 1);
+        mbar_init(&sm.acc_empty, 4);  // the four epilogue warps have read the accumulator
         sm.abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -191,89 +208,111 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
+        // `it` counts the CTA's K' stages over all its tiles (ring slot it % kStages)
         if (lane == 0) {
-            const int tile_a = m0 / 128, tile_b = n0 / 128;
-            const bool two_b = tile_b + 1 < a.sfb_tiles;
-            const uint32_t tx = kABytes + kBBytes + kSfaBytes + (two_b ? 2 : 1) * 512;
-            int issued = 0;
-            for (int ks = 0; ks < nst; ++ks) {
-                const int s = ks % kStages;
-                const uint32_t ph = (ks / kStages) & 1;
-                if (!mbar_wait(&sm.empty[s], ph ^ 1, abort)) break;
-                if (a.starve == ks + 1) continue;  // test hook: this stage never arrives
-                mbar_expect_tx(&sm.full[s], tx);
-                tma_load_2d(sm.a[s], &tmap_a, &sm.full[s], ks * kBK, m0);
-                tma_load_2d(sm.b[s], &tmap_b, &sm.full[s], ks * kBK, n0);
-                bulk_load(sm.sfa[s], a.sfa + ((int64_t)tile_a * nst + ks) * 512, 512, &sm.full[s]);
-                bulk_load(sm.sfb[s], a.sfb + ((int64_t)tile_b * nst + ks) * 512, 512, &sm.full[s]);
-                if (two_b) bulk_load(sm.sfb[s] + 512, a.sfb + ((int64_t)(tile_b + 1) * nst + ks) * 512, 512, &sm.full[s]);
-                issued = ks + 1;
+            int it = 0, issued = 0;
+            bool go = true;
+            for (int id = blockIdx.x; id < tiles && go; id += gridDim.x) {
+                int m0, n0;
+                tile_origin(id, m0, n0);
+                const int tile_a = m0 / 128, tile_b = n0 / 128;
+                const bool two_b = tile_b + 1 < a.sfb_tiles;
+                const uint32_t tx = kABytes + kBBytes + kSfaBytes + (two_b ? 2 : 1) * 512;
+                for (int ks = 0; ks < nst; ++ks, ++it) {
+                    const int s = it % kStages;
+                    const uint32_t ph = (it / kStages) & 1;
+                    if (!mbar_wait(&sm.empty[s], ph ^ 1, abort)) {
+                        go = false;
+                        break;
+                    }
+                    if (a.starve == it + 1) continue;  // test hook: this stage never arrives
+                    mbar_expect_tx(&sm.full[s], tx);
+                    tma_load_2d(sm.a[s], &tmap_a, &sm.full[s], ks * kBK, m0);
+                    tma_load_2d(sm.b[s], &tmap_b, &sm.full[s], ks * kBK, n0);
+                    bulk_load(sm.sfa[s], a.sfa + ((int64_t)tile_a * nst + ks) * 512, 512, &sm.full[s]);
+                    bulk_load(sm.sfb[s], a.sfb + ((int64_t)tile_b * nst + ks) * 512, 512, &sm.full[s]);
+                    if (two_b)
+                        bulk_load(sm.sfb[s] + 512, a.sfb + ((int64_t)(tile_b + 1) * nst + ks) * 512, 512, &sm.full[s]);
+                    issued = it + 1;
+                }
             }
             // drain: every stage this thread issued must have landed before the CTA exits
-            for (int ks = (issued > kStages ? issued - kStages : 0); ks < issued; ++ks) {
-                if (a.starve == ks + 1) continue;
-                const int s = ks % kStages;
+            for (int k = (issued > kStages ? issued - kStages : 0); k < issued; ++k) {
+                if (a.starve == k + 1) continue;
                 const long long t0 = clock64();
-                while (!mbar_try_wait(&sm.full[s], (ks / kStages) & 1) && clock64() - t0 < kWaitCycles) {
+                while (!mbar_try_wait(&sm.full[k % kStages], (k / kStages) & 1) && clock64() - t0 < kWaitCycles) {
                 }
             }
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
-            int committed = 0;
-            for (int ks = 0; ks < nst; ++ks) {
-                const int s = ks % kStages;
-                const uint32_t ph = (ks / kStages) & 1;
-                if (!mbar_wait(&sm.full[s], ph, abort)) break;
+            int it = 0, committed = 0, lt = 0;
+            bool go = true;
+            for (int id = blockIdx.x; id < tiles && go; id += gridDim.x, ++lt) {
+                // the accumulator is free once the epilogue has read the previous tile
+                if (lt > 0 && !mbar_wait(&sm.acc_empty, (lt - 1) & 1, abort)) break;
                 fence_after();
-                const uint32_t sfa_t = tmem + kSfCol + 12 * s, sfb_t = sfa_t + 4;
-                tmem_cp_sf(sfa_t, desc_sf(su32(sm.sfa[s])));
-                tmem_cp_sf(sfb_t, desc_sf(su32(sm.sfb[s])));
-                tmem_cp_sf(sfb_t + 4, desc_sf(su32(sm.sfb[s] + 512)));
-                const uint32_t a_addr = su32(sm.a[s]), b_addr = su32(sm.b[s]);
-                if (ks < a.st4) {  // four 4-bit blocks, one plane each
+                for (int ks = 0; ks < nst; ++ks, ++it) {
+                    const int s = it % kStages;
+                    const uint32_t ph = (it / kStages) & 1;
+                    if (!mbar_wait(&sm.full[s], ph, abort)) {
+                        go = false;
+                        break;
+                    }
+                    fence_after();
+                    const uint32_t sfa_t = tmem + kSfCol + 12 * s, sfb_t = sfa_t + 4;
+                    tmem_cp_sf(sfa_t, desc_sf(su32(sm.sfa[s])));
+                    tmem_cp_sf(sfb_t, desc_sf(su32(sm.sfb[s])));
+                    tmem_cp_sf(sfb_t + 4, desc_sf(su32(sm.sfb[s] + 512)));
+                    const uint32_t a_addr = su32(sm.a[s]), b_addr = su32(sm.b[s]);
+                    if (ks < a.st4) {  // four 4-bit blocks, one plane each
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        mma_mx(tmem + kAccCol, desc_sw128(a_addr + 32 * q), desc_sw128(b_addr + 32 * q), idesc(q, q),
-                               sfa_t, sfb_t, (ks > 0 || q > 0) ? 1u : 0u);
-                } else {  // two 6/8-bit blocks, high and low plane each
+                        for (int q = 0; q < 4; ++q)
+                            mma_mx(tmem + kAccCol, desc_sw128(a_addr + 32 * q), desc_sw128(b_addr + 32 * q),
+                                   idesc(q, q), sfa_t, sfb_t, (ks > 0 || q > 0) ? 1u : 0u);
+                    } else {  // two 6/8-bit blocks, high and low plane each
 #pragma unroll
-                    for (int j = 0; j < 2; ++j)
+                        for (int j = 0; j < 2; ++j)
 #pragma unroll
-                        for (int pp = 0; pp < 4; ++pp) {
-                            const int pa = pp >> 1, pb = pp & 1;
-                            mma_mx(tmem + kAccCol, desc_sw128(a_addr + 64 * j + 32 * pa),
-                                   desc_sw128(b_addr + 64 * j + 32 * pb), idesc(j, j), sfa_t, sfb_t,
-                                   (ks > 0 || j > 0 || pp > 0) ? 1u : 0u);
-                        }
+                            for (int pp = 0; pp < 4; ++pp) {
+                                const int pa = pp >> 1, pb = pp & 1;
+                                mma_mx(tmem + kAccCol, desc_sw128(a_addr + 64 * j + 32 * pa),
+                                       desc_sw128(b_addr + 64 * j + 32 * pb), idesc(j, j), sfa_t, sfb_t,
+                                       (ks > 0 || j > 0 || pp > 0) ? 1u : 0u);
+                            }
+                    }
+                    mma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
+                    committed = it + 1;
                 }
-                mma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
-                committed = ks + 1;
+                if (go) mma_commit(&sm.acc_full);  // the tile's accumulator is complete
             }
-            if (committed == nst) mma_commit(&sm.acc_full);
             // drain: wait (bounded) until the tensor core has finished what was issued
             if (committed > 0) {
-                const int ks = committed - 1;
+                const int k = committed - 1;
                 const long long t0 = clock64();
-                while (!mbar_try_wait(&sm.empty[ks % kStages], (ks / kStages) & 1) && clock64() - t0 < kWaitCycles) {
+                while (!mbar_try_wait(&sm.empty[k % kStages], (k / kStages) & 1) && clock64() - t0 < kWaitCycles) {
                 }
             }
         }
     } else {
         // ------------------------------------------------ epilogue (warps 2..5)
         const int quad = warp & 3;  // TMEM lane quadrant this warp may access
-        // one lane polls for the whole main loop, then every lane takes its own
-        // acquiring test; the decision is warp-uniform (tcgen05.ld is .sync.aligned)
-        bool ok = true;
-        if (lane == 0) ok = mbar_wait(&sm.acc_full, 0, abort);
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        if (ok) mbar_try_wait(&sm.acc_full, 0);
-        if (ok) {
+        const bool vec = ((a.ld_y & 3) == 0) && ((reinterpret_cast<uintptr_t>(a.y) & 15) == 0);
+        int lt = 0;
+        for (int id = blockIdx.x; id < tiles; id += gridDim.x, ++lt) {
+            int m0, n0;
+            tile_origin(id, m0, n0);
+            // one lane polls for the main loop, then every lane takes its own
+            // acquiring test; the decision is warp-uniform (tcgen05.ld is .sync.aligned)
+            bool ok = true;
+            if (lane == 0) ok = mbar_wait(&sm.acc_full, lt & 1, abort);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) break;
+            mbar_try_wait(&sm.acc_full, lt & 1);
             fence_after();
             const int row = m0 + 32 * quad + lane;
             float *yrow = a.y + (int64_t)row * a.ld_y;
-            const bool vec = ((a.ld_y & 3) == 0) && ((reinterpret_cast<uintptr_t>(a.y) & 15) == 0);
 #pragma unroll 1
             for (int c = 0; c < kBN / 32; ++c) {
                 uint32_t r[32];
@@ -292,6 +331,9 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
                     }
                 }
             }
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.acc_empty);  // this warp's quarter of the accumulator is read
         }
     }
 
@@ -331,8 +373,13 @@ int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packe
     const size_t smem = sizeof(Smem) + 1024;
     cudaError_t e = cudaFuncSetAttribute(gemm_prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(prefill smem)");
-    dim3 grid((unsigned)((N + kBN - 1) / kBN), (unsigned)((M + kBM - 1) / kBM));
-    if (grid.y > 65535) return fail(MXS_ERR_SHAPE, "M too large for the prefill grid");
+    const int64_t tiles = ((N + kBN - 1) / kBN) * ((M + kBM - 1) / kBM);
+    if (tiles > 0x7FFFFFFF) return fail(MXS_ERR_SHAPE, "M x N too large for the prefill grid");
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return cuda_fail(e, "cudaDeviceGetAttribute(SM count)");
+    dim3 grid((unsigned)std::min<int64_t>(tiles, std::max(1, sms)), 1);  // one persistent CTA per SM
     gemm_prefill_kernel<<<grid, 192, smem, st>>>(ta, tb, a);
     return cuda_fail(cudaGetLastError(), "gemm_prefill_kernel launch");
 }
