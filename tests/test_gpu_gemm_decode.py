@@ -239,3 +239,33 @@ def test_linear_decode_group(torch, M, shapes):
         U.check_gemm(got, ref, ab)
         single = mxs.linear_decode(x, bits, packed, N).cpu().numpy()
         U.check_gemm(got, single.astype(np.float64), ab)
+
+
+@pytest.mark.parametrize("M,N,nb", [(16, 1000, 128), (3, 4096, 448)])
+def test_linear_decode_workspace_garbage_reuse_and_graph_replay(torch, M, N, nb):
+    """The fused layer's workspace holds only what the same call writes: a
+    workspace full of garbage, the same workspace reused, and a CUDA graph
+    replaying the same call all give the same y, bit for bit."""
+    g = I.rng(70, M, N, nb)
+    bits = I.width_map(nb, 0.8, 0.15, 0.05, g)
+    xb, wb, codes, scales, packed = layer(torch, M, 32 * nb, N, bits, g)
+    x = U.to_dev_bf16(torch, xb)
+    ws = torch.randint(0, 256, (mxs.act_planes_bytes(M, 32 * nb, bits),), dtype=torch.uint8, device="cuda")
+    ys = [mxs.linear_decode(x, bits, packed, N, workspace=ws).cpu().numpy() for _ in range(3)]
+    ref, ab = oracle_full(xb, wb, bits)
+    U.check_gemm(ys[0], ref, ab)
+    assert all(np.array_equal(ys[0], y) for y in ys[1:])
+    y = torch.empty((M, N), dtype=torch.float32, device="cuda")
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        mxs.linear_decode(x, bits, packed, N, y=y, workspace=ws, stream=s)
+    s.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=s):
+        mxs.linear_decode(x, bits, packed, N, y=y, workspace=ws, stream=s)
+    for _ in range(3):
+        y.fill_(float("nan"))
+        graph.replay()
+        torch.cuda.synchronize()
+        assert np.array_equal(y.cpu().numpy(), ys[0])
