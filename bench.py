@@ -335,8 +335,8 @@ def run_ours(args):
         gemm_bytes = step_bytes
     launches_per_step = 2 * len(items)
     STAGES = [[0, 1, 2], [3], [4, 5], [6]]  # q k v | o | gate up | down: the projections of a stage share an input
-    if args.path == "grouped":
-        launches_per_step = len(items) + len(items) // 7 * len(STAGES)
+    if args.path == "grouped":  # per stage one quantizer launch and one GEMM launch
+        launches_per_step = 2 * len(items) // 7 * len(STAGES)
 
     # ---- the step as one CUDA graph.  Inputs are independent synthetic draws, so
     # for each M the graph runs all activation quantizations, then all GEMMs;
@@ -488,7 +488,7 @@ def run_ours(args):
                        "path": {"planes": "quantize to MMA planes, then GEMM over the planes (TMA)",
                                 "fused": "mxs_linear_decode: quantize + GEMM chained by programmatic dependent launch",
                                 "grouped": "mxs_linear_decode_group for q/k/v and gate/up (one GEMM launch per "
-                                           "group, the quantizers chained before it), mxs_linear_decode for o, down",
+                                           "group, after one quantizer launch for the group), mxs_linear_decode for o, down",
                                 "codes": "quantize to packed codes, GEMM over the codes"}[args.path],
                        "projections": [p[0] for p in I.LLAMA3_8B], "map_4_6_8": list(MAP),
                        "parallelism": f"replicas x{ws}", "l2": "inputs larger than L2 (packed weights "

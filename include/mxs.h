@@ -258,8 +258,8 @@ MXS_API int mxs_pack_weight_permuted(const void *w_bf16, int64_t N, int64_t K, i
  * weights, output and planes workspace), but their GEMMs are one kernel
  * launch: the set-up, the wait for the activations and the teardown are paid
  * once, and the CTAs are shared out among the problems by their weight bytes.
- * The activations of every problem are quantized first (one quantizer launch
- * each, chained by programmatic dependent launch), then the grouped GEMM.
+ * The activations of all problems are quantized first, in one quantizer
+ * launch, then the grouped GEMM runs as its programmatic dependent.
  * Same operands, layouts and contract as mxs_linear_decode (weights static;
  * 1 <= count <= 3; M <= 16, the same for every problem); every problem needs
  * its own workspace (mxs_act_planes_bytes(M, K, bits) bytes).  The K split of

@@ -110,6 +110,9 @@ int pack_weight_impl(const void *w, int64_t N, int64_t K, int64_t ld_w, const in
                      int rounding, int layout, void *packed, void *stream);
 int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rounding, void *codes,
                     uint8_t *scales, void *planes, cudaStream_t st, const int32_t *perm = nullptr);
+// the activations of up to three decode problems to MMA planes in one launch
+int launch_quantize_group(const Plan *const *plans, const void *const *x, const int64_t *ld, int64_t M, int rounding,
+                          void *const *planes, int count, cudaStream_t st);
 int launch_pack_weight(const Plan &p, const void *w, int64_t N, int64_t ld, int rounding, bool planes,
                        void *packed, cudaStream_t st, const int32_t *perm = nullptr);
 int64_t decode_workspace_bytes(const Plan &p, int64_t M, int64_t N);

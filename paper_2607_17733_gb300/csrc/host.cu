@@ -302,10 +302,12 @@ int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t 
     int rc = check_device();
     if (rc) return rc;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
-    for (int i = 0; i < count; ++i) {
-        rc = launch_quantize(plans[i], probs[i].x, M, probs[i].ld_x, rounding, nullptr, nullptr, probs[i].workspace, st);
-        if (rc) return rc;
-    }
+    const void *xs[3];
+    int64_t lds[3];
+    void *pls[3];
+    for (int i = 0; i < count; ++i) xs[i] = probs[i].x, lds[i] = probs[i].ld_x, pls[i] = probs[i].workspace;
+    rc = launch_quantize_group(pp, xs, lds, M, rounding, pls, count, st);  // one quantizer launch for the group
+    if (rc) return rc;
     rc = launch_gemm_decode_group(pp, planes, packed, N, y, ld_y, count, M, true, st);
     for (int i = 0; rc < 0 && i < count; ++i) {  // no grouped plan: one launch per problem
         const int r = launch_gemm_decode(plans[i], nullptr, nullptr, planes[i], packed[i], M, N[i], y[i], ld_y[i],

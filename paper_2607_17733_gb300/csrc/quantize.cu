@@ -79,15 +79,7 @@ __device__ __forceinline__ uint32_t bf2_clamp(uint32_t w, uint32_t hi, uint32_t 
 }
 
 template <bool kCodes, bool kPlanes, bool kRhaz, bool kPerm>
-__global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_constant__ Plan p,
-                                                                   const __grid_constant__ QuantArgs a) {
-    // Programmatic dependent launch, both ways: a decode GEMM launched after
-    // this kernel may start now (it waits for this grid before reading the
-    // planes), and this grid waits for the kernel before it (which may write
-    // x or still read the output buffers) before touching memory.
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-
+__device__ __forceinline__ void quantize_rows(const Plan &p, const QuantArgs &a) {
     // work slot vs -> real slot (or plane padding), its plane offset and its
     // scale byte (K' stage st, byte q of the stage's scale word)
     const int vs = blockIdx.x * blockDim.x + threadIdx.x;
@@ -289,7 +281,85 @@ __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_
     }
 }
 
+// Programmatic dependent launch, both ways: a decode GEMM launched after
+// these kernels may start at once (it waits for them before reading the
+// planes), and they wait for the kernel before them (which may write x or
+// still read the output buffers) before touching memory.
+template <bool kCodes, bool kPlanes, bool kRhaz, bool kPerm>
+__global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_constant__ Plan p,
+                                                                   const __grid_constant__ QuantArgs a) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    quantize_rows<kCodes, kPlanes, kRhaz, kPerm>(p, a);
+}
+
+// The activations of up to three decode layers that share a GEMM launch,
+// quantized to MMA planes in one launch (blockIdx.z = problem): one link in
+// the launch chain instead of one per problem.
+struct QuantGroup {
+    Plan p[3];
+    QuantArgs a[3];
+};
+template <bool kRhaz>
+__global__ void __launch_bounds__(kCtaThreads) quantize_act_group_kernel(const __grid_constant__ QuantGroup g) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    quantize_rows<false, true, kRhaz, false>(g.p[blockIdx.z], g.a[blockIdx.z]);
+}
+
+// CTA shape for rows of V work slots: one CTA of whole warps for short rows
+// (several rows to a CTA), else the fewest CTAs of at most 256 threads
+void quant_shape(int V, int64_t M, int &nx, int &tx, int &ry, int64_t &gy) {
+    nx = 1, ry = 1;
+    if (V <= kCtaThreads) {
+        tx = (V + 31) / 32 * 32;
+        ry = kCtaThreads / tx;
+    } else {
+        nx = (V + kCtaThreads - 1) / kCtaThreads;
+        tx = ((V + nx - 1) / nx + 31) / 32 * 32;
+    }
+    gy = std::min<int64_t>((M + ry - 1) / ry, 65535);
+}
+
 }  // namespace
+
+int launch_quantize_group(const Plan *const *plans, const void *const *x, const int64_t *ld, int64_t M, int rounding,
+                          void *const *planes, int count, cudaStream_t st) {
+    if (count < 1 || count > 3) return fail(MXS_ERR_INVALID_ARG, "quantize group of %d", count);
+    thread_local QuantGroup g;  // host staging of the parameter block (the launch copies it)
+    static_assert(sizeof(QuantGroup) < 32000, "kernel parameter block too large");
+    int Vmax = 0;
+    for (int i = 0; i < 3; ++i) {
+        const int k = i < count ? i : 0;
+        const Plan &p = *plans[k];
+        g.p[i] = p;
+        QuantArgs &a = g.a[i];
+        a = QuantArgs{};
+        a.x = static_cast<const uint16_t *>(x[k]);
+        a.M = M;
+        a.ld = ld[k];
+        a.planes = static_cast<uint8_t *>(planes[k]);
+        a.sf = a.planes + align256(M * p.kp);
+        a.V = 4 * p.st4 + 2 * ((p.n68 + 1) / 2);
+        Vmax = std::max(Vmax, a.V);
+    }
+    if (M == 0 || Vmax == 0) return MXS_OK;
+    int nx, tx, ry;
+    int64_t gy;
+    quant_shape(Vmax, M, nx, tx, ry, gy);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)nx, (unsigned)gy, (unsigned)count);
+    cfg.blockDim = dim3((unsigned)tx, (unsigned)ry, 1);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = rounding == MXS_RHAZ ? cudaLaunchKernelEx(&cfg, quantize_act_group_kernel<true>, g)
+                                               : cudaLaunchKernelEx(&cfg, quantize_act_group_kernel<false>, g);
+    return cuda_fail(e, "quantize_act_group_kernel launch");
+}
 
 int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rounding, void *codes,
                     uint8_t *scales, void *planes, cudaStream_t st, const int32_t *perm) {
@@ -304,17 +374,9 @@ int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rou
     a.sf = planes ? a.planes + align256(M * p.kp) : nullptr;
     a.V = planes ? 4 * p.st4 + 2 * ((p.n68 + 1) / 2) : p.nb;
     if (M == 0 || a.V == 0) return MXS_OK;
-    // a row's V lanes: one CTA of whole warps for short rows (several rows
-    // to a CTA), else the fewest CTAs of at most 256 threads, evenly filled
-    int nx = 1, tx, ry = 1;
-    if (a.V <= kCtaThreads) {
-        tx = (a.V + 31) / 32 * 32;
-        ry = kCtaThreads / tx;
-    } else {
-        nx = (a.V + kCtaThreads - 1) / kCtaThreads;
-        tx = ((a.V + nx - 1) / nx + 31) / 32 * 32;
-    }
-    const int64_t gy = std::min<int64_t>((M + ry - 1) / ry, 65535);
+    int nx, tx, ry;
+    int64_t gy;
+    quant_shape(a.V, M, nx, tx, ry, gy);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)nx, (unsigned)gy, 1);
     cfg.blockDim = dim3((unsigned)tx, (unsigned)ry, 1);
