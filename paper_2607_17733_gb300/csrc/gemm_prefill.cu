@@ -22,6 +22,8 @@
 // Every mbarrier wait is bounded; on expiry the kernel records MXS_ERR_TIMEOUT
 // in a device status word, stops issuing work, drains what it issued and frees
 // its tensor memory before returning.
+#include <cstring>
+
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -49,6 +51,7 @@ struct PrefillArgs {
     int64_t ld_y;
     int M, N, nst, st4, sfb_tiles;
     int starve;  // test hook: >0 makes the producer skip stage `starve-1` (the wait then times out)
+    int tma_y;   // y is written by TMA stores through tmap_y (16-byte aligned rows), else by plain stores
 };
 
 struct Smem {
@@ -56,6 +59,7 @@ struct Smem {
     uint8_t b[kStages][kBBytes];
     uint8_t sfa[kStages][kSfaBytes];
     uint8_t sfb[kStages][kSfbBytes];
+    uint8_t stage_y[4][32 * 128];  // per epilogue warp: a 32 x 32 fp32 output block, 128-byte swizzle (TMA store)
     uint64_t full[kStages], empty[kStages], acc_full, acc_empty;
     uint32_t tmem_base;
     int abort;
@@ -145,6 +149,17 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar))
                  : "memory");
 }
+// smem -> global tile store through a tensor map (clipped at the tensor's edges)
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, const void *src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(map),
+                 "r"(su32(src)), "r"(x), "r"(y)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// generic-proxy shared-memory writes -> visible to the bulk copy engine
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -162,6 +177,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
 
 __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_constant__ CUtensorMap tmap_a,
                                                               const __grid_constant__ CUtensorMap tmap_b,
+                                                              const __grid_constant__ CUtensorMap tmap_y,
                                                               const __grid_constant__ PrefillArgs a) {
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment for the 128B-swizzled operand tiles
@@ -299,6 +315,7 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
         // ------------------------------------------------ epilogue (warps 2..5)
         const int quad = warp & 3;  // TMEM lane quadrant this warp may access
         const bool vec = ((a.ld_y & 3) == 0) && ((reinterpret_cast<uintptr_t>(a.y) & 15) == 0);
+        uint8_t *stg = sm.stage_y[quad];
         int lt = 0;
         for (int id = blockIdx.x; id < tiles; id += gridDim.x, ++lt) {
             int m0, n0;
@@ -311,14 +328,37 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
             if (!ok) break;
             mbar_try_wait(&sm.acc_full, lt & 1);
             fence_after();
-            const int row = m0 + 32 * quad + lane;
+            const int row0 = m0 + 32 * quad, row = row0 + lane;
             float *yrow = a.y + (int64_t)row * a.ld_y;
 #pragma unroll 1
             for (int c = 0; c < kBN / 32; ++c) {
                 uint32_t r[32];
                 tmem_ld32(tmem + ((uint32_t)(32 * quad) << 16) + kAccCol + 32 * c, r);
+                if (c == kBN / 32 - 1) {  // the whole accumulator is in registers: the next tile may start
+                    fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sm.acc_empty);
+                }
                 const int n = n0 + 32 * c;
-                if (row < a.M) {
+                if (a.tma_y) {
+                    // 32 rows x 32 columns through the staging block: each lane
+                    // writes its row (16-byte chunk j at chunk j ^ (row & 7)),
+                    // one TMA store writes the block as whole 128-byte rows
+                    if (row0 < a.M && n < a.N) {
+                        if (lane == 0) bulk_wait_read0();  // the previous store has read the block
+                        __syncwarp();
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            *reinterpret_cast<uint4 *>(stg + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                                make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+                        fence_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(&tmap_y, stg, n, row0);
+                            bulk_commit();
+                        }
+                    }
+                } else if (row < a.M) {
                     if (vec && n + 32 <= a.N) {
 #pragma unroll
                         for (int i = 0; i < 8; ++i)
@@ -331,10 +371,8 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
                     }
                 }
             }
-            fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.acc_empty);  // this warp's quarter of the accumulator is read
         }
+        if (lane == 0) bulk_wait0();  // the stores have finished reading (and writing) before the CTA ends
     }
 
     fence_before();
@@ -370,6 +408,15 @@ int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packe
     a.st4 = p.st4;
     a.sfb_tiles = (int)((N + 127) / 128);
     a.starve = starve;
+    // y by TMA stores when its rows are 16-byte aligned (else plain stores)
+    CUtensorMap ty;
+    a.tma_y = ((ld_y & 3) == 0) && ((reinterpret_cast<uintptr_t>(y) & 15) == 0);
+    if (a.tma_y) {
+        rc = make_f32_out_map(&ty, y, M, N, ld_y);
+        if (rc) return rc;
+    } else {
+        std::memcpy(&ty, &ta, sizeof(CUtensorMap));  // unused
+    }
     const size_t smem = sizeof(Smem) + 1024;
     cudaError_t e = cudaFuncSetAttribute(gemm_prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(prefill smem)");
@@ -380,7 +427,7 @@ int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packe
     if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return cuda_fail(e, "cudaDeviceGetAttribute(SM count)");
     dim3 grid((unsigned)std::min<int64_t>(tiles, std::max(1, sms)), 1);  // one persistent CTA per SM
-    gemm_prefill_kernel<<<grid, 192, smem, st>>>(ta, tb, a);
+    gemm_prefill_kernel<<<grid, 192, smem, st>>>(ta, tb, ty, a);
     return cuda_fail(cudaGetLastError(), "gemm_prefill_kernel launch");
 }
 

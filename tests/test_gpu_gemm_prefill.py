@@ -49,14 +49,18 @@ def test_prefill_small(torch, M, N, nb, mp):
     print(f"prefill M={M} N={N} K={32 * nb} map={mp}: max err/abssum {err:.2e}")
 
 
-def test_prefill_through_mxs_gemm_and_stride(torch):
+@pytest.mark.parametrize("pad", [64, 3])
+def test_prefill_through_mxs_gemm_and_stride(torch, pad):
+    """Ragged M and N, y a view with row stride N + pad: rows of 16-byte
+    multiples go out through TMA stores (clipped at N and M), other strides
+    through plain stores; the padding columns stay untouched."""
     g = I.rng(21)
     bits = I.width_map(32, 0.8, 0.15, 0.05, g)
-    M, N = 200, 384
+    M, N = 200, 384 - 40
     xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=50.0)
     wb = I.normal_bf16((N, 1024), 0.02, g)
     planes, packed = prep(torch, xb, wb, bits)
-    y = torch.full((M, N + 64), -3.0, device="cuda")
+    y = torch.full((M, N + pad), -3.0, device="cuda")
     mxs.gemm(None, None, planes, bits, packed, N, w_layout=mxs.W_COMPACT_AND_PLANES, y=y[:, :N], M=M)
     yh = y.cpu().numpy()
     assert np.all(yh[:, N:] == -3.0)
