@@ -60,11 +60,17 @@
  *   MMA planes (layout MXS_W_COMPACT_AND_PLANES for weights, the `planes`
  *     output of mxs_quantize_act for activations), Kp = 128*(ceil(n4/4) +
  *     ceil((n6+n8)/2)):
- *       P [rows, Kp] e4m3: 4-bit slot s at bytes [32s, +32) = m/4; padding to
- *       a multiple of 4 slots is zero; 6/8-bit slot j at 128*ceil(n4/4)+64j:
- *       high digit then low digit (32 B each); b=6: m = 8h+l, digits h/2, l/16;
- *       b=8: m = 16h+l, digits h/4, l/64 (l >= 0), so that the two digits add
- *       up to m*2^-(b-2) and the block scale S applies to both unchanged.
+ *       P [rows, Kp]: 4-bit slot s at bytes [32s, +32) = e4m3 m/4; padding
+ *       to a multiple of 4 slots is zero; 6/8-bit slot j at 64 bytes from
+ *       128*ceil(n4/4)+64j, in one of two forms:
+ *         digit form (activations with M <= 16: the decode GEMM's operand):
+ *         high digit then low digit (e4m3, 32 B each); b=6: m = 8h+l, digits
+ *         h/2, l/16; b=8: m = 16h+l, digits h/4, l/64 (l >= 0), so that the
+ *         two digits add up to m*2^-(b-2) and the block scale S applies to
+ *         both unchanged;
+ *         bf16 form (activations with M > 16 and weights: the prefill GEMM's
+ *         operand): element i at +2i is the bf16 value m*2^(S-127-(b-2))
+ *         (exact), 0x7FC0 (NaN) in a block with S = 255.
  *       SF at align256(P + rows*Kp): per 128-row tile and 128-byte K' stage,
  *       512 B ordered [i<32][w<4][q<4] = S of row 128*tile+32w+i, slot 4*st+q
  *       (4-bit stages) or 2*(st-ceil(n4/4))+q for q<2 (6/8-bit stages); every
@@ -127,7 +133,9 @@ MXS_API int64_t mxs_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K, const 
  * Appendix A.2 activations quantized on the fly) and writes
  *   codes  [M, mxs_act_row_bytes]  packed codes (may be NULL)
  *   scales [M, K/32]               scale bytes by slot (NULL iff codes NULL)
- *   planes mxs_act_planes_bytes    MMA planes + scale tiles (may be NULL)
+ *   planes mxs_act_planes_bytes    MMA planes + scale tiles (may be NULL); 6/8-bit
+ *                                  blocks in digit form for M <= 16 (decode),
+ *                                  bf16 form for M > 16 (prefill)
  * At least one of codes / planes must be non-NULL. */
 MXS_API int mxs_quantize_act(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x,
                      const uint8_t *bits, int rounding,
@@ -206,14 +214,15 @@ MXS_API int mxs_linear_decode_noalloc(const void *x_bf16, int64_t M, int64_t K, 
                                       int rounding, const void *packed_w, int64_t N, float *y, int64_t ld_y,
                                       void *stream);
 
-/* Prefill path only (any M >= 1, efficient for M >= 128): the tensor-core
- * kernel over the MMA planes of the activations (mxs_quantize_act `planes`)
- * and of the weights (packed with MXS_W_COMPACT_AND_PLANES).  Sec. 6: the
- * mixed widths are executed on a fixed-width tensor core by splitting each
- * 6/8-bit mantissa into two exactly representable e4m3 digits (4 MMAs per
- * block pair, 1 for 4-bit blocks); scales are applied per 32-element block by
- * the block-scaled MMA (UE8M0).  Waits inside the kernel are bounded (about
- * 2 s); on expiry it records MXS_ERR_TIMEOUT (see mxs_device_status). */
+/* Prefill path only (M > 16; MXS_ERR_SHAPE for 1 <= M <= 16, whose planes
+ * hold the decode form): the tensor-core kernel over the MMA planes of the
+ * activations (mxs_quantize_act `planes`) and of the weights (packed with
+ * MXS_W_COMPACT_AND_PLANES).  The mixed widths run on fixed-width tensor
+ * cores in exact forms accumulated into one fp32 accumulator: 4-bit blocks as
+ * e4m3 m/4 on the block-scaled FP8 MMA (UE8M0 scale per 32 elements, one MMA
+ * per block), 6/8-bit blocks as their bf16 values on the bf16 MMA (two K=16
+ * MMAs per block).  Waits inside the kernel are bounded (about 2 s); on
+ * expiry it records MXS_ERR_TIMEOUT (see mxs_device_status). */
 MXS_API int mxs_gemm_prefill(const void *act_planes, const uint8_t *bits, const void *packed_w,
                              int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, void *stream);
 

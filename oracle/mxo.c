@@ -336,13 +336,19 @@ static int64_t weight_compact(int64_t N, int64_t n4, int64_t n68)
     return align256((N + 127) / 128 * group_bytes(n4, n68));
 }
 
-/* Planes: for every row, Kp = 128*(ceil(n4/4) + ceil(n68/2)) e4m3 bytes.
+/* Planes: for every row, Kp = 128*(ceil(n4/4) + ceil(n68/2)) bytes.
  * 4-bit slot s: bytes [32s, 32s+32) = e4m3(m/4).  Slots n4..4*ceil(n4/4)-1
- * are zero padding.  6/8-bit slot j at P68 = 128*ceil(n4/4): bytes
- * [P68+64j, +32) = high digit, [P68+64j+32, +32) = low digit, with
- * b=6: m = 8h + l (l in 0..7),  high = h/2, low = l/16;
- * b=8: m = 16h + l (l in 0..15), high = h/4, low = l/64.
- * so that high + low = m * 2^-(b-2) and the E8M0 scale S applies to both.
+ * are zero padding.  6/8-bit slot j at P68 = 128*ceil(n4/4), bytes
+ * [P68+64j, +64), in one of two forms:
+ *  - digit form: [P68+64j, +32) = high digit, [P68+64j+32, +32) = low digit
+ *    (e4m3), with
+ *      b=6: m = 8h + l (l in 0..7),  high = h/2, low = l/16;
+ *      b=8: m = 16h + l (l in 0..15), high = h/4, low = l/64.
+ *    so that high + low = m * 2^-(b-2) and the E8M0 scale S applies to both;
+ *  - bf16 form: element i is the bf16 value m * 2^(S-127-(b-2)) (exact: |m|
+ *    has at most 7 significant bits and bf16 keeps 8, with fp32's exponent
+ *    range and subnormals), little-endian at P68+64j+2i; a block with S = 255
+ *    (NaN/Inf) holds the bf16 NaN 0x7FC0.
  * Scale tiles SF: for row tile tau (128 rows) and stage st (one 128-byte
  * K' step: 4 slots of 4-bit or 2 slots of 6/8-bit), 512 bytes ordered
  * [i in 0..31][w in 0..3][q in 0..3]: the byte is S of row 128tau+32w+i,
@@ -389,6 +395,29 @@ int mxo_e4m3_encode(double v)
     return (sign ? 0x80 : 0) | code;
 }
 
+/* bf16 (1 sign, 8 exponent bits with bias 127, 7 fraction bits) encoding of a
+ * value that is exactly representable; returns -1 otherwise. */
+int mxo_bf16_encode(double v)
+{
+    if (v == 0.0) return signbit(v) ? 0x8000 : 0x0000;
+    int sign = v < 0.0;
+    double a = fabs(v);
+    int e;
+    double f = frexp(a, &e);
+    int E = e - 1;
+    int code;
+    if (E >= -126) { /* normal: a = (1 + k/128) * 2^E */
+        double k = (2.0 * f - 1.0) * 128.0;
+        if (k != floor(k) || E + 127 > 254) return -1;
+        code = ((E + 127) << 7) | (int)k;
+    } else { /* subnormal: a = k/128 * 2^-126 */
+        double k = ldexp(a, 133);
+        if (k != floor(k) || k < 1.0 || k > 127.0) return -1;
+        code = (int)k;
+    }
+    return (sign ? 0x8000 : 0) | code;
+}
+
 static int plane_digits(int b, int m, double *hi, double *lo)
 {
     if (b == 4) { *hi = m / 4.0; *lo = 0.0; return 1; }
@@ -400,9 +429,10 @@ static int plane_digits(int b, int m, double *hi, double *lo)
     return 2;
 }
 
-/* Planes [R, Kp] and scale tiles for R rows quantized with map bits. */
+/* Planes [R, Kp] and scale tiles for R rows quantized with map bits; 6/8-bit
+ * blocks in digit form (bf16_68 = 0) or bf16 form (bf16_68 = 1). */
 int mxo_planes(int64_t R, int64_t K, const uint8_t *bits, const uint8_t *scales,
-               const int8_t *codes, uint8_t *planes, uint8_t *sf)
+               const int8_t *codes, uint8_t *planes, uint8_t *sf, int bf16_68)
 {
     const int64_t nb = K / MXO_BLOCK;
     int32_t *sb = (int32_t *)malloc(sizeof(int32_t) * (size_t)(nb > 0 ? nb : 1));
@@ -417,6 +447,17 @@ int mxo_planes(int64_t R, int64_t K, const uint8_t *bits, const uint8_t *scales,
         for (int64_t s = 0; s < nb; ++s) {
             const int64_t kb = sb[s];
             const int b = bits[kb];
+            if (s >= n4 && bf16_68) {
+                const int S = scales[r * nb + kb];
+                for (int i = 0; i < MXO_BLOCK; ++i) {
+                    const int m = codes[r * K + kb * MXO_BLOCK + i];
+                    const int v = S == 255 ? 0x7FC0 : mxo_bf16_encode(ldexp((double)m, S - 127 - (b - 2)));
+                    if (v < 0) err = 1;
+                    planes[r * kp + p68 + 64 * (s - n4) + 2 * i] = (uint8_t)(v & 0xFF);
+                    planes[r * kp + p68 + 64 * (s - n4) + 2 * i + 1] = (uint8_t)((v >> 8) & 0xFF);
+                }
+                continue;
+            }
             for (int i = 0; i < MXO_BLOCK; ++i) {
                 double hi, lo;
                 plane_digits(b, codes[r * K + kb * MXO_BLOCK + i], &hi, &lo);
@@ -494,7 +535,7 @@ int mxo_pack_weight(int64_t N, int64_t K, const uint8_t *bits, const uint8_t *sc
     if (with_planes) {
         const int64_t kp = kp_bytes(n4, n68);
         const int64_t psf = align256(compact + N * kp);
-        err = mxo_planes(N, K, bits, scales, codes, out + compact, out + psf) != 0;
+        err = mxo_planes(N, K, bits, scales, codes, out + compact, out + psf, 1) != 0;  /* prefill operand */
     }
     free(sb);
     return err ? -1 : 0;

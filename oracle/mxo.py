@@ -74,7 +74,7 @@ def _load():
         lib.mxo_weight_bytes.restype = I64
         lib.mxo_e4m3_encode.argtypes = [ctypes.c_double]
         lib.mxo_e4m3_encode.restype = I
-        lib.mxo_planes.argtypes = [I64, I64, P, P, P, P, P]
+        lib.mxo_planes.argtypes = [I64, I64, P, P, P, P, P, I]
         lib.mxo_planes.restype = I
         lib.mxo_pack_weight.argtypes = [I64, I64, P, P, P, I, P]
         lib.mxo_pack_weight.restype = I
@@ -228,8 +228,10 @@ def plane_shape(bits):
     return 128 * nst, nst
 
 
-def planes(bits, scales, codes):
-    """(planes uint8 [R, Kp], scale tiles uint8 [ceil(R/128), nst, 512])."""
+def planes(bits, scales, codes, bf16_68: bool = False):
+    """(planes uint8 [R, Kp], scale tiles uint8 [ceil(R/128), nst, 512]).
+    6/8-bit blocks as high/low e4m3 digits, or (bf16_68) as bf16 values
+    m * 2^(S-127-(b-2)); see mxo.c."""
     bits = _c(bits, np.uint8)
     scales = _c(scales, np.uint8)
     codes = _c(codes, np.int8)
@@ -237,6 +239,6 @@ def planes(bits, scales, codes):
     kp, nst = plane_shape(bits)
     pl = np.zeros((R, kp), np.uint8)
     sf = np.zeros(((R + 127) // 128, nst, 512), np.uint8)
-    if _load().mxo_planes(R, K, _p(bits), _p(scales), _p(codes), _p(pl), _p(sf)) != 0:
+    if _load().mxo_planes(R, K, _p(bits), _p(scales), _p(codes), _p(pl), _p(sf), int(bool(bf16_68))) != 0:
         raise ValueError("mxo_planes failed")
     return pl, sf

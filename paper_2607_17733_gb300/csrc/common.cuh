@@ -88,6 +88,13 @@ __device__ __forceinline__ uint16_t e4m3x2(float lo, float hi) {
     return r;
 }
 
+// bf16 pair of two exactly representable values (lo in the low half)
+__device__ __forceinline__ uint32_t bf16x2(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
 // 2^e as fp32 for e in [-149, 127] (subnormal below -126), exact.
 __device__ __forceinline__ float pow2f(int e) {
     return e >= -126 ? __int_as_float((e + 127) << 23) : __int_as_float(1 << (e + 149 < 0 ? 0 : e + 149));

@@ -4,14 +4,15 @@
 // y[m,n] = sum over 32-element K-blocks of 2^(Ea+Ew) * sum_i (ma_i 2^-(b-2)) *
 // (mw_i 2^-(b-2)): the MXINT product of Sec. 2 with the widths of Sec. 4.1.
 // sm_103a has no integer tcgen05 MMA, so the integer mantissas enter the
-// block-scaled FP8 MMA (kind::mxf8f6f4, e4m3 x e4m3, one UE8M0 scale per 32
-// K-elements) as exact e4m3 "digit planes" -- the decomposition into high- and
-// low-precision parts that Sec. 6 describes for mixed-width execution:
-//   4-bit block:    one plane  m/4;
-//   6/8-bit block:  two planes, m*2^-(b-2) = high + low (both exact in e4m3),
-//                   four MMAs (hi*hi, hi*lo, lo*hi, lo*lo).
-// Every plane product is an exact small integer sum scaled by the block's own
-// scale bytes; the tensor core accumulates it into fp32 TMEM.
+// tensor core in exact floating-point forms, one accumulator for both:
+//   4-bit block:    one e4m3 plane m/4 on the block-scaled FP8 MMA
+//                   (kind::mxf8f6f4, one UE8M0 scale per 32 K-elements);
+//   6/8-bit block:  its values m * 2^(E-(b-2)) in bf16 (|m| <= 127 has at
+//                   most 7 significant bits, bf16 keeps 8 and fp32's exponent
+//                   range) on the bf16 MMA (kind::f16): two K=16 MMAs per
+//                   block, where high/low e4m3 digits would take four FP8
+//                   MMAs (Sec. 6's high/low split, kept for decode).
+// Every product is exact; the tensor core accumulates in fp32 TMEM.
 //
 // Structure (one 128x256 output tile per CTA, 192 threads):
 //   warp 0     TMA producer: 128-byte K' stages of A and W planes (128B swizzle)
@@ -140,6 +141,17 @@ __device__ __forceinline__ void mma_mx(uint32_t d, uint64_t a, uint64_t b, uint3
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
         " tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%5], [%6], p;\n}" ::"r"(d),
         "l"(a), "l"(b), "r"(id), "r"(accum), "r"(sfa), "r"(sfb)
+        : "memory");
+}
+// Instruction descriptor, kind::f16: f32 accumulator (bits 4-5 = 1), A and B
+// bf16 (bits 7-9, 10-12 = 1), K-major, N>>3 at 17, M>>4 at 24.
+constexpr uint32_t kIdescBf16 =
+    (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+__device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t accum) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %3, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %4, p;\n}" ::"r"(d),
+        "l"(a), "l"(b), "r"(accum), "r"(kIdescBf16)
         : "memory");
 }
 __device__ __forceinline__ void tmem_cp_sf(uint32_t taddr, uint64_t desc) {
@@ -298,26 +310,21 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
                         break;
                     }
                     fence_after();
-                    const uint32_t sfa_t = tmem + kSfCol + 12 * s, sfb_t = sfa_t + 4;
-                    tmem_cp_sf(sfa_t, desc_sf(su32(sm.sfa[s])));
-                    tmem_cp_sf(sfb_t, desc_sf(su32(sm.sfb[s])));
-                    tmem_cp_sf(sfb_t + 4, desc_sf(su32(sm.sfb[s] + 512)));
                     const uint32_t a_addr = su32(sm.a[s]), b_addr = su32(sm.b[s]);
-                    if (ks < a.st4) {  // four 4-bit blocks, one plane each
+                    if (ks < a.st4) {  // four 4-bit blocks, one e4m3 plane each, block-scaled
+                        const uint32_t sfa_t = tmem + kSfCol + 12 * s, sfb_t = sfa_t + 4;
+                        tmem_cp_sf(sfa_t, desc_sf(su32(sm.sfa[s])));
+                        tmem_cp_sf(sfb_t, desc_sf(su32(sm.sfb[s])));
+                        tmem_cp_sf(sfb_t + 4, desc_sf(su32(sm.sfb[s] + 512)));
 #pragma unroll
                         for (int q = 0; q < 4; ++q)
                             mma_mx(tmem + kAccCol, desc_sw128(a_addr + 32 * q), desc_sw128(b_addr + 32 * q),
                                    idesc(q, q), sfa_t, sfb_t, (ks > 0 || q > 0) ? 1u : 0u);
-                    } else {  // two 6/8-bit blocks, high and low plane each
+                    } else {  // two 6/8-bit blocks as bf16 values (scales inside): four K=16 MMAs
 #pragma unroll
-                        for (int j = 0; j < 2; ++j)
-#pragma unroll
-                            for (int pp = 0; pp < 4; ++pp) {
-                                const int pa = pp >> 1, pb = pp & 1;
-                                mma_mx(tmem + kAccCol, desc_sw128(a_addr + 64 * j + 32 * pa),
-                                       desc_sw128(b_addr + 64 * j + 32 * pb), idesc(j, j), sfa_t, sfb_t,
-                                       (ks > 0 || j > 0 || pp > 0) ? 1u : 0u);
-                            }
+                        for (int q = 0; q < 4; ++q)
+                            mma_bf16(tmem + kAccCol, desc_sw128(a_addr + 32 * q), desc_sw128(b_addr + 32 * q),
+                                     (ks > 0 || q > 0) ? 1u : 0u);
                     }
                     mma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
                     committed = it + 1;

@@ -382,6 +382,8 @@ static int prefill_checked(const void *act_planes, const uint8_t *bits, const vo
     int rc = build_plan(bits, K, &p);
     if (rc) return rc;
     if (M < 0 || N < 0) return fail(MXS_ERR_SHAPE, "M=%lld N=%lld", (long long)M, (long long)N);
+    if (M > 0 && M <= 16)  // such planes hold the decode GEMM's digit form of 6/8-bit blocks
+        return fail(MXS_ERR_SHAPE, "the prefill path takes M > 16 (M=%lld): use the decode path", (long long)M);
     if (!act_planes || !packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
     if (ld_y < N) return fail(MXS_ERR_INVALID_ARG, "ld_y=%lld < N", (long long)ld_y);
     if (!aligned16(act_planes) || !aligned16(packed_w) || (reinterpret_cast<uintptr_t>(y) & 3))

@@ -5,8 +5,8 @@
 // block).  One thread owns one (row, slot) block: it loads the 32 bf16 values
 // with four 128-bit loads and writes the row's sign-magnitude codes and scale
 // byte into its 128-row group (read by the decode kernel), and optionally the
-// e4m3
-// digit planes and scale tiles read by the tensor-core prefill kernel.  The
+// planes and scale tiles read by the tensor-core prefill kernel (4-bit blocks
+// as e4m3 m/4, 6/8-bit blocks as their bf16 values).  The
 // buffer is cleared first, so padding rows and slots read as zero.  This runs
 // once per layer and is not on the timed path.
 #include "common.cuh"
@@ -103,23 +103,13 @@ __global__ void __launch_bounds__(256) pack_weight_kernel(const __grid_constant_
             }
             st = s >> 2;
             q = s & 3;
-        } else {
+        } else {  // the block's values m * 2^(S-127-(b-2)) in bf16 (exact), NaN for S = 255
             const int j = s - p.n4;
-            const int sh = b == 6 ? 3 : 4;
-            const float fh = b == 6 ? 0.5f : 0.25f, fl = b == 6 ? 0.0625f : 0.015625f;
-            uint32_t *hi = reinterpret_cast<uint32_t *>(prow + 128 * (int64_t)p.st4 + 64 * (int64_t)j);
-            uint32_t *lo = hi + 8;
+            uint32_t *dst = reinterpret_cast<uint32_t *>(prow + 128 * (int64_t)p.st4 + 64 * (int64_t)j);
+            const float f = pow2f(S - 125 - b);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                int hd[4], ld[4];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    hd[k] = m[4 * i + k] >> sh;
-                    ld[k] = m[4 * i + k] & ((1 << sh) - 1);
-                }
-                hi[i] = e4m3x2(fh * hd[0], fh * hd[1]) | ((uint32_t)e4m3x2(fh * hd[2], fh * hd[3]) << 16);
-                lo[i] = e4m3x2(fl * ld[0], fl * ld[1]) | ((uint32_t)e4m3x2(fl * ld[2], fl * ld[3]) << 16);
-            }
+            for (int i = 0; i < 16; ++i)
+                dst[i] = S == 255 ? 0x7FC07FC0u : bf16x2((float)m[2 * i] * f, (float)m[2 * i + 1] * f);
             st = p.st4 + (j >> 1);
             q = j & 1;
         }

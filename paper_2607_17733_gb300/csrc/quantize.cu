@@ -46,6 +46,7 @@ struct QuantArgs {
     int V;  // work slots per row (with plane padding when planes are written)
     uint8_t *codes, *scales, *planes, *sf;
     const int32_t *perm;  // column order (Alg. 3): block kb holds columns perm[32 kb ..], or nullptr
+    int bf16_68;          // planes of 6/8-bit blocks as bf16 values (the prefill operand), else e4m3 digits
 };
 
 // low bytes of four words, in order
@@ -160,6 +161,7 @@ __device__ __forceinline__ void quantize_rows(const Plan &p, const QuantArgs &a)
         }
 
         uint4 pl[4];  // 4-bit: plane halves in pl[0..1]; 6/8-bit: hi halves pl[0..1], lo halves pl[2..3]
+                      // (bf16 form: elements 0-15 in pl[0..1], 16-31 in pl[2..3])
         uint4 cd[2];  // codes: 4-bit in cd[0]; 8-bit halves in cd[0..1]
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -219,6 +221,15 @@ __device__ __forceinline__ void quantize_rows(const Plan &p, const QuantArgs &a)
                     }
                     pl[h] = make_uint4(c[0] | (c[1] << 16), c[2] | (c[3] << 16), c[4] | (c[5] << 16),
                                        c[6] | (c[7] << 16));
+                } else if (a.bf16_68) {  // the block's values m * 2^(S-127-(b-2)) in bf16 (exact)
+                    const float fs = pow2f(S - 125 - b);
+                    uint32_t cw[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        cw[i] = S == 255 ? 0x7FC07FC0u
+                                         : bf16x2((tf[2 * i] - kMagic) * fs, (tf[2 * i + 1] - kMagic) * fs);
+                    pl[2 * h] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
+                    pl[2 * h + 1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
                 } else {  // m = 2^sh * hi + lo: planes hi * 2^sh * fl and lo * fl
                     const uint32_t mask = b == 6 ? 7u : 15u;
                     const float fl = b == 6 ? 0.0625f : 0.015625f;
@@ -372,6 +383,7 @@ int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rou
     a.scales = scales;
     a.planes = static_cast<uint8_t *>(planes);
     a.sf = planes ? a.planes + align256(M * p.kp) : nullptr;
+    a.bf16_68 = M > 16;  // more than 16 rows are the prefill GEMM's operand
     a.V = planes ? 4 * p.st4 + 2 * ((p.n68 + 1) / 2) : p.nb;
     if (M == 0 || a.V == 0) return MXS_OK;
     int nx, tx, ry;

@@ -103,24 +103,16 @@ def e4m3_value(code):
 E4M3_TABLE = np.array([e4m3_value(c) for c in range(256)])
 
 
-def decode_planes(bits, planes, sf):
-    """planes [R,Kp] + scale tiles -> (scales [R,nb], codes [R,K]) natural order."""
+def decode_planes(bits, planes, sf, bf16_68=False):
+    """planes [R,Kp] + scale tiles -> (scales [R,nb], codes [R,K]) natural order.
+    6/8-bit blocks as high/low e4m3 digits, or (bf16_68) as bf16 values
+    m * 2^(S-127-(b-2))."""
     sb, (n4, n6, n8) = slot_blocks(bits)
     n68 = n6 + n8
     st4 = (n4 + 3) // 4
     nst = st4 + (n68 + 1) // 2
     R = planes.shape[0]
     nb = len(bits)
-    codes = np.zeros((R, 32 * nb), np.int8)
-    vals = E4M3_TABLE[planes]
-    for s, kb in enumerate(sb):
-        b = int(bits[kb])
-        if s < n4:
-            v = vals[:, 32 * s:32 * s + 32]
-        else:
-            off = 128 * st4 + 64 * (s - n4)
-            v = vals[:, off:off + 32] + vals[:, off + 32:off + 64]
-        codes[:, 32 * kb:32 * kb + 32] = np.rint(v * 2.0 ** (b - 2)).astype(np.int8)
     # scale tiles: [tau][st][i][w][q] -> row 128 tau + 32 w + i
     tiles = sf.reshape(-1, nst, 32, 4, 4)
     scales = np.zeros((R, nb), np.uint8)
@@ -132,4 +124,21 @@ def decode_planes(bits, planes, sf):
         col = tiles[:, st, :, :, qq]            # [tau, i, w]
         rows = col.transpose(0, 2, 1).reshape(-1)  # row = 128 tau + 32 w + i
         scales[:, kb] = rows[:R]
+    codes = np.zeros((R, 32 * nb), np.int8)
+    vals = E4M3_TABLE[planes]
+    for s, kb in enumerate(sb):
+        b = int(bits[kb])
+        if s < n4:
+            v = vals[:, 32 * s:32 * s + 32]
+        elif bf16_68:
+            off = 128 * st4 + 64 * (s - n4)
+            h = planes[:, off:off + 64].copy().view(np.uint16).astype(np.uint32) << 16
+            f = h.view(np.float32).astype(np.float64)
+            e = scales[:, kb].astype(np.float64) - 127.0
+            v = f * np.exp2(-e)[:, None]
+            v = np.where(scales[:, kb][:, None] == 255, 0.0, v)  # NaN blocks hold zero codes
+        else:
+            off = 128 * st4 + 64 * (s - n4)
+            v = vals[:, off:off + 32] + vals[:, off + 32:off + 64]
+        codes[:, 32 * kb:32 * kb + 32] = np.rint(v * 2.0 ** (b - 2)).astype(np.int8)
     return scales, codes

@@ -32,7 +32,7 @@ def run_quantize(torch, xb, bits, rounding=mxs.RNE, planes=True, ld=None):
 def oracle_quantize(xb, bits, rounding=mxo.RNE):
     s, c = mxo.quantize_bf16(xb, bits, rounding)
     pc, ps = mxo.pack_act(bits, s, c)
-    pl, sf = mxo.planes(bits, s, c)
+    pl, sf = mxo.planes(bits, s, c, bf16_68=xb.shape[0] > 16)  # more than 16 rows: the prefill operand form
     return pc, ps, pl, sf
 
 

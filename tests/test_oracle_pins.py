@@ -318,6 +318,31 @@ def test_plane_digits_cover_every_code(b):
     assert np.all(lo >= 0)
 
 
+@pytest.mark.parametrize("b", [6, 8])
+def test_plane_bf16_form_is_the_exact_block_value(b):
+    """bf16 form of a 6/8-bit block: every m in [-Q, Q] under scale bytes
+    from the bottom (subnormal results) to the top of the range is the bf16
+    whose value is exactly m * 2^(S-127-(b-2)) (compared with numpy's exact
+    fp64 ldexp), and the NaN scale byte gives bf16 NaN."""
+    Q = 2 ** (b - 1) - 1
+    bits = np.full(1, b, np.uint8)
+    m = np.arange(-Q, Q + 1)
+    for S in (0, 1, 7, 100, 127, 200, 254, 255):
+        codes = np.zeros((2 * Q + 1, 32), np.int8)
+        codes[:, 0] = m
+        codes[:, 31] = -m
+        scales = np.full((2 * Q + 1, 1), S, np.uint8)
+        pl, _ = mxo.planes(bits, scales, codes, bf16_68=True)
+        h = pl[:, :64].copy().view(np.uint16)
+        got = (h.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+        if S == 255:
+            assert np.all(h == 0x7FC0)
+            continue
+        want = np.ldexp(m.astype(np.float64), S - 127 - (b - 2))
+        assert np.array_equal(got[:, 0], want) and np.array_equal(got[:, 31], -want)
+        assert np.all(got[:, 1:31] == 0)
+
+
 def _random_quantized(seed, R, nb, p=(0.6, 0.25, 0.15)):
     g = I.rng(seed, 7)
     bits = I.width_map(nb, *p, g)
@@ -346,8 +371,11 @@ def test_pack_weight_round_trip(N):
     pl = buf[compact:compact + N * kp].reshape(N, kp)
     sf_off = mxformat.align256(compact + N * kp)
     sf = buf[sf_off:sf_off + ((N + 127) // 128) * nst * 512]
-    s3, c3 = mxformat.decode_planes(bits, pl, sf)
+    s3, c3 = mxformat.decode_planes(bits, pl, sf, bf16_68=True)  # weight planes: 6/8-bit blocks as bf16
     assert np.array_equal(s3, scales) and np.array_equal(c3, codes)
+    pd, sfd = mxo.planes(bits, scales, codes)  # digit form (decode operand)
+    s4, c4 = mxformat.decode_planes(bits, pd, sfd.reshape(-1))
+    assert np.array_equal(s4, scales) and np.array_equal(c4, codes)
 
 
 def test_storage_accounting_matches_paper_scale_overhead():
