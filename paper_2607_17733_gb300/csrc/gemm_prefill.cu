@@ -36,13 +36,21 @@ __device__ int g_prefill_status;  // sticky MXS_ERR_TIMEOUT, read by mxs_device_
 
 namespace {
 
-constexpr int kBM = 128, kBN = 256, kBK = 128;  // tile rows (A), tile rows (W), K' bytes per stage
-constexpr int kStages = 4;
+// Output tiles of 128 x BN, BN = 256, or 128 when 256-wide tiles would leave
+// SMs idle (fewer tiles than SMs).  Ring stages: 4 of 48 KB (BN = 256) or 6 of
+// 32 KB (BN = 128).
+constexpr int kBM = 128, kBK = 128;  // tile rows (A), K' bytes per stage
+template <int BN> struct Tile {
+    static constexpr int kStages = BN == 256 ? 4 : 6;
+    static constexpr int kBBytes = BN * kBK;
+    static constexpr int kSfbBytes = BN / 128 * 512;
+    static constexpr int kSfCols = 4 + BN / 32;  // TMEM columns per stage: SFA 4, SFB 4 per 128 rows
+};
 constexpr int kBandM = 16;  // row tiles per band of the tile order
-constexpr int kABytes = kBM * kBK, kBBytes = kBN * kBK;  // 16 KB, 32 KB
-constexpr int kSfaBytes = 512, kSfbBytes = 1024;
+constexpr int kABytes = kBM * kBK;  // 16 KB
+constexpr int kSfaBytes = 512;
 constexpr int kTmemCols = 512;
-constexpr int kAccCol = 0, kSfCol = 256;  // per stage: SFA 4 columns, SFB 8 columns
+constexpr int kAccCol = 0, kSfCol = 256;  // accumulator BN columns; scale factors from column 256
 constexpr long long kWaitCycles = 4000000000ll;  // ~2 s at the maximum SM clock  // 2 s bound on any single wait
 
 struct PrefillArgs {
@@ -55,13 +63,15 @@ struct PrefillArgs {
     int tma_y;   // y is written by TMA stores through tmap_y (16-byte aligned rows), else by plain stores
 };
 
+template <int BN>
 struct Smem {
-    uint8_t a[kStages][kABytes];
-    uint8_t b[kStages][kBBytes];
-    uint8_t sfa[kStages][kSfaBytes];
-    uint8_t sfb[kStages][kSfbBytes];
+    static constexpr int S = Tile<BN>::kStages;
+    uint8_t a[S][kABytes];
+    uint8_t b[S][Tile<BN>::kBBytes];
+    uint8_t sfa[S][kSfaBytes];
+    uint8_t sfb[S][Tile<BN>::kSfbBytes];
     uint8_t stage_y[4][32 * 128];  // per epilogue warp: a 32 x 32 fp32 output block, 128-byte swizzle (TMA store)
-    uint64_t full[kStages], empty[kStages], acc_full, acc_empty;
+    uint64_t full[S], empty[S], acc_full, acc_empty;
     uint32_t tmem_base;
     int abort;
 };
@@ -130,9 +140,10 @@ __device__ __forceinline__ uint64_t desc_sf(uint32_t addr) {  // 32 rows x 16 B,
 
 // Instruction descriptor, kind::mxf8f6f4: A/B e4m3 (0), K-major, N>>3 at 17,
 // UE8M0 scales (bit 23), M>>4 at 24, scale-factor byte ids at [4,6) (B) and [29,31) (A).
-constexpr uint32_t kIdesc = ((uint32_t)(kBN >> 3) << 17) | (1u << 23) | ((uint32_t)(kBM >> 4) << 24);
+template <int BN>
 __device__ __forceinline__ uint32_t idesc(int sfa_id, int sfb_id) {
-    return kIdesc | ((uint32_t)sfb_id << 4) | ((uint32_t)sfa_id << 29);
+    return ((uint32_t)(BN >> 3) << 17) | (1u << 23) | ((uint32_t)(kBM >> 4) << 24) | ((uint32_t)sfb_id << 4) |
+           ((uint32_t)sfa_id << 29);
 }
 
 __device__ __forceinline__ void mma_mx(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t sfa, uint32_t sfb,
@@ -145,13 +156,14 @@ __device__ __forceinline__ void mma_mx(uint32_t d, uint64_t a, uint64_t b, uint3
 }
 // Instruction descriptor, kind::f16: f32 accumulator (bits 4-5 = 1), A and B
 // bf16 (bits 7-9, 10-12 = 1), K-major, N>>3 at 17, M>>4 at 24.
-constexpr uint32_t kIdescBf16 =
-    (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+template <int BN>
 __device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t accum) {
+    constexpr uint32_t id =
+        (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
     asm volatile(
         "{\n .reg .pred p;\n setp.ne.b32 p, %3, 0;\n"
         " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %4, p;\n}" ::"r"(d),
-        "l"(a), "l"(b), "r"(accum), "r"(kIdescBf16)
+        "l"(a), "l"(b), "r"(accum), "r"(id)
         : "memory");
 }
 __device__ __forceinline__ void tmem_cp_sf(uint32_t taddr, uint64_t desc) {
@@ -208,6 +220,7 @@ __device__ __forceinline__ void tmem_ld128(uint32_t taddr, uint32_t (&r)[128]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+template <int BN>
 __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_constant__ CUtensorMap tmap_a,
                                                               const __grid_constant__ CUtensorMap tmap_b,
                                                               const __grid_constant__ CUtensorMap tmap_y,
@@ -215,7 +228,8 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment for the 128B-swizzled operand tiles
     const uint32_t base = su32(smem_raw);
-    Smem &sm = *reinterpret_cast<Smem *>(smem_raw + (((base + 1023) & ~1023u) - base));
+    constexpr int kStages = Tile<BN>::kStages;
+    Smem<BN> &sm = *reinterpret_cast<Smem<BN> *>(smem_raw + (((base + 1023) & ~1023u) - base));
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // Persistent: CTA c takes tiles c, c + gridDim.x, ... of the tile order:
@@ -223,13 +237,13 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
     // running at a time share few weight tiles (each read from DRAM about once
     // per band) and the band's activation tiles stay in L2.  The producer runs
     // ahead into the next tile while the epilogue drains the accumulator.
-    const int mt = (a.M + kBM - 1) / kBM, nt = (a.N + kBN - 1) / kBN, tiles = mt * nt;
+    const int mt = (a.M + kBM - 1) / kBM, nt = (a.N + BN - 1) / BN, tiles = mt * nt;
     auto tile_origin = [&](int id, int &m0, int &n0) {
         const int band = id / (kBandM * nt);
         const int first = band * kBandM, gm = min(kBandM, mt - first);
         const int in = id - band * kBandM * nt;
         m0 = (first + in % gm) * kBM;
-        n0 = (in / gm) * kBN;
+        n0 = (in / gm) * BN;
     };
     const int nst = a.nst;
 
@@ -265,8 +279,8 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
                 int m0, n0;
                 tile_origin(id, m0, n0);
                 const int tile_a = m0 / 128, tile_b = n0 / 128;
-                const bool two_b = tile_b + 1 < a.sfb_tiles;
-                const uint32_t tx = kABytes + kBBytes + kSfaBytes + (two_b ? 2 : 1) * 512;
+                const bool two_b = BN == 256 && tile_b + 1 < a.sfb_tiles;
+                const uint32_t tx = kABytes + Tile<BN>::kBBytes + kSfaBytes + (two_b ? 2 : 1) * 512;
                 for (int ks = 0; ks < nst; ++ks, ++it) {
                     const int s = it % kStages;
                     const uint32_t ph = (it / kStages) & 1;
@@ -312,19 +326,19 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
                     fence_after();
                     const uint32_t a_addr = su32(sm.a[s]), b_addr = su32(sm.b[s]);
                     if (ks < a.st4) {  // four 4-bit blocks, one e4m3 plane each, block-scaled
-                        const uint32_t sfa_t = tmem + kSfCol + 12 * s, sfb_t = sfa_t + 4;
+                        const uint32_t sfa_t = tmem + kSfCol + Tile<BN>::kSfCols * s, sfb_t = sfa_t + 4;
                         tmem_cp_sf(sfa_t, desc_sf(su32(sm.sfa[s])));
                         tmem_cp_sf(sfb_t, desc_sf(su32(sm.sfb[s])));
-                        tmem_cp_sf(sfb_t + 4, desc_sf(su32(sm.sfb[s] + 512)));
+                        if (BN == 256) tmem_cp_sf(sfb_t + 4, desc_sf(su32(sm.sfb[s] + 512)));
 #pragma unroll
                         for (int q = 0; q < 4; ++q)
                             mma_mx(tmem + kAccCol, desc_sw128(a_addr + 32 * q), desc_sw128(b_addr + 32 * q),
-                                   idesc(q, q), sfa_t, sfb_t, (ks > 0 || q > 0) ? 1u : 0u);
+                                   idesc<BN>(q, q), sfa_t, sfb_t, (ks > 0 || q > 0) ? 1u : 0u);
                     } else {  // two 6/8-bit blocks as bf16 values (scales inside): four K=16 MMAs
 #pragma unroll
                         for (int q = 0; q < 4; ++q)
-                            mma_bf16(tmem + kAccCol, desc_sw128(a_addr + 32 * q), desc_sw128(b_addr + 32 * q),
-                                     (ks > 0 || q > 0) ? 1u : 0u);
+                            mma_bf16<BN>(tmem + kAccCol, desc_sw128(a_addr + 32 * q), desc_sw128(b_addr + 32 * q),
+                                         (ks > 0 || q > 0) ? 1u : 0u);
                     }
                     mma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
                     committed = it + 1;
@@ -358,13 +372,13 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
             fence_after();
             const int row0 = m0 + 32 * quad, row = row0 + lane;
             float *yrow = a.y + (int64_t)row * a.ld_y;
-            // two halves of 128 columns: the accumulator is free for the next
-            // tile once the second half is in registers
+            // BN/128 parts of 128 columns: the accumulator is free for the next
+            // tile once the last part is in registers
 #pragma unroll 1
-            for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < BN / 128; ++h) {
                 uint32_t r[128];
                 tmem_ld128(tmem + ((uint32_t)(32 * quad) << 16) + kAccCol + 128 * h, r);
-                if (h == 1) {
+                if (h == BN / 128 - 1) {
                     fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&sm.acc_empty);
@@ -419,18 +433,39 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
     }
 }
 
+template <int BN>
+int launch_tiles(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap &ty, const PrefillArgs &a,
+                 int64_t tiles, int sms, cudaStream_t st) {
+    const size_t smem = sizeof(Smem<BN>) + 1024;
+    cudaError_t e = cudaFuncSetAttribute(gemm_prefill_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(prefill smem)");
+    dim3 grid((unsigned)std::min<int64_t>(tiles, std::max(1, sms)), 1);  // one persistent CTA per SM
+    gemm_prefill_kernel<BN><<<grid, 192, smem, st>>>(ta, tb, ty, a);
+    return cuda_fail(cudaGetLastError(), "gemm_prefill_kernel launch");
+}
+
 }  // namespace
 
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N, float *y,
                         int64_t ld_y, int starve, cudaStream_t st) {
     if (M > 0x7FFFFFF0 || N > 0x7FFFFFF0) return fail(MXS_ERR_SHAPE, "M or N too large");
+    int dev = 0, sms = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return cuda_fail(e, "cudaDeviceGetAttribute(SM count)");
+    // 256-wide tiles unless they would leave SMs idle
+    const int64_t mt = (M + kBM - 1) / kBM;
+    const int BN = mt * ((N + 255) / 256) >= sms ? 256 : 128;
+    const int64_t tiles = mt * ((N + BN - 1) / BN);
+    if (tiles > 0x7FFFFFFF) return fail(MXS_ERR_SHAPE, "M x N too large for the prefill grid");
     const uint8_t *ap = static_cast<const uint8_t *>(act_planes);
     const uint8_t *wb = static_cast<const uint8_t *>(packed_w);
     const WeightOffsets off = weight_offsets(p, N, true);
     CUtensorMap ta, tb;
     int rc = make_plane_map(&ta, ap, M, p.kp, kBM);
     if (rc) return rc;
-    rc = make_plane_map(&tb, wb + off.planes, N, p.kp, kBN);
+    rc = make_plane_map(&tb, wb + off.planes, N, p.kp, BN);
     if (rc) return rc;
     PrefillArgs a;
     a.sfa = ap + align256(M * p.kp);
@@ -452,18 +487,7 @@ int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packe
     } else {
         std::memcpy(&ty, &ta, sizeof(CUtensorMap));  // unused
     }
-    const size_t smem = sizeof(Smem) + 1024;
-    cudaError_t e = cudaFuncSetAttribute(gemm_prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(prefill smem)");
-    const int64_t tiles = ((N + kBN - 1) / kBN) * ((M + kBM - 1) / kBM);
-    if (tiles > 0x7FFFFFFF) return fail(MXS_ERR_SHAPE, "M x N too large for the prefill grid");
-    int dev = 0, sms = 0;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
-        return cuda_fail(e, "cudaDeviceGetAttribute(SM count)");
-    dim3 grid((unsigned)std::min<int64_t>(tiles, std::max(1, sms)), 1);  // one persistent CTA per SM
-    gemm_prefill_kernel<<<grid, 192, smem, st>>>(ta, tb, ty, a);
-    return cuda_fail(cudaGetLastError(), "gemm_prefill_kernel launch");
+    return BN == 256 ? launch_tiles<256>(ta, tb, ty, a, tiles, sms, st) : launch_tiles<128>(ta, tb, ty, a, tiles, sms, st);
 }
 
 int prefill_status(int *status, int reset, cudaStream_t st) {
