@@ -204,3 +204,13 @@ def test_decode_group_validation(L):
     assert call([prob(), prob(workspace=ws2, packed_w=FAKE + 4)]) == 4
     assert call([prob(), prob()]) == 1 and "share a workspace" in mxs.last_error()
     assert call([prob(N=-1)]) == 2
+
+
+def test_prefill_rejects_decode_sized_m(L):
+    """Planes of M <= 16 rows hold the decode form of 6/8-bit blocks, so the
+    prefill GEMM refuses them before any device call; M = 0 is a no-op."""
+    bits = np.full(4, 6, np.uint8)
+    b = bits.ctypes.data
+    for M in (1, 16):
+        assert L.mxs_gemm_prefill(FAKE, b, FAKE, M, 16, 128, FAKE, 16, None) == 2
+        assert "M > 16" in mxs.last_error()

@@ -49,6 +49,31 @@ def test_prefill_small(torch, M, N, nb, mp):
     print(f"prefill M={M} N={N} K={32 * nb} map={mp}: max err/abssum {err:.2e}")
 
 
+def test_prefill_special_blocks(torch):
+    """NaN and Inf in 4-, 6- and 8-bit blocks of activations and weights: the
+    outputs that read such a block are NaN (R5: scale byte 255, zero codes;
+    the bf16 form of a 6/8-bit block holds NaN), all others match the oracle;
+    all-zero and subnormal blocks quantize like any other."""
+    bits = np.array([4, 6, 8, 4, 6, 8, 4, 4], np.uint8)
+    g = I.rng(33)
+    M, N = 40, 150
+    xb = I.activations_bf16(M, bits, g, 0.0)
+    wb = I.normal_bf16((N, 32 * len(bits)), 0.02, g)
+    xb[3, 40] = 0x7FC0    # NaN in the 6-bit block of token 3
+    xb[7, 70] = 0x7F80    # +Inf in the 8-bit block of token 7
+    xb[11, 5] = 0xFF80    # -Inf in a 4-bit block of token 11
+    xb[20, 32 * 4:32 * 5] = 0        # an all-zero 6-bit block
+    xb[21, 32 * 2:32 * 3] = 0x0003   # a subnormal 8-bit block
+    wb[9, 32 * 5 + 3] = 0x7FC0       # NaN in the 8-bit block of output 9
+    planes, packed = prep(torch, xb, wb, bits)
+    y = mxs.gemm_prefill(planes, bits, packed, M, N).cpu().numpy()
+    ref, ab = oracle_entries(xb, wb, bits)
+    for r in (3, 7, 11):
+        assert np.all(np.isnan(y[r]))
+    assert np.all(np.isnan(y[:, 9]))
+    U.check_gemm(y, ref, ab)
+
+
 @pytest.mark.parametrize("pad", [64, 3])
 def test_prefill_through_mxs_gemm_and_stride(torch, pad):
     """Ragged M and N, y a view with row stride N + pad: rows of 16-byte
