@@ -591,7 +591,7 @@ def run_prefill(args):
         print(json.dumps({
             "metric": "mxint_prefill_gemm_tops", "value": value, "unit": "TOPS", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "e4m3 digit planes + f32",
+            "scaling": "weak", "vs_baseline": None, "dtype": "e4m3 (4-bit blocks) + bf16 (6/8-bit blocks), f32 accumulation",
             "data": "synthetic (seeded; W N(0,0.02), A N(0,1) with Student-t(3) outlier channels on 0.5% of K)",
             "config": {"workload": "llama3-8b-prefill", "M": M, "layers": L, "map_4_6_8": [0.8, 0.15, 0.05],
                        "l2": "inputs larger than L2"},
