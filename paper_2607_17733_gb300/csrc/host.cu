@@ -332,6 +332,36 @@ int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t 
     return rc;
 }
 
+int mxs_quantize_act_group(const mxs_quant_problem *probs, int count, int64_t M, int rounding, void *stream) {
+    if (!probs || count < 1 || count > 3) return fail(MXS_ERR_INVALID_ARG, "count=%d (1..3 problems)", count);
+    if (M < 0) return fail(MXS_ERR_SHAPE, "M=%lld", (long long)M);
+    if (rounding != MXS_RNE && rounding != MXS_RHAZ) return fail(MXS_ERR_INVALID_ARG, "rounding=%d", rounding);
+    Plan plans[3];
+    const Plan *pp[3];
+    const void *xs[3];
+    int64_t lds[3];
+    void *pls[3];
+    for (int i = 0; i < count; ++i) {
+        const mxs_quant_problem &q = probs[i];
+        int rc = build_plan(q.bits, q.K, &plans[i]);
+        if (rc) return rc;
+        if (!q.x || !q.planes) return fail(MXS_ERR_INVALID_ARG, "problem %d: NULL x or planes", i);
+        if (q.ld_x < q.K || q.ld_x % 8 != 0)
+            return fail(MXS_ERR_INVALID_ARG, "problem %d: ld_x=%lld must be >= K and a multiple of 8", i, (long long)q.ld_x);
+        if (!aligned16(q.x) || !aligned16(q.planes)) return fail(MXS_ERR_ALIGN, "problem %d: x and planes must be 16-byte aligned", i);
+        for (int j = 0; j < i; ++j)
+            if (probs[j].planes == q.planes) return fail(MXS_ERR_INVALID_ARG, "problems %d and %d share planes", j, i);
+        pp[i] = &plans[i];
+        xs[i] = q.x;
+        lds[i] = q.ld_x;
+        pls[i] = q.planes;
+    }
+    if (M == 0) return MXS_OK;
+    const int rc = check_device();
+    if (rc) return rc;
+    return launch_quantize_group(pp, xs, lds, M, rounding, pls, count, static_cast<cudaStream_t>(stream));
+}
+
 int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits, int rounding,
                       const void *packed_w, int64_t N, float *y, int64_t ld_y, void *ws, size_t ws_bytes,
                       void *stream) {

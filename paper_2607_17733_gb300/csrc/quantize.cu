@@ -304,9 +304,10 @@ __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_
     quantize_rows<kCodes, kPlanes, kRhaz, kPerm>(p, a);
 }
 
-// The activations of up to three decode layers that share a GEMM launch,
-// quantized to MMA planes in one launch (blockIdx.z = problem): one link in
-// the launch chain instead of one per problem.
+// The activations of up to three layers (a grouped decode GEMM, or prefill
+// layers that read one hidden state), quantized to MMA planes in one launch
+// (blockIdx.z = problem): one link in the launch chain instead of one per
+// problem.
 struct QuantGroup {
     Plan p[3];
     QuantArgs a[3];
@@ -352,6 +353,7 @@ int launch_quantize_group(const Plan *const *plans, const void *const *x, const 
         a.planes = static_cast<uint8_t *>(planes[k]);
         a.sf = a.planes + align256(M * p.kp);
         a.V = 4 * p.st4 + 2 * ((p.n68 + 1) / 2);
+        a.bf16_68 = M > 16;  // more than 16 rows are the prefill GEMM's operand
         Vmax = std::max(Vmax, a.V);
     }
     if (M == 0 || Vmax == 0) return MXS_OK;

@@ -28,7 +28,7 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode",
            "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer",
            "mxs_quantize_act_permuted", "mxs_pack_weight_permuted", "mxs_attention_decode_workspace_bytes",
-           "mxs_attention_decode", "mxs_linear_decode_group",
+           "mxs_attention_decode", "mxs_linear_decode_group", "mxs_quantize_act_group",
            "mxs_attention_decode_batch_workspace_bytes", "mxs_attention_decode_batch"]
 
 _lock = threading.Lock()
@@ -95,6 +95,8 @@ def lib() -> ctypes.CDLL:
         L.mxs_allocate_layer.restype = I
         L.mxs_linear_decode_group.argtypes = [P, I, I64, I, P]
         L.mxs_linear_decode_group.restype = I
+        L.mxs_quantize_act_group.argtypes = [P, I, I64, I, P]
+        L.mxs_quantize_act_group.restype = I
         L.mxs_attention_decode_workspace_bytes.argtypes = [I64, I64, I64]
         L.mxs_attention_decode_workspace_bytes.restype = I64
         L.mxs_attention_decode.argtypes = [P, I64, I64, I64, P, P, P, P, P, P, I64, ctypes.c_float, P, P, SZ, P]
@@ -294,6 +296,29 @@ def linear_decode_group(problems, rounding: int = RNE, stream=None):
         arr[i] = DecodeProblem(_ptr(x), x.shape[1], _ld(x), b.ptr, _ptr(packed_w), N, _ptr(y), _ld(y), _ptr(ws),
                                ws.numel() * ws.element_size())
     check(lib().mxs_linear_decode_group(ctypes.addressof(arr), len(problems), M, rounding, _stream(stream)))
+
+
+class QuantProblem(ctypes.Structure):
+    """ctypes mirror of mxs_quant_problem (include/mxs.h)."""
+    _fields_ = [("x", ctypes.c_void_p), ("K", ctypes.c_int64), ("ld_x", ctypes.c_int64), ("bits", ctypes.c_void_p),
+                ("planes", ctypes.c_void_p)]
+
+
+def quantize_act_group(problems, rounding: int = RNE, stream=None):
+    """MMA planes of up to three activations in one launch (mxs_quantize_act_group).
+    problems: sequence of (x [M, K] bf16, bits, planes uint8 of act_planes_bytes(M, K, bits)).
+    Returns the planes tensors."""
+    arr = (QuantProblem * len(problems))()
+    keep = []
+    M = problems[0][0].shape[0]
+    for i, (x, bits, planes) in enumerate(problems):
+        b = _Bits(bits)
+        keep.append(b)
+        if x.shape[0] != M:
+            raise ValueError("every problem of a group has the same M")
+        arr[i] = QuantProblem(_ptr(x), x.shape[1], _ld(x), b.ptr, _ptr(planes))
+    check(lib().mxs_quantize_act_group(ctypes.addressof(arr), len(problems), M, rounding, _stream(stream)))
+    return [p[2] for p in problems]
 
 
 def linear_decode_noalloc(x, bits, packed_w, N: int, rounding: int = RNE, y=None, stream=None):

@@ -214,3 +214,33 @@ def test_prefill_rejects_decode_sized_m(L):
     for M in (1, 16):
         assert L.mxs_gemm_prefill(FAKE, b, FAKE, M, 16, 128, FAKE, 16, None) == 2
         assert "M > 16" in mxs.last_error()
+
+
+def test_quantize_group_validation(L):
+    """mxs_quantize_act_group checks every problem before any device call."""
+    bits = np.full(4, 4, np.uint8)
+    b = bits.ctypes.data
+
+    def prob(**kw):
+        f = dict(x=FAKE, K=128, ld_x=128, bits=b, planes=FAKE)
+        f.update(kw)
+        return mxs.QuantProblem(**f)
+
+    def call(probs, M=4, rounding=0, count=None):
+        arr = (mxs.QuantProblem * max(1, len(probs)))(*probs)
+        return L.mxs_quantize_act_group(ctypes.addressof(arr), len(probs) if count is None else count, M,
+                                        rounding, None)
+
+    p2 = FAKE + (1 << 16)
+    bad = np.full(4, 5, np.uint8)
+    assert call([prob()], count=0) == 1
+    assert call([prob(), prob(planes=p2), prob(planes=2 * p2)], count=4) == 1
+    assert call([prob()], M=-1) == 2
+    assert call([prob()], rounding=2) == 1
+    assert call([prob(), prob(planes=p2, K=100)]) == 2
+    assert call([prob(), prob(planes=p2, bits=bad.ctypes.data)]) == 3
+    assert call([prob(), prob(planes=p2, ld_x=132)]) == 1
+    assert call([prob(), prob(planes=p2, x=None)]) == 1
+    assert call([prob(), prob(planes=p2 + 8)]) == 4
+    assert call([prob(), prob()]) == 1 and "share planes" in mxs.last_error()
+    assert call([prob()], M=0) == 0

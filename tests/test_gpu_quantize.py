@@ -155,3 +155,41 @@ def test_pack_weight_full_size_sampled(torch):
     torch.cuda.synchronize()
     s, c = mxo.quantize_bf16(wb, bits)
     assert np.array_equal(packed.cpu().numpy(), mxo.pack_weight(bits, s, c, True))
+
+
+@pytest.mark.parametrize("M", [5, 300])
+def test_quantize_group_matches_single_launches(torch, M):
+    """mxs_quantize_act_group writes, for every problem, the same planes and
+    scale tiles as mxs_quantize_act of that problem alone (three widths maps
+    and K's; digit form for M <= 16, bf16 form above)."""
+    shapes = [(4096, (0.8, 0.15, 0.05)), (1024, (0.5, 0.3, 0.2)), (2080, (0.9, 0.05, 0.05))]
+    probs, singles, xbs = [], [], []
+    for i, (K, p) in enumerate(shapes):
+        g = I.rng(90, M, K, i)
+        bits = I.width_map(K // 32, *p, g)
+        xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=40.0)
+        x = U.to_dev_bf16(torch, xb)
+        pl = torch.full((mxs.act_planes_bytes(M, K, bits),), 0xAB, dtype=torch.uint8, device="cuda")
+        probs.append((x, bits, pl))
+        xbs.append(xb)
+        _, _, one = mxs.quantize_act(x, bits, want_codes=False, want_planes=True)
+        singles.append(one)
+    mxs.quantize_act_group(probs)
+    torch.cuda.synchronize()
+    for (x, bits, pl), one, xb in zip(probs, singles, xbs):
+        K = x.shape[1]
+        kp = mxo.plane_shape(bits)[0]
+        got, want = pl.cpu().numpy(), one.cpu().numpy()
+        assert np.array_equal(got[:M * kp], want[:M * kp])
+        off = (M * kp + 255) // 256 * 256
+        nst = kp // 128
+        tiles_g = got[off:off + ((M + 127) // 128) * nst * 512].reshape(-1, nst, 32, 4, 4)
+        tiles_w = want[off:off + ((M + 127) // 128) * nst * 512].reshape(-1, nst, 32, 4, 4)
+        rows = 128 * np.arange(tiles_g.shape[0])[:, None, None, None, None] + 32 * np.arange(4)[None, None, None, :, None] \
+            + np.arange(32)[None, None, :, None, None]
+        valid = np.broadcast_to(rows < M, tiles_g.shape)
+        assert np.array_equal(tiles_g[valid], tiles_w[valid])
+        # and the oracle agrees
+        s_, c_ = mxo.quantize_bf16(xb, bits)
+        pl_o, _ = mxo.planes(bits, s_, c_, bf16_68=M > 16)
+        assert np.array_equal(got[:M * kp].reshape(M, kp), pl_o)
