@@ -141,6 +141,6 @@ int prefill_status(int *status, int reset, cudaStream_t st);
 // boxes of 128 bytes x box_rows rows, 128-byte swizzle, zero fill outside
 int make_plane_map(CUtensorMap *map, const void *base, int64_t rows, int64_t kp, int box_rows);
 // 2-D TMA map over an fp32 output y [rows, cols] (row stride ld elements, a
-// multiple of 4; base 16-byte aligned): 32 x 32 boxes, 128-byte swizzle
+// multiple of 4; base 16-byte aligned): boxes of 32 rows x 16 columns
 int make_f32_out_map(CUtensorMap *map, float *base, int64_t rows, int64_t cols, int64_t ld);
 }  // namespace mxs

@@ -14,12 +14,13 @@
 //                   MMAs (Sec. 6's high/low split, kept for decode).
 // Every product is exact; the tensor core accumulates in fp32 TMEM.
 //
-// Structure (one 128x256 output tile per CTA, 192 threads):
+// Structure (one 128x256 output tile per CTA, 320 threads):
 //   warp 0     TMA producer: 128-byte K' stages of A and W planes (128B swizzle)
 //              plus the scale tiles (1-D bulk copies), into a 4-stage ring;
 //   warp 1     TMEM owner and MMA issuer: tcgen05.cp scales -> TMEM, then the
 //              MMAs of the stage, tcgen05.commit frees the stage;
-//   warps 2-5  epilogue: tcgen05.ld the fp32 accumulator, store y.
+//   warps 2-9  epilogue: tcgen05.ld the fp32 accumulator (two warps per TMEM
+//              lane quarter, 128 columns each), TMA-store y.
 // Every mbarrier wait is bounded; on expiry the kernel records MXS_ERR_TIMEOUT
 // in a device status word, stops issuing work, drains what it issued and frees
 // its tensor memory before returning.
@@ -40,6 +41,7 @@ namespace {
 // SMs idle (fewer tiles than SMs).  Ring stages: 4 of 48 KB (BN = 256) or 6 of
 // 32 KB (BN = 128).
 constexpr int kBM = 128, kBK = 128;  // tile rows (A), K' bytes per stage
+constexpr int kPrefillThreads = 320;  // producer, MMA issuer, 8 epilogue warps (two per TMEM lane quarter)
 template <int BN> struct Tile {
     static constexpr int kStages = BN == 256 ? 4 : 6;
     static constexpr int kBBytes = BN * kBK;
@@ -70,7 +72,7 @@ struct Smem {
     uint8_t b[S][Tile<BN>::kBBytes];
     uint8_t sfa[S][kSfaBytes];
     uint8_t sfb[S][Tile<BN>::kSfbBytes];
-    uint8_t stage_y[4][32 * 128];  // per epilogue warp: a 32 x 32 fp32 output block, 128-byte swizzle (TMA store)
+    uint8_t stage_y[8][32 * 64];  // per epilogue warp: a 32 x 16 fp32 output block (TMA store)
     uint64_t full[S], empty[S], acc_full, acc_empty;
     uint32_t tmem_base;
     int abort;
@@ -221,7 +223,7 @@ __device__ __forceinline__ void tmem_ld128(uint32_t taddr, uint32_t (&r)[128]) {
 }
 
 template <int BN>
-__global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_constant__ CUtensorMap tmap_a,
+__global__ void __launch_bounds__(kPrefillThreads, 1) gemm_prefill_kernel(const __grid_constant__ CUtensorMap tmap_a,
                                                               const __grid_constant__ CUtensorMap tmap_b,
                                                               const __grid_constant__ CUtensorMap tmap_y,
                                                               const __grid_constant__ PrefillArgs a) {
@@ -253,7 +255,7 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
             mbar_init(&sm.empty[s], 1);
         }
         mbar_init(&sm.acc_full, 1);
-        mbar_init(&sm.acc_empty, 4);  // the four epilogue warps have read the accumulator
+        mbar_init(&sm.acc_empty, 4 * (BN / 128));  // the epilogue warps with columns have read them
         sm.abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -354,12 +356,16 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
             }
         }
     } else {
-        // ------------------------------------------------ epilogue (warps 2..5)
-        const int quad = warp & 3;  // TMEM lane quadrant this warp may access
+        // ------------------------------------------------ epilogue (warps 2..9)
+        // Warp w reads TMEM lane quarter w % 4 (the quarter a warp may access)
+        // and columns [128 h, 128 h + 128), h = (w - 2) / 4: one 128-column
+        // load, then the accumulator part is released and written out.
+        const int quad = warp & 3, half = (warp - 2) >> 2;
         const bool vec = ((a.ld_y & 3) == 0) && ((reinterpret_cast<uintptr_t>(a.y) & 15) == 0);
-        uint8_t *stg = sm.stage_y[quad];
+        uint8_t *stg = sm.stage_y[warp - 2];
         int lt = 0;
-        for (int id = blockIdx.x; id < tiles; id += gridDim.x, ++lt) {
+        // (128-wide tiles: the warps of the second column half have no work)
+        for (int id = half < BN / 128 ? (int)blockIdx.x : tiles; id < tiles; id += gridDim.x, ++lt) {
             int m0, n0;
             tile_origin(id, m0, n0);
             // one lane polls for the main loop, then every lane takes its own
@@ -372,51 +378,43 @@ __global__ void __launch_bounds__(192, 1) gemm_prefill_kernel(const __grid_const
             fence_after();
             const int row0 = m0 + 32 * quad, row = row0 + lane;
             float *yrow = a.y + (int64_t)row * a.ld_y;
-            // BN/128 parts of 128 columns: the accumulator is free for the next
-            // tile once the last part is in registers
-#pragma unroll 1
-            for (int h = 0; h < BN / 128; ++h) {
-                uint32_t r[128];
-                tmem_ld128(tmem + ((uint32_t)(32 * quad) << 16) + kAccCol + 128 * h, r);
-                if (h == BN / 128 - 1) {
-                    fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&sm.acc_empty);
-                }
+            uint32_t r[128];
+            tmem_ld128(tmem + ((uint32_t)(32 * quad) << 16) + kAccCol + 128 * half, r);
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.acc_empty);  // this part of the accumulator is in registers
 #pragma unroll
-                for (int cc = 0; cc < 4; ++cc) {
-                    const int n = n0 + 128 * h + 32 * cc;
-                    if (a.tma_y) {
-                        // 32 rows x 32 columns through the staging block: each lane
-                        // writes its row (16-byte chunk j at chunk j ^ (row & 7)),
-                        // one TMA store writes the block as whole 128-byte rows
-                        if (row0 < a.M && n < a.N) {
-                            if (lane == 0) bulk_wait_read0();  // the previous store has read the block
-                            __syncwarp();
+            for (int cc = 0; cc < 8; ++cc) {
+                const int n = n0 + 128 * half + 16 * cc;
+                if (a.tma_y) {
+                    // 32 rows x 16 columns through the staging block (row r at
+                    // 64 r), one TMA store writes it as 64-byte row pieces
+                    if (row0 < a.M && n < a.N) {
+                        if (lane == 0) bulk_wait_read0();  // the previous store has read the block
+                        __syncwarp();
 #pragma unroll
-                            for (int j = 0; j < 8; ++j)
-                                *reinterpret_cast<uint4 *>(stg + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-                                    make_uint4(r[32 * cc + 4 * j], r[32 * cc + 4 * j + 1], r[32 * cc + 4 * j + 2],
-                                               r[32 * cc + 4 * j + 3]);
-                            fence_async_smem();
-                            __syncwarp();
-                            if (lane == 0) {
-                                tma_store_2d(&tmap_y, stg, n, row0);
-                                bulk_commit();
-                            }
+                        for (int j = 0; j < 4; ++j)
+                            *reinterpret_cast<uint4 *>(stg + lane * 64 + 16 * j) =
+                                make_uint4(r[16 * cc + 4 * j], r[16 * cc + 4 * j + 1], r[16 * cc + 4 * j + 2],
+                                           r[16 * cc + 4 * j + 3]);
+                        fence_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(&tmap_y, stg, n, row0);
+                            bulk_commit();
                         }
-                    } else if (row < a.M) {
-                        if (vec && n + 32 <= a.N) {
+                    }
+                } else if (row < a.M) {
+                    if (vec && n + 16 <= a.N) {
 #pragma unroll
-                            for (int i = 0; i < 8; ++i)
-                                *reinterpret_cast<uint4 *>(yrow + n + 4 * i) =
-                                    make_uint4(r[32 * cc + 4 * i], r[32 * cc + 4 * i + 1], r[32 * cc + 4 * i + 2],
-                                               r[32 * cc + 4 * i + 3]);
-                        } else {
+                        for (int i = 0; i < 4; ++i)
+                            *reinterpret_cast<uint4 *>(yrow + n + 4 * i) =
+                                make_uint4(r[16 * cc + 4 * i], r[16 * cc + 4 * i + 1], r[16 * cc + 4 * i + 2],
+                                           r[16 * cc + 4 * i + 3]);
+                    } else {
 #pragma unroll
-                            for (int i = 0; i < 32; ++i)
-                                if (n + i < a.N) yrow[n + i] = __uint_as_float(r[32 * cc + i]);
-                        }
+                        for (int i = 0; i < 16; ++i)
+                            if (n + i < a.N) yrow[n + i] = __uint_as_float(r[16 * cc + i]);
                     }
                 }
             }
@@ -440,7 +438,7 @@ int launch_tiles(const CUtensorMap &ta, const CUtensorMap &tb, const CUtensorMap
     cudaError_t e = cudaFuncSetAttribute(gemm_prefill_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(prefill smem)");
     dim3 grid((unsigned)std::min<int64_t>(tiles, std::max(1, sms)), 1);  // one persistent CTA per SM
-    gemm_prefill_kernel<BN><<<grid, 192, smem, st>>>(ta, tb, ty, a);
+    gemm_prefill_kernel<BN><<<grid, kPrefillThreads, smem, st>>>(ta, tb, ty, a);
     return cuda_fail(cudaGetLastError(), "gemm_prefill_kernel launch");
 }
 
