@@ -157,8 +157,8 @@ def test_pack_weight_full_size_sampled(torch):
     assert np.array_equal(packed.cpu().numpy(), mxo.pack_weight(bits, s, c, True))
 
 
-@pytest.mark.parametrize("M", [5, 300])
-def test_quantize_group_matches_single_launches(torch, M):
+@pytest.mark.parametrize("M,rounding", [(5, mxs.RNE), (300, mxs.RNE), (300, mxs.RHAZ)])
+def test_quantize_group_matches_single_launches(torch, M, rounding):
     """mxs_quantize_act_group writes, for every problem, the same planes and
     scale tiles as mxs_quantize_act of that problem alone (three widths maps
     and K's; digit form for M <= 16, bf16 form above)."""
@@ -172,9 +172,9 @@ def test_quantize_group_matches_single_launches(torch, M):
         pl = torch.full((mxs.act_planes_bytes(M, K, bits),), 0xAB, dtype=torch.uint8, device="cuda")
         probs.append((x, bits, pl))
         xbs.append(xb)
-        _, _, one = mxs.quantize_act(x, bits, want_codes=False, want_planes=True)
+        _, _, one = mxs.quantize_act(x, bits, rounding=rounding, want_codes=False, want_planes=True)
         singles.append(one)
-    mxs.quantize_act_group(probs)
+    mxs.quantize_act_group(probs, rounding=rounding)
     torch.cuda.synchronize()
     for (x, bits, pl), one, xb in zip(probs, singles, xbs):
         K = x.shape[1]
@@ -190,6 +190,6 @@ def test_quantize_group_matches_single_launches(torch, M):
         valid = np.broadcast_to(rows < M, tiles_g.shape)
         assert np.array_equal(tiles_g[valid], tiles_w[valid])
         # and the oracle agrees
-        s_, c_ = mxo.quantize_bf16(xb, bits)
+        s_, c_ = mxo.quantize_bf16(xb, bits, mxo.RHAZ if rounding == mxs.RHAZ else mxo.RNE)
         pl_o, _ = mxo.planes(bits, s_, c_, bf16_68=M > 16)
         assert np.array_equal(got[:M * kp].reshape(M, kp), pl_o)
