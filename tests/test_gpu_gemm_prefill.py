@@ -112,6 +112,27 @@ def test_prefill_full_size_sampled(torch, shape):
     print(f"prefill {name}: max err/abssum {err:.2e}")
 
 
+@pytest.mark.parametrize("maps", ["u6", "u8", "50/30/20-clustered"])
+def test_prefill_sweep_shape_sampled(torch, maps):
+    """Bitwidth-sweep shape K=8192, N=28672, M=4096 with the maps that are all
+    (or mostly) bf16-form 6/8-bit blocks, 1% outlier columns x50: 96 sampled
+    rows x 512 sampled columns against the oracle."""
+    K, N, M = 8192, 28672, 4096
+    g = I.rng(5, len(maps))
+    p = {"u6": (0, 1, 0), "u8": (0, 0, 1), "50/30/20-clustered": (0.5, 0.3, 0.2)}[maps]
+    bits = I.width_map(K // 32, *p, g, clustered=maps.endswith("clustered"))
+    xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=50.0)
+    wb = I.normal_bf16((N, K), 0.02, g)
+    planes, packed = prep(torch, xb, wb, bits)
+    y = mxs.gemm_prefill(planes, bits, packed, M, N).cpu().numpy()
+    rs = np.random.default_rng(3)
+    rows = np.sort(rs.choice(M, 96, replace=False))
+    cols = np.sort(rs.choice(N, 512, replace=False))
+    ref, ab = oracle_entries(xb, wb, bits, rows, cols)
+    err = U.check_gemm(y[np.ix_(rows, cols)], ref, ab)
+    print(f"prefill sweep {maps}: max err/abssum {err:.2e}")
+
+
 def test_prefill_bounded_wait_reports_timeout(torch):
     """A stage that is never loaded: the kernel gives up after its wait bound,
     records MXS_ERR_TIMEOUT, frees its tensor memory and the context stays usable."""
