@@ -287,15 +287,18 @@ typedef struct mxs_decode_problem {
     size_t ws_bytes;
 } mxs_decode_problem;
 MXS_API int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t M, int rounding, void *stream);
-/* mxs_quantize_act_group -- the MMA planes of up to three activations with M
- * rows each (the inputs of linear layers that read the same hidden state:
- * q, k and v; gate and up), each with its own width map, in one kernel
- * launch: byte for byte what mxs_quantize_act(x_i, M, K_i, ld_i, bits_i,
- * rounding, NULL, NULL, planes_i) writes (digit form for M <= 16, bf16 form
- * of the 6/8-bit blocks for M > 16), one link in the launch chain instead of
- * one per layer.  planes_i: device, mxs_act_planes_bytes(M, K_i, bits_i)
- * bytes, 16-byte aligned, distinct buffers.  1 <= count <= 3.  Errors as
- * mxs_quantize_act, per problem (the message names it). */
+/* mxs_quantize_act_group -- A1 (the activations of every linear layer are
+ * quantized on the fly, Appendix A.2; one width per 32-element block, Sec.
+ * 4.1) for up to three activations with M rows each (the inputs of linear
+ * layers that read the same hidden state: q, k and v; gate and up), each with
+ * its own width map, in one kernel launch: byte for byte what
+ * mxs_quantize_act(x_i, M, K_i, ld_i, bits_i, rounding, NULL, NULL, planes_i)
+ * writes (digit form for M <= 16, bf16 form of the 6/8-bit blocks for
+ * M > 16), one link in the launch chain instead of one per layer.
+ * planes_i: device, mxs_act_planes_bytes(M, K_i, bits_i) bytes, 16-byte
+ * aligned, distinct buffers.  1 <= count <= 3.  Asynchronous on `stream`
+ * (programmatic dependent launch as mxs_quantize_act); allocates nothing.
+ * Errors as mxs_quantize_act, per problem (the message names it). */
 typedef struct mxs_quant_problem {
     const void *x;         /* device, bf16 [M, K], row stride ld_x (>= K, a multiple of 8) */
     int64_t K, ld_x;
