@@ -1,21 +1,27 @@
 #!/usr/bin/env python
 """Benchmark of the MXINT mixed-precision linear layer (MXSens) on GB300.
 
-Default workload (LLaMA-3-8B-shaped decode): for M in {1, 4, 16} tokens, the
-seven projections (q, k, v, o: 4096x4096 / 4096x1024; gate, up: 4096x14336;
-down: 14336x4096) of all 32 decoder layers; width map 85/10/5 % (4/6/8 bits)
-per projection, weights N(0, 0.02), activations N(0, 1) with 1 % outlier
-columns x30.  One step = for every (M, layer, projection): quantize the
-activations (A1) and run the MXINT GEMM (A4); weights are packed once (A2).
-The step is captured in a CUDA graph and replayed.  The 4.2 GB of packed
-weights a step streams is far larger than L2, so no flush is needed.
+Default workload (LLaMA-2-70B-shaped, the largest configuration): hidden 8192,
+MLP 28672, GQA k/v 8192x1024; 80 synthetic decoder layers whose width maps
+run from 60 % 4-bit (layer 0) to 95 % 4-bit (layer 79), 8-bit blocks over the
+1 % outlier columns (x50) of the activations, weights N(0, 0.015).
 
-Metric: GB/s of algorithmic traffic (packed weights + bf16 activations read +
-fp32 outputs written) per second, whole job; TOPS (2*M*N*K per second) is
-reported beside it.
+  value (decode): for M in {1, 16} tokens, the seven projections of all 80
+    layers; per decoder layer one quantizer launch + one grouped GEMM launch
+    for q/k/v and for gate/up, and one fused quantize + GEMM for o and down.
+    Weights are packed once (A2, 44 GB); the step is captured in a CUDA graph
+    and replayed.  Metric: GB/s of algorithmic traffic (packed weights + bf16
+    activations read + fp32 outputs written) per second, whole job.
+  prefill (object in the same line): M = 4096 tokens through the seven
+    projections of 4 layers spread over the depth (0, 26, 53, 79); per stage
+    of projections that read one hidden state one quantizer launch to MMA
+    planes, then the tcgen05 GEMMs.  Effective TOPS = 2*M*N*K per second,
+    with the GEMMs' roofline and the quantizer's HBM roofline.
 
---impl reference times the CPU oracle (the paper publishes no kernel to run)
-on a bounded sample of the same workload, on the host cores.
+--workload also offers the LLaMA-3-8B decode / prefill / calibration / KV
+attention workloads.  --impl reference times the CPU oracle (the paper
+publishes no kernel to run) on a bounded sample of the same workload, on the
+host cores.
 """
 from __future__ import annotations
 
@@ -36,25 +42,70 @@ sys.path.insert(0, ROOT)
 
 from paper_2607_17733_gb300 import inputs as I  # noqa: E402
 
-DECODE_MS = (1, 4, 16)
-MAP = (0.85, 0.10, 0.05)
-W_SIGMA = 0.02
-OUTLIER_FRAC, OUTLIER_SCALE = 0.01, 30.0
 SEED = 2607
-SAMPLE_ROWS = 2048
+STAGES = [[0, 1, 2], [3], [4, 5], [6]]  # q k v | o | gate up | down: the projections of a stage share an input
+
+
+class Spec:
+    """A decode or prefill workload: the model's projection shapes, how many
+    decoder layers, the width map of each projection, the weight and
+    activation distributions."""
+
+    def __init__(self, name, shapes, layers, Ms, w_sigma, outlier_frac, outlier_scale, map_fn, student_t=False,
+                 layer_ids=None, sample_cols=2048):
+        self.name, self.shapes, self.layers, self.Ms = name, shapes, layers, tuple(Ms)
+        self.w_sigma, self.outlier_frac, self.outlier_scale = w_sigma, outlier_frac, outlier_scale
+        self.map_fn, self.student_t = map_fn, student_t
+        self.layer_ids = list(layer_ids) if layer_ids is not None else list(range(layers))
+        self.sample_cols = sample_cols
+
+    def bits(self, rank, l, pi, K):
+        return self.map_fn(K, l, self.layers, I.rng(SEED, rank, 70, l, pi))
+
+
+def _map_8b_decode(K, l, L, g):
+    return I.width_map(K // 32, 0.85, 0.10, 0.05, g)
+
+
+def _map_8b_prefill(K, l, L, g):
+    return I.width_map(K // 32, 0.80, 0.15, 0.05, g)
+
+
+def _map_70b(K, l, L, g):
+    return I.llama70b_layer_map(K, l, L, g)
+
+
+def spec_for(workload: str, layers=None) -> Spec:
+    if workload == "llama3-8b-decode":
+        return Spec("llama3-8b-decode", I.LLAMA3_8B, layers or 32, (1, 4, 16), 0.02, 0.01, 30.0, _map_8b_decode)
+    if workload == "llama3-8b-prefill":
+        return Spec("llama3-8b-prefill", I.LLAMA3_8B, layers or 8, (2048,), 0.02, 0.005, None, _map_8b_prefill,
+                    student_t=True, sample_cols=1024)
+    if workload == "llama2-70b-decode":
+        return Spec("llama2-70b-decode", I.LLAMA2_70B, layers or 80, (1, 16), 0.015, 0.01, 50.0, _map_70b,
+                    sample_cols=512)
+    if workload == "llama2-70b-prefill":
+        L = layers or 80
+        ids = sorted({int(round(v)) for v in np.linspace(0, L - 1, min(4, L))})
+        return Spec("llama2-70b-prefill", I.LLAMA2_70B, L, (4096,), 0.015, 0.01, 50.0, _map_70b,
+                    layer_ids=ids, sample_cols=512)
+    raise ValueError(workload)
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--layers", type=int, default=None,
-                    help="decoder layers per step (default 32 for decode, 8 for prefill)")
-    ap.add_argument("--workload", default="llama3-8b-decode",
-                    choices=["llama3-8b-decode", "llama3-8b-prefill", "llama3-8b-calibration",
+                    help="decoder layers of the model (default 80 for LLaMA-2-70B, 32 for LLaMA-3-8B decode, "
+                         "8 for LLaMA-3-8B prefill)")
+    ap.add_argument("--workload", default="llama2-70b",
+                    choices=["llama2-70b", "llama3-8b-decode", "llama3-8b-prefill", "llama3-8b-calibration",
                              "llama3-8b-decode-attention"])
+    ap.add_argument("--part", default="both", choices=["both", "decode", "prefill"],
+                    help="llama2-70b: run the decode part, the prefill part or both (one JSON line)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="grouped", choices=["planes", "fused", "codes", "grouped"],
                     help="decode activation path: quantize all projections to MMA planes, then the GEMMs "
@@ -182,137 +233,163 @@ def allreduce_max(v: float, ws: int) -> float:
 
 
 # --------------------------------------------------------------- CPU oracle sample
-_SAMPLE = None
+_SAMPLES = {}
 
 
-def _oracle_jobs(seed_rank: int = 0):
-    """Layer 0 of the workload for the oracle, the first min(N, 2048) output
-    rows of every projection: weights quantized once (offline packing is not
-    timed), activations for M = 1, 4, 16."""
-    global _SAMPLE
-    if _SAMPLE is None:
+def _oracle_jobs(spec: Spec, seed_rank: int = 0):
+    """The first timed layer of `spec` for the oracle: every projection's
+    first min(N, spec.sample_cols) output columns, weights quantized once
+    (offline packing is not timed), activations for every M of the spec (the
+    first 64 token rows of a prefill M)."""
+    key = (spec.name, seed_rank)
+    if key not in _SAMPLES:
         from oracle import mxo
         jobs = []
-        for pi, (name, K, N) in enumerate(I.LLAMA3_8B):
-            g = I.rng(SEED, seed_rank, 0, pi)
-            bits = I.width_map(K // 32, *MAP, g)
-            N = min(N, SAMPLE_ROWS)
-            w = I.normal_bf16((N, K), W_SIGMA, g)
+        l = spec.layer_ids[0]
+        for pi, (name, K, N) in enumerate(spec.shapes):
+            bits = spec.bits(seed_rank, l, pi, K)
+            N = min(N, spec.sample_cols)
+            w = I.normal_bf16((N, K), spec.w_sigma, I.rng(SEED, seed_rank, 71, l, pi))
             w_s, w_c = mxo.quantize_bf16(w, bits)
             del w
-            for M in DECODE_MS:
-                x = I.activations_bf16(M, bits, I.rng(SEED, seed_rank, 1, pi, M), OUTLIER_FRAC,
-                                       outlier_scale=OUTLIER_SCALE)
-                jobs.append((bits, x, w_s, w_c, K, N, M))
-        _SAMPLE = jobs
-    return _SAMPLE
+            for M in spec.Ms:
+                Ms = min(M, 64)
+                x = I.activations_bf16(Ms, bits, I.rng(SEED, seed_rank, 72, pi, M), spec.outlier_frac,
+                                       outlier_scale=spec.outlier_scale, student_t=spec.student_t)
+                jobs.append((bits, x, w_s, w_c, K, N, Ms))
+        _SAMPLES[key] = jobs
+    return _SAMPLES[key]
 
 
-def oracle_sample(min_seconds: float = 10.0):
-    """Time the oracle on a bounded sample of the step: the quantization and
-    exact GEMM of layer 0's seven projections at M = 1, 4, 16 (the first
-    min(N, 2048) output columns of each), passes
-    repeated until min_seconds have elapsed (at least one).  Returns (GB/s of
-    the same algorithmic traffic as the GPU step, seconds, threads, text)."""
+def oracle_sample(spec: Spec, min_seconds: float = 10.0):
+    """Time the oracle on a bounded sample of the step: the activation
+    quantization and exact GEMM of the jobs of _oracle_jobs, passes repeated
+    until min_seconds have elapsed (at least one).  Returns (rate, seconds,
+    threads, text, unit): GB/s of the same algorithmic traffic as the GPU
+    step for decode, effective TOPS for prefill."""
     from oracle import mxo
-    jobs = _oracle_jobs()
+    jobs = _oracle_jobs(spec)
     t0 = time.perf_counter()
-    nbytes = 0
-    passes = 0
+    nbytes = ops = passes = 0
     while True:
         for bits, x, w_s, w_c, K, N, M in jobs:
             a_s, a_c = mxo.quantize_bf16(x, bits)
             mxo.gemm(bits, a_c, a_s, w_c, w_s)
             n4 = int(np.sum(bits == 4))
             nbytes += N * (16 * n4 + 32 * (bits.size - n4) + bits.size) + M * K * 2 + M * N * 4
+            ops += 2 * M * N * K
         passes += 1
         if time.perf_counter() - t0 >= min_seconds:
             break
     dt = time.perf_counter() - t0
     threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    desc = (f"layer 0 (q/k/v/o/gate/up/down, first min(N,{SAMPLE_ROWS}) output columns) at M=1,4,16, "
-            f"{passes} pass(es): oracle "
-            f"activation quantization + exact GEMM, OpenMP over output rows")
-    return nbytes / dt / 1e9, dt, threads, desc
+    decode = spec.Ms[0] <= 16
+    desc = (f"layer {spec.layer_ids[0]} of {spec.name} (q/k/v/o/gate/up/down, first min(N,{spec.sample_cols}) "
+            "output columns" + (f") at M={','.join(map(str, spec.Ms))}" if decode else
+                                f", first 64 of {spec.Ms[0]} token rows)") +
+            f", {passes} pass(es): oracle activation quantization + exact GEMM, OpenMP over output rows")
+    if decode:
+        return nbytes / dt / 1e9, dt, threads, desc, "GB/s"
+    return ops / dt / 1e12, dt, threads, desc, "TOPS"
+
+
+def reference_spec(args) -> Spec | None:
+    if args.workload == "llama2-70b":
+        return spec_for("llama2-70b-prefill" if args.part == "prefill" else "llama2-70b-decode", args.layers)
+    if args.workload in ("llama3-8b-decode", "llama3-8b-prefill"):
+        return spec_for(args.workload, args.layers)
+    return None
 
 
 def run_reference(args):
     ws, rank, _ = dist_setup()
     if rank != 0:
         return
+    spec = reference_spec(args)
+    if spec is None:
+        print(json.dumps({"impl": "reference", "unavailable": f"the oracle arm times the GEMM workloads "
+                          f"(llama2-70b, llama3-8b-decode, llama3-8b-prefill), not {args.workload}"}), flush=True)
+        return
     for _ in range(args.warmup):
-        oracle_sample(min_seconds=0.0)
+        oracle_sample(spec, min_seconds=0.0)
     vals, secs = [], []
+    desc, threads, unit = "", 1, "GB/s"
     for _ in range(args.steps):
-        v, dt, threads, desc = oracle_sample(min_seconds=0.0)
+        v, dt, threads, desc, unit = oracle_sample(spec, min_seconds=0.0)
         vals.append(v)
         secs.append(dt)
     value = statistics.median(vals)
+    decode = unit == "GB/s"
     line = {
-        "impl": "reference", "metric": "mxint_decode_gemm_gbps", "value": value, "unit": "GB/s",
+        "impl": "reference", "metric": "mxint_decode_gemm_gbps" if decode else "mxint_prefill_gemm_tops",
+        "value": value, "unit": unit,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * statistics.median(secs), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int64+f64", "data": "synthetic",
-        "config": {"workload": "llama3-8b-decode (sample)", "layers": 1, "M": list(DECODE_MS)},
-        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": threads, "kind": "oracle", "sample": desc},
-        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "config": {"workload": f"{args.workload} (sample)", "layers": 1, "M": list(spec.Ms)},
+        "cpu_baseline": {"value": value, "unit": unit, "cores": threads, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
 
 
 # --------------------------------------------------------------- GPU arm
-def run_ours(args):
+def _gpu_setup():
     import torch
-
     ws, rank, local = dist_setup()
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     from paper_2607_17733_gb300 import build as B
     from paper_2607_17733_gb300 import mxs
-    from paper_2607_17733_gb300.runtime import MxLinear
     if not os.path.exists(mxs.LIB_PATH):
         B.build()
     mxs.lib()
+    return torch, ws, rank, dev
 
-    L = args.layers
+
+def _weight(torch, gen, dev, N, K, sigma, seed):
+    gen.manual_seed(seed)
+    return (torch.randn((N, K), generator=gen, device=dev, dtype=torch.float32) * sigma).to(torch.bfloat16)
+
+
+def run_decode(args, spec: Spec):
+    """Decode step of `spec`: for every M of the spec, the seven projections of
+    every layer (A1 + A4), weights packed once (A2), the step captured in a
+    CUDA graph.  Returns the JSON line (rank 0) or None."""
+    torch, ws, rank, dev = _gpu_setup()
+    from paper_2607_17733_gb300 import mxs
+    from paper_2607_17733_gb300.runtime import MxLinear
+
+    L = spec.layers
     # ---- weights: drawn on the GPU (seeded per layer/projection), packed once
     layers = []
     gen = torch.Generator(device=dev)
     for l in range(L):
         projs = []
-        for pi, (name, K, N) in enumerate(I.LLAMA3_8B):
-            bits = I.width_map(K // 32, *MAP, I.rng(SEED, rank, l, pi))
-            gen.manual_seed(SEED * 1_000_003 + rank * 10_007 + l * 101 + pi)
-            w = (torch.randn((N, K), generator=gen, device=dev, dtype=torch.float32) * W_SIGMA).to(torch.bfloat16)
-            projs.append(MxLinear(w, bits))
+        for pi, (name, K, N) in enumerate(spec.shapes):
+            w = _weight(torch, gen, dev, N, K, spec.w_sigma, SEED * 1_000_003 + rank * 10_007 + l * 101 + pi)
+            projs.append(MxLinear(w, spec.bits(rank, l, pi, K)))
             del w
         layers.append(projs)
     torch.cuda.synchronize()
 
     # ---- inputs: one contiguous pinned host block and one device block per step
     items = []  # (M, lin, x_dev, bufs)
-    x_sizes = []
-    for M in DECODE_MS:
-        for l in range(L):
-            for pi, lin in enumerate(layers[l]):
-                x_sizes.append(M * lin.K)
-    x_host = torch.empty(sum(x_sizes), dtype=torch.bfloat16, pin_memory=True)
+    x_total = sum(M * lin.K for M in spec.Ms for projs in layers for lin in projs)
+    x_host = torch.empty(x_total, dtype=torch.bfloat16, pin_memory=True)
     x_dev = torch.empty_like(x_host, device=dev)
     y_sizes = []
     off = 0
-    xi = 0
-    for M in DECODE_MS:
+    for M in spec.Ms:
         for l in range(L):
             for pi, lin in enumerate(layers[l]):
-                xb = I.activations_bf16(M, lin.bits, I.rng(SEED, rank, 2, M, l, pi), OUTLIER_FRAC,
-                                        outlier_scale=OUTLIER_SCALE)
+                xb = I.activations_bf16(M, lin.bits, I.rng(SEED, rank, 2, M, l, pi), spec.outlier_frac,
+                                        outlier_scale=spec.outlier_scale)
                 n = M * lin.K
                 x_host[off:off + n].copy_(torch.from_numpy(xb.view(np.int16).ravel()).view(torch.bfloat16))
-                bufs = lin.buffers(M, dev)
-                items.append((M, lin, x_dev[off:off + n].view(M, lin.K), bufs))
+                items.append((M, lin, x_dev[off:off + n].view(M, lin.K), lin.buffers(M, dev)))
                 y_sizes.append(M * lin.N)
                 off += n
-                xi += 1
     y_dev = torch.empty(sum(y_sizes), dtype=torch.float32, device=dev)
     y_host = torch.empty_like(y_dev, device="cpu", pin_memory=True)
     off = 0
@@ -333,18 +410,20 @@ def run_ours(args):
                          for M, lin, _, _ in items)
     else:  # the timed segment is quantize + GEMM: bf16 activations in, y out
         gemm_bytes = step_bytes
+    nproj = len(spec.shapes)
     launches_per_step = 2 * len(items)
-    STAGES = [[0, 1, 2], [3], [4, 5], [6]]  # q k v | o | gate up | down: the projections of a stage share an input
+    gemm_launches = len(items)
     if args.path == "grouped":  # per stage one quantizer launch and one GEMM launch
-        launches_per_step = 2 * len(items) // 7 * len(STAGES)
+        launches_per_step = 2 * len(items) // nproj * len(STAGES)
+        gemm_launches = len(items) // nproj * len(STAGES)
 
     # ---- the step as one CUDA graph.  Inputs are independent synthetic draws, so
     # for each M the graph runs all activation quantizations, then all GEMMs;
     # on one stream every kernel waits for the previous one either way.  Two
     # event nodes per M bracket the GEMM segment: the dominant kernel's time
-    # is read from them for every timed step, at 6 event nodes per step.
+    # is read from them for every timed step.
     capture_stream = torch.cuda.Stream(device=dev)
-    groups = [[it for it in items if it[0] == M] for M in DECODE_MS]
+    groups = [[it for it in items if it[0] == M] for M in spec.Ms]
 
     def make_step(events=None):
         def fn():
@@ -359,7 +438,7 @@ def run_ours(args):
                 if events is not None:
                     events[gi][0].record()
                 if args.path == "grouped":
-                    for base in range(0, len(grp), 7):
+                    for base in range(0, len(grp), nproj):
                         for stage in STAGES:
                             its = [grp[base + i] for i in stage]
                             if len(its) == 1:
@@ -398,7 +477,7 @@ def run_ours(args):
         torch.cuda.synchronize()
         if rank == 0:
             print(json.dumps({"eager_steps": args.steps, "launches_per_step": launches_per_step}), flush=True)
-        return
+        return None
 
     plain = capture(make_step())
     try:
@@ -409,16 +488,10 @@ def run_ours(args):
     except TypeError:  # torch without external events: time the plain graph only
         ev_sets, timed = None, [plain] * args.steps
 
-    for _ in range(args.warmup):
+    for _ in range(max(args.warmup, 3)):
         plain.replay()
     torch.cuda.synchronize()
-
-    gpu_id = None
-    try:
-        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid).replace("GPU-", "")
-    except Exception:
-        pass
-    sampler = ClockSampler(gpu_id)
+    sampler = ClockSampler(_gpu_uuid(torch, dev))
 
     # ---- timed region (device time, max over ranks)
     barrier(ws)
@@ -434,8 +507,7 @@ def run_ours(args):
     torch.cuda.synchronize()
     clocks = sampler.stop()
     barrier(ws)
-    ms = t0.elapsed_time(t1) / args.steps
-    ms = allreduce_max(ms, ws)
+    ms = allreduce_max(t0.elapsed_time(t1) / args.steps, ws)
     value = ws * step_bytes / (ms * 1e-3) / 1e9
     tops = ws * step_ops / (ms * 1e-3) / 1e12
 
@@ -445,15 +517,16 @@ def run_ours(args):
     if ev_sets is not None:
         gemm_ms = sum(s.elapsed_time(e) for evs in ev_sets for s, e in evs) / len(ev_sets)  # per step
         achieved = gemm_bytes / (gemm_ms * 1e-3) / 1e9
-        traffic = profile_traffic("gemm_decode.cu", "gemm_decode_llama3_8b_decode.md")
+        prof = "gemm_decode_llama2_70b_decode.md" if spec.name.startswith("llama2-70b") \
+            else "gemm_decode_llama3_8b_decode.md"
         roofline = {"kernel": "gemm_decode_kernel" + (" + quantize_act_kernel (PDL chain)"
                                                       if args.path in ("fused", "grouped") else f" ({args.path} path)"),
                     "bound": "hbm", "achieved": achieved,
                     "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": achieved / pk["hbm_gbs"],
-                    "peak_source": pk["source"], "traffic": traffic,
+                    "peak_source": pk["source"] + " (HBM copy)",
+                    "traffic": profile_traffic("gemm_decode.cu", prof),
                     "bytes_per_step": gemm_bytes, "gemm_ms_per_step": gemm_ms,
-                    "gemm_launches_per_step": len(items) // 7 * len(STAGES) if args.path == "grouped" else len(items),
-                    "share_of_step": gemm_ms / ms}
+                    "gemm_launches_per_step": gemm_launches, "share_of_step": gemm_ms / ms}
 
     # ---- end to end through the public API with host buffers
     barrier(ws)
@@ -475,114 +548,134 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        v, dt, threads, desc = oracle_sample()
-        cpu = {"value": v, "unit": "GB/s", "cores": threads, "kind": "oracle", "sample": desc, "seconds": dt}
+        v, dt, threads, desc, unit = oracle_sample(spec)
+        cpu = {"value": v, "unit": unit, "cores": threads, "kind": "oracle", "sample": desc, "seconds": dt}
+    w_bytes = sum(lin.weight_bytes for p in layers for lin in p)
+    del plain, timed, layers, items, x_dev, y_dev
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    if rank != 0:
+        return None
+    maps = ("4-bit share from 60% (layer 0) to 95% (last layer), 8-bit blocks over the 1% outlier columns, "
+            "the rest 6-bit" if spec.map_fn is _map_70b else "85/10/5 % (4/6/8 bits)")
+    return {
+        "metric": "mxint_decode_gemm_gbps", "value": value, "unit": "GB/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int8+f32",
+        "data": f"synthetic (seeded; weights N(0,{spec.w_sigma}), activations N(0,1) with "
+                f"{100 * spec.outlier_frac:g}% outlier columns x{spec.outlier_scale:g})",
+        "config": {"workload": spec.name, "M": list(spec.Ms), "layers": L,
+                   "path": {"planes": "quantize to MMA planes, then GEMM over the planes (TMA)",
+                            "fused": "mxs_linear_decode: quantize + GEMM chained by programmatic dependent launch",
+                            "grouped": "mxs_linear_decode_group for q/k/v and gate/up (one GEMM launch per "
+                                       "group, after one quantizer launch for the group), mxs_linear_decode for o, down",
+                            "codes": "quantize to packed codes, GEMM over the codes"}[args.path],
+                   "projections": [p[0] for p in spec.shapes], "maps": maps,
+                   "parallelism": f"replicas x{ws}", "l2": "inputs larger than L2 (packed weights "
+                   f"{w_bytes / 1e9:.2f} GB per M per step)"},
+        "tops": tops,
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks,
+    }
 
-    if rank == 0:
-        line = {
-            "metric": "mxint_decode_gemm_gbps", "value": value, "unit": "GB/s", "n_gpus": ws,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "int8+f32",
-            "data": "synthetic (seeded; weights N(0,0.02), activations N(0,1) with 1% outlier columns x30)",
-            "config": {"workload": "llama3-8b-decode", "M": list(DECODE_MS), "layers": L,
-                       "path": {"planes": "quantize to MMA planes, then GEMM over the planes (TMA)",
-                                "fused": "mxs_linear_decode: quantize + GEMM chained by programmatic dependent launch",
-                                "grouped": "mxs_linear_decode_group for q/k/v and gate/up (one GEMM launch per "
-                                           "group, after one quantizer launch for the group), mxs_linear_decode for o, down",
-                                "codes": "quantize to packed codes, GEMM over the codes"}[args.path],
-                       "projections": [p[0] for p in I.LLAMA3_8B], "map_4_6_8": list(MAP),
-                       "parallelism": f"replicas x{ws}", "l2": "inputs larger than L2 (packed weights "
-                       f"{sum(lin.weight_bytes for p in layers for lin in p) / 1e9:.2f} GB per step)"},
-            "tops": tops,
-            "roofline": roofline,
-            "cpu_baseline": cpu,
-            "e2e": e2e,
-            "gpu_launches": launches_per_step * args.steps,
-            "clocks": clocks,
-        }
-        print(json.dumps(line), flush=True)
+
+def _gpu_uuid(torch, dev):
+    try:
+        return "GPU-" + str(torch.cuda.get_device_properties(dev).uuid).replace("GPU-", "")
+    except Exception:
+        return None
 
 
-def run_prefill(args):
-    """LLaMA-3-8B-shaped prefill: M = 2048 tokens through q/k/v/o/gate/up/down of
-    `layers` layers, map 80/15/5, activations N(0,1) with Student-t(3) outlier
-    channels on 0.5 % of K.  Per stage of a layer (q/k/v, o, gate/up, down: the
-    projections of a stage read one hidden state): one quantizer launch to MMA
-    planes (A1) for its projections, then their tcgen05 GEMMs (A3).  Metric:
-    effective TOPS = 2*M*N*K / s, whole job."""
-    import torch
-
-    ws, rank, local = dist_setup()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    from paper_2607_17733_gb300 import build as B
+def run_prefill_part(args, spec: Spec):
+    """Prefill step of `spec` (M = spec.Ms[0] tokens) through the seven
+    projections of the layers spec.layer_ids.  Per stage of a layer (q/k/v,
+    o, gate/up, down: the projections of a stage read one hidden state): one
+    quantizer launch to MMA planes (A1) for its projections, then their
+    tcgen05 GEMMs (A3).  Metric: effective TOPS = 2*M*N*K / s, whole job.
+    Returns the JSON object (rank 0) or None."""
+    torch, ws, rank, dev = _gpu_setup()
     from paper_2607_17733_gb300 import mxs
     from paper_2607_17733_gb300.runtime import MxLinear
-    if not os.path.exists(mxs.LIB_PATH):
-        B.build()
-    mxs.lib()
-    M = 2048
-    L = args.layers or 8
+    M = spec.Ms[0]
     gen = torch.Generator(device=dev)
     items = []
-    for l in range(L):
-        for pi, (name, K, N) in enumerate(I.LLAMA3_8B):
-            bits = I.width_map(K // 32, 0.80, 0.15, 0.05, I.rng(SEED, rank, 3, l, pi))
-            gen.manual_seed(SEED * 7 + rank * 10_007 + l * 101 + pi)
-            w = (torch.randn((N, K), generator=gen, device=dev, dtype=torch.float32) * W_SIGMA).to(torch.bfloat16)
-            lin = MxLinear(w, bits, with_planes=True)
+    for l in spec.layer_ids:
+        for pi, (name, K, N) in enumerate(spec.shapes):
+            w = _weight(torch, gen, dev, N, K, spec.w_sigma, SEED * 7 + rank * 10_007 + l * 101 + pi)
+            bits = spec.bits(rank, l, pi, K)
+            items.append((MxLinear(w, bits, with_planes=True), bits))
             del w
-            items.append((lin, bits))
-    planes, ys = [], []
+    xs, planes, ys = [], [], []
     for idx, (lin, bits) in enumerate(items):
-        # N(0,1) activations, 0.5 % of K channels (inside 8-bit blocks) redrawn from
-        # a Student-t(3) = Z / sqrt(chi2_3 / 3); drawn on the GPU from a seeded stream
+        # N(0,1) activations with outlier columns inside the 8-bit blocks: scaled,
+        # or redrawn from a Student-t(3) = Z / sqrt(chi2_3 / 3); drawn on the GPU
         gen.manual_seed(SEED * 13 + rank * 10_007 + idx)
         x = torch.randn((M, lin.K), generator=gen, device=dev, dtype=torch.float32)
-        cols = torch.from_numpy(I.outlier_columns(bits, int(np.floor(0.005 * lin.K + 0.5)),
-                                                  I.rng(SEED, rank, 6, idx))).to(dev)
-        z = torch.randn((M, cols.numel(), 4), generator=gen, device=dev, dtype=torch.float32)
-        x[:, cols] = z[..., 0] / torch.sqrt((z[..., 1:] ** 2).sum(-1) / 3.0)
-        x = x.to(torch.bfloat16)
-        planes.append((x, torch.empty(mxs.act_planes_bytes(M, lin.K, bits), dtype=torch.uint8, device=dev)))
+        n_out = int(np.floor(spec.outlier_frac * lin.K + 0.5))
+        cols = torch.from_numpy(I.outlier_columns(bits, n_out, I.rng(SEED, rank, 6, idx))).to(dev)
+        if spec.student_t:
+            z = torch.randn((M, cols.numel(), 4), generator=gen, device=dev, dtype=torch.float32)
+            x[:, cols] = z[..., 0] / torch.sqrt((z[..., 1:] ** 2).sum(-1) / 3.0)
+        else:
+            x[:, cols] *= spec.outlier_scale
+        xs.append(x.to(torch.bfloat16))
+        del x
+        planes.append(torch.empty(mxs.act_planes_bytes(M, lin.K, bits), dtype=torch.uint8, device=dev))
         ys.append(torch.empty((M, lin.N), dtype=torch.float32, device=dev))
     torch.cuda.synchronize()
+    nproj = len(spec.shapes)
     step_ops = sum(2 * M * lin.N * lin.K for lin, _ in items)
-
-    # the projections of a stage read one hidden state (q/k/v; gate/up): their
-    # activations are quantized by one launch, then their GEMMs run
-    PSTAGES = [[0, 1, 2], [3], [4, 5], [6]]
-    n_launch = len(items) + len(items) // 7 * len(PSTAGES)
+    # tensor work as issued: a 4-bit K' stage is four K=32 FP8 MMAs, a 6/8-bit stage
+    # four K=16 bf16 MMAs of the same cost: 2*M*N*128 per K' stage, in FP8 units
+    nst = []
+    for lin, bits in items:
+        n4 = int(np.sum(bits == 4))
+        nst.append((n4 + 3) // 4 + (bits.size - n4 + 1) // 2)
+    issued_ops = sum(2 * M * lin.N * 128 * s for (lin, _), s in zip(items, nst))
+    q_bytes = sum(2 * M * lin.K + pl.numel() for (lin, _), pl in zip(items, planes))
+    n_launch = len(items) + len(items) // nproj * len(STAGES)
 
     def fn(events=None):
-        for base in range(0, len(items), 7):
-            for stage in PSTAGES:
+        for base in range(0, len(items), nproj):
+            for si, stage in enumerate(STAGES):
                 idxs = [base + i for i in stage]
+                if events is not None:
+                    events["q"][base // nproj * len(STAGES) + si][0].record()
                 if len(idxs) == 1:
-                    x, pl = planes[idxs[0]]
-                    mxs.quantize_act(x, items[idxs[0]][1], planes=pl, want_codes=False)
+                    mxs.quantize_act(xs[idxs[0]], items[idxs[0]][1], planes=planes[idxs[0]], want_codes=False)
                 else:
-                    mxs.quantize_act_group([(planes[i][0], items[i][1], planes[i][1]) for i in idxs])
+                    mxs.quantize_act_group([(xs[i], items[i][1], planes[i]) for i in idxs])
+                if events is not None:
+                    events["q"][base // nproj * len(STAGES) + si][1].record()
                 for idx in idxs:
                     lin, bits = items[idx]
                     if events is not None:
-                        events[idx][0].record()
-                    mxs.gemm_prefill(planes[idx][1], bits, lin.packed, M, lin.N, y=ys[idx])
+                        events["g"][idx][0].record()
+                    mxs.gemm_prefill(planes[idx], bits, lin.packed, M, lin.N, y=ys[idx])
                     if events is not None:
-                        events[idx][1].record()
+                        events["g"][idx][1].record()
 
     if args.eager:
         for _ in range(args.warmup + args.steps):
             fn()
         torch.cuda.synchronize()
-        print(json.dumps({"eager_steps": args.steps, "launches_per_step": n_launch}), flush=True)
-        return
-    for _ in range(args.warmup):
+        if rank == 0:
+            print(json.dumps({"eager_steps": args.steps, "launches_per_step": n_launch}), flush=True)
+        return None
+    for _ in range(max(args.warmup, 3)):
         fn()
     torch.cuda.synchronize()
-    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in items]
-           for _ in range(args.steps)]
-    sampler = ClockSampler(None)
+
+    def evpair():
+        return (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+
+    steps = max(1, min(args.steps, 20))
+    evs = [{"g": [evpair() for _ in items], "q": [evpair() for _ in range(len(items) // nproj * len(STAGES))]}
+           for _ in range(steps)]
+    sampler = ClockSampler(_gpu_uuid(torch, dev))
     barrier(ws)
     torch.cuda.synchronize()
     sampler.start()
@@ -590,31 +683,92 @@ def run_prefill(args):
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record()
-    for k in range(args.steps):
+    for k in range(steps):
         fn(evs[k])
     t1.record()
     torch.cuda.synchronize()
     clocks = sampler.stop()
-    ms = allreduce_max(t0.elapsed_time(t1) / args.steps, ws)
-    gemm_ms = sum(s.elapsed_time(e) for ev in evs for s, e in ev) / args.steps
+    ms = allreduce_max(t0.elapsed_time(t1) / steps, ws)
+    gemm_ms = sum(s.elapsed_time(e) for ev in evs for s, e in ev["g"]) / steps
+    quant_ms = sum(s.elapsed_time(e) for ev in evs for s, e in ev["q"]) / steps
     pk = peaks()
     fp8_peak = 2.0 * pk["bf16_tflops"]
     achieved = step_ops / (gemm_ms * 1e-3) / 1e12
+    issued = issued_ops / (gemm_ms * 1e-3) / 1e12
     value = ws * step_ops / (ms * 1e-3) / 1e12
-    if rank == 0:
-        print(json.dumps({
-            "metric": "mxint_prefill_gemm_tops", "value": value, "unit": "TOPS", "n_gpus": ws,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "e4m3 (4-bit blocks) + bf16 (6/8-bit blocks), f32 accumulation",
-            "data": "synthetic (seeded; W N(0,0.02), A N(0,1) with Student-t(3) outlier channels on 0.5% of K)",
-            "config": {"workload": "llama3-8b-prefill", "M": M, "layers": L, "map_4_6_8": [0.8, 0.15, 0.05],
-                       "l2": "inputs larger than L2"},
-            "roofline": {"kernel": "gemm_prefill_kernel", "bound": "tensor", "achieved": achieved,
-                         "peak": fp8_peak, "unit": "TFLOP/s", "frac": achieved / fp8_peak,
-                         "peak_source": pk["source"] + " bf16 x 2 (fp8/bf16 nominal ratio)",
-                         "traffic": profile_traffic("gemm_prefill.cu", "gemm_prefill_llama3_8b_prefill.md"),
-                         "gemm_ms_per_step": gemm_ms, "share_of_step": gemm_ms / ms},
-            "gpu_launches": n_launch * args.steps, "clocks": clocks}), flush=True)
+    q_gbs = q_bytes / (quant_ms * 1e-3) / 1e9
+
+    # end to end: the step's activations from pinned host memory, every output back
+    x_host = [x.cpu().pin_memory() for x in xs]
+    y_host = [torch.empty(tuple(y.shape), dtype=torch.float32).pin_memory() for y in ys]
+    barrier(ws)
+    torch.cuda.synchronize()
+    e2e_steps = max(1, min(steps, 5))
+    t0.record()
+    for _ in range(e2e_steps):
+        for xh, x in zip(x_host, xs):
+            x.copy_(xh, non_blocking=True)
+        fn()
+        for yh, y in zip(y_host, ys):
+            yh.copy_(y, non_blocking=True)
+    t1.record()
+    torch.cuda.synchronize()
+    e2e_ms = allreduce_max(t0.elapsed_time(t1) / e2e_steps, ws)
+    e2e = {"value": ws * step_ops / (e2e_ms * 1e-3) / 1e12, "unit": "TOPS",
+           "h2d_bytes_per_step": sum(x.numel() * 2 for x in xs), "d2h_bytes_per_step": sum(y.numel() * 4 for y in ys),
+           "ms_per_step": e2e_ms}
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        v, dt, threads, desc, unit = oracle_sample(spec)
+        cpu = {"value": v, "unit": unit, "cores": threads, "kind": "oracle", "sample": desc, "seconds": dt}
+    q_launches = len(items) // nproj * len(STAGES)
+    del items, xs, planes, ys, x_host, y_host
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    if rank != 0:
+        return None
+    prof = "gemm_prefill_llama2_70b_prefill.md" if spec.name.startswith("llama2-70b") \
+        else "gemm_prefill_llama3_8b_prefill.md"
+    return {
+        "metric": "mxint_prefill_gemm_tops", "value": value, "unit": "TOPS", "n_gpus": ws,
+        "steps": steps, "warmup": max(args.warmup, 3), "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "e4m3 (4-bit blocks) + bf16 (6/8-bit blocks), f32 accumulation",
+        "data": f"synthetic (seeded; W N(0,{spec.w_sigma}), A N(0,1) with " +
+                ("Student-t(3) outlier channels" if spec.student_t else f"outlier columns x{spec.outlier_scale:g}") +
+                f" on {100 * spec.outlier_frac:g}% of K)",
+        "config": {"workload": spec.name, "M": M, "layers": spec.layer_ids, "of_layers": spec.layers,
+                   "l2": "inputs larger than L2"},
+        "roofline": {"kernel": "gemm_prefill_kernel", "bound": "tensor", "achieved": achieved,
+                     "peak": fp8_peak, "unit": "TFLOP/s", "frac": achieved / fp8_peak,
+                     "peak_source": pk["source"] + " bf16 x 2 (fp8/bf16 nominal ratio)",
+                     "issued_fp8_equivalent": issued, "issued_frac": issued / fp8_peak,
+                     "traffic": profile_traffic("gemm_prefill.cu", prof),
+                     "gemm_ms_per_step": gemm_ms, "share_of_step": gemm_ms / ms},
+        "quantizer": {"kernel": "quantize_act_group_kernel / quantize_act_kernel (bf16 in, MMA planes out)",
+                      "bound": "hbm", "achieved": q_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                      "frac": q_gbs / pk["hbm_gbs"], "bytes_per_step": q_bytes, "ms_per_step": quant_ms,
+                      "launches_per_step": q_launches},
+        "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": n_launch * steps, "clocks": clocks}
+
+
+def run_llama70b(args):
+    """The default workload: LLaMA-2-70B decode (the line's value) and
+    prefill (its `prefill` object)."""
+    line = None
+    if args.part in ("both", "decode"):
+        line = run_decode(args, spec_for("llama2-70b-decode", args.layers))
+    if args.part in ("both", "prefill"):
+        pre = run_prefill_part(args, spec_for("llama2-70b-prefill", args.layers))
+        if line is None:
+            line = pre
+        elif pre is not None:
+            line["prefill"] = pre
+    if line is not None:
+        if "config" in line:
+            line["config"]["workload"] = "llama2-70b" + ("" if args.part == "both" else f" ({args.part})")
+        print(json.dumps(line), flush=True)
 
 
 CALIB_SEQ, CALIB_BATCH = 2048, 8  # a calibration sample is a 2048-token sequence; 8 samples per call
@@ -940,16 +1094,20 @@ def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload == "llama2-70b":
+        run_llama70b(args)
     elif args.workload == "llama3-8b-prefill":
-        run_prefill(args)
+        line = run_prefill_part(args, spec_for("llama3-8b-prefill", args.layers))
+        if line is not None:
+            print(json.dumps(line), flush=True)
     elif args.workload == "llama3-8b-calibration":
         run_calibration(args)
     elif args.workload == "llama3-8b-decode-attention":
         run_attention(args)
     else:
-        if args.layers is None:
-            args.layers = 32
-        run_ours(args)
+        line = run_decode(args, spec_for("llama3-8b-decode", args.layers))
+        if line is not None:
+            print(json.dumps(line), flush=True)
 
 
 if __name__ == "__main__":
