@@ -93,7 +93,7 @@ extern "C" {
 #define MXS_API
 #endif
 
-#define MXS_VERSION 1
+#define MXS_VERSION 2
 #define MXS_MAX_K 65536 /* K/32 <= 2048 blocks */
 
 enum mxs_status {
@@ -118,13 +118,22 @@ MXS_API int mxs_version(void);
 
 /* ---------------------------------------------------------------- sizes
  * Bytes the caller must provide.  They touch no device and return a negative
- * mxs_status (e.g. -MXS_ERR_BITS) for invalid arguments. */
+ * mxs_status (e.g. -MXS_ERR_BITS) for invalid arguments.  The storage they
+ * count is the paper's: b bits per element for a b-bit block (one width per
+ * 32-element block, Sec. 4.1) plus one 8-bit shared exponent per block, i.e.
+ * +0.25 bit per element (Sec. 5.1), laid out as the format above.
+ *   mxs_act_row_bytes    code bytes of one activation row: 16*n4 + 32*(n6+n8)
+ *   mxs_act_codes_bytes  M rows of codes (the scales are a separate [M, K/32])
+ *   mxs_act_planes_bytes activation MMA planes + scale tiles, one buffer with
+ *                        the tiles at align256(M*Kp)
+ *   mxs_weight_bytes     the weight buffer of mxs_pack_weight for `layout`
+ *   mxs_gemm_workspace_bytes  scratch of mxs_gemm / mxs_gemm_decode (0 for
+ *                        the current kernels; kept so callers need not change
+ *                        if a kernel ever needs one) */
 MXS_API int64_t mxs_act_row_bytes(int64_t K, const uint8_t *bits);
 MXS_API int64_t mxs_act_codes_bytes(int64_t M, int64_t K, const uint8_t *bits);
-/* activation planes + their scale tiles (one buffer; SF at align256(M*Kp)) */
 MXS_API int64_t mxs_act_planes_bytes(int64_t M, int64_t K, const uint8_t *bits);
 MXS_API int64_t mxs_weight_bytes(int64_t N, int64_t K, const uint8_t *bits, int layout);
-/* scratch for mxs_gemm / mxs_gemm_decode: split-K partial sums (fp32). */
 MXS_API int64_t mxs_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K, const uint8_t *bits);
 
 /* ---------------------------------------------------------------- A1: activation quantization
@@ -142,18 +151,29 @@ MXS_API int mxs_quantize_act(const void *x_bf16, int64_t M, int64_t K, int64_t l
                      void *codes, uint8_t *scales, void *planes, void *stream);
 
 /* ---------------------------------------------------------------- A2: weight packing (offline)
- * Quantizes W (bf16 [N,K] row stride ld_w, the nn.Linear convention) with the
- * same rules and writes the weight buffer (mxs_weight_bytes(N,K,bits,layout)
- * bytes).  Run once per layer. */
+ * The paper quantizes the weights of every linear layer with the same MXINT
+ * rule as the activations (Appendix A.2), under the layer's one width map
+ * (Sec. 4.1), and stores each block at its width plus the 8-bit exponent
+ * (Sec. 5.1).  Quantizes W (bf16 [N,K] row stride ld_w >= K, a multiple of 8;
+ * the nn.Linear convention) with those rules and writes the weight buffer
+ * (mxs_weight_bytes(N,K,bits,layout) bytes, caller-allocated device memory,
+ * fully overwritten).  Run once per layer, offline.  Errors: MXS_ERR_SHAPE,
+ * MXS_ERR_BITS, MXS_ERR_INVALID_ARG (NULL, rounding, layout, ld_w),
+ * MXS_ERR_ALIGN (w, packed), MXS_ERR_CUDA. */
 MXS_API int mxs_pack_weight(const void *w_bf16, int64_t N, int64_t K, int64_t ld_w,
                     const uint8_t *bits, int rounding, int layout,
                     void *packed, void *stream);
 
 /* ---------------------------------------------------------------- A3/A4: GEMM
+ * The MXINT product (Sec. 2): within a block the integer mantissas multiply
+ * and add exactly under the two shared scales, and the blocks' terms
+ * 2^(Ea'+Ew') * D add up to y; the widths come one per block (Sec. 4.1).
  * y [M,N] fp32 (row stride ld_y >= N, elements) = x W^T over the quantized
- * operands.  act_bits must equal w_bits (the paper allocates one map per
- * linear layer and applies it to W and A); other pairs return
- * MXS_ERR_UNSUPPORTED.  `w_layout` is the layout W was packed with.
+ * operands.  act_bits must equal w_bits: the paper's Alg. 3 returns one
+ * column allocation per linear layer, derived from one Hessian diagonal that
+ * serves both operands (Sec. 3.1), so one map applies to W and A; maps that
+ * differ return MXS_ERR_UNSUPPORTED.  `w_layout` is the layout W was packed
+ * with.
  * mxs_gemm picks the decode kernel for M <= 16 (over act_planes when given,
  * else over codes/scales) and the tensor-core prefill kernel otherwise (needs
  * act_planes and a weight packed with MXS_W_COMPACT_AND_PLANES).  workspace may be NULL when
@@ -203,8 +223,11 @@ MXS_API int mxs_linear_decode(const void *x_bf16, int64_t M, int64_t K, int64_t 
  * allocates nothing.  Sizes whose planes exceed 2 MiB
  * (mxs_act_planes_bytes(M, K, bits) > 2 MiB; M <= 16 fits for K <= 49152
  * with any map) return MXS_ERR_BUFFER.  The first call on each device looks
- * up the array's device address (cudaGetSymbolAddress, current device):
- * make that first call before any stream capture.  All calls share the one
+ * up the array's device address (cudaGetSymbolAddress, current device) and
+ * keeps it for the life of the process: make that first call before any
+ * stream capture, and do not reset the device (cudaDeviceReset, or anything
+ * else that destroys its primary context) after it, since the kept address
+ * would then be stale.  All calls share the one
  * array and leave their planes in it: calls ordered on one stream are safe
  * (each waits for the one before it as mxs_linear_decode does), calls that
  * overlap on the GPU (other streams, other host threads) race and give wrong
@@ -241,6 +264,19 @@ MXS_API int mxs_device_status(int *status, int reset, void *stream);
 MXS_API int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits, const void *packed_w,
                                     int64_t M, int64_t N, int64_t K, float *y, int64_t ld_y, int stage,
                                     void *stream);
+
+/* Test hook for the decode kernel's bounded waits (failure handling of this
+ * library; the paper has no counterpart): mxs_gemm_decode over
+ * activation planes (M in 1..16), except that every CTA skips the weight copy
+ * of its copy chunk `chunk` (1-based, in the CTA's streaming order), so the
+ * converter warps' wait for it runs out.  Each CTA then records
+ * MXS_ERR_TIMEOUT, stops its quads, waits (bounded) for what it issued and for
+ * any slices its cluster partners sent it, frees its tensor memory and
+ * returns; y is left partly unwritten.  No device fault or hang is involved;
+ * the context stays usable.  Errors as mxs_gemm_decode, MXS_ERR_INVALID_ARG
+ * for chunk < 1. */
+MXS_API int mxs_test_decode_starve(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M,
+                                   int64_t N, int64_t K, float *y, int64_t ld_y, int chunk, void *stream);
 
 /* mxs_quantize_act_permuted / mxs_pack_weight_permuted -- the layer's
  * columns in the order of the allocation (Alg. 3 returns column lists, and the
@@ -295,8 +331,9 @@ MXS_API int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, 
  * mxs_quantize_act(x_i, M, K_i, ld_i, bits_i, rounding, NULL, NULL, planes_i)
  * writes (digit form for M <= 16, bf16 form of the 6/8-bit blocks for
  * M > 16), one link in the launch chain instead of one per layer.
- * planes_i: device, mxs_act_planes_bytes(M, K_i, bits_i) bytes, 16-byte
- * aligned, distinct buffers.  1 <= count <= 3.  Asynchronous on `stream`
+ * planes_i: device, at least mxs_act_planes_bytes(M, K_i, bits_i) bytes
+ * (planes_bytes_i says how many the caller has), 16-byte aligned, distinct
+ * buffers.  1 <= count <= 3.  Asynchronous on `stream`
  * (programmatic dependent launch as mxs_quantize_act); allocates nothing.
  * Errors as mxs_quantize_act, per problem (the message names it). */
 typedef struct mxs_quant_problem {
@@ -304,6 +341,7 @@ typedef struct mxs_quant_problem {
     int64_t K, ld_x;
     const uint8_t *bits;   /* host, K/32 widths */
     void *planes;          /* device, the MMA planes + scale tiles */
+    size_t planes_bytes;   /* size of `planes`; MXS_ERR_BUFFER below mxs_act_planes_bytes(M, K, bits) */
 } mxs_quant_problem;
 MXS_API int mxs_quantize_act_group(const mxs_quant_problem *probs, int count, int64_t M, int rounding, void *stream);
 

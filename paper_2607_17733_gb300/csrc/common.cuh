@@ -126,8 +126,10 @@ int64_t decode_workspace_bytes(const Plan &p, int64_t M, int64_t N);
 // decode GEMM over packed codes + scales (act_planes NULL) or over the
 // activation MMA planes (codes/scales NULL); pdl: the launch may overlap the
 // tail of the previous kernel on the stream (programmatic dependent launch)
+// starve > 0 (test hook): every CTA skips the weight copy of its chunk starve-1
 int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, const void *act_planes,
-                       const void *packed, int64_t M, int64_t N, float *y, int64_t ld_y, bool pdl, cudaStream_t st);
+                       const void *packed, int64_t M, int64_t N, float *y, int64_t ld_y, bool pdl, cudaStream_t st,
+                       int starve = 0);
 // up to three decode GEMMs (planes mode) in one launch; returns -1, with no
 // error recorded, when no cluster size fits every problem
 int launch_gemm_decode_group(const Plan *const *plans, const void *const *act_planes, const void *const *packed,

@@ -94,6 +94,7 @@ struct DecodeArgs {
     int ring, slot_bytes;  // copy chunks in flight, bytes per ring slot (a multiple of 1024)
     int w_off;             // weights' offset in a slot: after the streamed token tiles (planes mode), else 0
     int accumulate;        // add into y (a later K pass) instead of storing
+    int starve;            // test hook: > 0 makes every CTA skip the weight copy of its chunk starve-1
     int64_t GB;            // bytes of one 128-row weight group
 };
 
@@ -410,6 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
     // converted by quad qc % kQuads (ring is a multiple of kQuads, so each slot
     // has one consumer, which takes its slots in order)
     auto issue = [&](int qc) {
+        if (a.starve == qc + 1) return;  // test hook: this chunk never arrives (its converters' wait runs out)
         const int gi = qc / nchunks, k = qc - gi * nchunks;
         const int s = qc % a.ring;
         int lo, hi, lo2, hi2;
@@ -524,7 +526,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         // residue's last ring / kQuads chunks that exist)
         if (role != 2)
             for (int qc = nx - kQuads, n = 0; qc >= 0 && n < a.ring / kQuads; qc -= kQuads, ++n)
-                if (qc < total) drain_wait(role == 0 ? &full_c[qc % a.ring] : &full_t[qc % a.ring], (qc / a.ring) & 1);
+                if (qc < total && !(role == 0 && a.starve == qc + 1))
+                    drain_wait(role == 0 ? &full_c[qc % a.ring] : &full_t[qc % a.ring], (qc / a.ring) & 1);
     } else if (warp >= kWorkerWarp0) {
         // ------------------------------------------------------------ worker quads
         // quad j = warps 5+5j .. 9+5j: four converters (one per tensor-memory lane
@@ -793,6 +796,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
         if (a.GS > 1) cluster_wait();
         const int qtr = warp & 3;
         const int r = 32 * qtr + lane;
+        // cluster mode: the group whose slices the receive barrier is armed for
+        // and this CTA has not yet taken (-1: none).  Partners may send them
+        // whatever state this CTA is in, so a CTA that gives up waits (bounded)
+        // for them before it leaves: no copy may land in a CTA that has exited.
+        int rx_gi = a.GS > 1 ? 0 : -1;
         int gi = 0;
         for (int g = bx; g < a.G; g += gx, ++gi) {
             const int b = gi & 1;
@@ -843,6 +851,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
             if (!__shfl_sync(0xffffffffu, sent, 0)) break;  // whole warp
             // the other ranks' slices of this rank's rows arrived by bulk copy
             if (!warp_wait(xfull, gi & 1, abort)) break;
+            rx_gi = -1;
             const int lr = r - (int)rank * R;  // row within this rank's slice
             if (lr >= 0 && lr < R) {
                 float sum[16];
@@ -874,8 +883,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                     }
                 }
                 if (!__shfl_sync(0xffffffffu, freed, 0)) break;  // whole warp
+                rx_gi = gi + 1;
             }
         }
+        // gave up with the receive barrier armed: the slices partners have sent
+        // (or still send) land before this CTA exits
+        if (rx_gi >= 0 && et == 0) drain_wait(xfull, rx_gi & 1);
     }
 
     // No CTA leaves while a partner may still copy into or out of its memory:
@@ -1119,9 +1132,11 @@ int launch_gemm_decode_group(const Plan *const *plans, const void *const *act_pl
 }
 
 int launch_gemm_decode(const Plan &p, const void *codes, const uint8_t *scales, const void *act_planes,
-                       const void *packed, int64_t M, int64_t N, float *y, int64_t ld_y, bool pdl, cudaStream_t st) {
+                       const void *packed, int64_t M, int64_t N, float *y, int64_t ld_y, bool pdl, cudaStream_t st,
+                       int starve) {
     if (N > (int64_t)0x7FFFFFF0) return fail(MXS_ERR_SHAPE, "N too large");
     DecodeArgs a = {};
+    a.starve = starve;
     a.codes = static_cast<const uint8_t *>(codes);
     a.scales = scales;
     a.w = static_cast<const uint8_t *>(packed);

@@ -349,6 +349,10 @@ int mxs_quantize_act_group(const mxs_quant_problem *probs, int count, int64_t M,
         if (q.ld_x < q.K || q.ld_x % 8 != 0)
             return fail(MXS_ERR_INVALID_ARG, "problem %d: ld_x=%lld must be >= K and a multiple of 8", i, (long long)q.ld_x);
         if (!aligned16(q.x) || !aligned16(q.planes)) return fail(MXS_ERR_ALIGN, "problem %d: x and planes must be 16-byte aligned", i);
+        const int64_t need = align256(align256(M * plans[i].kp) + (M + 127) / 128 * plans[i].nst * 512);
+        if ((int64_t)q.planes_bytes < need)
+            return fail(MXS_ERR_BUFFER, "problem %d: planes of %lld bytes needed, %zu given", i, (long long)need,
+                        q.planes_bytes);
         for (int j = 0; j < i; ++j)
             if (probs[j].planes == q.planes) return fail(MXS_ERR_INVALID_ARG, "problems %d and %d share planes", j, i);
         pp[i] = &plans[i];
@@ -426,6 +430,22 @@ static int prefill_checked(const void *act_planes, const uint8_t *bits, const vo
 int mxs_gemm_prefill(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M, int64_t N,
                      int64_t K, float *y, int64_t ld_y, void *stream) {
     return prefill_checked(act_planes, bits, packed_w, M, N, K, y, ld_y, 0, stream);
+}
+
+int mxs_test_decode_starve(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M, int64_t N,
+                           int64_t K, float *y, int64_t ld_y, int chunk, void *stream) {
+    Plan p;
+    int rc = build_plan(bits, K, &p);
+    if (rc) return rc;
+    if (chunk < 1) return fail(MXS_ERR_INVALID_ARG, "chunk=%d must be >= 1", chunk);
+    if (M < 1 || M > 16 || N < 1) return fail(MXS_ERR_SHAPE, "M=%lld (1..16), N=%lld", (long long)M, (long long)N);
+    if (!act_planes || !packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
+    if (ld_y < N) return fail(MXS_ERR_INVALID_ARG, "ld_y=%lld < N", (long long)ld_y);
+    if (!aligned16(act_planes) || !aligned16(packed_w) || (reinterpret_cast<uintptr_t>(y) & 3))
+        return fail(MXS_ERR_ALIGN, "act_planes/packed_w must be 16-byte aligned, y 4-byte aligned");
+    if ((rc = check_device())) return rc;
+    return launch_gemm_decode(p, nullptr, nullptr, act_planes, packed_w, M, N, y, ld_y, false,
+                              static_cast<cudaStream_t>(stream), chunk);
 }
 
 int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M, int64_t N,

@@ -25,7 +25,8 @@ LIB_PATH = os.path.join(_HERE, "libmxs.so")
 EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_bytes",
            "mxs_act_planes_bytes", "mxs_weight_bytes", "mxs_gemm_workspace_bytes",
            "mxs_quantize_act", "mxs_pack_weight", "mxs_gemm", "mxs_gemm_decode",
-           "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_linear_decode",
+           "mxs_gemm_prefill", "mxs_device_status", "mxs_test_prefill_starve", "mxs_test_decode_starve",
+           "mxs_linear_decode",
            "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer",
            "mxs_quantize_act_permuted", "mxs_pack_weight_permuted", "mxs_attention_decode_workspace_bytes",
            "mxs_attention_decode", "mxs_linear_decode_group", "mxs_quantize_act_group",
@@ -84,6 +85,8 @@ def lib() -> ctypes.CDLL:
         L.mxs_gemm_prefill.restype = I
         L.mxs_test_prefill_starve.argtypes = [P, P, P, I64, I64, I64, P, I64, I, P]
         L.mxs_test_prefill_starve.restype = I
+        L.mxs_test_decode_starve.argtypes = [P, P, P, I64, I64, I64, P, I64, I, P]
+        L.mxs_test_decode_starve.restype = I
         L.mxs_device_status.argtypes = [ctypes.POINTER(ctypes.c_int), I, P]
         L.mxs_device_status.restype = I
         D = ctypes.c_double
@@ -225,7 +228,9 @@ def gemm(codes, scales, planes, bits, packed_w, N: int, w_layout: int = W_COMPAC
     b = _Bits(bits)
     K = 32 * len(b) if K is None else K
     if M is None:
-        M = (codes if codes is not None else planes).shape[0] if codes is not None else M
+        if codes is None:
+            raise ValueError("gemm over activation planes needs M= (a planes buffer is flat)")
+        M = codes.shape[0]
     dev = packed_w.device
     if y is None:
         y = torch.empty((M, N), dtype=torch.float32, device=dev)
@@ -301,7 +306,7 @@ def linear_decode_group(problems, rounding: int = RNE, stream=None):
 class QuantProblem(ctypes.Structure):
     """ctypes mirror of mxs_quant_problem (include/mxs.h)."""
     _fields_ = [("x", ctypes.c_void_p), ("K", ctypes.c_int64), ("ld_x", ctypes.c_int64), ("bits", ctypes.c_void_p),
-                ("planes", ctypes.c_void_p)]
+                ("planes", ctypes.c_void_p), ("planes_bytes", ctypes.c_size_t)]
 
 
 def quantize_act_group(problems, rounding: int = RNE, stream=None):
@@ -316,7 +321,7 @@ def quantize_act_group(problems, rounding: int = RNE, stream=None):
         keep.append(b)
         if x.shape[0] != M:
             raise ValueError("every problem of a group has the same M")
-        arr[i] = QuantProblem(_ptr(x), x.shape[1], _ld(x), b.ptr, _ptr(planes))
+        arr[i] = QuantProblem(_ptr(x), x.shape[1], _ld(x), b.ptr, _ptr(planes), planes.numel() * planes.element_size())
     check(lib().mxs_quantize_act_group(ctypes.addressof(arr), len(problems), M, rounding, _stream(stream)))
     return [p[2] for p in problems]
 
@@ -356,6 +361,19 @@ def test_prefill_starve(planes, bits, packed_w, M: int, N: int, stage: int, y=No
         y = torch.zeros((M, N), dtype=torch.float32, device=packed_w.device)
     check(lib().mxs_test_prefill_starve(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), _ld(y),
                                         int(stage), _stream(stream)))
+    return y
+
+
+def test_decode_starve(planes, bits, packed_w, M: int, N: int, chunk: int, y=None, stream=None):
+    """Test hook: the decode kernel over activation planes with every CTA's
+    copy chunk `chunk` (1-based) never loaded."""
+    import torch
+    b = _Bits(bits)
+    K = 32 * len(b)
+    if y is None:
+        y = torch.zeros((M, N), dtype=torch.float32, device=packed_w.device)
+    check(lib().mxs_test_decode_starve(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), _ld(y),
+                                       int(chunk), _stream(stream)))
     return y
 
 

@@ -33,7 +33,7 @@ def test_every_declared_function_is_exported(L):
     for n in names:
         assert hasattr(L, n), n
     assert sorted(mxs.EXPORTS) == names
-    assert L.mxs_version() == 1
+    assert L.mxs_version() == 2
 
 
 def _bits(nb, seed=0, p=(0.7, 0.2, 0.1)):
@@ -222,7 +222,7 @@ def test_quantize_group_validation(L):
     b = bits.ctypes.data
 
     def prob(**kw):
-        f = dict(x=FAKE, K=128, ld_x=128, bits=b, planes=FAKE)
+        f = dict(x=FAKE, K=128, ld_x=128, bits=b, planes=FAKE, planes_bytes=1 << 16)
         f.update(kw)
         return mxs.QuantProblem(**f)
 
@@ -242,5 +242,7 @@ def test_quantize_group_validation(L):
     assert call([prob(), prob(planes=p2, ld_x=132)]) == 1
     assert call([prob(), prob(planes=p2, x=None)]) == 1
     assert call([prob(), prob(planes=p2 + 8)]) == 4
+    need = mxs.act_planes_bytes(4, 128, bits)
+    assert call([prob(), prob(planes=p2, planes_bytes=need - 1)]) == 5 and "problem 1" in mxs.last_error()
     assert call([prob(), prob()]) == 1 and "share planes" in mxs.last_error()
     assert call([prob()], M=0) == 0

@@ -269,3 +269,23 @@ def test_linear_decode_workspace_garbage_reuse_and_graph_replay(torch, M, N, nb)
         graph.replay()
         torch.cuda.synchronize()
         assert np.array_equal(y.cpu().numpy(), ys[0])
+
+
+def test_decode_bounded_wait_reports_timeout(torch):
+    """A weight chunk that never arrives, in a launch the planner splits over a
+    thread-block cluster (N = 1024: 8 row groups, K = 8192): every CTA's
+    converters give up after the wait bound, the kernel records
+    MXS_ERR_TIMEOUT, drains what it issued, frees its tensor memory and
+    returns; the context stays usable and the next decode call is exact."""
+    M, N, K = 16, 1024, 8192
+    g = I.rng(43)
+    bits = I.width_map(K // 32, 0.8, 0.15, 0.05, g)
+    xb, wb, codes, scales, packed = layer(torch, M, K, N, bits, g)
+    _, _, planes = mxs.quantize_act(U.to_dev_bf16(torch, xb), bits, want_codes=False, want_planes=True)
+    assert mxs.device_status(reset=True) in (0, 7)
+    mxs.test_decode_starve(planes, bits, packed, M, N, chunk=1)
+    assert mxs.device_status(reset=True) == 7
+    assert mxs.device_status() == 0
+    y = mxs.gemm_decode(None, None, bits, packed, N, planes=planes, M=M).cpu().numpy()
+    ref, ab = oracle_full(xb, wb, bits)
+    U.check_gemm(y, ref, ab)

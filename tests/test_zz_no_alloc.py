@@ -27,24 +27,24 @@ def torch():
     return U.torch_or_skip()
 
 
-def _layer(torch, M, K, N, p, seed):
+def _layer(torch, M, K, N, p, seed, rounding=mxs.RNE):
     g = I.rng(70, seed)
     bits = I.width_map(K // 32, *p, g)
     xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=30.0)
     wb = I.normal_bf16((N, K), 0.02, g)
-    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits, rounding=rounding)
     torch.cuda.synchronize()  # weights are static before the first decode call
     return bits, xb, wb, packed
 
 
-def _noalloc(torch, x, bits, packed, N):
+def _noalloc(torch, x, bits, packed, N, rounding=mxs.RNE):
     """One call straight through the C ABI (no workspace argument exists)."""
     L = mxs.lib()
     M, K = x.shape
     y = torch.full((M, N), float("nan"), device="cuda")
     b = np.ascontiguousarray(bits, np.uint8)
     rc = L.mxs_linear_decode_noalloc(ctypes.c_void_p(x.data_ptr()), M, K, x.stride(0),
-                                     b.ctypes.data_as(ctypes.c_void_p), mxs.RNE, ctypes.c_void_p(packed.data_ptr()),
+                                     b.ctypes.data_as(ctypes.c_void_p), rounding, ctypes.c_void_p(packed.data_ptr()),
                                      N, ctypes.c_void_p(y.data_ptr()), y.stride(0), None)
     assert rc == 0, mxs.last_error()
     return y
@@ -67,3 +67,23 @@ def test_noalloc_matches_workspace_path_on_two_calls_in_a_row(torch):
         w_s, w_c = mxo.quantize_bf16(wb, bits)
         _, abssum = mxo.gemm(bits, a_c, a_s, w_c, w_s)
         U.check_gemm(y.cpu().numpy(), y_ws.astype(np.float64), abssum)
+
+
+def test_noalloc_at_the_size_limit_under_both_roundings(torch):
+    """The largest planes the array holds in practice: 16 tokens, K = 49152,
+    every block 8-bit (1,966,080 of the 2 MiB), under ties-to-even and
+    ties-away rounding, two calls in a row against the workspace path."""
+    M, K, N = 16, 49152, 256
+    bits_all8 = np.full(K // 32, 8, np.uint8)
+    assert 1_900_000 < mxs.act_planes_bytes(M, K, bits_all8) <= 2 << 20
+    for rounding in (mxs.RHAZ, mxs.RNE):
+        bits, xb, wb, packed = _layer(torch, M, K, N, (0, 0, 1), 9, rounding)
+        assert np.all(bits == 8)
+        x = U.to_dev_bf16(torch, xb)
+        y_na = _noalloc(torch, x, bits, packed, N, rounding)
+        y_ws = mxs.linear_decode(x, bits, packed, N, rounding=rounding).cpu().numpy()
+        a_s, a_c = mxo.quantize_bf16(xb, bits, rounding=rounding)
+        w_s, w_c = mxo.quantize_bf16(wb, bits, rounding=rounding)
+        ref, abssum = mxo.gemm(bits, a_c, a_s, w_c, w_s)
+        U.check_gemm(y_na.cpu().numpy(), y_ws.astype(np.float64), abssum)
+        U.check_gemm(y_na.cpu().numpy(), ref, abssum)
