@@ -589,6 +589,34 @@ def _gpu_uuid(torch, dev):
         return None
 
 
+def probe_peaks(torch):
+    """Tensor-core rates measured on this GPU with mxs_probe_mma (one CTA per
+    SM, back-to-back MMAs over zero operands, best of three launches): the
+    block-scaled FP8 MMA the prefill GEMM issues for 4-bit blocks, the bf16
+    MMA it issues for 6/8-bit blocks (both M = 128, N = 256), and the legacy
+    mma.sync s8 rate (this part's INT8 tensor path).  TFLOP/s (TOPS for s8)."""
+    from paper_2607_17733_gb300 import mxs
+    out = {}
+    for name, kind, n, iters in (("fp8_block_scaled_tflops", mxs.PROBE_FP8, 256, 20000),
+                                 ("bf16_tflops", mxs.PROBE_BF16, 256, 20000),
+                                 ("s8_mma_sync_tops", mxs.PROBE_S8_MMA_SYNC, 16, 100000)):
+        for _ in range(2):
+            mxs.probe_mma(kind, n, iters)
+        torch.cuda.synchronize()
+        best = 0.0
+        for _ in range(3):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            flop = mxs.probe_mma(kind, n, iters)
+            e1.record()
+            torch.cuda.synchronize()
+            best = max(best, flop / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+        out[name] = best
+    if mxs.probe_status(reset=True) != 0:
+        return {}
+    return out
+
+
 def run_prefill_part(args, spec: Spec):
     """Prefill step of `spec` (M = spec.Ms[0] tokens) through the seven
     projections of the layers spec.layer_ids.  Per stage of a layer (q/k/v,
@@ -698,6 +726,8 @@ def run_prefill_part(args, spec: Spec):
     value = ws * step_ops / (ms * 1e-3) / 1e12
     q_gbs = q_bytes / (quant_ms * 1e-3) / 1e9
 
+    probes = probe_peaks(torch) if rank == 0 else {}
+
     # end to end: the step's activations from pinned host memory, every output back
     x_host = [x.cpu().pin_memory() for x in xs]
     y_host = [torch.empty(tuple(y.shape), dtype=torch.float32).pin_memory() for y in ys]
@@ -743,6 +773,10 @@ def run_prefill_part(args, spec: Spec):
                      "peak": fp8_peak, "unit": "TFLOP/s", "frac": achieved / fp8_peak,
                      "peak_source": pk["source"] + " bf16 x 2 (fp8/bf16 nominal ratio)",
                      "issued_fp8_equivalent": issued, "issued_frac": issued / fp8_peak,
+                     "probe": probes,
+                     "frac_of_probe_fp8": achieved / probes["fp8_block_scaled_tflops"] if probes else None,
+                     "issued_frac_of_probe_fp8": issued / probes["fp8_block_scaled_tflops"] if probes else None,
+                     "frac_of_s8_mma_sync": achieved / probes["s8_mma_sync_tops"] if probes else None,
                      "traffic": profile_traffic("gemm_prefill.cu", prof),
                      "gemm_ms_per_step": gemm_ms, "share_of_step": gemm_ms / ms},
         "quantizer": {"kernel": "quantize_act_group_kernel / quantize_act_kernel (bf16 in, MMA planes out)",

@@ -398,6 +398,30 @@ MXS_API int mxs_attention_decode_batch(const void *q_bf16, int64_t B, int64_t H,
                                        const int32_t *lengths, int64_t T_cap, float scale, float *out,
                                        void *workspace, size_t ws_bytes, void *stream);
 
+/* ---------------------------------------------------------------- tensor-core rate probes
+ * Measurement only (not on the layer's path; the paper has no counterpart):
+ * the denominators of the GEMMs' rooflines, and the cost of the small MMAs
+ * the decode GEMM issues.  One CTA per SM; thread 0 of each issues `iters`
+ * MMAs back to back into one tensor-memory accumulator over all-zero
+ * operands, commits them and waits (bounded) for completion:
+ *   kind 0  tcgen05.mma kind::mxf8f6f4 block_scale (e4m3, UE8M0 per 32),
+ *           M = 128, N = n, K = 32, A and B in shared memory (the prefill
+ *           GEMM's 4-bit instruction);
+ *   kind 1  the same with A in tensor memory (the decode GEMM's instruction);
+ *   kind 2  tcgen05.mma kind::f16 (bf16 -> fp32), M = 128, N = n, K = 16;
+ *   kind 3  legacy warp MMA mma.sync m16n8k32 s8 -> s32 on four warps per
+ *           CTA (n ignored): the INT8 tensor rate of this part.
+ * n: a multiple of 16 in [16, 256].  *flop receives the launch's operations
+ * (2*M*N*K per MMA); time the launch with events on `stream`.  cycles
+ * (device int64 [SM count], 8-byte aligned, or NULL) receives each CTA's
+ * clock cycles from its first MMA to its wait's end (kinds 0-2) or its
+ * loop (kind 3).  Asynchronous.  Errors: MXS_ERR_INVALID_ARG (kind 0..3, n,
+ * iters outside [1, 2^32], flop NULL), MXS_ERR_ALIGN, MXS_ERR_CUDA.
+ * mxs_probe_status synchronises the device and reads (reset != 0: clears)
+ * the probes' status word: MXS_ERR_TIMEOUT if a wait ran out. */
+MXS_API int mxs_probe_mma(int kind, int n, int64_t iters, int64_t *cycles, double *flop, void *stream);
+MXS_API int mxs_probe_status(int *status, int reset);
+
 /* ---------------------------------------------------------------- offline allocation
  * Calibration that produces the width maps (Alg. 1, Alg. 3, Theorem 1).  Not
  * on the inference path; run once per model over calibration activations.

@@ -79,6 +79,12 @@ constexpr int kMinSmem = 116 * 1024;   // one CTA per SM (each allocates all of 
 constexpr int kQuadBar0 = 8;           // named barriers 8..11: one per quad
 constexpr int kCodesBar = 12;          // named barrier of the token prologue (codes mode)
 constexpr long long kWaitCycles = 4000000000ll;  // ~2 s at the maximum SM clock
+#ifndef MXS_POLL_SLEEP_NS
+#define MXS_POLL_SLEEP_NS 64
+#endif
+// the producer warp's pause after a pass over its slots that moved nothing:
+// its polling would otherwise take issue slots from the converter warps
+constexpr unsigned kPollSleepNs = MXS_POLL_SLEEP_NS;
 
 struct DecodeArgs {
     const uint8_t *codes;   // [M, row_bytes] packed activation codes (codes mode)
@@ -519,6 +525,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                     atomicExch(&g_decode_status, MXS_ERR_TIMEOUT);
                 }
                 break;
+            } else if (kPollSleepNs > 0) {
+                __nanosleep(kPollSleepNs);
             }
         }
         // copies still in flight land in shared memory before the CTA exits:

@@ -30,7 +30,8 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_linear_decode_noalloc", "mxs_column_sensitivity", "mxs_allocation_r", "mxs_allocate_layer",
            "mxs_quantize_act_permuted", "mxs_pack_weight_permuted", "mxs_attention_decode_workspace_bytes",
            "mxs_attention_decode", "mxs_linear_decode_group", "mxs_quantize_act_group",
-           "mxs_attention_decode_batch_workspace_bytes", "mxs_attention_decode_batch"]
+           "mxs_attention_decode_batch_workspace_bytes", "mxs_attention_decode_batch", "mxs_probe_mma",
+           "mxs_probe_status"]
 
 _lock = threading.Lock()
 _lib = None
@@ -109,6 +110,10 @@ def lib() -> ctypes.CDLL:
         L.mxs_attention_decode_batch.argtypes = [P, I64, I64, I64, I64, P, P, P, P, P, P, P, I64, ctypes.c_float, P, P,
                                                  SZ, P]
         L.mxs_attention_decode_batch.restype = I
+        L.mxs_probe_mma.argtypes = [I, I, I64, P, ctypes.POINTER(ctypes.c_double), P]
+        L.mxs_probe_mma.restype = I
+        L.mxs_probe_status.argtypes = [ctypes.POINTER(ctypes.c_int), I]
+        L.mxs_probe_status.restype = I
         _lib = L
         return L
 
@@ -462,3 +467,20 @@ def attention_decode_batch(q, H_kv: int, k_codes, k_scales, k_bits, v_codes, v_s
 
 def attention_batch_workspace_bytes(B: int, T_cap: int, H: int, D: int) -> int:
     return _size(lib().mxs_attention_decode_batch_workspace_bytes(B, T_cap, H, D))
+
+
+# ---------------------------------------------------------------- tensor-core rate probes
+PROBE_FP8, PROBE_FP8_TMEM_A, PROBE_BF16, PROBE_S8_MMA_SYNC = 0, 1, 2, 3
+
+
+def probe_mma(kind: int, n: int, iters: int, cycles=None, stream=None) -> float:
+    """Launch the rate probe (mxs_probe_mma); returns the launch's FLOPs."""
+    flop = ctypes.c_double()
+    check(lib().mxs_probe_mma(int(kind), int(n), int(iters), _ptr(cycles), ctypes.byref(flop), _stream(stream)))
+    return flop.value
+
+
+def probe_status(reset: bool = False) -> int:
+    st = ctypes.c_int(0)
+    check(lib().mxs_probe_status(ctypes.byref(st), int(reset)))
+    return st.value

@@ -246,3 +246,15 @@ def test_quantize_group_validation(L):
     assert call([prob(), prob(planes=p2, planes_bytes=need - 1)]) == 5 and "problem 1" in mxs.last_error()
     assert call([prob(), prob()]) == 1 and "share planes" in mxs.last_error()
     assert call([prob()], M=0) == 0
+
+
+def test_probe_validation(L):
+    """The rate probe checks its arguments before any device call."""
+    f = ctypes.c_double()
+    assert L.mxs_probe_mma(4, 16, 10, None, ctypes.byref(f), None) == 1
+    assert L.mxs_probe_mma(0, 24, 10, None, ctypes.byref(f), None) == 1
+    assert L.mxs_probe_mma(0, 272, 10, None, ctypes.byref(f), None) == 1
+    assert L.mxs_probe_mma(1, 16, 0, None, ctypes.byref(f), None) == 1
+    assert L.mxs_probe_mma(2, 16, 10, None, None, None) == 1
+    assert L.mxs_probe_mma(0, 16, 10, FAKE + 4, ctypes.byref(f), None) == 4
+    assert L.mxs_probe_status(None, 0) == 1
