@@ -136,6 +136,16 @@ int launch_gemm_decode_group(const Plan *const *plans, const void *const *act_pl
                              const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, bool pdl,
                              cudaStream_t st);
 int decode_status(int *status, int reset);
+// Decode shapes of at most kGemvMaxM tokens: the activations' quantization
+// fused into a CUDA-core GEMM (dp4a integer dots, fp32 fold), up to three
+// problems that read x_i (bf16 [M, K_i], row stride ld_x_i) in one launch.
+#ifndef MXS_GEMV_MAX_M
+#define MXS_GEMV_MAX_M 4
+#endif
+constexpr int kGemvMaxM = MXS_GEMV_MAX_M;
+int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int64_t *ld_x, const void *const *packed,
+                       const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, int rounding,
+                       bool pdl, cudaStream_t st);
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N,
                         float *y, int64_t ld_y, int starve, cudaStream_t st);
 int prefill_status(int *status, int reset, cudaStream_t st);
