@@ -411,10 +411,13 @@ def run_decode(args, spec: Spec):
     else:  # the timed segment is quantize + GEMM: bf16 activations in, y out
         gemm_bytes = step_bytes
     nproj = len(spec.shapes)
-    launches_per_step = 2 * len(items)
+    # M = 1 through mxs_linear_decode(_group): one kernel (quantization fused);
+    # otherwise a quantizer launch and a GEMM launch
+    per_gemm = {M: (1 if (M == 1 and args.path in ("fused", "grouped")) else 2) for M in spec.Ms}
+    launches_per_step = sum(per_gemm[M] for M, _, _, _ in items)
     gemm_launches = len(items)
-    if args.path == "grouped":  # per stage one quantizer launch and one GEMM launch
-        launches_per_step = 2 * len(items) // nproj * len(STAGES)
+    if args.path == "grouped":  # per stage one GEMM launch, after one quantizer launch when M > 1
+        launches_per_step = sum(per_gemm[M] for M in spec.Ms) * spec.layers * len(STAGES)
         gemm_launches = len(items) // nproj * len(STAGES)
 
     # ---- the step as one CUDA graph.  Inputs are independent synthetic draws, so
@@ -519,8 +522,9 @@ def run_decode(args, spec: Spec):
         achieved = gemm_bytes / (gemm_ms * 1e-3) / 1e9
         prof = "gemm_decode_llama2_70b_decode.md" if spec.name.startswith("llama2-70b") \
             else "gemm_decode_llama3_8b_decode.md"
-        roofline = {"kernel": "gemm_decode_kernel" + (" + quantize_act_kernel (PDL chain)"
-                                                      if args.path in ("fused", "grouped") else f" ({args.path} path)"),
+        roofline = {"kernel": ("gemv_decode_kernel for M = 1 (quantization fused), gemm_decode_kernel + "
+                               "quantize_act_kernel (PDL chain) for M > 1" if args.path in ("fused", "grouped")
+                               else f"gemm_decode_kernel ({args.path} path)"),
                     "bound": "hbm", "achieved": achieved,
                     "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": achieved / pk["hbm_gbs"],
                     "peak_source": pk["source"] + " (HBM copy)",
@@ -568,7 +572,8 @@ def run_decode(args, spec: Spec):
                    "path": {"planes": "quantize to MMA planes, then GEMM over the planes (TMA)",
                             "fused": "mxs_linear_decode: quantize + GEMM chained by programmatic dependent launch",
                             "grouped": "mxs_linear_decode_group for q/k/v and gate/up (one GEMM launch per "
-                                       "group, after one quantizer launch for the group), mxs_linear_decode for o, down",
+                                       "group), mxs_linear_decode for o, down; M = 1: the CUDA-core GEMM with "
+                                       "the quantization fused, else one quantizer launch before each tensor-core GEMM",
                             "codes": "quantize to packed codes, GEMM over the codes"}[args.path],
                    "projections": [p[0] for p in spec.shapes], "maps": maps,
                    "parallelism": f"replicas x{ws}", "l2": "inputs larger than L2 (packed weights "

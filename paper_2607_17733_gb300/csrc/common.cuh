@@ -139,8 +139,10 @@ int decode_status(int *status, int reset);
 // Decode shapes of at most kGemvMaxM tokens: the activations' quantization
 // fused into a CUDA-core GEMM (dp4a integer dots, fp32 fold), up to three
 // problems that read x_i (bf16 [M, K_i], row stride ld_x_i) in one launch.
+// The kernel takes 1 <= M <= 4; the library routes M = 1 to it by default
+// (beyond one token the tensor-core path is faster, as measured on GB300).
 #ifndef MXS_GEMV_MAX_M
-#define MXS_GEMV_MAX_M 4
+#define MXS_GEMV_MAX_M 1
 #endif
 constexpr int kGemvMaxM = MXS_GEMV_MAX_M;
 int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int64_t *ld_x, const void *const *packed,

@@ -320,7 +320,7 @@ int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t 
     int64_t lds[3];
     void *pls[3];
     for (int i = 0; i < count; ++i) xs[i] = probs[i].x, lds[i] = probs[i].ld_x, pls[i] = probs[i].workspace;
-    if (M <= kGemvMaxM)  // a few tokens: quantization fused into the CUDA-core GEMM (no planes)
+    if (M <= kGemvMaxM)  // one token: quantization fused into the CUDA-core GEMM (no planes)
         return launch_gemv_decode(pp, xs, lds, packed, N, y, ld_y, count, M, rounding, true, st);
     rc = launch_quantize_group(pp, xs, lds, M, rounding, pls, count, st);  // one quantizer launch for the group
     if (rc) return rc;
@@ -388,7 +388,7 @@ int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const u
     if (M == 0 || N == 0) return MXS_OK;
     if ((rc = check_device())) return rc;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (M <= kGemvMaxM) {  // a few tokens: quantization fused into the CUDA-core GEMM (no planes)
+    if (M <= kGemvMaxM) {  // one token: quantization fused into the CUDA-core GEMM (no planes)
         const Plan *pp = &p;
         return launch_gemv_decode(&pp, &x, &ld_x, &packed_w, &N, &y, &ld_y, 1, M, rounding, true, st);
     }

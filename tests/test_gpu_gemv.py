@@ -1,8 +1,8 @@
-"""Decode with at most four tokens: the activations' quantization fused into
-the CUDA-core GEMM (mxs_linear_decode and mxs_linear_decode_group take this
-path for M <= 4) against the exact oracle; ragged shapes, K split over
-cluster ranks, NaN blocks, ties-away rounding, block scales over +-20
-binades, grouped problems."""
+"""Decode with one to four tokens through mxs_linear_decode and
+mxs_linear_decode_group (M = 1: the activations' quantization fused into the
+CUDA-core GEMM; M = 2..4: quantizer + tensor-core GEMM) against the exact
+oracle; ragged shapes, K split over cluster ranks, NaN blocks, ties-away
+rounding, block scales over +-20 binades, grouped problems."""
 import numpy as np
 import pytest
 
