@@ -62,15 +62,9 @@
  *     ceil((n6+n8)/2)):
  *       P [rows, Kp]: 4-bit slot s at bytes [32s, +32) = e4m3 m/4; padding
  *       to a multiple of 4 slots is zero; 6/8-bit slot j at 64 bytes from
- *       128*ceil(n4/4)+64j, in one of two forms:
- *         digit form (activations with M <= 16: the decode GEMM's operand):
- *         high digit then low digit (e4m3, 32 B each); b=6: m = 8h+l, digits
- *         h/2, l/16; b=8: m = 16h+l, digits h/4, l/64 (l >= 0), so that the
- *         two digits add up to m*2^-(b-2) and the block scale S applies to
- *         both unchanged;
- *         bf16 form (activations with M > 16 and weights: the prefill GEMM's
- *         operand): element i at +2i is the bf16 value m*2^(S-127-(b-2))
- *         (exact), 0x7FC0 (NaN) in a block with S = 255.
+ *       128*ceil(n4/4)+64j: element i at +2i is the bf16 value
+ *       m*2^(S-127-(b-2)) (exact), 0x7FC0 (NaN) in a block with S = 255
+ *       (for weights and activations of every M: the operand of both GEMMs).
  *       SF at align256(P + rows*Kp): per 128-row tile and 128-byte K' stage,
  *       512 B ordered [i<32][w<4][q<4] = S of row 128*tile+32w+i, slot 4*st+q
  *       (4-bit stages) or 2*(st-ceil(n4/4))+q for q<2 (6/8-bit stages); every
@@ -142,9 +136,7 @@ MXS_API int64_t mxs_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K, const 
  * Appendix A.2 activations quantized on the fly) and writes
  *   codes  [M, mxs_act_row_bytes]  packed codes (may be NULL)
  *   scales [M, K/32]               scale bytes by slot (NULL iff codes NULL)
- *   planes mxs_act_planes_bytes    MMA planes + scale tiles (may be NULL); 6/8-bit
- *                                  blocks in digit form for M <= 16 (decode),
- *                                  bf16 form for M > 16 (prefill)
+ *   planes mxs_act_planes_bytes    MMA planes + scale tiles (may be NULL)
  * At least one of codes / planes must be non-NULL. */
 MXS_API int mxs_quantize_act(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x,
                      const uint8_t *bits, int rounding,
@@ -184,9 +176,10 @@ MXS_API int mxs_gemm(const void *act_codes, const uint8_t *act_scales, const voi
              void *workspace, size_t ws_bytes, void *stream);
 
 /* Decode path only (M <= 16): weights streamed once from the compact layout by
- * bulk copies into shared memory, converted there to exact e4m3 digits and
- * multiplied on the block-scaled tensor-core MMA (tcgen05, fp32 accumulation
- * in tensor memory); when K is split over a thread-block cluster the partial
+ * bulk copies into shared memory, converted there to exact e4m3 values
+ * (4-bit blocks, on the block-scaled FP8 MMA) or bf16 values (6/8-bit blocks,
+ * on the bf16 MMA) and multiplied on the tensor cores (tcgen05, fp32
+ * accumulation in tensor memory); when K is split over a thread-block cluster the partial
  * tiles are added in rank order.  The activations are given EITHER as packed
  * codes + scales (act_planes NULL) OR as the MMA planes written by
  * mxs_quantize_act (codes and scales NULL; faster: the operand is loaded by
@@ -329,8 +322,7 @@ MXS_API int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, 
  * layers that read the same hidden state: q, k and v; gate and up), each with
  * its own width map, in one kernel launch: byte for byte what
  * mxs_quantize_act(x_i, M, K_i, ld_i, bits_i, rounding, NULL, NULL, planes_i)
- * writes (digit form for M <= 16, bf16 form of the 6/8-bit blocks for
- * M > 16), one link in the launch chain instead of one per layer.
+ * writes, one link in the launch chain instead of one per layer.
  * planes_i: device, at least mxs_act_planes_bytes(M, K_i, bits_i) bytes
  * (planes_bytes_i says how many the caller has), 16-byte aligned, distinct
  * buffers.  1 <= count <= 3.  Asynchronous on `stream`

@@ -8,21 +8,24 @@
 // Decode reads every weight byte once, so the kernel streams the weights in
 // their compact form (4-bit nibbles, 6/8-bit bytes) and does all arithmetic on
 // the tensor core:
-//   * the block-scaled FP8 MMA (tcgen05.mma kind::mxf8f6f4, scale_vec::1X)
-//     with 128 weight rows as the A operand -- in tensor memory -- and the
-//     <= 16 tokens as the N = 16 B operand in shared memory; per-block scales
-//     are applied by the hardware and the sum over K stays in fp32
-//     tensor-memory accumulators;
-//   * a weight code of magnitude <= 15 is fed as the e4m3 byte
+//   * 128 weight rows are the A operand -- in tensor memory -- and the <= 16
+//     tokens the N = 16 B operand in shared memory; the sum over K stays in
+//     fp32 tensor-memory accumulators;
+//   * a 4-bit block runs on the block-scaled FP8 MMA (tcgen05.mma
+//     kind::mxf8f6f4, scale_vec::1X): its weight code is fed as the e4m3 byte
 //     (sign << 7) | |m|, whose value is |m| * 2^-9 (subnormals and the first
-//     binade); 6/8-bit codes split as |m| = 16h + l into two such digits
-//     (Sec. 6: high- and low-precision parts multiplied separately).  The
-//     fixed-point weight of each digit goes into the E8M0 scale byte (+7 for
-//     a 4-bit code, +9/+5 for the high/low digit of a 6-bit code, +7/+3 for
-//     an 8-bit one), so every MMA term is exact;
+//     binade), with the code's fixed-point weight in the E8M0 scale byte (+7),
+//     and the hardware applies the per-block scales;
+//   * a 6/8-bit block runs on the bf16 MMA (kind::f16, two K = 16 MMAs): its
+//     codes become the exact bf16 values m * 2^(Sw-127-(b-2)) (two integer
+//     operations and one exact bf16 subtraction per two codes), and the
+//     token operand holds the activations' bf16 values the same way; every
+//     MMA term is exact.  (Two e4m3 digits per code on both sides, Sec. 6's
+//     high/low split, took four FP8 MMAs per block: the MMA's fixed issue
+//     cost makes two bf16 MMAs cheaper);
 //   * the token operand is the activations' MMA-plane form (the layout the
-//     prefill GEMM reads: e4m3 values m/4, or a high and a low digit, under
-//     the block's own scale byte).  It is either loaded by TMA from planes
+//     prefill GEMM reads: e4m3 values m/4 under the block's own scale byte,
+//     or bf16 values).  It is either loaded by TMA from planes
 //     written by mxs_quantize_act -- the launch may then overlap the kernel
 //     before it (programmatic dependent launch) -- or built in the prologue
 //     from packed codes.
@@ -32,8 +35,8 @@
 // a shared-memory ring with cp.async.bulk (about 17 KB per copy, up to eight
 // in flight: the ring, not registers, holds the bytes in flight).  Four quads
 // of four worker warps take the chunks round robin; each warp converts its 32
-// rows (its tensor-memory lane quarter) of a stage and writes the e4m3 digits
-// straight into the quad's A tile in tensor memory (tcgen05.st), the quad
+// rows (its tensor-memory lane quarter) of a stage and writes the e4m3 or
+// bf16 values straight into the quad's A tile in tensor memory (tcgen05.st), the quad
 // meets at a hardware named barrier, and one thread issues the stage's MMAs
 // into the quad's accumulator.  Quads never wait for one another; the
 // epilogue warps add the quads' partial accumulators in quad order (a fixed
@@ -48,8 +51,9 @@
 // drains what it issued and frees tensor memory.  The quads' named barrier
 // carries an AND of the four warps' status, so a warp that gave up stops its
 // quad at the next stage instead of leaving the others at the barrier.
-// Weight scale bytes above 245 (|w| >= 2^118) saturate at 254 after the digit
-// shift.
+// Weight scale bytes above 247 of a 4-bit block (|w| >= 2^120) saturate at
+// 254 after the shift, as do those above 251 (6-bit) and 253 (8-bit) in the
+// bf16 exponent.
 #include <algorithm>
 #include <cstring>
 #include <cooperative_groups.h>
@@ -242,6 +246,18 @@ constexpr uint32_t kIdesc = ((uint32_t)(16 >> 3) << 17) | (1u << 23) | ((uint32_
 __device__ __forceinline__ constexpr uint32_t idesc(int sfa_id, int sfb_id) {
     return kIdesc | ((uint32_t)sfb_id << 4) | ((uint32_t)sfa_id << 29);
 }
+// kind::f16, bf16 x bf16, K-major, N = 16, M = 128, f32 accumulator
+constexpr uint32_t kIdescF16 =
+    (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(16 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+// the bf16 MMA with the A operand in tensor memory (K-major: row i in lane i,
+// two 16-bit elements per 32-bit column)
+__device__ __forceinline__ void mma_f16_t(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t accum) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %3, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %4, p;\n}" ::"r"(d),
+        "r"(a_tmem), "l"(b), "r"(accum), "r"(kIdescF16)
+        : "memory");
+}
 // the same with the A operand in tensor memory (K-major: row i in lane i, four
 // 8-bit elements per 32-bit column)
 __device__ __forceinline__ void mma_mx_t(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t id, uint32_t sfa,
@@ -284,14 +300,27 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
 // byte offset of 16-byte chunk c (0..7) of row r in a 128B-swizzled K-major tile
 __device__ __forceinline__ uint32_t sw128(int r, int c) { return (r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4); }
 
-// e4m3 digit bytes (sign << 7) | |m| of the four low / four high
+// e4m3 bytes (sign << 7) | |m| of the four low / four high
 // sign-magnitude nibbles (s << 3) | |m| held in a word
 __device__ __forceinline__ uint32_t lo_nib(uint32_t w) { return (w & 0x07070707u) | ((w << 4) & 0x80808080u); }
 __device__ __forceinline__ uint32_t hi_nib(uint32_t w) { return ((w >> 4) & 0x07070707u) | (w & 0x80808080u); }
-// high (|m| >> 4) and low (|m| & 15) digit of four sign-magnitude 8-bit codes
-__device__ __forceinline__ uint32_t hi_digit(uint32_t x) { return ((x >> 4) & 0x07070707u) | (x & 0x80808080u); }
-__device__ __forceinline__ uint32_t lo_digit(uint32_t x) { return x & 0x8F8F8F8Fu; }
-// four scale bytes carrying their digits' fixed-point weights (shift per byte
+// bf16 pair of two 7-bit sign-magnitude codes (s << 7) | m spread by prmt
+// into the 16-bit lanes of t (the code in the low byte, its sign replicated
+// in the high one): with eb = E in each lane's exponent field, (s | E | m) -
+// (s | E) = +-m * 2^(E-134), exact (a NaN when eb holds the NaN pattern)
+__device__ __forceinline__ uint32_t bf16_codes(uint32_t t, uint32_t eb) {
+    const uint32_t y = (t & 0x807F807Fu) | eb;
+    const uint32_t o = (t & 0x80008000u) | eb;
+    uint32_t d;
+    asm("fma.rn.bf16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(o), "r"(0xBF80BF80u), "r"(y));  // y - o
+    return d;
+}
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+    return d;
+}
+// four scale bytes carrying their codes' fixed-point weights (shift per byte
 // in `add`), saturating at 254; 255 (NaN) stays
 __device__ __forceinline__ uint32_t shifted4(uint32_t S4, uint32_t add) {
     const uint32_t t = __vminu4(__vaddus4(S4, add), 0xFEFEFEFEu);
@@ -597,47 +626,35 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                             }
                             sfw = shifted4(sb, 0x07070707u);
                         } else {
-                            uint4 v0[2], v1[2];
-                            uint32_t sb = 0, add = 0;
+                            // two 6/8-bit slots as bf16 values m * 2^(Sw-127-(b-2)) (the scale inside,
+                            // no scale tile): row r's 32 codes of slot h at K' bytes 64h .. 64h+63
 #pragma unroll
                             for (int h = 0; h < 2; ++h) {
-                                v0[h] = v1[h] = make_uint4(0, 0, 0, 0);
+                                uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
+                                uint32_t eb = (1u << 7) | (1u << 23);  // absent slot: zeros
                                 if (h < nsl) {
-                                    v0[h] = *reinterpret_cast<const uint4 *>(s0 + 4224 * h + 32 * r);
-                                    v1[h] = *reinterpret_cast<const uint4 *>(s0 + 4224 * h + 32 * r + 16);
-                                    sb |= (uint32_t)s0[4224 * h + 4096 + r] * (0x0101u << (16 * h));
-                                    // byte 2h: the high digit's shift, byte 2h+1: the low digit's
-                                    add |= (slot_width(p, lo + h) == 6 ? 0x0509u : 0x0307u) << (16 * h);
+                                    v0 = *reinterpret_cast<const uint4 *>(s0 + 4224 * h + 32 * r);
+                                    v1 = *reinterpret_cast<const uint4 *>(s0 + 4224 * h + 32 * r + 16);
+                                    const int Sw = s0[4224 * h + 4096 + r];
+                                    // exponent field E = Sw + 7 - (b - 2), so that m * 2^(E-134) is the value
+                                    const uint32_t E = (uint32_t)min(Sw + 9 - slot_width(p, lo + h), 254);
+                                    eb = Sw == 255 ? 0x7FC07FC0u : (E << 7) | (E << 23);
+                                }
+                                const uint32_t w[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+                                for (int i = 0; i < 8; ++i) {  // word i: elements 4i .. 4i+3
+                                    d[16 * h + 2 * i] = bf16_codes(prmt(w[i], 0u, 0x9180u), eb);
+                                    d[16 * h + 2 * i + 1] = bf16_codes(prmt(w[i], 0u, 0xB3A2u), eb);
                                 }
                             }
-#pragma unroll
-                            for (int h = 0; h < 2; ++h) {
-                                // high digits at K' bytes 64h.., low digits at 64h+32..
-                                d[16 * h + 0] = hi_digit(v0[h].x);
-                                d[16 * h + 1] = hi_digit(v0[h].y);
-                                d[16 * h + 2] = hi_digit(v0[h].z);
-                                d[16 * h + 3] = hi_digit(v0[h].w);
-                                d[16 * h + 4] = hi_digit(v1[h].x);
-                                d[16 * h + 5] = hi_digit(v1[h].y);
-                                d[16 * h + 6] = hi_digit(v1[h].z);
-                                d[16 * h + 7] = hi_digit(v1[h].w);
-                                d[16 * h + 8] = lo_digit(v0[h].x);
-                                d[16 * h + 9] = lo_digit(v0[h].y);
-                                d[16 * h + 10] = lo_digit(v0[h].z);
-                                d[16 * h + 11] = lo_digit(v0[h].w);
-                                d[16 * h + 12] = lo_digit(v1[h].x);
-                                d[16 * h + 13] = lo_digit(v1[h].y);
-                                d[16 * h + 14] = lo_digit(v1[h].z);
-                                d[16 * h + 15] = lo_digit(v1[h].w);
-                            }
-                            sfw = shifted4(sb, add);
+                            sfw = 0;
                         }
                         if (st == st_end - 1) {
                             // the chunk's last stage is in registers: its weight bytes are free
                             __syncwarp();
                             if (lane == 0) mbar_arrive(&empty_c[s]);
                         }
-                        // absent slots: zero digits (their scale bytes do not matter)
+                        // absent slots: zero values (their scale bytes do not matter)
                         // the row's 128 K' bytes into its lane of the quad's A tile (32 columns)
                         tmem_st32(tmem + a_lane + kACol + 32 * (2 * j + buf), d);
                         // scale tile: row r = 32 qtr + lane at lane `lane`, column qtr; byte = sf id
@@ -672,10 +689,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                             fence_after();
                             const uint32_t sfa_t = tmem + kSfaCol + 4 * (2 * j + buf);
                             const uint32_t sfb_t = tmem + kSfbCol + 4 * (2 * j + buf);
-                            tmem_cp_sf(sfa_t, dsfa + 32 * buf);
-                            // token scales: the chunk's tile (planes mode) or the resident one
-                            tmem_cp_sf(sfb_t, from_planes ? desc_sf(su32(slot_base + 2 * kTokBytes)) + 32 * (st - 2 * k)
-                                                          : dsfb + 32 * st);
+                            if (st < S.st4) {
+                                tmem_cp_sf(sfa_t, dsfa + 32 * buf);
+                                // token scales: the chunk's tile (planes mode) or the resident one
+                                tmem_cp_sf(sfb_t, from_planes ? desc_sf(su32(slot_base + 2 * kTokBytes)) +
+                                                                    32 * (st - 2 * k)
+                                                              : dsfb + 32 * st);
+                            }
                             const uint32_t acc = tmem + kAccCol + kAccCols * (2 * j + b);
                             const uint32_t aT = tmem + kACol + 32 * (2 * j + buf);
                             const uint64_t db = from_planes
@@ -683,22 +703,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
                                                     : dB + (uint64_t)(st * (kTokBytes >> 4));
                             const uint32_t accum = first ? 0u : 1u;
                             if (st < S.st4) {
-                                // slot q: weight digits at columns 8q.. (K' bytes 32q..), token values at 32q..
+                                // slot q: weight values at columns 8q.. (K' bytes 32q..), token values at 32q..
                                 mma_mx_t(acc, aT, db, idesc(0, 0), sfa_t, sfb_t, accum);
                                 mma_mx_t(acc, aT + 8, db + 2, idesc(1, 1), sfa_t, sfb_t, 1u);
                                 mma_mx_t(acc, aT + 16, db + 4, idesc(2, 2), sfa_t, sfb_t, 1u);
                                 mma_mx_t(acc, aT + 24, db + 6, idesc(3, 3), sfa_t, sfb_t, 1u);
                             } else {
-                                // slot h: weight digit pa (high, low) at K' bytes 64h + 32pa under scale
-                                // 2h + pa; token digit pb at 64h + 32pb under the slot's scale byte h
-                                mma_mx_t(acc, aT, db, idesc(0, 0), sfa_t, sfb_t, accum);
-                                mma_mx_t(acc, aT, db + 2, idesc(0, 0), sfa_t, sfb_t, 1u);
-                                mma_mx_t(acc, aT + 8, db, idesc(1, 0), sfa_t, sfb_t, 1u);
-                                mma_mx_t(acc, aT + 8, db + 2, idesc(1, 0), sfa_t, sfb_t, 1u);
-                                mma_mx_t(acc, aT + 16, db + 4, idesc(2, 1), sfa_t, sfb_t, 1u);
-                                mma_mx_t(acc, aT + 16, db + 6, idesc(2, 1), sfa_t, sfb_t, 1u);
-                                mma_mx_t(acc, aT + 24, db + 4, idesc(3, 1), sfa_t, sfb_t, 1u);
-                                mma_mx_t(acc, aT + 24, db + 6, idesc(3, 1), sfa_t, sfb_t, 1u);
+                                // two 6/8-bit slots as bf16 values on both sides (scales inside):
+                                // four K = 16 MMAs over K' bytes 32q .. 32q+31
+                                mma_f16_t(acc, aT, db, accum);
+                                mma_f16_t(acc, aT + 8, db + 2, 1u);
+                                mma_f16_t(acc, aT + 16, db + 4, 1u);
+                                mma_f16_t(acc, aT + 24, db + 6, 1u);
                             }
                             mma_commit(&a_free[2 * j + buf]);  // A tile + scale tiles free once read
                             if (from_planes && st == st_end - 1) mma_commit(&empty_t[s]);  // token tiles free once read
@@ -751,27 +767,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_decode_kernel(const __grid_c
 #pragma unroll
                     for (int i = 0; i < 32; ++i) m[i] = (int)(int8_t)(w8[i >> 2] >> (8 * (i & 3)));
                 }
-                // the plane form of the prefill layout: m/4 (4-bit), or a high digit
-                // floor(m / 2^sh) and a low digit m mod 2^sh, scaled so that they sum
-                // to m * 2^-(b-2) (6/8-bit)
+                // the plane form: m/4 (4-bit, block-scaled), or the bf16 values
+                // m * 2^(Sa-127-(b-2)) (6/8-bit; NaN for a NaN block)
                 uint32_t d0[8], d1[8];
-                const int sh = b == 6 ? 3 : 4;
-                const float fh = b == 6 ? 0.5f : 0.25f, fl = b == 6 ? 0.0625f : 0.015625f;
+                const float fv = b == 4 ? 0.25f : (Sa == 255 ? __int_as_float(0x7FC00000) : pow2f((int)Sa - 125 - b));
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     if (b == 4) {
-                        d0[i] = e4m3x2(0.25f * m[4 * i], 0.25f * m[4 * i + 1]) |
-                                ((uint32_t)e4m3x2(0.25f * m[4 * i + 2], 0.25f * m[4 * i + 3]) << 16);
+                        d0[i] = e4m3x2(fv * m[4 * i], fv * m[4 * i + 1]) |
+                                ((uint32_t)e4m3x2(fv * m[4 * i + 2], fv * m[4 * i + 3]) << 16);
                         d1[i] = 0;
                     } else {
-                        int hd[4], ld[4];
-#pragma unroll
-                        for (int k = 0; k < 4; ++k) {
-                            hd[k] = m[4 * i + k] >> sh;
-                            ld[k] = m[4 * i + k] & ((1 << sh) - 1);
-                        }
-                        d0[i] = e4m3x2(fh * hd[0], fh * hd[1]) | ((uint32_t)e4m3x2(fh * hd[2], fh * hd[3]) << 16);
-                        d1[i] = e4m3x2(fl * ld[0], fl * ld[1]) | ((uint32_t)e4m3x2(fl * ld[2], fl * ld[3]) << 16);
+                        d0[i] = bf16x2(fv * m[2 * i], fv * m[2 * i + 1]);            // elements 0..15
+                        d1[i] = bf16x2(fv * m[16 + 2 * i], fv * m[17 + 2 * i]);      // elements 16..31
                     }
                 }
                 int st, pos, sfid;

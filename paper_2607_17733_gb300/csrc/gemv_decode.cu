@@ -29,9 +29,9 @@
 // product is exact: |D| < 2^20 times a power of two).  The sets' sums are
 // added in set order; cluster ranks write theirs into rank 0's shared memory
 // (distributed shared-memory stores, then a cluster barrier) and rank 0 adds
-// them in rank order: deterministic.  One thread streams the group's weight
-// bytes into L2 ahead of the loads (bulk L2 prefetches), so the loads are L2
-// hits.
+// them in rank order: deterministic.  Lanes of warp 0 stream the group's
+// weight bytes into L2 ahead of the loads (bulk L2 prefetches, issued in
+// turn), so the loads are L2 hits.
 #include <algorithm>
 #include <cstring>
 #include <cooperative_groups.h>
@@ -54,7 +54,14 @@ constexpr int kGMaxProblems = 3;
 #endif
 constexpr int kPrefetchAhead = MXS_GEMV_AHEAD_KB * 1024;  // bytes of the weight stream kept in flight to L2
 constexpr int kUnroll4 = MXS_GEMV_UNROLL;  // 4-bit slots a thread loads before it computes
-constexpr int kPrefetchChunk = 16 * 1024;
+#ifndef MXS_GEMV_PF_KB
+#define MXS_GEMV_PF_KB 64
+#endif
+#ifndef MXS_GEMV_PF_LANES
+#define MXS_GEMV_PF_LANES 1
+#endif
+constexpr int kPrefetchChunk = MXS_GEMV_PF_KB * 1024;  // bytes per bulk L2 prefetch
+constexpr int kPfLanes = MXS_GEMV_PF_LANES;            // lanes of warp 0 that issue them, in turn
 
 struct GemvProblem {
     const uint16_t *x;  // bf16 [M, K], row stride ld_x
@@ -145,11 +152,13 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
     const int64_t head = imin64(rbytes, kPrefetchAhead);
     int64_t pf = 0;     // bytes of the current group's range prefetched
     bool next_out = false;  // the next group's head has been prefetched
+    // the prefetch state is kept alike in lanes 0 .. kPfLanes-1; chunk i of a
+    // range is issued by lane i % kPfLanes
     auto prefetch_range = [&](const uint8_t *base, int64_t from, int64_t to) {
-        for (int64_t q = from; q < to; q += kPrefetchChunk)
+        for (int64_t q = from + (int64_t)tid * kPrefetchChunk; q < to; q += (int64_t)kPfLanes * kPrefetchChunk)
             prefetch_l2(base + q, (uint32_t)imin64(kPrefetchChunk, to - q));
     };
-    if (tid == 0 && ngroups > 0) {
+    if (tid < kPfLanes && ngroups > 0) {
         prefetch_range(P.w + (int64_t)bx * P.GB + r0, 0, head);
         pf = head;
     }
@@ -206,12 +215,12 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
         float acc[MT];
 #pragma unroll
         for (int t = 0; t < MT; ++t) acc[t] = 0.0f;
-        if (tid == 0 && gi > 0) {  // the head of this group went out with the previous one
+        if (tid < kPfLanes && gi > 0) {  // the head of this group went out with the previous one
             pf = next_out ? head : 0;
             next_out = false;
         }
         auto advance = [&](int64_t done) {
-            if (tid != 0) return;
+            if (tid >= kPfLanes) return;
             const int64_t to = imin64(rbytes, done + kPrefetchAhead);
             if (pf < to) {
                 prefetch_range(rng, pf, to);
@@ -303,7 +312,7 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
                 }
             }
         }
-        advance(rbytes);  // (thread 0) the rest of this range and the next group's head
+        advance(rbytes);  // (the prefetch lanes) the rest of this range and the next group's head
 
         // ---- the sets' sums in set order, then the ranks' in rank order
 #pragma unroll

@@ -4,8 +4,9 @@
 // Appendix A.2 (activations of every linear layer are quantized at run time).
 // One lane owns one 32-element block: it issues its four 128-bit loads
 // together, finds the block maximum with packed bf16 max instructions, and
-// writes its block's packed codes (16 B of nibbles or 32 B of int8), its e4m3
-// MMA planes (32 B per digit plane) and its scale byte.  The work is
+// writes its block's packed codes (16 B of nibbles or 32 B of int8), its MMA
+// plane (32 B of e4m3 m/4 for a 4-bit block, 64 B of bf16 values for a
+// 6/8-bit one) and its scale byte.  The work is
 // enumerated in slot (grouped) order, so a warp writes 32 consecutive slots
 // of one row and the lanes of one K' stage combine their scale bytes into
 // one 32-bit word of the scale tile.  The grid is rows x slots.
@@ -22,9 +23,8 @@
 //    this holds) and its low bits are m in two's complement.  Ties away from
 //    zero instead floor |y| + 1/2 with a round-toward-zero addition of 2^23
 //    (|y| + 1/2 is exact wherever its floor is not 0).
-//  * The MMA digits come from the same word: lo = m mod 2^sh is read from its
-//    low bits, hi = (m - lo) / 2^sh by exact float arithmetic, and both are
-//    converted to e4m3 exactly.
+//  * The MMA planes come from the same word: m/4 converted to e4m3, or
+//    m * 2^(S-127-(b-2)) converted to bf16, both exactly.
 // Blocks whose maximum is below 2^-119 (S < 8) take a slower path: 2^(b-2-E)
 // is then not a normal float, so x is first scaled by 2^8 (exact) and the
 // clamp is done in float.
@@ -37,7 +37,6 @@ namespace {
 
 constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23: C + m has m in its low bits
 constexpr float kTwo23 = 8388608.0f;
-constexpr float kTwo22 = 4194304.0f;
 constexpr int kCtaThreads = 256;
 
 struct QuantArgs {
@@ -46,7 +45,6 @@ struct QuantArgs {
     int V;  // work slots per row (with plane padding when planes are written)
     uint8_t *codes, *scales, *planes, *sf;
     const int32_t *perm;  // column order (Alg. 3): block kb holds columns perm[32 kb ..], or nullptr
-    int bf16_68;          // planes of 6/8-bit blocks as bf16 values (the prefill operand), else e4m3 digits
 };
 
 // low bytes of four words, in order
@@ -65,12 +63,6 @@ __device__ __forceinline__ void fma2(float &d0, float &d1, float a0, float a1, f
         " fma.rn.f32x2 d, a, b, c;\n mov.b64 {%0, %1}, d;\n}"
         : "=f"(d0), "=f"(d1)
         : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
-}
-__device__ __forceinline__ void sub2(float &d0, float &d1, float a0, float a1, float b0, float b1) {
-    asm("{\n .reg .b64 a, b, d;\n mov.b64 a, {%2, %3};\n mov.b64 b, {%4, %5};\n"
-        " sub.rn.f32x2 d, a, b;\n mov.b64 {%0, %1}, d;\n}"
-        : "=f"(d0), "=f"(d1)
-        : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
 }
 __device__ __forceinline__ uint32_t bf2_clamp(uint32_t w, uint32_t hi, uint32_t lo) {
     uint32_t r;
@@ -104,8 +96,8 @@ __device__ __forceinline__ void quantize_rows(const Plan &p, const QuantArgs &a)
     }
     const bool in_row = vs < a.V;
     const bool live = in_row && s >= 0;
-    // padding slots are written as zero digits: one plane in the 4-bit
-    // region, two in the 6/8-bit region
+    // padding slots are written as zeros: 32 plane bytes in the 4-bit region,
+    // 64 in the 6/8-bit region
     const int b = s >= 0 ? slot_width(p, s) : (vs < 4 * p.st4 ? 4 : 8);
     const float Q = (float)((1 << (b - 1)) - 1);
     const int kb = live ? p.slot_block[s] : 0;
@@ -221,7 +213,7 @@ __device__ __forceinline__ void quantize_rows(const Plan &p, const QuantArgs &a)
                     }
                     pl[h] = make_uint4(c[0] | (c[1] << 16), c[2] | (c[3] << 16), c[4] | (c[5] << 16),
                                        c[6] | (c[7] << 16));
-                } else if (a.bf16_68) {  // the block's values m * 2^(S-127-(b-2)) in bf16 (exact)
+                } else {  // the block's values m * 2^(S-127-(b-2)) in bf16 (exact)
                     const float fs = pow2f(S - 125 - b);
                     uint32_t cw[8];
 #pragma unroll
@@ -230,26 +222,6 @@ __device__ __forceinline__ void quantize_rows(const Plan &p, const QuantArgs &a)
                                          : bf16x2((tf[2 * i] - kMagic) * fs, (tf[2 * i + 1] - kMagic) * fs);
                     pl[2 * h] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
                     pl[2 * h + 1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
-                } else {  // m = 2^sh * hi + lo: planes hi * 2^sh * fl and lo * fl
-                    const uint32_t mask = b == 6 ? 7u : 15u;
-                    const float fl = b == 6 ? 0.0625f : 0.015625f;
-                    uint32_t ch[8], cl[8];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int j = 2 * i;
-                        const float L0 = __uint_as_float((tb[j] & mask) | 0x4B000000u);  // 2^23 + lo
-                        const float L1 = __uint_as_float((tb[j + 1] & mask) | 0x4B000000u);
-                        float hs0, hs1, ls0, ls1, d0, d1;
-                        fma2(ls0, ls1, L0, L1, fl, fl, -fl * kTwo23, -fl * kTwo23);
-                        sub2(d0, d1, tf[j], tf[j + 1], L0, L1);  // 2^22 + (m - lo), exact
-                        fma2(hs0, hs1, d0, d1, fl, fl, -fl * kTwo22, -fl * kTwo22);
-                        ch[i] = e4m3x2(hs0, hs1);
-                        cl[i] = e4m3x2(ls0, ls1);
-                    }
-                    pl[h] = make_uint4(ch[0] | (ch[1] << 16), ch[2] | (ch[3] << 16), ch[4] | (ch[5] << 16),
-                                       ch[6] | (ch[7] << 16));
-                    pl[2 + h] = make_uint4(cl[0] | (cl[1] << 16), cl[2] | (cl[3] << 16), cl[4] | (cl[5] << 16),
-                                           cl[6] | (cl[7] << 16));
                 }
             }
         }
@@ -353,7 +325,6 @@ int launch_quantize_group(const Plan *const *plans, const void *const *x, const 
         a.planes = static_cast<uint8_t *>(planes[k]);
         a.sf = a.planes + align256(M * p.kp);
         a.V = 4 * p.st4 + 2 * ((p.n68 + 1) / 2);
-        a.bf16_68 = M > 16;  // more than 16 rows are the prefill GEMM's operand
         Vmax = std::max(Vmax, a.V);
     }
     if (M == 0 || Vmax == 0) return MXS_OK;
@@ -385,7 +356,6 @@ int launch_quantize(const Plan &p, const void *x, int64_t M, int64_t ld, int rou
     a.scales = scales;
     a.planes = static_cast<uint8_t *>(planes);
     a.sf = planes ? a.planes + align256(M * p.kp) : nullptr;
-    a.bf16_68 = M > 16;  // more than 16 rows are the prefill GEMM's operand
     a.V = planes ? 4 * p.st4 + 2 * ((p.n68 + 1) / 2) : p.nb;
     if (M == 0 || a.V == 0) return MXS_OK;
     int nx, tx, ry;

@@ -32,7 +32,7 @@ def run_quantize(torch, xb, bits, rounding=mxs.RNE, planes=True, ld=None):
 def oracle_quantize(xb, bits, rounding=mxo.RNE):
     s, c = mxo.quantize_bf16(xb, bits, rounding)
     pc, ps = mxo.pack_act(bits, s, c)
-    pl, sf = mxo.planes(bits, s, c, bf16_68=xb.shape[0] > 16)  # more than 16 rows: the prefill operand form
+    pl, sf = mxo.planes(bits, s, c, bf16_68=True)  # 6/8-bit blocks as bf16 values, the operand of both GEMMs
     return pc, ps, pl, sf
 
 
@@ -161,7 +161,7 @@ def test_pack_weight_full_size_sampled(torch):
 def test_quantize_group_matches_single_launches(torch, M, rounding):
     """mxs_quantize_act_group writes, for every problem, the same planes and
     scale tiles as mxs_quantize_act of that problem alone (three widths maps
-    and K's; digit form for M <= 16, bf16 form above)."""
+    and K's)."""
     shapes = [(4096, (0.8, 0.15, 0.05)), (1024, (0.5, 0.3, 0.2)), (2080, (0.9, 0.05, 0.05))]
     probs, singles, xbs = [], [], []
     for i, (K, p) in enumerate(shapes):
@@ -191,5 +191,5 @@ def test_quantize_group_matches_single_launches(torch, M, rounding):
         assert np.array_equal(tiles_g[valid], tiles_w[valid])
         # and the oracle agrees
         s_, c_ = mxo.quantize_bf16(xb, bits, mxo.RHAZ if rounding == mxs.RHAZ else mxo.RNE)
-        pl_o, _ = mxo.planes(bits, s_, c_, bf16_68=M > 16)
+        pl_o, _ = mxo.planes(bits, s_, c_, bf16_68=True)
         assert np.array_equal(got[:M * kp].reshape(M, kp), pl_o)
