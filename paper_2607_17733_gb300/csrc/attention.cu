@@ -39,6 +39,9 @@
 namespace mxs {
 namespace {
 
+#ifndef MXS_ATT_MIN_CTAS
+#define MXS_ATT_MIN_CTAS 3
+#endif
 constexpr int kTile = 64;          // tokens per ring stage (16 per warp)
 constexpr int kWarps = 4;
 constexpr int kThreads = 32 * kWarps;
@@ -169,7 +172,7 @@ __device__ __forceinline__ int kpair_dim(int b, int r, int hi) {
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 3) attention_decode_kernel(const __grid_constant__ AttnArgs a) {
+__global__ void __launch_bounds__(kThreads, MXS_ATT_MIN_CTAS) attention_decode_kernel(const __grid_constant__ AttnArgs a) {
     constexpr int NBH = D / 32;      // blocks per head
     constexpr int KSTEPS = D / 16;   // k-steps of the score MMA
     constexpr int NT = D / 8;        // n-tiles of the weighted-sum MMA (= dims of a V segment)
