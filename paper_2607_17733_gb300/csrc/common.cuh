@@ -136,6 +136,7 @@ int launch_gemm_decode_group(const Plan *const *plans, const void *const *act_pl
                              const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, bool pdl,
                              cudaStream_t st);
 int decode_status(int *status, int reset);
+int gemv_status(int *status, int reset);
 // Decode shapes of at most kGemvMaxM tokens: the activations' quantization
 // fused into a CUDA-core GEMM (dp4a integer dots, fp32 fold), up to three
 // problems that read x_i (bf16 [M, K_i], row stride ld_x_i) in one launch.

@@ -464,10 +464,11 @@ int mxs_device_status(int *status, int reset, void *stream) {
     if (!status) return fail(MXS_ERR_INVALID_ARG, "status is NULL");
     int rc = check_device();
     if (rc) return rc;
-    int a = 0, b = 0;
+    int a = 0, b = 0, c = 0;
     if ((rc = prefill_status(&a, reset, static_cast<cudaStream_t>(stream)))) return rc;
     if ((rc = decode_status(&b, reset))) return rc;
-    *status = a ? a : b;
+    if ((rc = gemv_status(&c, reset))) return rc;
+    *status = a ? a : (b ? b : c);
     return MXS_OK;
 }
 
