@@ -87,7 +87,7 @@ extern "C" {
 #define MXS_API
 #endif
 
-#define MXS_VERSION 2
+#define MXS_VERSION 3
 #define MXS_MAX_K 65536 /* K/32 <= 2048 blocks */
 
 enum mxs_status {
@@ -127,6 +127,12 @@ MXS_API int mxs_version(void);
 MXS_API int64_t mxs_act_row_bytes(int64_t K, const uint8_t *bits);
 MXS_API int64_t mxs_act_codes_bytes(int64_t M, int64_t K, const uint8_t *bits);
 MXS_API int64_t mxs_act_planes_bytes(int64_t M, int64_t K, const uint8_t *bits);
+/* Workspace of mxs_linear_decode (and of each problem of
+ * mxs_linear_decode_group) for M tokens, K columns, N output rows: for M = 1
+ * the CUDA-core path's arrival counters (8 bytes per 128 rows) and partial
+ * sums (256 KiB); otherwise mxs_act_planes_bytes(M, K, bits).  Negative
+ * error code on bad arguments. */
+MXS_API int64_t mxs_linear_decode_workspace_bytes(int64_t M, int64_t K, int64_t N, const uint8_t *bits);
 MXS_API int64_t mxs_weight_bytes(int64_t N, int64_t K, const uint8_t *bits, int layout);
 MXS_API int64_t mxs_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K, const uint8_t *bits);
 
@@ -189,19 +195,31 @@ MXS_API int mxs_gemm_decode(const void *act_codes, const uint8_t *act_scales, co
                     const uint8_t *bits, const void *packed_w, int64_t M, int64_t N, int64_t K,
                     float *y, int64_t ld_y, void *workspace, size_t ws_bytes, void *stream);
 
-/* A1 + A4 for one linear layer at decode (M <= 16): quantizes x (bf16 [M,K],
- * row stride ld_x elements) with `bits` and `rounding` into MMA planes in
- * `workspace` (at least mxs_act_planes_bytes(M, K, bits) bytes, 16-byte
- * aligned; the same planes mxs_quantize_act writes) and returns
- * y [M,N] fp32 = x W^T like mxs_gemm_decode.  Two kernels on `stream`; the
- * GEMM is launched as a programmatic dependent of the quantizer, so its
- * weight stream starts while the activations are quantized -- and, in a chain
- * of such calls, while the previous layer finishes (Appendix A.2: activations
- * are quantized on the fly).  Hence packed_w must not be written by work that
- * is still in flight on `stream` when the call is made (weights are static;
- * pack them, then synchronise, before the first use).  x, y and the workspace
- * have the ordinary stream semantics; the workspace may be reused by the next
- * call on the same stream. */
+/* A1 + A4 for one linear layer at decode (M <= 16): y [M,N] fp32 = x W^T
+ * like mxs_gemm_decode, x bf16 [M,K] (row stride ld_x elements) quantized
+ * on the fly with `bits` and `rounding` (Appendix A.2: activations are
+ * quantized on the fly).  `workspace`: device, 16-byte aligned, at least
+ * mxs_linear_decode_workspace_bytes(M, K, N, bits) bytes, any prior contents.
+ *   M = 1: one kernel.  Its prologue quantizes x (the rule of
+ *     mxs_quantize_act) and its CUDA cores form the integer block dots from
+ *     the packed codes.  Every CTA streams an equal share of the weight bytes;
+ *     the CTAs that share a 128-row group leave their partial sums and a
+ *     tagged arrival count in the workspace, and the last to arrive adds the
+ *     partials in a fixed order (results do not depend on timing).
+ *   M > 1: the quantizer writes the activations' MMA planes into the
+ *     workspace (the planes mxs_quantize_act writes), then the tensor-core
+ *     GEMM reads them.
+ * The GEMM is launched as a programmatic dependent of the kernel before it,
+ * so its weight stream starts while the activations are produced -- in a
+ * chain of such calls, while the previous layer finishes.  Hence packed_w
+ * must not be written by work that is still in flight on `stream` when the
+ * call is made (weights are static; pack them, then synchronise, before the
+ * first use).  x, y and the workspace have the ordinary stream semantics; the
+ * workspace may be reused by the next call on the same stream (two calls in
+ * flight at once on one workspace race).  After MXS_ERR_TIMEOUT
+ * (mxs_device_status) a workspace may hold a partial count of the failed
+ * call: rewrite it (e.g. zero it) before it serves a CUDA graph that replays
+ * the failed call. */
 MXS_API int mxs_linear_decode(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits,
                               int rounding, const void *packed_w, int64_t N, float *y, int64_t ld_y,
                               void *workspace, size_t ws_bytes, void *stream);
@@ -213,9 +231,10 @@ MXS_API int mxs_linear_decode(const void *x_bf16, int64_t M, int64_t K, int64_t 
  * and launches as mxs_linear_decode, but the activation planes live in a
  * fixed 2 MiB array inside the library (a __device__ variable every GPU that
  * loads the library holds until exit) instead of a caller workspace; the call
- * allocates nothing.  Sizes whose planes exceed 2 MiB
- * (mxs_act_planes_bytes(M, K, bits) > 2 MiB; M <= 16 fits for K <= 49152
- * with any map) return MXS_ERR_BUFFER.  The first call on each device looks
+ * allocates nothing.  Sizes whose workspace exceeds 2 MiB
+ * (mxs_linear_decode_workspace_bytes(M, K, N, bits) > 2 MiB; M <= 16 fits
+ * for K <= 49152 with any map, M = 1 for N up to about 29 million) return
+ * MXS_ERR_BUFFER.  The first call on each device looks
  * up the array's device address (cudaGetSymbolAddress, current device) and
  * keeps it for the life of the process: make that first call before any
  * stream capture, and do not reset the device (cudaDeviceReset, or anything
@@ -225,7 +244,8 @@ MXS_API int mxs_linear_decode(const void *x_bf16, int64_t M, int64_t K, int64_t 
  * (each waits for the one before it as mxs_linear_decode does), calls that
  * overlap on the GPU (other streams, other host threads) race and give wrong
  * results.  Nothing in the array has to start at zero: every byte the GEMM
- * reads is written by the same call's quantizer. */
+ * reads is written by the same call (the one-token path's arrival counts are
+ * tagged per call). */
 MXS_API int mxs_linear_decode_noalloc(const void *x_bf16, int64_t M, int64_t K, int64_t ld_x, const uint8_t *bits,
                                       int rounding, const void *packed_w, int64_t N, float *y, int64_t ld_y,
                                       void *stream);
@@ -271,6 +291,17 @@ MXS_API int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits,
 MXS_API int mxs_test_decode_starve(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M,
                                    int64_t N, int64_t K, float *y, int64_t ld_y, int chunk, void *stream);
 
+/* Test hook (host only, no device): the one-token decode path's work split
+ * for `count` (1..3) problems of K[i] columns, width map bits[i] and N[i]
+ * rows on `sms` SMs.  Writes each problem's CTA count to ncta[i] and, for
+ * every CTA in launch order, four ints to spans (room for 4 * 256): its first
+ * 128-row group, the first slot (32-element block, in the plan's slot order)
+ * it takes there, its last group, and the slot where it stops there (the
+ * group's block count when it takes the group to its end).  Returns the
+ * number of CTAs, or minus an error code. */
+MXS_API int mxs_test_gemv_split(const int64_t *K, const uint8_t *const *bits, const int64_t *N, int count, int sms,
+                                int32_t *ncta, int32_t *spans);
+
 /* mxs_quantize_act_permuted / mxs_pack_weight_permuted -- the layer's
  * columns in the order of the allocation (Alg. 3 returns column lists, and the
  * 32 most sensitive columns form one 8-bit block only once they are placed
@@ -300,7 +331,7 @@ MXS_API int mxs_pack_weight_permuted(const void *w_bf16, int64_t N, int64_t K, i
  * launch, then the grouped GEMM runs as its programmatic dependent.
  * Same operands, layouts and contract as mxs_linear_decode (weights static;
  * 1 <= count <= 3; M <= 16, the same for every problem); every problem needs
- * its own workspace (mxs_act_planes_bytes(M, K, bits) bytes).  The K split of
+ * its own workspace (mxs_linear_decode_workspace_bytes(M, K, N, bits) bytes).  The K split of
  * a problem may differ from its single launch, so results agree with
  * mxs_linear_decode to fp32 rounding, not bit for bit.  Errors as
  * mxs_linear_decode, per problem (the message names it). */

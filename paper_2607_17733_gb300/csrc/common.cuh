@@ -146,9 +146,12 @@ int gemv_status(int *status, int reset);
 #define MXS_GEMV_MAX_M 1
 #endif
 constexpr int kGemvMaxM = MXS_GEMV_MAX_M;
+// ws_i: device workspace of at least gemv_workspace_bytes(M, N_i) bytes
+// (arrival counters and partial sums; any prior contents).
 int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int64_t *ld_x, const void *const *packed,
-                       const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, int rounding,
-                       bool pdl, cudaStream_t st);
+                       const int64_t *N, float *const *y, const int64_t *ld_y, void *const *ws,
+                       const size_t *ws_bytes, int count, int64_t M, int rounding, bool pdl, cudaStream_t st);
+int64_t gemv_workspace_bytes(int64_t M, int64_t N);
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N,
                         float *y, int64_t ld_y, int starve, cudaStream_t st);
 int prefill_status(int *status, int reset, cudaStream_t st);

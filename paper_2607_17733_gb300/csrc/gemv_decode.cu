@@ -18,34 +18,54 @@
 // but 3.6 ms at M = 4 against 2.43 ms), so the library sends it
 // M <= kGemvMaxM (1) tokens.
 //
-// Work.  A CTA owns 128-row weight groups (and, in a thread-block cluster, a
-// K range of them).  Prologue: it quantizes the activations of its K range
-// (x is bf16; the rule, bit for bit, of mxs_quantize_act) into shared memory
-// as int8 codes and scale bytes, in slot order.  One lane of a producer warp
-// streams the group's K range into a ring of shared-memory stages with
-// cp.async.bulk (sixteen 4-bit slots or eight 6/8-bit slots, about 34 KB per
-// stage, four stages in flight), starting before the wait for the kernel
-// before (the weights are static).  Main loop: consumer thread t of four sets
-// of 128 is weight row t % 128, and set t / 128 takes the slots
-// lo + t / 128 + 4j of a stage; per slot it reads its row's codes (16 or 32
-// bytes) and scale byte from the stage, forms the integer dots with dp4a
-// straight from the sign-magnitude codes (two integer operations and two dp4a
-// per four codes) and adds 2^(Ea'+Ew') * D into an fp32 accumulator per token
-// (the product is exact: |D| < 2^20 times a power of two).  Copies in flight
-// keep HBM busy; the consumers' integer work is what bounds the kernel.  The
-// sets' sums are added in set order; cluster ranks write theirs into rank 0's
-// shared memory (distributed shared-memory stores, then a cluster barrier)
-// and rank 0 adds them in rank order: deterministic.  Every wait on a stage is
-// bounded: on expiry the kernel records MXS_ERR_TIMEOUT (mxs_device_status),
-// skips the rest of its arithmetic while still taking its barriers, and waits
-// for its copies.
+// Work split.  The packed weights of a problem are one stream of W bytes
+// (128-row groups, each a run of 32-element slots).  Each CTA of the launch
+// takes an equal share of the bytes -- the k-th of ncta ranges, cut at slot
+// boundaries -- whatever the number of row groups, so that every SM streams
+// the same bytes (a split by whole groups or by clusters along K leaves SMs
+// idle whenever the groups do not divide the SM count).  A range covers whole
+// groups, whose rows the CTA writes to y, and partial groups at its ends,
+// whose per-row partial sums it writes to the caller's workspace; the last of
+// a group's CTAs to arrive (an arrival counter in the workspace) adds the
+// partials in CTA order and writes y: deterministic, independent of timing.
+// A CTA takes its partial groups first and hands their sums to a hand-off
+// warp (workspace stores, a release fence, one compare-and-swap, and for the
+// last arriver the ordered sum), so that the latency of that exchange overlaps
+// the streaming of the rest of its range.  (Measured on the 70B layers: with
+// one CTA per SM and equal bytes, q/k/v, o, gate/up and down took 18.1, 15.9,
+// 53.8 and 37.0 us against 19.7, 14.7, 53.8 and 38.5 us with whole groups
+// per CTA split along K over thread-block clusters, whose counts cannot match
+// 152 SMs for 64 or 80 row groups.)
+//
+// Per CTA.  Prologue: it quantizes the activations of the slots its range
+// takes (x is bf16; the rule, bit for bit, of mxs_quantize_act; four threads
+// per block, the block maximum by shuffles) into shared memory as int8 codes
+// and scale bytes.  One lane of a producer warp streams the range into a ring of
+// shared-memory stages with cp.async.bulk (sixteen 4-bit slots or eight
+// 6/8-bit slots, about 34 KB per stage, four stages in flight), starting
+// before the wait for the kernel before (the weights are static).  Main loop:
+// consumer thread t of four sets of 128 is weight row t % 128, and set t / 128
+// takes the slots lo + t / 128 + 4j of a stage; per slot it reads its row's
+// codes (16 or 32 bytes) and scale byte from the stage, forms the integer dots
+// with dp4a straight from the sign-magnitude codes and adds 2^(Ea'+Ew') * D
+// into an fp32 accumulator per token (the product is exact: |D| < 2^20 times
+// a power of two).  The sets' sums are added in set order.  Every wait on a
+// stage is bounded: on expiry the kernel records MXS_ERR_TIMEOUT
+// (mxs_device_status), skips the rest of its arithmetic and waits for its
+// copies.
+//
+// Arrival counters are 64-bit words holding a 48-bit tag, a number the host
+// draws afresh for every call, and a 16-bit count.  A CTA that finds another
+// tag takes the count for zero, and the last arriver leaves (tag, 0), so the
+// workspace needs no preparation: garbage, planes of an earlier call with
+// M > 1, or the counters of an earlier call all read as zero (unless a stale
+// word carries this call's 48-bit tag), and a CUDA graph that replays one call
+// finds its own tag with count zero.
 #include <algorithm>
+#include <atomic>
 #include <cstring>
-#include <cooperative_groups.h>
 
 #include "common.cuh"
-
-namespace cg = cooperative_groups;
 
 namespace mxs {
 
@@ -56,7 +76,8 @@ namespace {
 constexpr int kGSets = 4;                    // consumer sets; a set is 128 threads, one per weight row
 constexpr int kConsumers = 4 * kGSets;       // consumer warps
 constexpr int kCThreads = 32 * kConsumers;   // 512
-constexpr int kGThreads = kCThreads + 32;    // + the producer warp
+constexpr int kGThreads = kCThreads + 64;    // + the producer warp and the hand-off warp
+constexpr int kFixWarp = kConsumers + 1;
 constexpr int kGMaxProblems = 3;
 #ifndef MXS_GEMV_RING
 #define MXS_GEMV_RING 4
@@ -65,26 +86,61 @@ constexpr int kRing = MXS_GEMV_RING;         // shared-memory stages in flight
 constexpr int kSlots4 = 16, kSlots68 = 8;    // slots per stage: four (two) per consumer set
 constexpr int kStageBytes = 2176 * kSlots4;  // 34816 >= 8 x 4224
 constexpr long long kWaitCycles = 4000000000ll;  // ~2 s at the maximum SM clock
+constexpr int64_t kMinCtaBytes = 32768;      // a CTA streams at least this much (and more than one slot)
+constexpr int kGemvMaxCtas = 256;            // CTAs per launch at most (sizes the partial-sum area)
 
 struct GemvProblem {
-    const uint16_t *x;  // bf16 [M, K], row stride ld_x
-    const uint8_t *w;   // packed weights (compact part)
+    const uint16_t *x;           // bf16 [M, K], row stride ld_x
+    const uint8_t *w;            // packed weights (compact part)
     float *y;
-    int64_t ld_x, ld_y, GB;
-    int N, G, GS, nb, n4, n6;
-    int bound[9];       // cluster rank r owns slots [bound[r], bound[r+1])
-    int cta0, ncta;
+    unsigned long long *cnt;     // workspace: arrival counters [G]
+    float *rec;                  // workspace: partial sums [ncta][2][MT][128]
+    int64_t ld_x, ld_y, GB, W;   // W = G * GB, the problem's weight bytes
+    int N, G, nb, n4, n6;
+    int cta0, ncta;              // the problem's CTAs [cta0, cta0 + ncta)
 };
 struct GemvParams {
     GemvProblem prob[kGMaxProblems];
     uint16_t slot_block[kGMaxProblems][kMaxNb];  // slot -> block of each problem's plan
+    int4 span[kGemvMaxCtas];  // per CTA: first group, its first slot, last group, end slot in it
+    unsigned long long tag;   // this call's counter tag (48 bits, nonzero)
     int nprob, M, rhaz;
 };
 
 __host__ __device__ __forceinline__ int64_t slot_off_g(int n4, int s) {
     return s < n4 ? 2176 * (int64_t)s : 2176 * (int64_t)n4 + 4224 * (int64_t)(s - n4);
 }
-// stage k of a rank's slot range [c0, c1), 4-bit slots [c0, e4): slots [lo, hi)
+// the slot that starts at byte `off` of a group (off a slot boundary, off <= GB)
+__host__ __device__ __forceinline__ int slot_at(int n4, int64_t off) {
+    const int64_t b4 = 2176 * (int64_t)n4;
+    return off <= b4 ? (int)(off / 2176) : n4 + (int)((off - b4) / 4224);
+}
+// start of CTA k's range: the first slot boundary at or after k * W / ncta
+__host__ __device__ __forceinline__ int64_t cta_start(int k, int ncta, int64_t W, int64_t GB, int n4) {
+    if (k >= ncta) return W;
+    const int64_t b = W * k / ncta, g = b / GB, rem = b - g * GB, b4 = 2176 * (int64_t)n4;
+    const int64_t off = rem <= b4 ? (rem + 2175) / 2176 * 2176 : b4 + (rem - b4 + 4223) / 4224 * 4224;
+    return g * GB + off;
+}
+// the CTAs of a problem whose ranges meet group g: [first, last] (sp: the
+// problem's rows of the span table, n CTAs; nb slots per group)
+__host__ __device__ __forceinline__ int first_cta(const int4 *sp, int n, int g) {
+    int lo = 0, hi = n - 1;  // the last CTA that starts at or before the group's first byte
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) / 2;
+        if (sp[mid].x < g || (sp[mid].x == g && sp[mid].y == 0)) lo = mid; else hi = mid - 1;
+    }
+    return lo;
+}
+__host__ __device__ __forceinline__ int last_cta(const int4 *sp, int n, int g, int nb) {
+    int lo = 0, hi = n - 1;  // the first CTA that ends at or after the group's last byte
+    while (lo < hi) {
+        const int mid = (lo + hi) / 2;
+        if (sp[mid].z > g || (sp[mid].z == g && sp[mid].w == nb)) hi = mid; else lo = mid + 1;
+    }
+    return lo;
+}
+// stage k of a slot range [c0, c1), 4-bit slots [c0, e4): slots [lo, hi)
 __host__ __device__ __forceinline__ void stage_range(int c0, int e4, int c1, int k, int &lo, int &hi) {
     const int n4s = (e4 - c0 + kSlots4 - 1) / kSlots4;
     if (k < n4s) {
@@ -98,19 +154,17 @@ __host__ __device__ __forceinline__ void stage_range(int c0, int e4, int c1, int
 __host__ __device__ __forceinline__ int stage_count(int c0, int e4, int c1) {
     return (e4 - c0 + kSlots4 - 1) / kSlots4 + (c1 - e4 + kSlots68 - 1) / kSlots68;
 }
-// shared memory: the cluster exchange first (its offset is the same in every
-// rank), the sets' partial sums, the barriers and abort flag, the stage ring
-// (128-byte aligned), the token codes and scale bytes
-__host__ __device__ __forceinline__ size_t off_part(int GS, int MT) { return (size_t)2 * GS * MT * 128 * 4; }
-__host__ __device__ __forceinline__ size_t off_bars(int GS, int MT) {
-    return off_part(GS, MT) + (size_t)kGSets * MT * 128 * 4;
+// shared memory: the sets' partial sums, the sums of the (at most two)
+// partial segments for the hand-off warp, the barriers and flags, the stage
+// ring (128-byte aligned), the token codes and scale bytes
+__host__ __device__ __forceinline__ size_t off_fix(int MT) { return (size_t)kGSets * MT * 128 * 4; }
+__host__ __device__ __forceinline__ size_t off_bars(int MT) { return off_fix(MT) + (size_t)2 * MT * 128 * 4; }
+__host__ __device__ __forceinline__ size_t off_ring(int MT) {
+    return (off_bars(MT) + (2 * kRing + 2) * 8 + 16 + 127) / 128 * 128;
 }
-__host__ __device__ __forceinline__ size_t off_ring(int GS, int MT) {
-    return (off_bars(GS, MT) + 2 * kRing * 8 + 16 + 127) / 128 * 128;
-}
-__host__ __device__ __forceinline__ size_t off_tok(int GS, int MT) {
-    return off_ring(GS, MT) + (size_t)kRing * kStageBytes;
-}
+__host__ __device__ __forceinline__ size_t off_tok(int MT) { return off_ring(MT) + (size_t)kRing * kStageBytes; }
+__host__ __device__ __forceinline__ int64_t rec_bytes(int ncta, int MT) { return (int64_t)ncta * 2 * MT * 128 * 4; }
+__host__ __device__ __forceinline__ int64_t cnt_bytes(int64_t G) { return (8 * G + 255) / 256 * 256; }
 
 __device__ __forceinline__ uint32_t su32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
@@ -167,16 +221,6 @@ __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t b
                  : "memory");
 }
 __device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
-__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
-    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
-}
-__device__ __forceinline__ uint32_t map_rank(const void *p, uint32_t rank) {
-    uint32_t ra;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(su32(p)), "r"(rank));
-    return ra;
-}
-__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release;" ::: "memory"); }
-__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire;" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
     uint32_t d;
@@ -269,29 +313,78 @@ __device__ __forceinline__ void slot68(const uint8_t *sl, int r, int b, const in
     }
 }
 
+// The token slots a CTA needs: its own slots [sp.y, sp.w) when its range
+// lies in one group; [sp.y, nb) then [0, sp.w) when it ends in the next group
+// before the slot it started at; else all.  Slot s is token slot
+// (s - q0) mod nb of ns.
+__host__ __device__ __forceinline__ void token_slots(int4 sp, int nb, int &q0, int &ns) {
+    if (sp.x == sp.z) {
+        q0 = sp.y, ns = sp.w - sp.y;
+    } else if (sp.z == sp.x + 1 && sp.w <= sp.y) {
+        q0 = sp.y, ns = nb - sp.y + sp.w;
+    } else {
+        q0 = 0, ns = nb;
+    }
+}
+
+// A CTA's segments (group, slots [sa, sb)) in processing order: the partial
+// groups first -- the tail of its first group, then the head of its last --
+// so that their hand-off to the workspace overlaps the whole groups that
+// follow; then the whole groups in order.
+struct Segs {
+    int n, np;         // segments; partial ones first
+    int gfull;         // the first whole group
+    int4 part0, part1;  // partial segments (group, sa, sb, side)
+};
+__device__ __forceinline__ Segs segments(int4 sp, int nb) {
+    Segs s;
+    s.part0 = s.part1 = make_int4(0, 0, 0, 0);
+    if (sp.x == sp.z) {
+        const bool whole = sp.y == 0 && sp.w == nb;
+        s.np = whole ? 0 : 1;
+        s.part0 = make_int4(sp.x, sp.y, sp.w, 0);
+        s.gfull = whole ? sp.x : sp.x + 1;
+        s.n = 1;
+        return s;
+    }
+    const bool lead = sp.y > 0, trail = sp.w < nb;
+    const int4 head = make_int4(sp.x, sp.y, nb, 0), tail = make_int4(sp.z, 0, sp.w, 1);
+    s.part0 = lead ? head : tail;
+    s.part1 = tail;
+    s.np = (lead ? 1 : 0) + (trail ? 1 : 0);
+    s.gfull = sp.x + (lead ? 1 : 0);
+    s.n = s.np + (sp.z - (trail ? 1 : 0)) - s.gfull + 1;
+    return s;
+}
+__device__ __forceinline__ int4 segment(const Segs &s, int i, int nb) {
+    if (i < s.np) return i == 0 ? s.part0 : s.part1;
+    return make_int4(s.gfull + (i - s.np), 0, nb, 0);
+}
+
 template <int MT>
 __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_constant__ GemvParams gp) {
     int pi = 0;
     while (pi + 1 < gp.nprob && (int)blockIdx.x >= gp.prob[pi + 1].cta0) ++pi;
     const GemvProblem &P = gp.prob[pi];
     const uint16_t *sblk = gp.slot_block[pi];
-    const int bx = (int)blockIdx.x - P.cta0, gx = P.ncta, GS = P.GS;
-    const uint32_t rank = GS > 1 ? cg::this_cluster().block_rank() : 0;
-    const int c0 = P.bound[rank], c1 = P.bound[rank + 1], ns = c1 - c0;
-    const int e4 = max(c0, min(c1, P.n4));  // 4-bit slots [c0, e4), 6/8-bit slots [e4, c1)
-    const int nst = stage_count(c0, e4, c1);
+    const int kc = (int)blockIdx.x - P.cta0;  // the CTA's index within its problem
+    const int4 sp = gp.span[blockIdx.x];      // groups sp.x .. sp.z; slots from sp.y in the first, to sp.w in the last
+    const Segs segs = segments(sp, P.nb);
     const int M = gp.M, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int ngroups = bx < P.G ? (P.G - 1 - bx) / gx + 1 : 0;
+    int q0, ns;
+    token_slots(sp, P.nb, q0, ns);
 
     extern __shared__ __align__(128) uint8_t smem[];
-    float *xbuf = reinterpret_cast<float *>(smem);                          // [2][GS][MT][128] (read in rank 0)
-    float *part = reinterpret_cast<float *>(smem + off_part(GS, MT));       // [sets][MT][128]
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + off_bars(GS, MT));  // [kRing]
-    uint64_t *empty = full + kRing;                                          // [kRing]
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(empty + kRing);
-    uint8_t *ring = smem + off_ring(GS, MT);                                // [kRing][kStageBytes]
-    int8_t *tcode = reinterpret_cast<int8_t *>(smem + off_tok(GS, MT));    // [ns][MT][32] token codes
+    float *part = reinterpret_cast<float *>(smem);                           // [sets][MT][128]
+    float *fixbuf = reinterpret_cast<float *>(smem + off_fix(MT));           // [2][MT][128]
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + off_bars(MT));       // [kRing]
+    uint64_t *empty = full + kRing;                                           // [kRing]
+    uint64_t *fix_ready = empty + kRing;                                      // [2]
+    volatile int *flags = reinterpret_cast<volatile int *>(fix_ready + 2);    // abort
+    uint8_t *ring = smem + off_ring(MT);                                     // [kRing][kStageBytes]
+    int8_t *tcode = reinterpret_cast<int8_t *>(smem + off_tok(MT));          // [ns][MT][32] token codes
     uint8_t *tsc = reinterpret_cast<uint8_t *>(tcode) + (size_t)ns * MT * 32;  // [ns][MT] token scale bytes
+    volatile int *abort_flag = flags;
 
     if (tid == 0) {
         asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -299,25 +392,27 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], kConsumers);
         }
-        *abort_flag = 0;
+        mbar_init(&fix_ready[0], kGSets);  // the four warps of set 0
+        mbar_init(&fix_ready[1], kGSets);
+        flags[0] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
 
     if (warp == kConsumers) {
-        // ---- producer: the weight bytes of [c0, c1) of each group, stage by
-        // stage (the weights are static: no wait for the kernel before).  Its
-        // cluster barriers run one phase late, so that the copies run ahead:
-        // phase 0 is the consumers' start, phase gi + 1 the end of group gi.
+        // ---- producer: the range's weight bytes, stage by stage (the weights
+        // are static: no wait for the kernel before)
         int ctr = 0;
-        bool ok = true;
-        if (GS > 1) cluster_arrive();  // phase 0
-        for (int gi = 0; gi < ngroups; ++gi) {
-            if (lane == 0 && ok) {
-                const uint8_t *base = P.w + (int64_t)(bx + gi * gx) * P.GB;
+        if (lane == 0) {
+            bool ok = true;
+            for (int si = 0; si < segs.n && ok; ++si) {
+                const int4 sg = segment(segs, si, P.nb);
+                const int sa = sg.y, sb = sg.z, e4 = max(sa, min(sb, P.n4));
+                const int nst = stage_count(sa, e4, sb);
+                const uint8_t *base = P.w + (int64_t)sg.x * P.GB;
                 for (int k = 0; k < nst; ++k, ++ctr) {
                     int lo, hi;
-                    stage_range(c0, e4, c1, k, lo, hi);
+                    stage_range(sa, e4, sb, k, lo, hi);
                     const int i = ctr % kRing;
                     const uint32_t n = (uint32_t)(ctr / kRing);
                     if (*abort_flag || (n > 0 && !mbar_wait(&empty[i], (n - 1) & 1, abort_flag))) {
@@ -330,13 +425,9 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
                     bulk_load(ring + (size_t)i * kStageBytes, base + off, bytes, &full[i]);
                 }
             }
-            __syncwarp();
-            if (GS > 1) {  // wait for phase gi, arrive for gi + 1
-                cluster_wait();
-                cluster_arrive();
-            }
         }
-        if (GS > 1) cluster_wait();  // the last phase
+        __syncwarp();
+        named_sync(2, kGThreads);  // the consumers are done
         if (lane == 0 && *abort_flag)  // drain: the last copy issued into each ring slot
             for (int i = 0; i < kRing && i < ctr; ++i) {
                 const int last = i + (ctr - 1 - i) / kRing * kRing;
@@ -345,83 +436,164 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
         return;
     }
 
-    // ---- consumers.  Prologue: the activations of slots [c0, c1) as int8
-    // codes (mxs_quantize_act's rule); x may come from the kernel before
-    // (programmatic dependent launch)
+    if (warp == kFixWarp) {
+        // ---- the hand-off of the partial segments: this CTA's sums into the
+        // workspace, one arrival on the group's counter (release: a fence
+        // after the stores), and, for the last of the group's CTAs to arrive,
+        // the sum of all of them in CTA order into y.  The consumers go on
+        // with the next segment meanwhile.
+        const int4 *pspan = gp.span + P.cta0;
+        for (int pseg = 0; pseg < segs.np; ++pseg) {
+            const int4 sg = pseg == 0 ? segs.part0 : segs.part1;
+            const int g = sg.x;
+            int kf = 0, kl = 0;
+            unsigned long long cur = 0;
+            if (lane == 0) {  // ahead of the wait: the contributors and the counter word
+                kf = first_cta(pspan, P.ncta, g);
+                kl = last_cta(pspan, P.ncta, g, P.nb);
+                cur = atomicAdd(P.cnt + g, 0ull);
+            }
+            if (!warp_wait(&fix_ready[pseg], 0, abort_flag) || *abort_flag) break;
+            for (int rr = lane; rr < 128; rr += 32)
+#pragma unroll
+                for (int t = 0; t < MT; ++t)
+                    P.rec[((size_t)(kc * 2 + sg.w) * MT + t) * 128 + rr] = fixbuf[(pseg * MT + t) * 128 + rr];
+            __syncwarp();
+            int last = 0;
+            if (lane == 0) {
+                const unsigned long long want = (unsigned long long)(kl - kf + 1);
+                unsigned long long *cw = P.cnt + g;
+                bool done = false;
+                asm volatile("fence.acq_rel.gpu;" ::: "memory");
+                for (int it = 0; it < (1 << 20) && !done; ++it) {
+                    const unsigned long long c = (cur >> 16) == gp.tag ? (cur & 0xFFFFull) + 1 : 1;
+                    const unsigned long long prev = atomicCAS(cw, cur, (gp.tag << 16) | c);
+                    if (prev == cur) {
+                        done = true;
+                        last = c == want;
+                    } else {
+                        cur = prev;
+                    }
+                }
+                if (!done) {
+                    *abort_flag = 1;
+                    atomicExch(&g_gemv_status, MXS_ERR_TIMEOUT);
+                }
+                if (last) {
+                    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+                    // (tag, 0): what a replay of this call expects to find
+                    asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(cw), "l"(gp.tag << 16) : "memory");
+                }
+            }
+            last = __shfl_sync(0xffffffffu, last, 0);
+            kf = __shfl_sync(0xffffffffu, kf, 0);
+            kl = __shfl_sync(0xffffffffu, kl, 0);
+            if (!last) continue;
+            // rows lane + 32u: every contributor's four rows in flight at once,
+            // then added in CTA order
+#pragma unroll
+            for (int t = 0; t < MT; ++t) {
+                if (t >= M) continue;
+                float v[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+                for (int k0 = kf; k0 <= kl; k0 += 4) {
+                    float pv[4][4];
+#pragma unroll
+                    for (int d = 0; d < 4; ++d) {
+                        const int kk = k0 + d;
+                        const int sd = kk <= kl && pspan[kk].x < g ? 1 : 0;  // g is that CTA's last group
+                        const float *src = P.rec + ((size_t)(kk * 2 + sd) * MT + t) * 128 + lane;
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) pv[d][u] = kk <= kl ? __ldcg(src + 32 * u) : 0.0f;
+                    }
+#pragma unroll
+                    for (int d = 0; d < 4; ++d)
+#pragma unroll
+                        for (int u = 0; u < 4; ++u)
+                            if (k0 + d <= kl) v[u] = k0 + d == kf ? pv[d][u] : v[u] + pv[d][u];
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int n = 128 * g + lane + 32 * u;
+                    if (n < P.N) P.y[(int64_t)t * P.ld_y + n] = v[u];
+                }
+            }
+        }
+        named_sync(2, kGThreads);
+        return;
+    }
+
+    // ---- consumers.  Prologue: the activations of the CTA's token slots as
+    // int8 codes (mxs_quantize_act's rule), four threads per block of a
+    // token; x may come from the kernel before (programmatic dependent launch)
     const int set = tid >> 7, r = tid & 127;
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    for (int i = tid; i < ns * MT; i += kCThreads) {
-        const int j = i / MT, t = i - j * MT, s = c0 + j;
-        uint4 *dst = reinterpret_cast<uint4 *>(tcode + ((size_t)j * MT + t) * 32);
-        if (t >= M) {
-            dst[0] = dst[1] = make_uint4(0, 0, 0, 0);
-            tsc[j * MT + t] = 0;
-            continue;
+    const int nq = ns * MT * 4;
+    for (int base = 0; base < nq; base += kCThreads) {  // the same trip count in every thread
+        const int i = base + tid;
+        const int q = i & 3, jt = i >> 2, j = jt / MT, t = jt - j * MT;
+        const int s = q0 + j < P.nb ? q0 + j : q0 + j - P.nb;
+        const bool act = i < nq;
+        uint4 u = make_uint4(0, 0, 0, 0);
+        int b = 8;
+        if (act) {
+            b = s < P.n4 ? 4 : (s < P.n4 + P.n6 ? 6 : 8);
+            if (t < M)
+                u = __ldg(reinterpret_cast<const uint4 *>(P.x + (int64_t)t * P.ld_x + 32 * (int64_t)sblk[s]) + q);
         }
-        const int b = s < P.n4 ? 4 : (s < P.n4 + P.n6 ? 6 : 8);
-        const uint4 *src = reinterpret_cast<const uint4 *>(P.x + (int64_t)t * P.ld_x + 32 * (int64_t)sblk[s]);
-        uint32_t h[32];
+        const uint32_t h[8] = {u.x & 0xFFFFu, u.x >> 16, u.y & 0xFFFFu, u.y >> 16,
+                               u.z & 0xFFFFu, u.z >> 16, u.w & 0xFFFFu, u.w >> 16};
         uint32_t mag = 0;
 #pragma unroll
-        for (int v = 0; v < 4; ++v) {
-            const uint4 u = __ldg(src + v);
-            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+        for (int k = 0; k < 8; ++k) mag = max(mag, h[k] & 0x7FFFu);
+        mag = max(mag, __shfl_xor_sync(0xffffffffu, mag, 1));  // the four threads of the block
+        mag = max(mag, __shfl_xor_sync(0xffffffffu, mag, 2));
+        const int S = (int)(mag >> 7);
+        if (act) {
+            uint32_t c0 = 0, c1 = 0;
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-                h[8 * v + 2 * k] = w4[k] & 0xFFFF;
-                h[8 * v + 2 * k + 1] = w4[k] >> 16;
+                const int m0 = S == 255 ? 0 : quant_elem(h[k], S, b, gp.rhaz);
+                const int m1 = S == 255 ? 0 : quant_elem(h[4 + k], S, b, gp.rhaz);
+                c0 |= (uint32_t)(m0 & 0xFF) << (8 * k);
+                c1 |= (uint32_t)(m1 & 0xFF) << (8 * k);
             }
+            *reinterpret_cast<uint2 *>(tcode + (size_t)jt * 32 + 8 * q) = make_uint2(c0, c1);
+            if (q == 0) tsc[jt] = (uint8_t)S;
         }
-#pragma unroll
-        for (int k = 0; k < 32; ++k) mag = max(mag, h[k] & 0x7FFF);
-        const int S = (int)(mag >> 7);
-        uint32_t cw[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            cw[k] = 0;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int m = S == 255 ? 0 : quant_elem(h[4 * k + q], S, b, gp.rhaz);
-                cw[k] |= (uint32_t)(m & 0xFF) << (8 * q);
-            }
-        }
-        dst[0] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
-        dst[1] = make_uint4(cw[4], cw[5], cw[6], cw[7]);
-        tsc[j * MT + t] = (uint8_t)S;
     }
     named_sync(1, kCThreads);
-    if (GS > 1) {  // phase 0: every rank runs before the first store into rank 0
-        cluster_arrive();
-        cluster_wait();
-    }
 
     bool aborted = false;
     int ctr = 0;
-    for (int gi = 0; gi < ngroups; ++gi) {
-        const int g = bx + gi * gx;
+    for (int si = 0; si < segs.n; ++si) {
+        const int4 sg = segment(segs, si, P.nb);
+        const int g = sg.x, sa = sg.y, sb = sg.z, e4 = max(sa, min(sb, P.n4));
+        const int nst = stage_count(sa, e4, sb);
+        const bool whole = sa == 0 && sb == P.nb;
         float acc[MT];
 #pragma unroll
         for (int t = 0; t < MT; ++t) acc[t] = 0.0f;
         for (int k = 0; k < nst; ++k, ++ctr) {
             int lo, hi;
-            stage_range(c0, e4, c1, k, lo, hi);
+            stage_range(sa, e4, sb, k, lo, hi);
             const int i = ctr % kRing;
             if (!aborted && !warp_wait(&full[i], (uint32_t)(ctr / kRing) & 1, abort_flag)) aborted = true;
             if (!aborted) {
-                const uint8_t *sb = ring + (size_t)i * kStageBytes;
+                const uint8_t *sb8 = ring + (size_t)i * kStageBytes;
                 if (lo < P.n4) {
 #pragma unroll
-                    for (int j = 0; j < kSlots4 / kGSets; ++j) {
-                        const int s = lo + set + kGSets * j;
-                        if (s < hi) slot4<MT>(sb + 2176 * (s - lo), r, tcode + (size_t)(s - c0) * MT * 32,
-                                              tsc + (s - c0) * MT, acc);
+                    for (int jj = 0; jj < kSlots4 / kGSets; ++jj) {
+                        const int s = lo + set + kGSets * jj;
+                        const int ts = s >= q0 ? s - q0 : s - q0 + P.nb;
+                        if (s < hi) slot4<MT>(sb8 + 2176 * (s - lo), r, tcode + (size_t)ts * MT * 32, tsc + ts * MT, acc);
                     }
                 } else {
 #pragma unroll
-                    for (int j = 0; j < kSlots68 / kGSets; ++j) {
-                        const int s = lo + set + kGSets * j;
-                        if (s < hi) slot68<MT>(sb + 4224 * (s - lo), r, s < P.n4 + P.n6 ? 6 : 8,
-                                               tcode + (size_t)(s - c0) * MT * 32, tsc + (s - c0) * MT, acc);
+                    for (int jj = 0; jj < kSlots68 / kGSets; ++jj) {
+                        const int s = lo + set + kGSets * jj;
+                        const int ts = s >= q0 ? s - q0 : s - q0 + P.nb;
+                        if (s < hi) slot68<MT>(sb8 + 4224 * (s - lo), r, s < P.n4 + P.n6 ? 6 : 8,
+                                               tcode + (size_t)ts * MT * 32, tsc + ts * MT, acc);
                     }
                 }
             }
@@ -429,12 +601,12 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
             if (lane == 0) mbar_arrive(&empty[i]);
         }
 
-        // ---- the sets' sums in set order, then the ranks' in rank order
+        // ---- the sets' sums in set order
 #pragma unroll
         for (int t = 0; t < MT; ++t) part[(set * MT + t) * 128 + r] = acc[t];
         named_sync(1, kCThreads);
         float val[MT];
-        if (set == 0) {
+        if (set == 0)
 #pragma unroll
             for (int t = 0; t < MT; ++t) {
                 float v = part[t * 128 + r];
@@ -442,55 +614,25 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
                 for (int k = 1; k < kGSets; ++k) v += part[(k * MT + t) * 128 + r];
                 val[t] = v;
             }
-        }
-        const int n = 128 * g + r;
-        if (GS == 1) {
-            if (set == 0 && n < P.N && !aborted)
+        if (set == 0) {
+            const int n = 128 * g + r;
+            if (!whole) {  // part of the group: to the hand-off warp
+#pragma unroll
+                for (int t = 0; t < MT; ++t) fixbuf[(si * MT + t) * 128 + r] = val[t];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&fix_ready[si]);
+            } else if (n < P.N && !*abort_flag) {  // the whole group: straight to y
 #pragma unroll
                 for (int t = 0; t < MT; ++t)
                     if (t < M) P.y[(int64_t)t * P.ld_y + n] = val[t];
-        } else {
-            float *xb = xbuf + (gi & 1) * GS * MT * 128;
-            if (set == 0)
-#pragma unroll
-                for (int t = 0; t < MT; ++t) st_cluster_f32(map_rank(xb + (rank * MT + t) * 128 + r, 0), val[t]);
-            cluster_arrive();  // phase gi + 1: every rank's partial sums are in rank 0
-            cluster_wait();
-            if (rank == 0 && set == 0 && n < P.N && !aborted)
-#pragma unroll
-                for (int t = 0; t < MT; ++t) {
-                    if (t >= M) continue;
-                    float v = xb[t * 128 + r];
-                    for (int k = 1; k < GS; ++k) v += xb[(k * MT + t) * 128 + r];
-                    P.y[(int64_t)t * P.ld_y + n] = v;
-                }
+            }
         }
-        named_sync(1, kCThreads);  // `part` is reused by the next group
+        named_sync(1, kCThreads);  // `part` is reused by the next segment
     }
+    named_sync(2, kGThreads);  // with the producer, which drains after an abort
 }
 
 // ------------------------------------------------------------------ host side
-int gemv_stage_lo(const Plan &p, int sg) {
-    return sg <= p.st4 ? std::min(4 * sg, p.n4) : std::min(p.n4 + 2 * (sg - p.st4), p.nb);
-}
-
-// slot boundaries of `parts` K ranges of about the same packed bytes (stage-aligned)
-void gemv_split(const Plan &p, int parts, int *bound) {
-    const int g1 = p.nst;
-    const int64_t total = slot_off_g(p.n4, gemv_stage_lo(p, g1));
-    int gb[9];
-    gb[0] = 0;
-    for (int r = 1; r < parts; ++r) {
-        int s = gb[r - 1] + 1;
-        while (s < g1 - (parts - r) && slot_off_g(p.n4, gemv_stage_lo(p, s)) * parts < total * r) ++s;
-        gb[r] = s;
-    }
-    gb[parts] = g1;
-    for (int r = 0; r <= parts; ++r) bound[r] = gemv_stage_lo(p, gb[r]);
-}
-
-size_t gemv_smem(int ns, int MT, int GS) { return off_tok(GS, MT) + ((size_t)ns * MT * 33 + 15) / 16 * 16; }
-
 int sms_now() {
     static int cached = 0;
     if (!cached) {
@@ -504,8 +646,50 @@ int sms_now() {
     return cached;
 }
 
+int mt_of(int64_t M) { return M == 1 ? 1 : (M == 2 ? 2 : 4); }
+
+// CTAs per problem for a launch of `count` problems of W[i] weight bytes on
+// `sms` SMs: one CTA each, then one at a time to the problem with the most
+// bytes per CTA, each problem keeping at least kMinCtaBytes (and more than
+// one 6/8-bit slot) per CTA.
+void gemv_split_ctas(const int64_t *W, int count, int sms, int *ncta) {
+    const int total = std::max(count, std::min(sms, kGemvMaxCtas));
+    int64_t cap[kGMaxProblems];
+    int used = 0;
+    for (int i = 0; i < count; ++i) {
+        cap[i] = std::max<int64_t>(1, std::min<int64_t>(W[i] / 4225, W[i] / kMinCtaBytes));
+        ncta[i] = 1;
+        ++used;
+    }
+    while (used < total) {
+        int best = -1;
+        double bw = -1.0;
+        for (int i = 0; i < count; ++i)
+            if (ncta[i] < cap[i] && (double)W[i] / ncta[i] > bw) bw = (double)W[i] / ncta[i], best = i;
+        if (best < 0) break;
+        ++ncta[best];
+        ++used;
+    }
+}
+
+// the span of CTA k of n over a problem (groups of GB bytes, n4 4-bit slots
+// of nb): first group, its first slot, last group, end slot in it
+void gemv_span(int k, int n, int64_t W, int64_t GB, int n4, int nb, int *out) {
+    (void)nb;
+    const int64_t a = cta_start(k, n, W, GB, n4), b = cta_start(k + 1, n, W, GB, n4);
+    const int64_t g0 = a / GB, g1 = (b - 1) / GB;
+    out[0] = (int)g0;
+    out[1] = slot_at(n4, a - g0 * GB);
+    out[2] = (int)g1;
+    out[3] = slot_at(n4, b - g1 * GB);
+}
 
 }  // namespace
+
+int64_t gemv_workspace_bytes(int64_t M, int64_t N) {
+    const int64_t G = (N + 127) / 128;
+    return cnt_bytes(G) + rec_bytes(kGemvMaxCtas, mt_of(M));
+}
 
 int gemv_status(int *status, int reset) {
     int v = 0;
@@ -521,104 +705,78 @@ int gemv_status(int *status, int reset) {
 }
 
 int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int64_t *ld_x, const void *const *packed,
-                       const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, int rounding,
-                       bool pdl, cudaStream_t st) {
+                       const int64_t *N, float *const *y, const int64_t *ld_y, void *const *ws,
+                       const size_t *ws_bytes, int count, int64_t M, int rounding, bool pdl, cudaStream_t st) {
     if (count < 1 || count > kGMaxProblems) return fail(MXS_ERR_INVALID_ARG, "count=%d (1..%d)", count, kGMaxProblems);
     if (M < 1 || M > kGemvMaxM) return fail(MXS_ERR_SHAPE, "the CUDA-core decode path takes 1 <= M <= %d", kGemvMaxM);
-    const int MT = M == 1 ? 1 : (M == 2 ? 2 : 4);
-    const int sms = sms_now();
-    int64_t G[kGMaxProblems], bytes[kGMaxProblems];
+    const int MT = mt_of(M);
+    int64_t G[kGMaxProblems], GB[kGMaxProblems], W[kGMaxProblems];
     for (int i = 0; i < count; ++i) {
         if (N[i] > (int64_t)0x7FFFFFF0) return fail(MXS_ERR_SHAPE, "N too large");
-        G[i] = weight_offsets(*plans[i], N[i], false).G;
-        bytes[i] = weight_offsets(*plans[i], N[i], false).GB;
+        const WeightOffsets wo = weight_offsets(*plans[i], N[i], false);
+        G[i] = wo.G;
+        GB[i] = wo.GB;
+        W[i] = G[i] * GB[i];
     }
-    // One cluster size for the launch.  A CTA's time is about its groups x the
-    // bytes of its K range of one group (the stream), plus a fixed cost per
-    // group and, in a cluster, per cluster barrier; CTAs are handed one at a
-    // time to the problem whose slowest CTA costs most.
-    auto cost = [&](int i, int GS, int n) {
-        const double rounds = (double)((G[i] + n - 1) / n);
-        return rounds * ((double)bytes[i] / GS / 40.0 + (GS > 1 ? 3000.0 : 1500.0));  // ~40 bytes per cycle per SM
-    };
-    double best = 1e300;
-    int bestGS = 1, bestn[kGMaxProblems] = {};
-    for (int GS = 1; GS <= 8; GS *= 2) {
-        bool ok = sms / GS >= count;
-        for (int i = 0; i < count && ok; ++i) {
-            ok = GS <= plans[i]->nst;
-            if (!ok) break;
-            int bound[9], most = 0;
-            gemv_split(*plans[i], GS, bound);
-            for (int r = 0; r < GS; ++r) most = std::max(most, bound[r + 1] - bound[r]);
-            ok = gemv_smem(most, MT, GS) <= (size_t)200 * 1024;
-        }
-        if (!ok) continue;
-        int n[kGMaxProblems], used = count;
-        for (int i = 0; i < count; ++i) n[i] = 1;
-        while (used < sms / GS) {
-            int worst = -1;
-            double wc = -1.0;
-            for (int i = 0; i < count; ++i)
-                if (n[i] < G[i] && cost(i, GS, n[i]) > wc) wc = cost(i, GS, n[i]), worst = i;
-            if (worst < 0) break;
-            ++n[worst];
-            ++used;
-        }
-        double c = 0.0;
-        for (int i = 0; i < count; ++i) c = std::max(c, cost(i, GS, n[i]));
-        if (c < best * 0.98) {
-            best = c;
-            bestGS = GS;
-            for (int i = 0; i < count; ++i) bestn[i] = n[i];
-        }
-    }
-    if (best >= 1e299) return fail(MXS_ERR_SHAPE, "decode: K too large for the CUDA-core path");
-    // the parameter block carries the slot tables (a few KB): built on the host
+    int ncta[kGMaxProblems];
+    gemv_split_ctas(W, count, sms_now(), ncta);
+    // the parameter block carries the slot tables and the spans (about 17 KB): built on the host
     static thread_local GemvParams gp;
     std::memset(&gp, 0, sizeof(gp));
+    static std::atomic<unsigned long long> tags{0};
+    unsigned long long tag = 0;
+    while (tag == 0) tag = (tags.fetch_add(1) + 1) & 0xFFFFFFFFFFFFull;
+    gp.tag = tag;
     gp.nprob = count;
     gp.M = (int)M;
     gp.rhaz = rounding == MXS_RHAZ;
     int cta = 0, max_ns = 0;
     for (int i = 0; i < count; ++i) {
         const Plan &p = *plans[i];
+        const int64_t need = cnt_bytes(G[i]) + rec_bytes(ncta[i], MT);
+        if ((int64_t)ws_bytes[i] < need || !ws[i])
+            return fail(MXS_ERR_BUFFER, "problem %d: workspace of %lld bytes needed, %zu given", i, (long long)need,
+                        ws_bytes[i]);
         GemvProblem &P = gp.prob[i];
         P.x = static_cast<const uint16_t *>(x[i]);
         P.w = static_cast<const uint8_t *>(packed[i]);
         P.y = y[i];
+        P.cnt = static_cast<unsigned long long *>(ws[i]);
+        P.rec = reinterpret_cast<float *>(static_cast<uint8_t *>(ws[i]) + cnt_bytes(G[i]));
         P.ld_x = ld_x[i];
         P.ld_y = ld_y[i];
-        P.GB = bytes[i];
+        P.GB = GB[i];
+        P.W = W[i];
         P.N = (int)N[i];
         P.G = (int)G[i];
-        P.GS = bestGS;
         P.nb = p.nb, P.n4 = p.n4, P.n6 = p.n6;
-        gemv_split(p, bestGS, P.bound);
-        for (int r = bestGS + 1; r < 9; ++r) P.bound[r] = P.bound[bestGS];
-        for (int r = 0; r < bestGS; ++r) max_ns = std::max(max_ns, P.bound[r + 1] - P.bound[r]);
         P.cta0 = cta;
-        P.ncta = bestn[i];
-        cta += bestn[i];
+        P.ncta = ncta[i];
+        for (int k = 0; k < ncta[i]; ++k) {
+            int sp[4];
+            gemv_span(k, ncta[i], W[i], GB[i], p.n4, p.nb, sp);
+            gp.span[cta + k] = make_int4(sp[0], sp[1], sp[2], sp[3]);
+            int q0, ns;
+            token_slots(make_int4(sp[0], sp[1], sp[2], sp[3]), p.nb, q0, ns);
+            max_ns = std::max(max_ns, ns);
+        }
+        cta += ncta[i];
         std::memcpy(gp.slot_block[i], p.slot_block, sizeof(uint16_t) * (size_t)p.nb);
     }
-    const size_t smem = gemv_smem(max_ns, MT, bestGS);
+    const size_t smem = off_tok(MT) + ((size_t)max_ns * MT * 33 + 15) / 16 * 16;
+    if (smem > (size_t)227 * 1024)
+        return fail(MXS_ERR_SHAPE, "decode: K too large for the CUDA-core path at M=%lld", (long long)M);
     using Kernel = void (*)(GemvParams);
     const Kernel k = MT == 1 ? gemv_decode_kernel<1> : (MT == 2 ? gemv_decode_kernel<2> : gemv_decode_kernel<4>);
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(gemv smem)");
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)cta, (unsigned)bestGS, 1);
+    cfg.gridDim = dim3((unsigned)cta, 1, 1);
     cfg.blockDim = dim3(kGThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[2];
+    cudaLaunchAttribute attr[1];
     int na = 0;
-    attr[na].id = cudaLaunchAttributeClusterDimension;
-    attr[na].val.clusterDim.x = 1;
-    attr[na].val.clusterDim.y = (unsigned)bestGS;
-    attr[na].val.clusterDim.z = 1;
-    ++na;
     if (pdl) {
         attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr[na].val.programmaticStreamSerializationAllowed = 1;
@@ -631,3 +789,30 @@ int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int
 }
 
 }  // namespace mxs
+
+using namespace mxs;
+
+int mxs_test_gemv_split(const int64_t *K, const uint8_t *const *bits, const int64_t *N, int count, int sms,
+                        int32_t *ncta, int32_t *spans) {
+    if (!K || !bits || !N || !ncta || !spans) return -fail(MXS_ERR_INVALID_ARG, "NULL argument");
+    if (count < 1 || count > kGMaxProblems || sms < 1)
+        return -fail(MXS_ERR_INVALID_ARG, "count=%d (1..%d), sms=%d", count, kGMaxProblems, sms);
+    int64_t W[kGMaxProblems], GB[kGMaxProblems];
+    Plan plans[kGMaxProblems];
+    for (int i = 0; i < count; ++i) {
+        const int rc = build_plan(bits[i], K[i], &plans[i]);
+        if (rc) return -rc;
+        if (N[i] < 1 || N[i] > (int64_t)0x7FFFFFF0) return -fail(MXS_ERR_SHAPE, "N=%lld", (long long)N[i]);
+        const WeightOffsets wo = weight_offsets(plans[i], N[i], false);
+        GB[i] = wo.GB;
+        W[i] = wo.G * wo.GB;
+    }
+    int n[kGMaxProblems];
+    gemv_split_ctas(W, count, sms, n);
+    int cta = 0;
+    for (int i = 0; i < count; ++i) {
+        ncta[i] = n[i];
+        for (int k = 0; k < n[i]; ++k, ++cta) gemv_span(k, n[i], W[i], GB[i], plans[i].n4, plans[i].nb, spans + 4 * cta);
+    }
+    return cta;
+}

@@ -164,6 +164,17 @@ int64_t mxs_weight_bytes(int64_t N, int64_t K, const uint8_t *bits, int layout) 
     return rc ? -rc : weight_offsets(p, N, layout == MXS_W_COMPACT_AND_PLANES).total;
 }
 
+int64_t mxs_linear_decode_workspace_bytes(int64_t M, int64_t K, int64_t N, const uint8_t *bits) {
+    if (M < 0 || N < 0) return -fail(MXS_ERR_SHAPE, "M=%lld N=%lld", (long long)M, (long long)N);
+    if (M >= 1 && M <= kGemvMaxM) {  // the CUDA-core path: arrival counters and partial sums
+        Plan p;
+        const int rc = build_plan(bits, K, &p);
+        if (rc) return -rc;
+        return gemv_workspace_bytes(M, N);
+    }
+    return mxs_act_planes_bytes(M, K, bits);
+}
+
 int64_t mxs_gemm_workspace_bytes(int64_t M, int64_t N, int64_t K, const uint8_t *bits) {
     if (M < 0 || N < 0) return -fail(MXS_ERR_SHAPE, "M/N < 0");
     Plan p;
@@ -286,7 +297,9 @@ int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t 
         if (q.ld_x < q.K || q.ld_x % 8 != 0)
             return fail(MXS_ERR_INVALID_ARG, "problem %d: ld_x=%lld must be >= K and a multiple of 8", i, (long long)q.ld_x);
         if (q.ld_y < q.N) return fail(MXS_ERR_INVALID_ARG, "problem %d: ld_y=%lld < N", i, (long long)q.ld_y);
-        const int64_t need = align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);  // mxs_act_planes_bytes
+        const int64_t need = M >= 1 && M <= kGemvMaxM
+                                 ? gemv_workspace_bytes(M, q.N)
+                                 : align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);  // the planes
         if ((int64_t)q.ws_bytes < need || (need > 0 && !q.workspace))
             return fail(MXS_ERR_BUFFER, "problem %d: workspace of %lld bytes needed, %zu given", i, (long long)need,
                         q.ws_bytes);
@@ -319,9 +332,11 @@ int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t 
     const void *xs[3];
     int64_t lds[3];
     void *pls[3];
-    for (int i = 0; i < count; ++i) xs[i] = probs[i].x, lds[i] = probs[i].ld_x, pls[i] = probs[i].workspace;
+    size_t wsb[3];
+    for (int i = 0; i < count; ++i)
+        xs[i] = probs[i].x, lds[i] = probs[i].ld_x, pls[i] = probs[i].workspace, wsb[i] = probs[i].ws_bytes;
     if (M <= kGemvMaxM)  // one token: quantization fused into the CUDA-core GEMM (no planes)
-        return launch_gemv_decode(pp, xs, lds, packed, N, y, ld_y, count, M, rounding, true, st);
+        return launch_gemv_decode(pp, xs, lds, packed, N, y, ld_y, pls, wsb, count, M, rounding, true, st);
     rc = launch_quantize_group(pp, xs, lds, M, rounding, pls, count, st);  // one quantizer launch for the group
     if (rc) return rc;
     rc = launch_gemm_decode_group(pp, planes, packed, N, y, ld_y, count, M, true, st);
@@ -380,7 +395,9 @@ int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const u
     if (!x || !packed_w || !y) return fail(MXS_ERR_INVALID_ARG, "NULL operand");
     if (ld_x < K || ld_x % 8 != 0) return fail(MXS_ERR_INVALID_ARG, "ld_x=%lld must be >= K and a multiple of 8", (long long)ld_x);
     if (ld_y < N) return fail(MXS_ERR_INVALID_ARG, "ld_y=%lld < N", (long long)ld_y);
-    const int64_t need = align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);  // mxs_act_planes_bytes
+    const int64_t need = M >= 1 && M <= kGemvMaxM
+                             ? gemv_workspace_bytes(M, N)
+                             : align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);  // the planes
     if ((int64_t)ws_bytes < need || (need > 0 && !ws))
         return fail(MXS_ERR_BUFFER, "workspace of %lld bytes needed, %zu given", (long long)need, ws_bytes);
     if (!aligned16(x) || !aligned16(packed_w) || (ws && !aligned16(ws)) || (reinterpret_cast<uintptr_t>(y) & 3))
@@ -390,7 +407,8 @@ int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const u
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (M <= kGemvMaxM) {  // one token: quantization fused into the CUDA-core GEMM (no planes)
         const Plan *pp = &p;
-        return launch_gemv_decode(&pp, &x, &ld_x, &packed_w, &N, &y, &ld_y, 1, M, rounding, true, st);
+        return launch_gemv_decode(&pp, &x, &ld_x, &packed_w, &N, &y, &ld_y, &ws, &ws_bytes, 1, M, rounding, true,
+                                  st);
     }
     rc = launch_quantize(p, x, M, ld_x, rounding, nullptr, nullptr, ws, st);
     if (rc) return rc;

@@ -1,7 +1,8 @@
 // noalloc.cu -- mxs_linear_decode for callers that cannot allocate device
 // memory.
 //
-// mxs_linear_decode needs a scratch buffer for the activations' MMA planes,
+// mxs_linear_decode needs a scratch buffer (the activations' MMA planes, or
+// for one token the arrival counters and partial sums of the CUDA-core path),
 // which its caller allocates.  Some callers cannot: code that runs where
 // cudaMalloc is not allowed or not wanted -- an allocator-free runtime that
 // owns all device memory up front, a plug-in whose host framework forbids
@@ -58,13 +59,13 @@ int mxs_linear_decode_noalloc(const void *x, int64_t M, int64_t K, int64_t ld_x,
                               const void *packed_w, int64_t N, float *y, int64_t ld_y, void *stream) {
     // the checks that need no device come first
     if (M > 16) return fail(MXS_ERR_SHAPE, "the fused decode path takes M <= 16 (M=%lld)", (long long)M);
-    const int64_t need = mxs_act_planes_bytes(M, K, bits);
+    const int64_t need = mxs_linear_decode_workspace_bytes(M, K, N, bits);
     if (need < 0) return (int)-need;  // the size query has set the message
     if ((uint64_t)need > kScratchBytes)
         return fail(MXS_ERR_BUFFER,
-                    "mxs_linear_decode_noalloc: M=%lld, K=%lld need %lld bytes of scratch; its built-in scratch holds "
-                    "%zu (use mxs_linear_decode with a workspace)",
-                    (long long)M, (long long)K, (long long)need, kScratchBytes);
+                    "mxs_linear_decode_noalloc: M=%lld, K=%lld, N=%lld need %lld bytes of scratch; its built-in "
+                    "scratch holds %zu (use mxs_linear_decode with a workspace)",
+                    (long long)M, (long long)K, (long long)N, (long long)need, kScratchBytes);
     if (M == 0) return mxs_linear_decode(x, M, K, ld_x, bits, rounding, packed_w, N, y, ld_y, nullptr, 0, stream);
     int rc = check_device();
     if (rc) return rc;

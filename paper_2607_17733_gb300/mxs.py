@@ -31,7 +31,7 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_quantize_act_permuted", "mxs_pack_weight_permuted", "mxs_attention_decode_workspace_bytes",
            "mxs_attention_decode", "mxs_linear_decode_group", "mxs_quantize_act_group",
            "mxs_attention_decode_batch_workspace_bytes", "mxs_attention_decode_batch", "mxs_probe_mma",
-           "mxs_probe_status"]
+           "mxs_probe_status", "mxs_linear_decode_workspace_bytes", "mxs_test_gemv_split"]
 
 _lock = threading.Lock()
 _lib = None
@@ -114,6 +114,10 @@ def lib() -> ctypes.CDLL:
         L.mxs_probe_mma.restype = I
         L.mxs_probe_status.argtypes = [ctypes.POINTER(ctypes.c_int), I]
         L.mxs_probe_status.restype = I
+        L.mxs_linear_decode_workspace_bytes.argtypes = [I64, I64, I64, P]
+        L.mxs_linear_decode_workspace_bytes.restype = I64
+        L.mxs_test_gemv_split.argtypes = [P, P, P, I, I, P, P]
+        L.mxs_test_gemv_split.restype = I
         _lib = L
         return L
 
@@ -175,6 +179,13 @@ def act_codes_bytes(M: int, K: int, bits) -> int:
 def act_planes_bytes(M: int, K: int, bits) -> int:
     b = _Bits(bits)
     return _size(lib().mxs_act_planes_bytes(M, K, b.ptr))
+
+
+def linear_decode_workspace_bytes(M: int, K: int, N: int, bits) -> int:
+    """Workspace bytes of linear_decode / each problem of linear_decode_group
+    (mxs_linear_decode_workspace_bytes)."""
+    b = _Bits(bits)
+    return _size(lib().mxs_linear_decode_workspace_bytes(M, K, N, b.ptr))
 
 
 def weight_bytes(N: int, K: int, bits, layout: int = W_COMPACT) -> int:
@@ -270,15 +281,16 @@ def gemm_decode(codes, scales, bits, packed_w, N: int, y=None, workspace=None, s
 
 def linear_decode(x, bits, packed_w, N: int, rounding: int = RNE, y=None, workspace=None, stream=None):
     """Activation quantization + decode GEMM (M <= 16) in one call: y [M, N]
-    fp32.  workspace: uint8 of at least act_planes_bytes(M, K, bits) bytes
-    (allocated when None)."""
+    fp32.  workspace: uint8 of at least linear_decode_workspace_bytes(M, K, N,
+    bits) bytes (allocated when None)."""
     import torch
     b = _Bits(bits)
     M, K = x.shape
     if y is None:
         y = torch.empty((M, N), dtype=torch.float32, device=packed_w.device)
     if workspace is None:
-        workspace = torch.empty(max(act_planes_bytes(M, K, b.arr), 16), dtype=torch.uint8, device=packed_w.device)
+        workspace = torch.empty(max(linear_decode_workspace_bytes(M, K, N, b.arr), 16), dtype=torch.uint8,
+                                device=packed_w.device)
     ws_bytes = workspace.numel() * workspace.element_size()
     check(lib().mxs_linear_decode(_ptr(x), M, K, _ld(x), b.ptr, rounding, _ptr(packed_w), N, _ptr(y),
                                   _ld(y), _ptr(workspace), ws_bytes, _stream(stream)))

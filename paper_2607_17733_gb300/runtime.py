@@ -39,9 +39,10 @@ class MxLinear:
             "scales": torch.empty((M, self.K // 32), dtype=torch.uint8, device=device),
             "y": torch.empty((M, self.N), dtype=torch.float32, device=device),
             "ws": None,
-            # MMA planes of the activations, written and read inside fused()
-            "planes": torch.empty(max(mxs.act_planes_bytes(M, self.K, self.bits), 16), dtype=torch.uint8,
-                                  device=device) if M <= 16 else None,
+            # the workspace of fused(): the activations' MMA planes (M > 1), the
+            # CUDA-core path's arrival counters and partial sums (M = 1)
+            "planes": torch.empty(max(mxs.linear_decode_workspace_bytes(M, self.K, self.N, self.bits), 16),
+                                  dtype=torch.uint8, device=device) if M <= 16 else None,
         }
 
     def quantize(self, x: torch.Tensor, bufs: dict):

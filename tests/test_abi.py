@@ -33,7 +33,7 @@ def test_every_declared_function_is_exported(L):
     for n in names:
         assert hasattr(L, n), n
     assert sorted(mxs.EXPORTS) == names
-    assert L.mxs_version() == 2
+    assert L.mxs_version() == 3
 
 
 def _bits(nb, seed=0, p=(0.7, 0.2, 0.1)):

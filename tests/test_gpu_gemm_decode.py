@@ -228,7 +228,7 @@ def test_linear_decode_group(torch, M, shapes):
         packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
         x = U.to_dev_bf16(torch, xb)
         y = torch.full((M, N), float("nan"), device="cuda")
-        ws = torch.empty(mxs.act_planes_bytes(M, K, bits), dtype=torch.uint8, device="cuda")
+        ws = torch.empty(mxs.linear_decode_workspace_bytes(M, K, N, bits), dtype=torch.uint8, device="cuda")
         probs.append((x, bits, packed, N, y, ws))
         refs.append(oracle_full(xb, wb, bits))
     torch.cuda.synchronize()  # weights are static before the first decode call
@@ -241,16 +241,18 @@ def test_linear_decode_group(torch, M, shapes):
         U.check_gemm(got, single.astype(np.float64), ab)
 
 
-@pytest.mark.parametrize("M,N,nb", [(16, 1000, 128), (3, 4096, 448)])
+@pytest.mark.parametrize("M,N,nb", [(16, 1000, 128), (3, 4096, 448), (1, 3000, 448), (1, 8192, 256)])
 def test_linear_decode_workspace_garbage_reuse_and_graph_replay(torch, M, N, nb):
-    """The fused layer's workspace holds only what the same call writes: a
-    workspace full of garbage, the same workspace reused, and a CUDA graph
-    replaying the same call all give the same y, bit for bit."""
+    """The fused layer needs nothing prepared in its workspace: a workspace
+    full of garbage, the same workspace reused, and a CUDA graph replaying the
+    same call all give the same y, bit for bit (M = 1: the arrival counts of
+    the CTAs that share a row group are tagged per call)."""
     g = I.rng(70, M, N, nb)
     bits = I.width_map(nb, 0.8, 0.15, 0.05, g)
     xb, wb, codes, scales, packed = layer(torch, M, 32 * nb, N, bits, g)
     x = U.to_dev_bf16(torch, xb)
-    ws = torch.randint(0, 256, (mxs.act_planes_bytes(M, 32 * nb, bits),), dtype=torch.uint8, device="cuda")
+    ws = torch.randint(0, 256, (mxs.linear_decode_workspace_bytes(M, 32 * nb, N, bits),), dtype=torch.uint8,
+                       device="cuda")
     ys = [mxs.linear_decode(x, bits, packed, N, workspace=ws).cpu().numpy() for _ in range(3)]
     ref, ab = oracle_full(xb, wb, bits)
     U.check_gemm(ys[0], ref, ab)

@@ -73,7 +73,7 @@ def test_gemv_group_and_repeat(torch):
         wb = I.normal_bf16((N, K), 0.02, g)
         packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
         y = torch.full((M, N), float("nan"), device="cuda")
-        ws = torch.empty(mxs.act_planes_bytes(M, K, bits), dtype=torch.uint8, device="cuda")
+        ws = torch.empty(mxs.linear_decode_workspace_bytes(M, K, N, bits), dtype=torch.uint8, device="cuda")
         probs.append((U.to_dev_bf16(torch, xb), bits, packed, N, y, ws))
         refs.append(_ref(xb, wb, bits))
     torch.cuda.synchronize()
