@@ -299,6 +299,12 @@ MXS_API int mxs_test_decode_starve(const void *act_planes, const uint8_t *bits, 
  * it takes there, its last group, and the slot where it stops there (the
  * group's block count when it takes the group to its end).  Returns the
  * number of CTAs, or minus an error code. */
+/* Test hook: the one-token decode kernel's ring of weight stages.  stages =
+ * 2 or 3 caps it at that many stages for the calls that follow in this
+ * process (the kernel drops to fewer than four by itself only when a CTA's
+ * token codes need the shared memory: long K over several row groups);
+ * 0 restores the choice by size.  MXS_ERR_INVALID_ARG for other values. */
+MXS_API int mxs_test_gemv_ring(int stages);
 MXS_API int mxs_test_gemv_split(const int64_t *K, const uint8_t *const *bits, const int64_t *N, int count, int sms,
                                 int32_t *ncta, int32_t *spans);
 

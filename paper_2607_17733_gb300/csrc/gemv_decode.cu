@@ -40,12 +40,13 @@
 // Per CTA.  Prologue: it quantizes the activations of the slots its range
 // takes (x is bf16; the rule, bit for bit, of mxs_quantize_act; four threads
 // per block, the block maximum by shuffles) into shared memory as int8 codes
-// and scale bytes.  One lane of a producer warp streams the range into a ring of
-// shared-memory stages with cp.async.bulk (sixteen 4-bit slots or eight
-// 6/8-bit slots, about 34 KB per stage, four stages in flight), starting
+// and scale bytes.  One lane of a producer warp streams the range into a ring
+// of shared-memory stages with cp.async.bulk (eighteen 4-bit slots, 39 KB, or
+// six 6/8-bit slots, 25 KB, per stage; four stages in flight), starting
 // before the wait for the kernel before (the weights are static).  Main loop:
-// consumer thread t of four sets of 128 is weight row t % 128, and set t / 128
-// takes the slots lo + t / 128 + 4j of a stage; per slot it reads its row's
+// consumer thread t of six sets of 128 is weight row t % 128, and set t / 128
+// takes the slots lo + t / 128 + 6j of a stage (a full stage without a test
+// per slot); per slot it reads its row's
 // codes (16 or 32 bytes) and scale byte from the stage, forms the integer dots
 // with dp4a straight from the sign-magnitude codes and adds 2^(Ea'+Ew') * D
 // into an fp32 accumulator per token (the product is exact: |D| < 2^20 times
@@ -73,18 +74,26 @@ __device__ int g_gemv_status;  // sticky MXS_ERR_TIMEOUT, read by mxs_device_sta
 
 namespace {
 
-constexpr int kGSets = 4;                    // consumer sets; a set is 128 threads, one per weight row
-constexpr int kConsumers = 4 * kGSets;       // consumer warps
-constexpr int kCThreads = 32 * kConsumers;   // 512
+#ifndef MXS_GEMV_SETS
+#define MXS_GEMV_SETS 6
+#endif
+constexpr int kGSets = MXS_GEMV_SETS;        // consumer sets; a set is 128 threads, one per weight row
+constexpr int kSetWarps = 4;                 // warps per set
+constexpr int kConsumers = kSetWarps * kGSets;  // consumer warps
+constexpr int kCThreads = 32 * kConsumers;   // 768
 constexpr int kGThreads = kCThreads + 64;    // + the producer warp and the hand-off warp
 constexpr int kFixWarp = kConsumers + 1;
 constexpr int kGMaxProblems = 3;
-#ifndef MXS_GEMV_RING
-#define MXS_GEMV_RING 4
+constexpr int kRing = 4;                     // shared-memory stages in flight (fewer when the tokens need the room)
+#ifndef MXS_GEMV_PER4
+#define MXS_GEMV_PER4 3
 #endif
-constexpr int kRing = MXS_GEMV_RING;         // shared-memory stages in flight
-constexpr int kSlots4 = 16, kSlots68 = 8;    // slots per stage: four (two) per consumer set
-constexpr int kStageBytes = 2176 * kSlots4;  // 34816 >= 8 x 4224
+#ifndef MXS_GEMV_PER68
+#define MXS_GEMV_PER68 1
+#endif
+constexpr int kSlots4 = MXS_GEMV_PER4 * kGSets;    // 4-bit slots per stage (18: three per set)
+constexpr int kSlots68 = MXS_GEMV_PER68 * kGSets;  // 6/8-bit slots per stage (6: one per set)
+constexpr int kStageBytes = 2176 * kSlots4 > 4224 * kSlots68 ? 2176 * kSlots4 : 4224 * kSlots68;  // 39168
 constexpr long long kWaitCycles = 4000000000ll;  // ~2 s at the maximum SM clock
 constexpr int64_t kMinCtaBytes = 32768;      // a CTA streams at least this much (and more than one slot)
 constexpr int kGemvMaxCtas = 256;            // CTAs per launch at most (sizes the partial-sum area)
@@ -162,7 +171,9 @@ __host__ __device__ __forceinline__ size_t off_bars(int MT) { return off_fix(MT)
 __host__ __device__ __forceinline__ size_t off_ring(int MT) {
     return (off_bars(MT) + (2 * kRing + 2) * 8 + 16 + 127) / 128 * 128;
 }
-__host__ __device__ __forceinline__ size_t off_tok(int MT) { return off_ring(MT) + (size_t)kRing * kStageBytes; }
+__host__ __device__ __forceinline__ size_t off_tok(int MT, int nring) {
+    return off_ring(MT) + (size_t)nring * kStageBytes;
+}
 __host__ __device__ __forceinline__ int64_t rec_bytes(int ncta, int MT) { return (int64_t)ncta * 2 * MT * 128 * 4; }
 __host__ __device__ __forceinline__ int64_t cnt_bytes(int64_t G) { return (8 * G + 255) / 256 * 256; }
 
@@ -361,7 +372,7 @@ __device__ __forceinline__ int4 segment(const Segs &s, int i, int nb) {
     return make_int4(s.gfull + (i - s.np), 0, nb, 0);
 }
 
-template <int MT>
+template <int MT, int NR>
 __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_constant__ GemvParams gp) {
     int pi = 0;
     while (pi + 1 < gp.nprob && (int)blockIdx.x >= gp.prob[pi + 1].cta0) ++pi;
@@ -382,18 +393,19 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
     uint64_t *fix_ready = empty + kRing;                                      // [2]
     volatile int *flags = reinterpret_cast<volatile int *>(fix_ready + 2);    // abort
     uint8_t *ring = smem + off_ring(MT);                                     // [kRing][kStageBytes]
-    int8_t *tcode = reinterpret_cast<int8_t *>(smem + off_tok(MT));          // [ns][MT][32] token codes
+    constexpr int nring = NR;                                                // stages in the ring
+    int8_t *tcode = reinterpret_cast<int8_t *>(smem + off_tok(MT, nring));   // [ns][MT][32] token codes
     uint8_t *tsc = reinterpret_cast<uint8_t *>(tcode) + (size_t)ns * MT * 32;  // [ns][MT] token scale bytes
     volatile int *abort_flag = flags;
 
     if (tid == 0) {
         asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-        for (int i = 0; i < kRing; ++i) {
+        for (int i = 0; i < nring; ++i) {
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], kConsumers);
         }
-        mbar_init(&fix_ready[0], kGSets);  // the four warps of set 0
-        mbar_init(&fix_ready[1], kGSets);
+        mbar_init(&fix_ready[0], kSetWarps);  // the warps of set 0
+        mbar_init(&fix_ready[1], kSetWarps);
         flags[0] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -402,7 +414,7 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
     if (warp == kConsumers) {
         // ---- producer: the range's weight bytes, stage by stage (the weights
         // are static: no wait for the kernel before)
-        int ctr = 0;
+        int ctr = 0, ri = 0, rn = 0;  // copies issued; ring slot and its use count
         if (lane == 0) {
             bool ok = true;
             for (int si = 0; si < segs.n && ok; ++si) {
@@ -410,28 +422,28 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
                 const int sa = sg.y, sb = sg.z, e4 = max(sa, min(sb, P.n4));
                 const int nst = stage_count(sa, e4, sb);
                 const uint8_t *base = P.w + (int64_t)sg.x * P.GB;
-                for (int k = 0; k < nst; ++k, ++ctr) {
+                for (int k = 0; k < nst; ++k) {
                     int lo, hi;
                     stage_range(sa, e4, sb, k, lo, hi);
-                    const int i = ctr % kRing;
-                    const uint32_t n = (uint32_t)(ctr / kRing);
-                    if (*abort_flag || (n > 0 && !mbar_wait(&empty[i], (n - 1) & 1, abort_flag))) {
+                    if (*abort_flag || (rn > 0 && !mbar_wait(&empty[ri], (uint32_t)(rn - 1) & 1, abort_flag))) {
                         ok = false;
                         break;
                     }
                     const int64_t off = slot_off_g(P.n4, lo);
                     const uint32_t bytes = (uint32_t)(slot_off_g(P.n4, hi) - off);
-                    mbar_expect_tx(&full[i], bytes);
-                    bulk_load(ring + (size_t)i * kStageBytes, base + off, bytes, &full[i]);
+                    mbar_expect_tx(&full[ri], bytes);
+                    bulk_load(ring + (size_t)ri * kStageBytes, base + off, bytes, &full[ri]);
+                    ++ctr;
+                    if (++ri == nring) ri = 0, ++rn;
                 }
             }
         }
         __syncwarp();
         named_sync(2, kGThreads);  // the consumers are done
         if (lane == 0 && *abort_flag)  // drain: the last copy issued into each ring slot
-            for (int i = 0; i < kRing && i < ctr; ++i) {
-                const int last = i + (ctr - 1 - i) / kRing * kRing;
-                drain_wait(&full[i], (uint32_t)(last / kRing) & 1);
+            for (int i = 0; i < nring && i < ctr; ++i) {
+                const int last = i + (ctr - 1 - i) / nring * nring;
+                drain_wait(&full[i], (uint32_t)(last / nring) & 1);
             }
         return;
     }
@@ -564,7 +576,7 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
     named_sync(1, kCThreads);
 
     bool aborted = false;
-    int ctr = 0;
+    int ri = 0, rn = 0;  // ring slot and its use count
     for (int si = 0; si < segs.n; ++si) {
         const int4 sg = segment(segs, si, P.nb);
         const int g = sg.x, sa = sg.y, sb = sg.z, e4 = max(sa, min(sb, P.n4));
@@ -573,14 +585,24 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
         float acc[MT];
 #pragma unroll
         for (int t = 0; t < MT; ++t) acc[t] = 0.0f;
-        for (int k = 0; k < nst; ++k, ++ctr) {
+        for (int k = 0; k < nst; ++k) {
             int lo, hi;
             stage_range(sa, e4, sb, k, lo, hi);
-            const int i = ctr % kRing;
-            if (!aborted && !warp_wait(&full[i], (uint32_t)(ctr / kRing) & 1, abort_flag)) aborted = true;
+            const int i = ri;
+            const uint32_t parity = (uint32_t)rn & 1;
+            if (++ri == nring) ri = 0, ++rn;
+            if (!aborted && !warp_wait(&full[i], parity, abort_flag)) aborted = true;
             if (!aborted) {
                 const uint8_t *sb8 = ring + (size_t)i * kStageBytes;
                 if (lo < P.n4) {
+                    if (hi - lo == kSlots4) {  // a full stage: no per-slot test
+#pragma unroll
+                        for (int jj = 0; jj < kSlots4 / kGSets; ++jj) {
+                            const int s = lo + set + kGSets * jj;
+                            const int ts = s >= q0 ? s - q0 : s - q0 + P.nb;
+                            slot4<MT>(sb8 + 2176 * (s - lo), r, tcode + (size_t)ts * MT * 32, tsc + ts * MT, acc);
+                        }
+                    } else
 #pragma unroll
                     for (int jj = 0; jj < kSlots4 / kGSets; ++jj) {
                         const int s = lo + set + kGSets * jj;
@@ -588,6 +610,15 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
                         if (s < hi) slot4<MT>(sb8 + 2176 * (s - lo), r, tcode + (size_t)ts * MT * 32, tsc + ts * MT, acc);
                     }
                 } else {
+                    if (hi - lo == kSlots68) {  // a full stage: no per-slot test
+#pragma unroll
+                        for (int jj = 0; jj < kSlots68 / kGSets; ++jj) {
+                            const int s = lo + set + kGSets * jj;
+                            const int ts = s >= q0 ? s - q0 : s - q0 + P.nb;
+                            slot68<MT>(sb8 + 4224 * (s - lo), r, s < P.n4 + P.n6 ? 6 : 8,
+                                       tcode + (size_t)ts * MT * 32, tsc + ts * MT, acc);
+                        }
+                    } else
 #pragma unroll
                     for (int jj = 0; jj < kSlots68 / kGSets; ++jj) {
                         const int s = lo + set + kGSets * jj;
@@ -647,6 +678,8 @@ int sms_now() {
 }
 
 int mt_of(int64_t M) { return M == 1 ? 1 : (M == 2 ? 2 : 4); }
+
+std::atomic<int> g_ring_override{0};  // mxs_test_gemv_ring: stages in the ring (0: chosen by size)
 
 // CTAs per problem for a launch of `count` problems of W[i] weight bytes on
 // `sms` SMs: one CTA each, then one at a time to the problem with the most
@@ -763,11 +796,22 @@ int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int
         cta += ncta[i];
         std::memcpy(gp.slot_block[i], p.slot_block, sizeof(uint16_t) * (size_t)p.nb);
     }
-    const size_t smem = off_tok(MT) + ((size_t)max_ns * MT * 33 + 15) / 16 * 16;
+    // four stages in flight, three or two when the token codes need the room
+    const size_t tok = ((size_t)max_ns * MT * 33 + 15) / 16 * 16;
+    int nring = kRing;
+    while (nring > 2 && off_tok(MT, nring) + tok > (size_t)227 * 1024) --nring;
+    const int forced = g_ring_override.load();
+    if (forced >= 2 && forced < nring) nring = forced;
+    const size_t smem = off_tok(MT, nring) + tok;
     if (smem > (size_t)227 * 1024)
         return fail(MXS_ERR_SHAPE, "decode: K too large for the CUDA-core path at M=%lld", (long long)M);
     using Kernel = void (*)(GemvParams);
-    const Kernel k = MT == 1 ? gemv_decode_kernel<1> : (MT == 2 ? gemv_decode_kernel<2> : gemv_decode_kernel<4>);
+    static const Kernel table[3][3] = {  // [MT 1, 2, 4][stages 2, 3, 4]
+        {gemv_decode_kernel<1, 2>, gemv_decode_kernel<1, 3>, gemv_decode_kernel<1, 4>},
+        {gemv_decode_kernel<2, 2>, gemv_decode_kernel<2, 3>, gemv_decode_kernel<2, 4>},
+        {gemv_decode_kernel<4, 2>, gemv_decode_kernel<4, 3>, gemv_decode_kernel<4, 4>}};
+    static_assert(kRing == 4, "the kernel table holds rings of 2..4 stages");
+    const Kernel k = table[MT == 1 ? 0 : (MT == 2 ? 1 : 2)][nring - 2];
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(gemv smem)");
     cudaLaunchConfig_t cfg = {};
@@ -815,4 +859,11 @@ int mxs_test_gemv_split(const int64_t *K, const uint8_t *const *bits, const int6
         for (int k = 0; k < n[i]; ++k, ++cta) gemv_span(k, n[i], W[i], GB[i], plans[i].n4, plans[i].nb, spans + 4 * cta);
     }
     return cta;
+}
+
+int mxs_test_gemv_ring(int stages) {
+    if (stages != 0 && (stages < 2 || stages > kRing))
+        return fail(MXS_ERR_INVALID_ARG, "stages=%d (0, or 2..%d)", stages, kRing);
+    g_ring_override.store(stages);
+    return MXS_OK;
 }

@@ -31,7 +31,8 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_quantize_act_permuted", "mxs_pack_weight_permuted", "mxs_attention_decode_workspace_bytes",
            "mxs_attention_decode", "mxs_linear_decode_group", "mxs_quantize_act_group",
            "mxs_attention_decode_batch_workspace_bytes", "mxs_attention_decode_batch", "mxs_probe_mma",
-           "mxs_probe_status", "mxs_linear_decode_workspace_bytes", "mxs_test_gemv_split"]
+           "mxs_probe_status", "mxs_linear_decode_workspace_bytes", "mxs_test_gemv_split",
+           "mxs_test_gemv_ring"]
 
 _lock = threading.Lock()
 _lib = None
@@ -118,6 +119,8 @@ def lib() -> ctypes.CDLL:
         L.mxs_linear_decode_workspace_bytes.restype = I64
         L.mxs_test_gemv_split.argtypes = [P, P, P, I, I, P, P]
         L.mxs_test_gemv_split.restype = I
+        L.mxs_test_gemv_ring.argtypes = [I]
+        L.mxs_test_gemv_ring.restype = I
         _lib = L
         return L
 

@@ -1,8 +1,9 @@
 """Decode with one to four tokens through mxs_linear_decode and
 mxs_linear_decode_group (M = 1: the activations' quantization fused into the
 CUDA-core GEMM; M = 2..4: quantizer + tensor-core GEMM) against the exact
-oracle; ragged shapes, K split over cluster ranks, NaN blocks, ties-away
-rounding, block scales over +-20 binades, grouped problems."""
+oracle; ragged shapes, row groups shared by several CTAs (their partial sums
+added by the last to arrive), NaN blocks, ties-away rounding, block scales
+over +-20 binades, grouped problems, shallow weight rings."""
 import numpy as np
 import pytest
 
@@ -84,3 +85,30 @@ def test_gemv_group_and_repeat(torch):
         got = y.cpu().numpy()
         assert np.array_equal(got, y0)
         U.check_gemm(got, ref, ab)
+
+
+@pytest.mark.parametrize("stages", [2, 3])
+def test_gemv_shallow_ring(torch, stages):
+    """The one-token kernel with two or three weight stages in its ring (what
+    it falls back to when a CTA's token codes need the shared memory): same
+    results, bit for bit, as with four, and within the bar of the oracle."""
+    L = mxs.lib()
+    M, N, nb = 1, 3000, 448
+    g = I.rng(84, stages)
+    bits = I.width_map(nb, 0.6, 0.3, 0.1, g)
+    xb = I.activations_bf16(M, bits, g, 0.01, outlier_scale=30.0)
+    wb = I.normal_bf16((N, 32 * nb), 0.02, g)
+    packed = mxs.pack_weight(U.to_dev_bf16(torch, wb), bits)
+    torch.cuda.synchronize()
+    x = U.to_dev_bf16(torch, xb)
+    y4 = mxs.linear_decode(x, bits, packed, N).cpu().numpy()
+    assert L.mxs_test_gemv_ring(stages) == 0
+    try:
+        ys = mxs.linear_decode(x, bits, packed, N).cpu().numpy()
+    finally:
+        assert L.mxs_test_gemv_ring(0) == 0
+    assert np.array_equal(ys, y4)
+    ref, ab = _ref(xb, wb, bits)
+    U.check_gemm(ys, ref, ab)
+    assert L.mxs_test_gemv_ring(1) == 1 and L.mxs_test_gemv_ring(5) == 1
+
