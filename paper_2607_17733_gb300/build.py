@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmxs.so")
-SOURCES = ["host.cu", "quantize.cu", "pack.cu", "gemm_decode.cu", "gemv_decode.cu", "gemm_prefill.cu", "noalloc.cu", "calib.cu", "attention.cu", "probe.cu"]
+SOURCES = ["host.cu", "quantize.cu", "pack.cu", "gemm_decode.cu", "gemv_decode.cu", "decode_tc.cu", "gemm_prefill.cu", "noalloc.cu", "calib.cu", "attention.cu", "probe.cu"]
 HEADERS = [os.path.join(CSRC, "common.cuh"), os.path.join(ROOT, "include", "mxs.h")]
 
 NVCC_FLAGS = [

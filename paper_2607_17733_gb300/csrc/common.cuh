@@ -152,6 +152,19 @@ int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int
                        const int64_t *N, float *const *y, const int64_t *ld_y, void *const *ws,
                        const size_t *ws_bytes, int count, int64_t M, int rounding, bool pdl, cudaStream_t st);
 int64_t gemv_workspace_bytes(int64_t M, int64_t N);
+// Decode shapes of kGemvMaxM < M <= 16 tokens through mxs_linear_decode(_group):
+// the quantizer writes the planes into ws_i, then the tensor-core kernel of
+// decode_tc.cu (an equal share of the weight bytes per CTA) runs as its
+// programmatic dependent.  ws_i: [planes][arrival counters][partial sums],
+// dtc_workspace_bytes(plan, M, N) bytes for the most CTAs (fewer fit a smaller one).
+#ifndef MXS_DECODE_TC
+#define MXS_DECODE_TC 1
+#endif
+int launch_decode_tc(const Plan *const *plans, void *const *ws, const size_t *ws_bytes, const void *const *packed,
+                     const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, bool pdl,
+                     cudaStream_t st);
+int64_t dtc_workspace_bytes(const Plan &p, int64_t M, int64_t N);
+int dtc_status(int *status, int reset);
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N,
                         float *y, int64_t ld_y, int starve, cudaStream_t st);
 int prefill_status(int *status, int reset, cudaStream_t st);

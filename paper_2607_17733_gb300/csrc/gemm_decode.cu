@@ -157,11 +157,15 @@ __device__ __forceinline__ bool test_phase(uint64_t *bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
+#ifndef MXS_DEC_SLEEP_NS
+#define MXS_DEC_SLEEP_NS 0
+#endif
 template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
     if (poll<kCluster>(bar, parity)) return true;
     const long long t0 = clock64();
     for (uint32_t i = 1;; ++i) {
+        if (MXS_DEC_SLEEP_NS > 0) __nanosleep(MXS_DEC_SLEEP_NS);
         if (poll<kCluster>(bar, parity)) return true;
         if ((i & 63) == 0) {  // the bound is checked every 64 polls
             if (*abort) return false;

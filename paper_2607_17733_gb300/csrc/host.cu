@@ -166,11 +166,12 @@ int64_t mxs_weight_bytes(int64_t N, int64_t K, const uint8_t *bits, int layout) 
 
 int64_t mxs_linear_decode_workspace_bytes(int64_t M, int64_t K, int64_t N, const uint8_t *bits) {
     if (M < 0 || N < 0) return -fail(MXS_ERR_SHAPE, "M=%lld N=%lld", (long long)M, (long long)N);
-    if (M >= 1 && M <= kGemvMaxM) {  // the CUDA-core path: arrival counters and partial sums
+    if (M >= 1 && M <= 16) {
         Plan p;
         const int rc = build_plan(bits, K, &p);
         if (rc) return -rc;
-        return gemv_workspace_bytes(M, N);
+        if (M <= kGemvMaxM) return gemv_workspace_bytes(M, N);  // the CUDA-core path: counters, partial sums
+        if (MXS_DECODE_TC) return dtc_workspace_bytes(p, M, N);  // planes, counters, partial sums
     }
     return mxs_act_planes_bytes(M, K, bits);
 }
@@ -276,6 +277,18 @@ int mxs_gemm_decode(const void *codes, const uint8_t *scales, const void *act_pl
                               static_cast<cudaStream_t>(stream));
 }
 
+// the tensor-core decode kernel of decode_tc.cu takes the problems when every
+// workspace holds, beyond its planes, the counters and one CTA's partial sums
+static bool dtc_fits(const Plan *const *plans, const size_t *ws_bytes, const int64_t *N, int count, int64_t M) {
+    for (int i = 0; i < count; ++i) {
+        const Plan &p = *plans[i];
+        const int64_t planes = align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);
+        const int64_t counters = (8 * ((N[i] + 127) / 128) + 255) / 256 * 256;
+        if ((int64_t)ws_bytes[i] < planes + counters + 2 * M * 128 * 4) return false;
+    }
+    return true;
+}
+
 int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t M, int rounding, void *stream) {
     if (!probs || count < 1 || count > 3) return fail(MXS_ERR_INVALID_ARG, "count=%d (1..3 problems)", count);
     if (M < 0) return fail(MXS_ERR_SHAPE, "M=%lld", (long long)M);
@@ -297,9 +310,11 @@ int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t 
         if (q.ld_x < q.K || q.ld_x % 8 != 0)
             return fail(MXS_ERR_INVALID_ARG, "problem %d: ld_x=%lld must be >= K and a multiple of 8", i, (long long)q.ld_x);
         if (q.ld_y < q.N) return fail(MXS_ERR_INVALID_ARG, "problem %d: ld_y=%lld < N", i, (long long)q.ld_y);
+        // the one-token path's counters and sums; else the planes (the tensor-core
+        // kernel fits its CTA count to what the workspace holds beyond them)
         const int64_t need = M >= 1 && M <= kGemvMaxM
                                  ? gemv_workspace_bytes(M, q.N)
-                                 : align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);  // the planes
+                                 : align256(align256(M * p.kp) + (M + 127) / 128 * p.nst * 512);
         if ((int64_t)q.ws_bytes < need || (need > 0 && !q.workspace))
             return fail(MXS_ERR_BUFFER, "problem %d: workspace of %lld bytes needed, %zu given", i, (long long)need,
                         q.ws_bytes);
@@ -339,6 +354,8 @@ int mxs_linear_decode_group(const mxs_decode_problem *probs, int count, int64_t 
         return launch_gemv_decode(pp, xs, lds, packed, N, y, ld_y, pls, wsb, count, M, rounding, true, st);
     rc = launch_quantize_group(pp, xs, lds, M, rounding, pls, count, st);  // one quantizer launch for the group
     if (rc) return rc;
+    if (MXS_DECODE_TC && M > kGemvMaxM && dtc_fits(pp, wsb, N, count, M))
+        return launch_decode_tc(pp, pls, wsb, packed, N, y, ld_y, count, M, true, st);
     rc = launch_gemm_decode_group(pp, planes, packed, N, y, ld_y, count, M, true, st);
     for (int i = 0; rc < 0 && i < count; ++i) {  // no grouped plan: one launch per problem
         const int r = launch_gemm_decode(plans[i], nullptr, nullptr, planes[i], packed[i], M, N[i], y[i], ld_y[i],
@@ -406,12 +423,15 @@ int mxs_linear_decode(const void *x, int64_t M, int64_t K, int64_t ld_x, const u
     if ((rc = check_device())) return rc;
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (M <= kGemvMaxM) {  // one token: quantization fused into the CUDA-core GEMM (no planes)
-        const Plan *pp = &p;
-        return launch_gemv_decode(&pp, &x, &ld_x, &packed_w, &N, &y, &ld_y, &ws, &ws_bytes, 1, M, rounding, true,
+        const Plan *pp1 = &p;
+        return launch_gemv_decode(&pp1, &x, &ld_x, &packed_w, &N, &y, &ld_y, &ws, &ws_bytes, 1, M, rounding, true,
                                   st);
     }
     rc = launch_quantize(p, x, M, ld_x, rounding, nullptr, nullptr, ws, st);
     if (rc) return rc;
+    const Plan *pp = &p;
+    if (MXS_DECODE_TC && dtc_fits(&pp, &ws_bytes, &N, 1, M))
+        return launch_decode_tc(&pp, &ws, &ws_bytes, &packed_w, &N, &y, &ld_y, 1, M, true, st);
     return launch_gemm_decode(p, nullptr, nullptr, ws, packed_w, M, N, y, ld_y, true, st);
 }
 
@@ -482,11 +502,12 @@ int mxs_device_status(int *status, int reset, void *stream) {
     if (!status) return fail(MXS_ERR_INVALID_ARG, "status is NULL");
     int rc = check_device();
     if (rc) return rc;
-    int a = 0, b = 0, c = 0;
+    int a = 0, b = 0, c = 0, d = 0;
     if ((rc = prefill_status(&a, reset, static_cast<cudaStream_t>(stream)))) return rc;
     if ((rc = decode_status(&b, reset))) return rc;
     if ((rc = gemv_status(&c, reset))) return rc;
-    *status = a ? a : (b ? b : c);
+    if ((rc = dtc_status(&d, reset))) return rc;
+    *status = a ? a : (b ? b : (c ? c : d));
     return MXS_OK;
 }
 

@@ -59,7 +59,10 @@ int mxs_linear_decode_noalloc(const void *x, int64_t M, int64_t K, int64_t ld_x,
                               const void *packed_w, int64_t N, float *y, int64_t ld_y, void *stream) {
     // the checks that need no device come first
     if (M > 16) return fail(MXS_ERR_SHAPE, "the fused decode path takes M <= 16 (M=%lld)", (long long)M);
-    const int64_t need = mxs_linear_decode_workspace_bytes(M, K, N, bits);
+    // one token: the CUDA-core path's counters and partial sums; more tokens:
+    // the planes (the tensor-core kernel fits its CTA count to the rest)
+    const int64_t need = M >= 1 && M <= kGemvMaxM ? mxs_linear_decode_workspace_bytes(M, K, N, bits)
+                                                  : mxs_act_planes_bytes(M, K, bits);
     if (need < 0) return (int)-need;  // the size query has set the message
     if ((uint64_t)need > kScratchBytes)
         return fail(MXS_ERR_BUFFER,
