@@ -200,19 +200,32 @@ __device__ __forceinline__ bool mbar_poll(uint64_t *bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
+#ifndef MXS_DTC_SUSPEND_NS
+#define MXS_DTC_SUSPEND_NS 1000
+#endif
+// the same test, but a thread whose phase is not complete is suspended until it
+// completes or `ns` nanoseconds pass: a waiting warp takes no issue slots from
+// the converters (a spinning one took most of them)
+__device__ __forceinline__ bool mbar_poll_sleep(uint64_t *bar, uint32_t parity, uint32_t ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(su32(bar)), "r"(parity), "r"(ns)
+        : "memory");
+    return ok != 0;
+}
 // bounded wait; on expiry the CTA's abort flag and the sticky status are set
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
     if (mbar_poll(bar, parity)) return true;
     const long long t0 = clock64();
-    for (uint32_t i = 1;; ++i) {
-        if (mbar_poll(bar, parity)) return true;
-        if ((i & 63) == 0) {
-            if (*abort) return false;
-            if (clock64() - t0 > kDWaitCycles) {
-                *abort = 1;
-                atomicExch(&g_dtc_status, MXS_ERR_TIMEOUT);
-                return false;
-            }
+    for (;;) {
+        if (mbar_poll_sleep(bar, parity, MXS_DTC_SUSPEND_NS)) return true;
+        if (*abort) return false;
+        if (clock64() - t0 > kDWaitCycles) {
+            *abort = 1;
+            atomicExch(&g_dtc_status, MXS_ERR_TIMEOUT);
+            return false;
         }
     }
 }
