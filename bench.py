@@ -522,13 +522,14 @@ def run_decode(args, spec: Spec):
         achieved = gemm_bytes / (gemm_ms * 1e-3) / 1e9
         prof = "gemm_decode_llama2_70b_decode.md" if spec.name.startswith("llama2-70b") \
             else "gemm_decode_llama3_8b_decode.md"
-        roofline = {"kernel": ("gemv_decode_kernel for M = 1 (quantization fused), gemm_decode_kernel + "
-                               "quantize_act_kernel (PDL chain) for M > 1" if args.path in ("fused", "grouped")
+        fused = args.path in ("fused", "grouped")
+        roofline = {"kernel": ("gemv_decode_kernel for M = 1 (quantization fused), decode_tc_kernel after "
+                               "quantize_act_kernel (PDL chain) for M > 1" if fused
                                else f"gemm_decode_kernel ({args.path} path)"),
                     "bound": "hbm", "achieved": achieved,
                     "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": achieved / pk["hbm_gbs"],
                     "peak_source": pk["source"] + " (HBM copy)",
-                    "traffic": profile_traffic("gemm_decode.cu", prof),
+                    "traffic": profile_traffic("decode_tc.cu" if fused else "gemm_decode.cu", prof),
                     "bytes_per_step": gemm_bytes, "gemm_ms_per_step": gemm_ms,
                     "gemm_launches_per_step": gemm_launches, "share_of_step": gemm_ms / ms}
 

@@ -450,6 +450,18 @@ MXS_API int mxs_attention_decode_batch(const void *q_bf16, int64_t B, int64_t H,
  * the probes' status word: MXS_ERR_TIMEOUT if a wait ran out. */
 MXS_API int mxs_probe_mma(int kind, int n, int64_t iters, int64_t *cycles, double *flop, void *stream);
 MXS_API int mxs_probe_status(int *status, int reset);
+/* Issue-rate probe for the decode GEMMs' MMAs (measurement only; the paper
+ * has no counterpart): on every SM, `issuers` warps (1, 2 or 4), one thread
+ * each, issue `iters` (a multiple of 4) MMAs back to back into four
+ * accumulators of their own: M = 128, N = 16, A in tensor memory, the A
+ * column and scale byte varying as in the decode kernels; kind 0 block-scaled
+ * e4m3 (kind::mxf8f6f4), 1 bf16 (kind::f16), 2 kind 0 with two scale-tile
+ * copies (tcgen05.cp) per four MMAs.  cycles (device int64 [SM count],
+ * 8-byte aligned, or NULL) receives issuer 0's clock cycles from its first
+ * MMA to its commit's completion; cycles / iters is the cost per MMA of one
+ * issuing thread.  Asynchronous.  Errors: MXS_ERR_INVALID_ARG, MXS_ERR_ALIGN,
+ * MXS_ERR_CUDA; status as mxs_probe_mma. */
+MXS_API int mxs_probe_mma_issue(int kind, int issuers, int64_t iters, int64_t *cycles, void *stream);
 
 /* ---------------------------------------------------------------- offline allocation
  * Calibration that produces the width maps (Alg. 1, Alg. 3, Theorem 1).  Not

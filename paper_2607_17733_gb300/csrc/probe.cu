@@ -159,6 +159,104 @@ __global__ void __launch_bounds__(kProbeThreads, 1) probe_mma_kernel(int kind, i
     }
 }
 
+// Issue rate of the decode GEMMs' MMAs: NW warps per CTA (one thread each)
+// issue `iters` MMAs back to back into four accumulators of their own, M = 128,
+// N = 16, A in tensor memory, the A column and the scale byte varying as in
+// the decode kernels.  KIND 0 block-scaled e4m3, 1 bf16, 2 kind 0 plus two
+// scale-tile copies per four MMAs.  Operands are zero.  Each issuer records
+// its cycles from its first MMA to its commit's completion.
+template <int KIND, int NW>
+__global__ void __launch_bounds__(kProbeThreads, 1) probe_issue_kernel(long long iters, long long *cycles) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t base = su32(smem_raw);
+    ProbeSmem &sm = *reinterpret_cast<ProbeSmem *>(smem_raw + (((base + 1023) & ~1023u) - base));
+    const int warp = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < (int)(sizeof(sm.a) + sizeof(sm.b) + sizeof(sm.sfa) + sizeof(sm.sfb)) / 16;
+         i += kProbeThreads)
+        reinterpret_cast<uint4 *>(sm.a)[i] = make_uint4(0, 0, 0, 0);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(&sm.bar)), "r"(NW) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(su32(&sm.tmem))
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = sm.tmem;
+    {  // zero the A tile in tensor memory: each warp its lane quarter, 32 columns
+        const uint32_t z = 0;
+        const uint32_t taddr = tmem + ((uint32_t)(32 * warp) << 16) + kATmemCol;
+        asm volatile(
+            "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,"
+            "%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1};" ::"r"(taddr),
+            "r"(z)
+            : "memory");
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    if ((threadIdx.x & 31) == 0 && warp < NW) {
+        const uint64_t db = desc_sw128(su32(sm.b)), dsa = desc_sf(su32(sm.sfa)), dsb = desc_sf(su32(sm.sfb));
+        const uint32_t sfa = tmem + kSfaCol, sfb = tmem + kSfbCol, a = tmem + kATmemCol;
+        const uint32_t acc0 = tmem + kAccCol + 64 * warp;  // four accumulators of 16 columns
+        if (KIND != 1) {
+            asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(sfa), "l"(dsa) : "memory");
+            asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(sfb), "l"(dsb) : "memory");
+        }
+        constexpr uint32_t id_mx = ((uint32_t)(16 >> 3) << 17) | (1u << 23) | ((uint32_t)(128 >> 4) << 24);
+        constexpr uint32_t id_bf =
+            (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(16 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+        const long long t0 = clock64();
+        for (long long i0 = 0; i0 < iters; i0 += 4) {
+            if (KIND == 2) {
+                asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(sfa), "l"(dsa) : "memory");
+                asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(sfb), "l"(dsb) : "memory");
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t acc = i0 > 0 ? 1u : 0u;
+                const uint32_t d = acc0 + 16 * q;
+                if (KIND == 1)
+                    asm volatile(
+                        "{\n .reg .pred p;\n setp.ne.b32 p, %3, 0;\n"
+                        " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %4, p;\n}" ::"r"(d),
+                        "r"(a + 8 * q), "l"(db + 2 * q), "r"(acc), "r"(id_bf)
+                        : "memory");
+                else
+                    asm volatile(
+                        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                        " tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], [%1], %2, %3, "
+                        "[%5], [%6], p;\n}" ::"r"(d),
+                        "r"(a + 8 * q), "l"(db + 2 * q), "r"(id_mx | ((uint32_t)q << 4) | ((uint32_t)q << 29)),
+                        "r"(acc), "r"(sfa), "r"(sfb)
+                        : "memory");
+            }
+        }
+        asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                         su32(&sm.bar))
+                     : "memory");
+        const long long tw = clock64();
+        bool done = false;
+        while (!(done = bar_done(&sm.bar, 0)) && clock64() - tw < kProbeWaitCycles) {
+        }
+        if (!done) atomicExch(&g_probe_status, MXS_ERR_TIMEOUT);
+        const long long t1 = clock64();
+        if (cycles && warp == 0) cycles[blockIdx.x] = t1 - t0;
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem) : "memory");
+    }
+}
+
 }  // namespace
 }  // namespace mxs
 
@@ -203,3 +301,27 @@ int mxs_probe_status(int *status, int reset) {
     }
     return MXS_OK;
 }
+
+int mxs_probe_mma_issue(int kind, int issuers, int64_t iters, int64_t *cycles, void *stream) {
+    if (kind < 0 || kind > 2) return fail(MXS_ERR_INVALID_ARG, "kind=%d (0..2)", kind);
+    if (issuers != 1 && issuers != 2 && issuers != 4) return fail(MXS_ERR_INVALID_ARG, "issuers=%d (1, 2, 4)", issuers);
+    if (iters < 4 || iters > (int64_t)1 << 32 || iters % 4) return fail(MXS_ERR_INVALID_ARG, "iters=%lld", (long long)iters);
+    if (cycles && (reinterpret_cast<uintptr_t>(cycles) & 7)) return fail(MXS_ERR_ALIGN, "cycles must be 8-byte aligned");
+    int rc = check_device();
+    if (rc) return rc;
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute(SM count)");
+    using K = void (*)(long long, long long *);
+    static const K table[3][3] = {{probe_issue_kernel<0, 1>, probe_issue_kernel<0, 2>, probe_issue_kernel<0, 4>},
+                                  {probe_issue_kernel<1, 1>, probe_issue_kernel<1, 2>, probe_issue_kernel<1, 4>},
+                                  {probe_issue_kernel<2, 1>, probe_issue_kernel<2, 2>, probe_issue_kernel<2, 4>}};
+    const K k = table[kind][issuers == 1 ? 0 : (issuers == 2 ? 1 : 2)];
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kProbeSmem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(probe smem)");
+    k<<<sms, kProbeThreads, kProbeSmem, static_cast<cudaStream_t>(stream)>>>((long long)iters,
+                                                                         reinterpret_cast<long long *>(cycles));
+    return cuda_fail(cudaGetLastError(), "probe_issue_kernel launch");
+}
+

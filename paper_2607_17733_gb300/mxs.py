@@ -32,7 +32,7 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_attention_decode", "mxs_linear_decode_group", "mxs_quantize_act_group",
            "mxs_attention_decode_batch_workspace_bytes", "mxs_attention_decode_batch", "mxs_probe_mma",
            "mxs_probe_status", "mxs_linear_decode_workspace_bytes", "mxs_test_gemv_split",
-           "mxs_test_gemv_ring"]
+           "mxs_test_gemv_ring", "mxs_probe_mma_issue"]
 
 _lock = threading.Lock()
 _lib = None
@@ -121,6 +121,8 @@ def lib() -> ctypes.CDLL:
         L.mxs_test_gemv_split.restype = I
         L.mxs_test_gemv_ring.argtypes = [I]
         L.mxs_test_gemv_ring.restype = I
+        L.mxs_probe_mma_issue.argtypes = [I, I, I64, P, P]
+        L.mxs_probe_mma_issue.restype = I
         _lib = L
         return L
 
