@@ -332,7 +332,10 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
 
 // e4m3 bytes (sign << 7) | |m| of the four low / four high sign-magnitude
 // nibbles (s << 3) | |m| held in a word
-__device__ __forceinline__ uint32_t lo_nib(uint32_t w) { return (w & 0x07070707u) | ((w << 4) & 0x80808080u); }
+// (the low nibble's sign, bit 3, becomes bit 7 by adding 120 where it is set:
+// n + 15 (n & 8) per byte never carries, n <= 15; an IMAD keeps the work off
+// the busier integer pipe)
+__device__ __forceinline__ uint32_t lo_nib(uint32_t w) { return (w & 0x0F0F0F0Fu) + (w & 0x08080808u) * 15u; }
 __device__ __forceinline__ uint32_t hi_nib(uint32_t w) { return ((w >> 4) & 0x07070707u) | (w & 0x80808080u); }
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
     uint32_t d;
@@ -349,12 +352,6 @@ __device__ __forceinline__ uint32_t bf16_codes(uint32_t t, uint32_t eb) {
     uint32_t d;
     asm("fma.rn.bf16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(o), "r"(0xBF80BF80u), "r"(y));  // y - o
     return d;
-}
-// four scale bytes carrying their codes' fixed-point weights (+add per byte),
-// saturating at 254; 255 (NaN) stays
-__device__ __forceinline__ uint32_t shifted4(uint32_t S4, uint32_t add) {
-    const uint32_t t = __vminu4(__vaddus4(S4, add), 0xFEFEFEFEu);
-    return t | __vcmpeq4(S4, 0xFFFFFFFFu);
 }
 
 // A CTA's segments (group, slots [sa, sb), side) in processing order: its
@@ -710,11 +707,12 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                 if (ok && gs >= kNA) ok = warp_wait(&a_free[buf], (uint32_t)(gs / kNA - 1) & 1, abort_flag);
                 if (ok && j < st.nps) {
                     const uint8_t *wst = ring + (size_t)s * kSlotBytes + kSlotTok + kSlotSf;  // the stage's weights
-                    const int64_t w0 = slot_off_d(P.n4, st.lo);
                     uint32_t d[32];
                     if (st.b4) {
-                        // plane stage ps: slots 4 ps .. 4 ps + 3 (those outside [lo, hi) are zeros)
+                        // plane stage ps: slots 4 ps .. 4 ps + 3 (those outside [lo, hi) are zeros),
+                        // 2176 bytes apart in the stage
                         const int ps = st.ps + j;
+                        const uint8_t *src0 = wst + 2176 * (4 * ps - st.lo);
                         uint4 v[4];
                         uint32_t sb = 0;
 #pragma unroll
@@ -722,9 +720,12 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                             const int sl = 4 * ps + q;
                             v[q] = make_uint4(0, 0, 0, 0);
                             if (sl >= st.lo && sl < st.hi) {
-                                const uint8_t *src = wst + (slot_off_d(P.n4, sl) - w0);
+                                const uint8_t *src = src0 + 2176 * q;
                                 v[q] = *reinterpret_cast<const uint4 *>(src + 16 * r);
-                                sb |= (uint32_t)src[2048 + r] << (8 * q);
+                                // the code's fixed-point weight in the scale byte: +7, at most
+                                // 254; 255 (NaN) stays
+                                const uint32_t S = src[2048 + r];
+                                sb |= (S == 255u ? 255u : min(S + 7u, 254u)) << (8 * q);
                             }
                         }
 #pragma unroll
@@ -740,19 +741,19 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                             d[8 * q + 7] = hi_nib(v[q].w);
                         }
                         // scale tile: row r = 32 qtr + lane at lane `lane`, column qtr; byte q = slot q
-                        *reinterpret_cast<uint32_t *>(sfa + (buf * kWin + j) * 512 + lane * 16 + qtr * 4) =
-                            shifted4(sb, 0x07070707u);
+                        *reinterpret_cast<uint32_t *>(sfa + (buf * kWin + j) * 512 + lane * 16 + qtr * 4) = sb;
                     } else {
                         // plane stage ps: slots n4 + 2 (ps - st4) + h, h = 0, 1, as bf16
                         // values m * 2^(Sw-127-(b-2)) (the scale inside)
                         const int q0 = P.n4 + 2 * (st.ps + j - P.st4);
+                        const uint8_t *src0 = wst + 4224 * (q0 - st.lo);
 #pragma unroll
                         for (int h = 0; h < 2; ++h) {
                             const int sl = q0 + h;
                             uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
                             uint32_t eb = (1u << 7) | (1u << 23);  // absent slot: zeros
                             if (sl >= st.lo && sl < st.hi) {
-                                const uint8_t *src = wst + (slot_off_d(P.n4, sl) - w0);
+                                const uint8_t *src = src0 + 4224 * h;
                                 v0 = *reinterpret_cast<const uint4 *>(src + 32 * r);
                                 v1 = *reinterpret_cast<const uint4 *>(src + 32 * r + 16);
                                 const int Sw = src[4096 + r];
