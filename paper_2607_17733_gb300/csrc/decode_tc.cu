@@ -229,13 +229,10 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
         }
     }
 }
-// whole-warp wait: lane 0 polls, then every lane takes its own acquiring test
+// whole-warp wait: every lane waits (its own acquiring test), and the warp goes
+// on only if all of them saw the phase
 __device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
-    bool ok = true;
-    if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort);
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    if (ok) mbar_poll(bar, parity);
-    return ok;
+    return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
 }
 __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
     const long long t0 = clock64();
@@ -715,11 +712,12 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                         const uint8_t *src0 = wst + 2176 * (4 * ps - st.lo);
                         uint4 v[4];
                         uint32_t sb = 0;
+                        const bool whole = 4 * ps >= st.lo && 4 * ps + 4 <= st.hi;  // all four slots present
 #pragma unroll
                         for (int q = 0; q < 4; ++q) {
                             const int sl = 4 * ps + q;
                             v[q] = make_uint4(0, 0, 0, 0);
-                            if (sl >= st.lo && sl < st.hi) {
+                            if (whole || (sl >= st.lo && sl < st.hi)) {
                                 const uint8_t *src = src0 + 2176 * q;
                                 v[q] = *reinterpret_cast<const uint4 *>(src + 16 * r);
                                 // the code's fixed-point weight in the scale byte: +7, at most
@@ -747,12 +745,13 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                         // values m * 2^(Sw-127-(b-2)) (the scale inside)
                         const int q0 = P.n4 + 2 * (st.ps + j - P.st4);
                         const uint8_t *src0 = wst + 4224 * (q0 - st.lo);
+                        const bool whole = q0 >= st.lo && q0 + 2 <= st.hi;  // both slots present
 #pragma unroll
                         for (int h = 0; h < 2; ++h) {
                             const int sl = q0 + h;
                             uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
                             uint32_t eb = (1u << 7) | (1u << 23);  // absent slot: zeros
-                            if (sl >= st.lo && sl < st.hi) {
+                            if (whole || (sl >= st.lo && sl < st.hi)) {
                                 const uint8_t *src = src0 + 4224 * h;
                                 v0 = *reinterpret_cast<const uint4 *>(src + 32 * r);
                                 v1 = *reinterpret_cast<const uint4 *>(src + 32 * r + 16);
