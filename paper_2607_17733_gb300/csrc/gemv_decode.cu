@@ -212,13 +212,10 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
         }
     }
 }
-// whole-warp wait: lane 0 polls, then every lane takes its own acquiring test
+// whole-warp wait: every lane waits (its own acquiring test), and the warp goes
+// on only if all of them saw the phase
 __device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
-    bool ok = true;
-    if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort);
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    if (ok) mbar_poll(bar, parity);
-    return ok;
+    return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
 }
 __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
     const long long t0 = clock64();
