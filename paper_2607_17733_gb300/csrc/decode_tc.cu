@@ -62,14 +62,18 @@ __device__ int g_dtc_status;  // sticky MXS_ERR_TIMEOUT, read by mxs_device_stat
 
 namespace {
 
-constexpr int kDThreads = 25 * 32;
-constexpr int kIssWarp0 = 1, kEpiWarp0 = 5, kConvWarp0 = 9, kConvWarps = 16;
-constexpr int kWin = 4;                         // plane stages per stage
+#ifndef MXS_DTC_WIN
+#define MXS_DTC_WIN 4
+#endif
+constexpr int kWin = MXS_DTC_WIN;               // plane stages per stage: one issuer and one converter quartet each
+constexpr int kIssWarp0 = 1, kEpiWarp0 = 1 + kWin, kConvWarp0 = kEpiWarp0 + 4, kConvWarps = 4 * kWin;
+constexpr int kDThreads = (kConvWarp0 + kConvWarps) * 32;  // 800 (25 warps)
 constexpr int kTokTile = 16 * 128;              // one plane stage of 16 token rows
-constexpr int kSlotTok = kWin * kTokTile;       // 8192: token tiles of a stage (1024-aligned)
-constexpr int kSlotSf = kWin * 512;             // 2048: their scale tiles
-constexpr int kSlotW = 16 * 2176;               // 34816 >= 8 x 4224: the weights
-constexpr int kSlotBytes = kSlotTok + kSlotSf + kSlotW;  // 45056 = 44 KiB
+constexpr int kSlotTok = kWin * kTokTile;       // token tiles of a stage (1024-aligned)
+constexpr int kSlotSf = kWin * 512;             // their scale tiles
+constexpr int kSlotW = 4 * kWin * 2176;         // >= 2 kWin x 4224: the weights
+constexpr int kSlotBytes = kSlotTok + kSlotSf + kSlotW;  // 45056 = 44 KiB for four plane stages
+static_assert(kSlotBytes % 1024 == 0 && kSlotW >= 2 * kWin * 4224, "ring slot");
 constexpr int kDMaxProblems = 3;
 constexpr int kDMaxCtas = 256;
 constexpr int64_t kDMinCtaBytes = 65536;
@@ -77,9 +81,13 @@ constexpr long long kDWaitCycles = 4000000000ll;  // ~2 s at the maximum SM cloc
 // tensor-memory columns: A tiles 128 buf (kNA buffers), accumulators
 // 256 + 64 ab + 16 j (one per issuer j), weight scale tiles 384 + 16 buf + 4 j,
 // token scale tiles 416 + 16 buf + 4 j
-constexpr int kNA = 2;
-constexpr uint32_t kAcc0 = 128 * kNA, kSfa0 = kAcc0 + 128, kSfb0 = kSfa0 + 16 * kNA, kTmemCols = 512;
-static_assert(kSfb0 + 16 * kNA <= kTmemCols, "tensor-memory columns");
+#ifndef MXS_DTC_NA
+#define MXS_DTC_NA 2
+#endif
+constexpr int kNA = MXS_DTC_NA;
+constexpr uint32_t kACols = 32 * kWin;  // one A tile
+constexpr uint32_t kAcc0 = kACols * kNA, kSfa0 = kAcc0 + 32 * kWin, kSfb0 = kSfa0 + 4 * kWin * kNA, kTmemCols = 512;
+static_assert(kSfb0 + 4 * kWin * kNA <= kTmemCols, "tensor-memory columns");
 
 struct DtcProblem {
     const uint8_t *w;              // packed weights (compact part)
@@ -156,6 +164,14 @@ __host__ __device__ __forceinline__ int stage_count_d(int sa, int sb, int n4) {
     const int p4 = e4 > sa ? (e4 + 3) / 4 - sa / 4 : 0;
     const int p8 = sb > a8 ? (sb - n4 + 1) / 2 - (a8 - n4) / 2 : 0;
     return (p4 + kWin - 1) / kWin + (p8 + kWin - 1) / kWin;
+}
+// the most plane stages any stage of a segment has (the first window of each
+// width run is the fullest)
+__host__ __device__ __forceinline__ int stage_npmax(int sa, int sb, int n4) {
+    const int e4 = max(sa, min(sb, n4)), a8 = max(sa, n4);
+    const int p4 = e4 > sa ? (e4 + 3) / 4 - sa / 4 : 0;
+    const int p8 = sb > a8 ? (sb - n4 + 1) / 2 - (a8 - n4) / 2 : 0;
+    return max(min(kWin, p4), min(kWin, p8));
 }
 __host__ __device__ __forceinline__ Stage stage_at(int sa, int sb, int n4, int st4, int k) {
     const int e4 = max(sa, min(sb, n4)), a8 = max(sa, n4);
@@ -448,7 +464,7 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
         // another, so each stream has its own lane.  A slot is refilled once the
         // MMAs of its last stage have run.
         int issued = 0;
-        if (lane < 6) {
+        if (lane <= kWin + 1) {
             if (lane > 0) asm volatile("griddepcontrol.wait;" ::: "memory");
             int gs = 0;
             bool ok = true;
@@ -484,7 +500,7 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
         }
         __syncwarp();
         named_sync(1, kDThreads);  // every role is done
-        if (lane < 6 && *abort_flag)  // drain: the last copies into each slot
+        if (lane <= kWin + 1 && *abort_flag)  // drain: the last copies into each slot
             for (int s = 0; s < NR && s < issued; ++s) {
                 const int last = s + (issued - 1 - s) / NR * NR;
                 drain_wait(lane == 0 ? &full_w[s] : &full_t[s], (uint32_t)(last / NR) & 1);
@@ -507,7 +523,7 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
             for (int si = 0; si < segs.n && ok; ++si) {
                 const int4 sg = segment_d(segs, si, P.nb);
                 const int nst = stage_count_d(sg.y, sg.z, P.n4), ab = si & 1;
-                const uint32_t acc = tmem + kAcc0 + 64 * ab + 16 * j;
+                const uint32_t acc = tmem + kAcc0 + 16 * kWin * ab + 16 * j;
                 bool first = true;
                 for (int k = 0; k < nst; ++k, ++gs) {
                     const Stage st = stage_at(sg.y, sg.z, P.n4, P.st4, k);
@@ -520,10 +536,10 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                         fence_after();
                         uint8_t *slot = ring + (size_t)s * kSlotBytes;
                         const uint64_t tj = desc_sw128(su32(slot)) + (uint64_t)(j * (kTokTile >> 4));
-                        const uint32_t aT = tmem + 128 * buf + 32 * j;
+                        const uint32_t aT = tmem + kACols * buf + 32 * j;
                         if (st.b4) {
-                            const uint32_t sfa_t = tmem + kSfa0 + 16 * buf + 4 * j;
-                            const uint32_t sfb_t = tmem + kSfb0 + 16 * buf + 4 * j;
+                            const uint32_t sfa_t = tmem + kSfa0 + 4 * kWin * buf + 4 * j;
+                            const uint32_t sfb_t = tmem + kSfb0 + 4 * kWin * buf + 4 * j;
                             tmem_cp_sf(sfa_t, desc_sf(su32(sfa + (buf * kWin + j) * 512)));
                             tmem_cp_sf(sfb_t, desc_sf(su32(slot + kSlotTok + j * 512)));
                             const int base = 4 * (st.ps + j);
@@ -598,19 +614,17 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
             fence_after();
             // issuer j's accumulator holds MMAs of this segment when one of its
             // stages has more than j plane stages (each has a slot in every one)
-            int npmax = 0;
-            for (int k = 0, nst = stage_count_d(sg.y, sg.z, P.n4); k < nst; ++k)
-                npmax = max(npmax, stage_at(sg.y, sg.z, P.n4, P.st4, k).nps);
+            const int npmax = stage_npmax(sg.y, sg.z, P.n4);
             float v[16];
             {
                 uint32_t u[16];
-                tmem_ld16(tmem + ((uint32_t)(32 * qtr) << 16) + kAcc0 + 64 * ab, u);
+                tmem_ld16(tmem + ((uint32_t)(32 * qtr) << 16) + kAcc0 + 16 * kWin * ab, u);
 #pragma unroll
                 for (int t = 0; t < 16; ++t) v[t] = __uint_as_float(u[t]);
             }
             for (int jj = 1; jj < npmax; ++jj) {  // in issuer order: deterministic
                 uint32_t u[16];
-                tmem_ld16(tmem + ((uint32_t)(32 * qtr) << 16) + kAcc0 + 64 * ab + 16 * jj, u);
+                tmem_ld16(tmem + ((uint32_t)(32 * qtr) << 16) + kAcc0 + 16 * kWin * ab + 16 * jj, u);
 #pragma unroll
                 for (int t = 0; t < 16; ++t) v[t] += __uint_as_float(u[t]);
             }
@@ -771,7 +785,7 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                     }
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&empty_w[s]);  // the stage's weight bytes are in registers
-                    tmem_st32(tmem + a_lane + 128 * buf + 32 * j, d);
+                    tmem_st32(tmem + a_lane + kACols * buf + 32 * j, d);
                     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                     fence_async_smem();
                     fence_before();
@@ -922,7 +936,10 @@ int launch_decode_tc(const Plan *const *plans, void *const *ws, const size_t *ws
         if (rc) return rc;
     }
     for (int i = count; i < kDMaxProblems; ++i) maps[i] = maps[0];
-    constexpr int NR = 4;
+#ifndef MXS_DTC_RING
+#define MXS_DTC_RING 4
+#endif
+    constexpr int NR = MXS_DTC_RING;
     const size_t smem = 1024 + (size_t)NR * kSlotBytes + kNA * kWin * 512 + (4 * NR + 2 * kNA + 4) * 8 + 32;
     auto k = decode_tc_kernel<NR>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
