@@ -291,22 +291,52 @@ MXS_API int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits,
 MXS_API int mxs_test_decode_starve(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M,
                                    int64_t N, int64_t K, float *y, int64_t ld_y, int chunk, void *stream);
 
-/* Test hook (host only, no device): the one-token decode path's work split
- * for `count` (1..3) problems of K[i] columns, width map bits[i] and N[i]
- * rows on `sms` SMs.  Writes each problem's CTA count to ncta[i] and, for
- * every CTA in launch order, four ints to spans (room for 4 * 256): its first
- * 128-row group, the first slot (32-element block, in the plan's slot order)
- * it takes there, its last group, and the slot where it stops there (the
- * group's block count when it takes the group to its end).  Returns the
- * number of CTAs, or minus an error code. */
+/* Test hook for the bounded waits of the two kernels mxs_linear_decode(_group)
+ * runs (failure handling of this library; the paper has no counterpart):
+ * arms the next launch of kernel 1 (the one-token CUDA-core GEMM, M = 1) or
+ * kernel 2 (the tensor-core GEMM for 2..16 tokens) so that every CTA skips
+ * the weight copy of its stage `stage` (1-based, in the CTA's streaming
+ * order; 0 disarms).  The consumers' wait for that stage runs out after ~2 s;
+ * each such CTA records MXS_ERR_TIMEOUT (mxs_device_status), stops its
+ * arithmetic, waits (bounded) for the copies it issued, frees its tensor
+ * memory and returns; y is left partly unwritten.  CTAs with fewer stages
+ * finish normally.  The arming is process-wide and taken by that one launch.
+ * No device fault or hang is involved; the context stays usable.
+ * MXS_ERR_INVALID_ARG for another kernel number or stage < 0. */
+MXS_API int mxs_test_decode_arm_starve(int kernel, int stage);
+
 /* Test hook: the one-token decode kernel's ring of weight stages.  stages =
  * 2 or 3 caps it at that many stages for the calls that follow in this
  * process (the kernel drops to fewer than four by itself only when a CTA's
  * token codes need the shared memory: long K over several row groups);
  * 0 restores the choice by size.  MXS_ERR_INVALID_ARG for other values. */
 MXS_API int mxs_test_gemv_ring(int stages);
+
+/* Test hook (host only, no device): the one-token decode path's work split
+ * for `count` (1..3) problems of K[i] columns, width map bits[i] and N[i]
+ * rows on `sms` SMs.  Writes each problem's CTA count to ncta[i] and, for
+ * every CTA in launch order, four ints to spans (room for 4 * 256): its first
+ * 128-row group, the first slot (32-element block, in the plan's slot order)
+ * it takes there, its last group, and the slot where it stops there (the
+ * group's block count when it takes the group to its end).  The ranges are
+ * balanced by weight: a 6/8-bit slot weighs its 4224 bytes, a 4-bit slot
+ * 2176 bytes times the build's weight (mxs_test_dtc_split_weight).  Returns
+ * the number of CTAs, or minus an error code. */
 MXS_API int mxs_test_gemv_split(const int64_t *K, const uint8_t *const *bits, const int64_t *N, int count, int sms,
                                 int32_t *ncta, int32_t *spans);
+
+/* Test hook (host only, no device): the same for the tensor-core decode path
+ * (2..16 tokens), whose ranges are cut at plane-stage boundaries (four 4-bit
+ * slots, two 6/8-bit slots, the end of the 4-bit run, the group's end) and
+ * balanced by weight: a 4-bit slot weighs its 2176 bytes, a 6/8-bit slot
+ * 4224 bytes times the build's weight (mxs_test_dtc_split_weight). */
+MXS_API int mxs_test_dtc_split(const int64_t *K, const uint8_t *const *bits, const int64_t *N, int count, int sms,
+                               int32_t *ncta, int32_t *spans);
+
+/* The split weights of this build, in percent: a 6/8-bit slot's in the
+ * tensor-core decode split (returned) and a 4-bit slot's in the one-token
+ * split (*cost4, if not NULL). */
+MXS_API int mxs_test_dtc_split_weight(int *cost4);
 
 /* mxs_quantize_act_permuted / mxs_pack_weight_permuted -- the layer's
  * columns in the order of the allocation (Alg. 3 returns column lists, and the

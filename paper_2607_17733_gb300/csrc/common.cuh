@@ -152,6 +152,10 @@ int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int
                        const int64_t *N, float *const *y, const int64_t *ld_y, void *const *ws,
                        const size_t *ws_bytes, int count, int64_t M, int rounding, bool pdl, cudaStream_t st);
 int64_t gemv_workspace_bytes(int64_t M, int64_t N);
+// test hook: the next launch of that kernel has every CTA skip the weight copy
+// of its stage `stage` (1-based; 0 disarms)
+void gemv_arm_starve(int stage);
+int gemv_split_cost4();  // the split's weight of a 4-bit slot, percent of its bytes
 // Decode shapes of kGemvMaxM < M <= 16 tokens through mxs_linear_decode(_group):
 // the quantizer writes the planes into ws_i, then the tensor-core kernel of
 // decode_tc.cu (an equal share of the weight bytes per CTA) runs as its
@@ -165,6 +169,8 @@ int launch_decode_tc(const Plan *const *plans, void *const *ws, const size_t *ws
                      cudaStream_t st);
 int64_t dtc_workspace_bytes(const Plan &p, int64_t M, int64_t N);
 int dtc_status(int *status, int reset);
+void dtc_arm_starve(int stage);  // as gemv_arm_starve
+int dtc_split_cost8();           // the split's weight of a 6/8-bit slot, percent of its bytes
 int launch_gemm_prefill(const Plan &p, const void *act_planes, const void *packed_w, int64_t M, int64_t N,
                         float *y, int64_t ld_y, int starve, cudaStream_t st);
 int prefill_status(int *status, int reset, cudaStream_t st);

@@ -104,6 +104,7 @@ struct DtcParams {
     int4 span[kDMaxCtas];          // per CTA: first group, its first slot, last group, end slot in it
     unsigned long long tag;        // this call's counter tag (48 bits, nonzero)
     int nprob, M;
+    int starve;                    // test hook: > 0 makes every CTA skip the weight copy of its stage starve-1
 };
 
 __host__ __device__ __forceinline__ int64_t slot_off_d(int n4, int s) {
@@ -113,23 +114,33 @@ __host__ __device__ __forceinline__ int slot_at_d(int n4, int64_t off) {
     const int64_t b4 = 2176 * (int64_t)n4;
     return off <= b4 ? (int)(off / 2176) : n4 + (int)((off - b4) / 4224);
 }
+#ifndef MXS_DTC_COST8
+#define MXS_DTC_COST8 100
+#endif
+// the work split's weight of a 6/8-bit slot, in percent of its bytes (a
+// 4-bit slot weighs its bytes): converting a 6/8-bit plane stage takes more
+// instructions per byte than a 4-bit one
+constexpr int64_t kCost8 = MXS_DTC_COST8;
+static_assert(kCost8 >= 50 && kCost8 <= 200, "split weight");
 // start of CTA k's range: the first plane-stage boundary (four 4-bit slots,
 // two 6/8-bit slots, the end of the 4-bit run, the group's end) at or after
-// k * W / ncta
+// the weighted position k * C / ncta (C: the problem's total weight)
 __host__ __device__ __forceinline__ int64_t dtc_start(int k, int ncta, int64_t W, int64_t GB, int n4, int nb) {
     if (k >= ncta) return W;
-    const int64_t b = W * k / ncta, g = b / GB, rem = b - g * GB, b4 = 2176 * (int64_t)n4;
+    const int64_t G = W / GB, w4 = 100 * 2176, w8 = kCost8 * 4224;
+    const int64_t CG = w4 * n4 + w8 * (nb - n4), b = G * CG * k / ncta;
+    const int64_t g = b / CG, rem = b - g * CG, c4 = w4 * n4;
     int64_t off;
-    if (rem <= b4) {
-        int64_t s = (rem + 2175) / 2176;
+    if (rem <= c4) {
+        int64_t s = (rem + w4 - 1) / w4;
         s = (s + 3) / 4 * 4;
         if (s > n4) s = n4;
         off = 2176 * s;
     } else {
-        int64_t t = (rem - b4 + 4223) / 4224;
+        int64_t t = (rem - c4 + w8 - 1) / w8;
         t = (t + 1) / 2 * 2;
         if (t > nb - n4) t = nb - n4;
-        off = b4 + 4224 * t;
+        off = 2176 * (int64_t)n4 + 4224 * t;
     }
     return g * GB + off;
 }
@@ -399,6 +410,63 @@ __device__ __forceinline__ int4 segment_d(const Segs &s, int i, int nb) {
     return make_int4(s.gfull + (i - s.np), 0, nb, 0);
 }
 
+// One arrival on a row group's counter word (tag << 16 | count) for the call
+// tagged `tag` (the caller's release fence comes first); returns the
+// arrival's count, 1-based, or 0 if the fallback ran out.  Tags grow call by
+// call, so the maximum turns an earlier call's word into (tag, 0) and one add
+// takes the count; a word that holds another tag even so (prior contents of
+// a workspace) goes through compare-and-swap, which reads it as count 0.
+__device__ __forceinline__ unsigned arrive_count(unsigned long long *cw, unsigned long long tag) {
+    atomicMax(cw, tag << 16);
+    unsigned long long cur = atomicAdd(cw, 1ull);
+    if ((cur >> 16) == tag) return (unsigned)(cur & 0xFFFFull) + 1;
+    cur += 1;  // the word after this add, as far as this thread knows
+    for (int it = 0; it < (1 << 20); ++it) {
+        const unsigned long long c = (cur >> 16) == tag ? (cur & 0xFFFFull) + 1 : 1;
+        const unsigned long long prev = atomicCAS(cw, cur, (tag << 16) | c);
+        if (prev == cur) return (unsigned)c;
+        cur = prev;
+    }
+    return 0;
+}
+
+// The last of row group g's CTAs to arrive, at the end of the kernel: every
+// contributor's partial sums (CTAs f..l, in CTA order) added for the group's
+// rows and the M tokens by all of the CTA's threads, a few outputs each with
+// the contributors' values in flight together.
+__device__ __forceinline__ void final_sum(const DtcProblem &P, const int4 *pspan, int M, int g, int f, int l) {
+    constexpr int kPer = (16 * 128 + kDThreads - 1) / kDThreads;  // outputs per thread
+    constexpr int kBatch = 8;                                      // contributors in flight
+    const int no = M * 128;
+    float acc[kPer];
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) acc[e] = 0.0f;
+    for (int k0 = f; k0 <= l; k0 += kBatch) {
+        float pv[kBatch][kPer];
+#pragma unroll
+        for (int d = 0; d < kBatch; ++d) {
+            const int kk = k0 + d;
+            const int sd = kk <= l && pspan[kk].x < g ? 1 : 0;  // g is that CTA's last group
+            const float *src = P.rec + (size_t)(kk * 2 + sd) * no;
+#pragma unroll
+            for (int e = 0; e < kPer; ++e) {
+                const int o = (int)threadIdx.x + e * kDThreads;
+                pv[d][e] = kk <= l && o < no ? __ldcg(src + o) : 0.0f;
+            }
+        }
+#pragma unroll
+        for (int d = 0; d < kBatch; ++d)
+#pragma unroll
+            for (int e = 0; e < kPer; ++e)
+                if (k0 + d <= l) acc[e] = k0 + d == f ? pv[d][e] : acc[e] + pv[d][e];
+    }
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) {
+        const int o = (int)threadIdx.x + e * kDThreads, n = 128 * g + (o & 127);
+        if (o < no && n < P.N) P.y[(int64_t)(o >> 7) * P.ld_y + n] = acc[e];
+    }
+}
+
 template <int NR>
 __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_constant__ DtcParams dp,
                                                                 const __grid_constant__ CUtensorMap map0,
@@ -422,7 +490,8 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
     uint64_t *full_t = full_w + NR, *freeb = full_t + NR, *empty_w = freeb + NR;
     uint64_t *a_full = empty_w + NR, *a_free = a_full + kNA, *acc_full = a_free + kNA, *acc_empty = acc_full + 2;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 2);
-    volatile int *flags = reinterpret_cast<volatile int *>(tmem_slot + 1);  // abort, last arriver, first, last CTA
+    // abort, last arriver, first and last CTA of its group, the final sum pending, its group
+    volatile int *flags = reinterpret_cast<volatile int *>(tmem_slot + 1);
     volatile int *abort_flag = flags;
 
     if (threadIdx.x == 0) {
@@ -441,7 +510,7 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
             mbar_init(&acc_full[i], kWin);  // each issuer's commit at the segment's end
             mbar_init(&acc_empty[i], 4);    // the four epilogue warps
         }
-        flags[0] = flags[1] = flags[2] = flags[3] = 0;
+        flags[0] = flags[1] = flags[2] = flags[3] = flags[4] = flags[5] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 0) {
@@ -456,6 +525,7 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
     fence_after();
     const uint32_t tmem = *tmem_slot;
 
+    int issued = 0;  // (producer lanes) copies issued, for the drain after an abort
     if (warp == 0) {
         // ---- producer: lane 0 the weights of each stage, lanes 1-4 its token
         // tiles (plane stage lane - 1 of the stage), lane 5 their scale tiles
@@ -463,21 +533,44 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
         // for it first).  Copies issued by one thread are served one after
         // another, so each stream has its own lane.  A slot is refilled once the
         // MMAs of its last stage have run.
-        int issued = 0;
+        int pre = 0;
+        if (lane == 0) {
+            // the weights of the ring's first NR stages at once, before the
+            // warp waits for the kernel before (a warp's lanes pass that wait
+            // together): their slots are free and the weights are static, so
+            // the converters fill the A tiles while the quantizer runs
+            int gs = 0;
+            for (int si = 0; si < segs.n && gs < NR && dp.starve != gs + 1; ++si) {
+                const int4 sg = segment_d(segs, si, P.nb);
+                const int nst = stage_count_d(sg.y, sg.z, P.n4);
+                for (int k = 0; k < nst && gs < NR && dp.starve != gs + 1; ++k, ++gs) {
+                    const Stage st = stage_at(sg.y, sg.z, P.n4, P.st4, k);
+                    const int64_t off = slot_off_d(P.n4, st.lo);
+                    const uint32_t bytes = (uint32_t)(slot_off_d(P.n4, st.hi) - off);
+                    mbar_expect_tx(&full_w[gs], bytes);
+                    bulk_load(ring + (size_t)gs * kSlotBytes + kSlotTok + kSlotSf, P.w + (int64_t)sg.x * P.GB + off,
+                              bytes, &full_w[gs]);
+                }
+            }
+            pre = issued = gs;
+        }
+        __syncwarp();
         if (lane <= kWin + 1) {
-            if (lane > 0) asm volatile("griddepcontrol.wait;" ::: "memory");
+            asm volatile("griddepcontrol.wait;" ::: "memory");  // the planes: written by the kernel before
             int gs = 0;
             bool ok = true;
             for (int si = 0; si < segs.n && ok; ++si) {
                 const int4 sg = segment_d(segs, si, P.nb);
                 const int nst = stage_count_d(sg.y, sg.z, P.n4);
                 for (int k = 0; k < nst; ++k, ++gs) {
+                    if (gs < pre) continue;  // (lane 0: issued above)
                     const Stage st = stage_at(sg.y, sg.z, P.n4, P.st4, k);
                     const int s = gs % NR;
                     // the weights' part of a slot is free once the converters have read
                     // it, the tokens' part once the MMAs have
                     uint64_t *fb = lane == 0 ? &empty_w[s] : &freeb[s];
-                    if (*abort_flag || (gs >= NR && !mbar_wait(fb, (uint32_t)(gs / NR - 1) & 1, abort_flag))) {
+                    if ((lane == 0 && dp.starve == gs + 1) || *abort_flag ||
+                        (gs >= NR && !mbar_wait(fb, (uint32_t)(gs / NR - 1) & 1, abort_flag))) {
                         ok = false;
                         break;
                     }
@@ -499,18 +592,7 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
             }
         }
         __syncwarp();
-        named_sync(1, kDThreads);  // every role is done
-        if (lane <= kWin + 1 && *abort_flag)  // drain: the last copies into each slot
-            for (int s = 0; s < NR && s < issued; ++s) {
-                const int last = s + (issued - 1 - s) / NR * NR;
-                drain_wait(lane == 0 ? &full_w[s] : &full_t[s], (uint32_t)(last / NR) & 1);
-            }
-        __syncwarp();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
-        return;
-    }
-
-    if (warp < kEpiWarp0) {
+    } else if (warp < kEpiWarp0) {
         // ---- the MMA issuers: issuer j (warp 1 + j, lane 0) issues the MMAs of
         // plane stage j of every stage into its own accumulator (an issuing
         // thread takes ~50 cycles per MMA whatever the other issuers do, so four
@@ -588,11 +670,7 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                 drain_wait(&a_free[committed % kNA], (uint32_t)(committed / kNA) & 1);
         }
         __syncwarp();
-        named_sync(1, kDThreads);
-        return;
-    }
-
-    if (warp < kConvWarp0) {
+    } else if (warp < kConvWarp0) {
         // ---- epilogue: accumulator row (= weight row) 32 * qtr + lane, columns = tokens
         const int qtr = warp & 3, r = 32 * qtr + lane, et = threadIdx.x - 32 * kEpiWarp0;
         const int4 *pspan = dp.span + P.cta0;
@@ -601,12 +679,10 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
             const int4 sg = segment_d(segs, si, P.nb);
             const int g = sg.x, ab = si & 1, n = 128 * g + r;
             const bool whole = sg.y == 0 && sg.z == P.nb;
-            unsigned long long cur = 0;
             int kf = 0, kl = 0;
-            if (!whole && et == 0) {  // ahead of the wait: the contributors and the counter word
+            if (!whole && et == 0) {  // ahead of the wait: the group's contributors
                 kf = first_cta_d(pspan, P.ncta, g);
                 kl = last_cta_d(pspan, P.ncta, g, P.nb);
-                cur = atomicAdd(P.cnt + g, 0ull);
             }
             // the four warps agree on going on (one that gave up would leave the
             // others at the named barrier)
@@ -640,7 +716,8 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
             }
             // part of the group: this CTA's sums into the workspace, one arrival
             // (release: a fence after the stores); the last of the group's CTAs
-            // to arrive adds all of them in CTA order
+            // to arrive adds all of them in CTA order (for the CTA's final
+            // segment, with all its threads once every role is done)
             float *mine = P.rec + (size_t)(kc * 2 + sg.w) * M * 128;
 #pragma unroll
             for (int t = 0; t < 16; ++t)
@@ -649,29 +726,25 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
             if (et == 0) {
                 int last = 0;
                 if (!*abort_flag) {
-                    const unsigned long long want = (unsigned long long)(kl - kf + 1);
                     unsigned long long *cw = P.cnt + g;
-                    bool done = false;
                     asm volatile("fence.acq_rel.gpu;" ::: "memory");
-                    for (int it = 0; it < (1 << 20) && !done; ++it) {
-                        const unsigned long long c = (cur >> 16) == dp.tag ? (cur & 0xFFFFull) + 1 : 1;
-                        const unsigned long long prev = atomicCAS(cw, cur, (dp.tag << 16) | c);
-                        if (prev == cur) {
-                            done = true;
-                            last = c == want;
-                        } else {
-                            cur = prev;
-                        }
-                    }
-                    if (!done) {
+                    const unsigned c = arrive_count(cw, dp.tag);
+                    if (c == 0) {
                         *abort_flag = 1;
                         atomicExch(&g_dtc_status, MXS_ERR_TIMEOUT);
                     }
+                    last = c == (unsigned)(kl - kf + 1);
                     if (last) {
                         asm volatile("fence.acq_rel.gpu;" ::: "memory");
+                        // (tag, 0): what a replay of this call expects to find
                         asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(cw), "l"(dp.tag << 16) : "memory");
                         flags[2] = kf;
                         flags[3] = kl;
+                        if (si == segs.n - 1) {  // the CTA's final segment: summed at the end
+                            flags[5] = g;
+                            flags[4] = 1;
+                            last = 0;
+                        }
                     }
                 }
                 flags[1] = last;
@@ -696,14 +769,10 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
             }
             named_sync(3, 128);  // the flags are reused by the next segment
         }
-        named_sync(1, kDThreads);
-        return;
-    }
-
-    // ---- converters: quartet j converts plane stage j of each stage for the
-    // 32 rows of its lane quarter into the A tile (tensor memory) and, for a
-    // 4-bit stage, the rows' scale bytes into the weight scale tile
-    {
+    } else {
+        // ---- converters: quartet j converts plane stage j of each stage for the
+        // 32 rows of its lane quarter into the A tile (tensor memory) and, for a
+        // 4-bit stage, the rows' scale bytes into the weight scale tile
         const int cw = warp - kConvWarp0, j = cw >> 2, qtr = warp & 3, r = 32 * qtr + lane;
         const uint32_t a_lane = (uint32_t)(32 * qtr) << 16;
         int gs = 0;
@@ -797,7 +866,18 @@ __global__ void __launch_bounds__(kDThreads, 1) decode_tc_kernel(const __grid_co
                 }
             }
         }
-        named_sync(1, kDThreads);
+    }
+
+    named_sync(1, kDThreads);  // every role is done
+    if (flags[4] && !*abort_flag) final_sum(P, dp.span + P.cta0, M, flags[5], flags[2], flags[3]);
+    if (warp == 0) {
+        if (lane <= kWin + 1 && *abort_flag)  // drain: the last copies into each slot
+            for (int s = 0; s < NR && s < issued; ++s) {
+                const int last = s + (issued - 1 - s) / NR * NR;
+                drain_wait(lane == 0 ? &full_w[s] : &full_t[s], (uint32_t)(last / NR) & 1);
+            }
+        __syncwarp();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
     }
 }
 
@@ -824,6 +904,7 @@ int64_t cnt_bytes_d(int64_t G) { return (8 * G + 255) / 256 * 256; }
 int64_t rec_bytes_d(int ncta, int64_t M) { return (int64_t)ncta * 2 * M * 128 * 4; }
 
 std::atomic<unsigned long long> g_dtc_tags{0};
+std::atomic<int> g_dtc_starve{0};  // mxs_test_decode_arm_starve: the next launch's skipped stage (1-based)
 
 }  // namespace
 
@@ -878,6 +959,9 @@ int dtc_status(int *status, int reset) {
     return MXS_OK;
 }
 
+void dtc_arm_starve(int stage) { g_dtc_starve.store(stage); }
+int dtc_split_cost8() { return (int)kCost8; }
+
 int launch_decode_tc(const Plan *const *plans, void *const *ws, const size_t *ws_bytes, const void *const *packed,
                      const int64_t *N, float *const *y, const int64_t *ld_y, int count, int64_t M, bool pdl,
                      cudaStream_t st) {
@@ -906,6 +990,7 @@ int launch_decode_tc(const Plan *const *plans, void *const *ws, const size_t *ws
     dp.tag = tag;
     dp.nprob = count;
     dp.M = (int)M;
+    dp.starve = g_dtc_starve.exchange(0);  // armed for this one launch
     CUtensorMap maps[kDMaxProblems];
     int cta = 0;
     for (int i = 0; i < count; ++i) {
@@ -940,7 +1025,7 @@ int launch_decode_tc(const Plan *const *plans, void *const *ws, const size_t *ws
 #define MXS_DTC_RING 4
 #endif
     constexpr int NR = MXS_DTC_RING;
-    const size_t smem = 1024 + (size_t)NR * kSlotBytes + kNA * kWin * 512 + (4 * NR + 2 * kNA + 4) * 8 + 32;
+    const size_t smem = 1024 + (size_t)NR * kSlotBytes + kNA * kWin * 512 + (4 * NR + 2 * kNA + 4) * 8 + 64;
     auto k = decode_tc_kernel<NR>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(decode_tc smem)");
@@ -963,3 +1048,32 @@ int launch_decode_tc(const Plan *const *plans, void *const *ws, const size_t *ws
 }
 
 }  // namespace mxs
+
+using namespace mxs;
+
+int mxs_test_dtc_split(const int64_t *K, const uint8_t *const *bits, const int64_t *N, int count, int sms,
+                       int32_t *ncta, int32_t *spans) {
+    if (!K || !bits || !N || !ncta || !spans) return -fail(MXS_ERR_INVALID_ARG, "NULL argument");
+    if (count < 1 || count > kDMaxProblems || sms < 1)
+        return -fail(MXS_ERR_INVALID_ARG, "count=%d (1..%d), sms=%d", count, kDMaxProblems, sms);
+    int64_t W[kDMaxProblems], GB[kDMaxProblems];
+    int cap_ws[kDMaxProblems];
+    Plan plans[kDMaxProblems];
+    for (int i = 0; i < count; ++i) {
+        const int rc = build_plan(bits[i], K[i], &plans[i]);
+        if (rc) return -rc;
+        if (N[i] < 1 || N[i] > (int64_t)0x7FFFFFF0) return -fail(MXS_ERR_SHAPE, "N=%lld", (long long)N[i]);
+        const WeightOffsets wo = weight_offsets(plans[i], N[i], false);
+        GB[i] = wo.GB;
+        W[i] = wo.G * wo.GB;
+        cap_ws[i] = kDMaxCtas;  // a workspace sized by dtc_workspace_bytes
+    }
+    int n[kDMaxProblems];
+    dtc_split_ctas(W, cap_ws, count, sms, n);
+    int cta = 0;
+    for (int i = 0; i < count; ++i) {
+        ncta[i] = n[i];
+        for (int k = 0; k < n[i]; ++k, ++cta) dtc_span(k, n[i], W[i], GB[i], plans[i].n4, plans[i].nb, spans + 4 * cta);
+    }
+    return cta;
+}

@@ -114,6 +114,7 @@ struct GemvParams {
     int4 span[kGemvMaxCtas];  // per CTA: first group, its first slot, last group, end slot in it
     unsigned long long tag;   // this call's counter tag (48 bits, nonzero)
     int nprob, M, rhaz;
+    int starve;               // test hook: > 0 makes every CTA's producer skip the copy of its stage starve-1
 };
 
 __host__ __device__ __forceinline__ int64_t slot_off_g(int n4, int s) {
@@ -124,11 +125,21 @@ __host__ __device__ __forceinline__ int slot_at(int n4, int64_t off) {
     const int64_t b4 = 2176 * (int64_t)n4;
     return off <= b4 ? (int)(off / 2176) : n4 + (int)((off - b4) / 4224);
 }
-// start of CTA k's range: the first slot boundary at or after k * W / ncta
+#ifndef MXS_GEMV_COST4
+#define MXS_GEMV_COST4 100
+#endif
+// the work split's weight of a 4-bit slot, in percent of its bytes (a 6/8-bit
+// slot weighs its bytes)
+constexpr int64_t kCost4 = MXS_GEMV_COST4;
+static_assert(kCost4 >= 50 && kCost4 <= 200, "split weight");
+// start of CTA k's range: the first slot boundary at or after the weighted
+// position k * C / ncta (C: the problem's total weight)
 __host__ __device__ __forceinline__ int64_t cta_start(int k, int ncta, int64_t W, int64_t GB, int n4) {
     if (k >= ncta) return W;
-    const int64_t b = W * k / ncta, g = b / GB, rem = b - g * GB, b4 = 2176 * (int64_t)n4;
-    const int64_t off = rem <= b4 ? (rem + 2175) / 2176 * 2176 : b4 + (rem - b4 + 4223) / 4224 * 4224;
+    const int64_t G = W / GB, nb68 = (GB - 2176 * (int64_t)n4) / 4224, w4 = kCost4 * 2176, w8 = 100 * 4224;
+    const int64_t CG = w4 * n4 + w8 * nb68, b = G * CG * k / ncta;
+    const int64_t g = b / CG, rem = b - g * CG, c4 = w4 * n4;
+    const int64_t off = rem <= c4 ? (rem + w4 - 1) / w4 * 2176 : 2176 * (int64_t)n4 + (rem - c4 + w8 - 1) / w8 * 4224;
     return g * GB + off;
 }
 // the CTAs of a problem whose ranges meet group g: [first, last] (sp: the
@@ -422,7 +433,8 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
                 for (int k = 0; k < nst; ++k) {
                     int lo, hi;
                     stage_range(sa, e4, sb, k, lo, hi);
-                    if (*abort_flag || (rn > 0 && !mbar_wait(&empty[ri], (uint32_t)(rn - 1) & 1, abort_flag))) {
+                    if (gp.starve == ctr + 1 || *abort_flag ||
+                        (rn > 0 && !mbar_wait(&empty[ri], (uint32_t)(rn - 1) & 1, abort_flag))) {
                         ok = false;
                         break;
                     }
@@ -677,6 +689,7 @@ int sms_now() {
 int mt_of(int64_t M) { return M == 1 ? 1 : (M == 2 ? 2 : 4); }
 
 std::atomic<int> g_ring_override{0};  // mxs_test_gemv_ring: stages in the ring (0: chosen by size)
+std::atomic<int> g_gemv_starve{0};    // mxs_test_decode_arm_starve: the next launch's skipped stage (1-based)
 
 // CTAs per problem for a launch of `count` problems of W[i] weight bytes on
 // `sms` SMs: one CTA each, then one at a time to the problem with the most
@@ -734,6 +747,9 @@ int gemv_status(int *status, int reset) {
     return MXS_OK;
 }
 
+void gemv_arm_starve(int stage) { g_gemv_starve.store(stage); }
+int gemv_split_cost4() { return (int)kCost4; }
+
 int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int64_t *ld_x, const void *const *packed,
                        const int64_t *N, float *const *y, const int64_t *ld_y, void *const *ws,
                        const size_t *ws_bytes, int count, int64_t M, int rounding, bool pdl, cudaStream_t st) {
@@ -760,6 +776,7 @@ int launch_gemv_decode(const Plan *const *plans, const void *const *x, const int
     gp.nprob = count;
     gp.M = (int)M;
     gp.rhaz = rounding == MXS_RHAZ;
+    gp.starve = g_gemv_starve.exchange(0);  // armed for this one launch
     int cta = 0, max_ns = 0;
     for (int i = 0; i < count; ++i) {
         const Plan &p = *plans[i];

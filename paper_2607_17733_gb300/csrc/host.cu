@@ -492,6 +492,21 @@ int mxs_test_decode_starve(const void *act_planes, const uint8_t *bits, const vo
                               static_cast<cudaStream_t>(stream), chunk);
 }
 
+int mxs_test_dtc_split_weight(int *cost4) {
+    if (cost4) *cost4 = gemv_split_cost4();
+    return dtc_split_cost8();
+}
+
+int mxs_test_decode_arm_starve(int kernel, int stage) {
+    if ((kernel != 1 && kernel != 2) || stage < 0)
+        return fail(MXS_ERR_INVALID_ARG, "kernel=%d (1 or 2), stage=%d (>= 0)", kernel, stage);
+    if (kernel == 1)
+        gemv_arm_starve(stage);
+    else
+        dtc_arm_starve(stage);
+    return MXS_OK;
+}
+
 int mxs_test_prefill_starve(const void *act_planes, const uint8_t *bits, const void *packed_w, int64_t M, int64_t N,
                             int64_t K, float *y, int64_t ld_y, int stage, void *stream) {
     if (stage < 1) return fail(MXS_ERR_INVALID_ARG, "stage=%d must be >= 1", stage);

@@ -291,11 +291,17 @@ __global__ void __launch_bounds__(kCtaThreads) quantize_act_group_kernel(const _
     quantize_rows<false, true, kRhaz, false>(g.p[blockIdx.z], g.a[blockIdx.z]);
 }
 
+#ifndef MXS_QUANT_WARP_CTAS
+#define MXS_QUANT_WARP_CTAS 1
+#endif
 // CTA shape for rows of V work slots: one CTA of whole warps for short rows
 // (several rows to a CTA), else the fewest CTAs of at most 256 threads
 void quant_shape(int V, int64_t M, int &nx, int &tx, int &ry, int64_t &gy) {
     nx = 1, ry = 1;
-    if (V <= kCtaThreads) {
+    if (MXS_QUANT_WARP_CTAS && M <= 16) {
+        tx = 32;
+        nx = (V + 31) / 32;
+    } else if (V <= kCtaThreads) {
         tx = (V + 31) / 32 * 32;
         ry = kCtaThreads / tx;
     } else {

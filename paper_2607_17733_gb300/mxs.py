@@ -32,7 +32,8 @@ EXPORTS = ["mxs_last_error", "mxs_version", "mxs_act_row_bytes", "mxs_act_codes_
            "mxs_attention_decode", "mxs_linear_decode_group", "mxs_quantize_act_group",
            "mxs_attention_decode_batch_workspace_bytes", "mxs_attention_decode_batch", "mxs_probe_mma",
            "mxs_probe_status", "mxs_linear_decode_workspace_bytes", "mxs_test_gemv_split",
-           "mxs_test_gemv_ring", "mxs_probe_mma_issue"]
+           "mxs_test_gemv_ring", "mxs_probe_mma_issue",
+           "mxs_test_decode_arm_starve", "mxs_test_dtc_split", "mxs_test_dtc_split_weight"]
 
 _lock = threading.Lock()
 _lib = None
@@ -119,8 +120,14 @@ def lib() -> ctypes.CDLL:
         L.mxs_linear_decode_workspace_bytes.restype = I64
         L.mxs_test_gemv_split.argtypes = [P, P, P, I, I, P, P]
         L.mxs_test_gemv_split.restype = I
+        L.mxs_test_dtc_split.argtypes = [P, P, P, I, I, P, P]
+        L.mxs_test_dtc_split.restype = I
+        L.mxs_test_dtc_split_weight.argtypes = [P]
+        L.mxs_test_dtc_split_weight.restype = I
         L.mxs_test_gemv_ring.argtypes = [I]
         L.mxs_test_gemv_ring.restype = I
+        L.mxs_test_decode_arm_starve.argtypes = [I, I]
+        L.mxs_test_decode_arm_starve.restype = I
         L.mxs_probe_mma_issue.argtypes = [I, I, I64, P, P]
         L.mxs_probe_mma_issue.restype = I
         _lib = L
@@ -397,6 +404,12 @@ def test_decode_starve(planes, bits, packed_w, M: int, N: int, chunk: int, y=Non
     check(lib().mxs_test_decode_starve(_ptr(planes), b.ptr, _ptr(packed_w), M, N, K, _ptr(y), _ld(y),
                                        int(chunk), _stream(stream)))
     return y
+
+
+def test_decode_arm_starve(kernel: int, stage: int):
+    """Test hook: the next launch of decode kernel `kernel` (1: one token,
+    2: tensor-core, 2..16 tokens) skips every CTA's weight stage `stage`."""
+    check(lib().mxs_test_decode_arm_starve(int(kernel), int(stage)))
 
 
 def device_status(reset: bool = False, stream=None) -> int:

@@ -258,3 +258,13 @@ def test_probe_validation(L):
     assert L.mxs_probe_mma(2, 16, 10, None, None, None) == 1
     assert L.mxs_probe_mma(0, 16, 10, FAKE + 4, ctypes.byref(f), None) == 4
     assert L.mxs_probe_status(None, 0) == 1
+
+
+def test_decode_arm_starve_validation(L):
+    """The decode kernels' starve hook takes kernel 1 or 2 and a stage >= 0
+    (host only: arming touches no device; 0 disarms)."""
+    assert L.mxs_test_decode_arm_starve(0, 1) == 1
+    assert L.mxs_test_decode_arm_starve(3, 1) == 1
+    assert L.mxs_test_decode_arm_starve(1, -1) == 1
+    assert L.mxs_test_decode_arm_starve(1, 0) == 0
+    assert L.mxs_test_decode_arm_starve(2, 0) == 0

@@ -17,7 +17,7 @@ from paper_2607_17733_gb300 import inputs as I
 from paper_2607_17733_gb300 import mxs
 
 
-def _split(problems, sms):
+def _split(problems, sms, hook="mxs_test_gemv_split"):
     """problems: [(K, bits, N)] -> (ncta list, spans [n, 4])."""
     L = mxs.lib()
     n = len(problems)
@@ -27,14 +27,26 @@ def _split(problems, sms):
     bp = (ctypes.c_void_p * n)(*[b.ctypes.data for b in keep])
     ncta = np.zeros(n, np.int32)
     spans = np.zeros((256, 4), np.int32)
-    total = L.mxs_test_gemv_split(Ks, bp, Ns, n, sms, ncta.ctypes.data, spans.ctypes.data)
+    total = getattr(L, hook)(Ks, bp, Ns, n, sms, ncta.ctypes.data, spans.ctypes.data)
     assert total > 0, mxs.last_error()
     assert total == int(ncta.sum())
     return [int(c) for c in ncta], spans[:total]
 
 
-def _check_problem(K, bits, N, spans):
-    """Each CTA's range, in bytes of the weight stream; the ranges tile it."""
+def _weights():
+    """The build's split weights (percent of a slot's bytes): 4-bit slots in
+    the one-token split, 6/8-bit slots in the tensor-core one."""
+    c4 = ctypes.c_int(0)
+    c8 = mxs.lib().mxs_test_dtc_split_weight(ctypes.byref(c4))
+    return c4.value, c8
+
+
+def _check_problem(K, bits, N, spans, w4=100, w8=100, stage=False):
+    """Each CTA's range, in bytes of the weight stream; the ranges tile it.
+    Returns their sizes in bytes and weights.  w4, w8: a slot's weight in
+    percent of its bytes; the weighted shares are equal up to the rounding of
+    each cut to the next slot (stage: to the next plane stage of four 4-bit or
+    two 6/8-bit slots, which each cut must then fall on)."""
     nb = K // 32
     n4 = int(np.sum(bits == 4))
     GB = 2176 * n4 + 4224 * (nb - n4)
@@ -44,20 +56,31 @@ def _check_problem(K, bits, N, spans):
     def off(s):  # byte offset of slot boundary s within a group
         return 2176 * s if s <= n4 else 2176 * n4 + 4224 * (s - n4)
 
+    def cost(s):  # weight of the group's slots before boundary s
+        return 2176 * w4 * min(s, n4) + 4224 * w8 * max(0, s - n4)
+
+    def on_stage(s):  # a plane-stage boundary of the group
+        return s in (n4, nb) or (s % 4 == 0 if s < n4 else (s - n4) % 2 == 0)
+
     pos = 0
-    sizes = []
-    for g0, s0, g1, s1 in spans:
+    sizes, costs = [], []
+    for g0, s0, g1, s1 in spans.tolist():  # Python ints: no fixed-width overflow
         assert 0 <= g0 <= g1 < G and 0 <= s0 < nb and 1 <= s1 <= nb
+        if stage:
+            assert on_stage(s0) and on_stage(s1)
         a, b = g0 * GB + off(s0), g1 * GB + off(s1)
         assert a == pos and b > a  # contiguous, nonempty
         sizes.append(b - a)
+        costs.append(g1 * cost(nb) + cost(s1) - g0 * cost(nb) - cost(s0))
         pos = b
     assert pos == W  # the whole stream, once
-    sizes = np.array(sizes)
-    # each share is the ideal W / n moved by less than one slot at either
-    # end (a 6/8-bit slot is the largest, 4224 bytes)
-    ideal = W / len(spans)
-    assert sizes.min() > ideal - 4224 - 1 and sizes.max() < ideal + 4224 + 1
+    sizes, costs = np.array(sizes), np.array(costs)
+    # each share is the ideal weight / n, each cut moved by less than one
+    # rounding step
+    ideal = G * cost(nb) / len(spans)
+    step = max(4 * 2176 * w4, 2 * 4224 * w8) if stage else max(2176 * w4, 4224 * w8)
+    assert costs.min() > ideal - step - 1 and costs.max() < ideal + step + 1
+    return sizes, costs
     # each CTA meets at most one group partly at either end; the CTAs that
     # share a group are a contiguous run
     for g in range(G):
@@ -82,7 +105,7 @@ def test_split_single(K, N, p, sms):
     bits = I.width_map(K // 32, *p, I.rng(401, K, N))
     ncta, spans = _split([(K, bits, N)], sms)
     assert 1 <= ncta[0] <= min(sms, 256)
-    sizes = _check_problem(K, bits, N, spans)
+    _check_problem(K, bits, N, spans, w4=_weights()[0])
     nb = K // 32
     n4 = int(np.sum(bits == 4))
     W = ((N + 127) // 128) * (2176 * n4 + 4224 * (nb - n4))
@@ -90,21 +113,48 @@ def test_split_single(K, N, p, sms):
     assert ncta[0] == min(sms, max(1, min(W // 4225, W // 32768)))
 
 
-def test_split_groups_share_the_sms_by_bytes():
+@pytest.mark.parametrize("hook", ["mxs_test_gemv_split", "mxs_test_dtc_split"])
+def test_split_groups_share_the_sms_by_bytes(hook):
     """q/k/v and gate/up of a 70B layer: the CTAs go to the problems in
-    proportion to their bytes, so the largest share per CTA is within a few
+    proportion to their bytes, so the heaviest share per CTA is within a few
     percent of the launch's average."""
+    w4, w8 = _weights()
+    kw = dict(w4=w4) if hook == "mxs_test_gemv_split" else dict(w8=w8, stage=True)
     for shapes in ([(8192, 8192), (8192, 1024), (8192, 1024)], [(8192, 28672), (8192, 28672)]):
         probs = [(K, I.llama70b_layer_map(K, 7, 80, I.rng(5, 0, i)), N) for i, (K, N) in enumerate(shapes)]
-        ncta, spans = _split(probs, 152)
+        ncta, spans = _split(probs, 152, hook)
         assert sum(ncta) == 152
         base, worst, total = 0, 0, 0
         for (K, bits, N), c in zip(probs, ncta):
-            sizes = _check_problem(K, bits, N, spans[base:base + c])
+            _, costs = _check_problem(K, bits, N, spans[base:base + c], **kw)
             base += c
-            worst = max(worst, sizes.max())
-            total += sizes.sum()
-        assert worst <= 1.05 * total / 152
+            worst = max(worst, costs.max())
+            total += costs.sum()
+        assert worst <= 1.06 * total / 152
+
+
+@pytest.mark.parametrize("K,N,p,sms", [
+    (8192, 8192, (0.6, 0.3, 0.1), 152),
+    (28672, 8192, (0.6, 0.3, 0.1), 152),
+    (8192, 28672, (0.95, 0.04, 0.01), 152),
+    (4096, 4096, (0.85, 0.1, 0.05), 148),
+    (4096, 14336, (0, 0, 1), 152),
+    (4096, 14336, (1, 0, 0), 152),
+    (32, 5, (1, 0, 0), 152),
+    (96, 300, (0, 1, 0), 152),
+    (65536, 129, (0.5, 0.3, 0.2), 152),
+    (1056, 700, (0.5, 0.3, 0.2), 152),      # odd runs: 4-bit and 6/8-bit ends off a plane stage
+])
+def test_dtc_split_single(K, N, p, sms):
+    """The tensor-core decode split: plane-stage cuts, shares of equal weight,
+    as many CTAs as the SMs unless a share would drop below 64 KB."""
+    bits = I.width_map(K // 32, *p, I.rng(402, K, N))
+    ncta, spans = _split([(K, bits, N)], sms, "mxs_test_dtc_split")
+    _check_problem(K, bits, N, spans, w8=_weights()[1], stage=True)
+    nb = K // 32
+    n4 = int(np.sum(bits == 4))
+    W = ((N + 127) // 128) * (2176 * n4 + 4224 * (nb - n4))
+    assert ncta[0] == min(sms, 256, max(1, min(W // 8705, W // 65536)))
 
 
 def test_split_rejects_bad_arguments():
