@@ -380,6 +380,26 @@ __device__ __forceinline__ int4 segment(const Segs &s, int i, int nb) {
     return make_int4(s.gfull + (i - s.np), 0, nb, 0);
 }
 
+// One arrival on a row group's counter word (tag << 16 | count) for the call
+// tagged `tag` (the caller's release fence comes first); returns the
+// arrival's count, 1-based, or 0 if the fallback ran out.  Tags grow call by
+// call, so the maximum turns an earlier call's word into (tag, 0) and one add
+// takes the count; a word that holds another tag even so (prior contents of
+// a workspace) goes through compare-and-swap, which reads it as count 0.
+__device__ __forceinline__ unsigned arrive_count(unsigned long long *cw, unsigned long long tag) {
+    atomicMax(cw, tag << 16);
+    unsigned long long cur = atomicAdd(cw, 1ull);
+    if ((cur >> 16) == tag) return (unsigned)(cur & 0xFFFFull) + 1;
+    cur += 1;  // the word after this add, as far as this thread knows
+    for (int it = 0; it < (1 << 20); ++it) {
+        const unsigned long long c = (cur >> 16) == tag ? (cur & 0xFFFFull) + 1 : 1;
+        const unsigned long long prev = atomicCAS(cw, cur, (tag << 16) | c);
+        if (prev == cur) return (unsigned)c;
+        cur = prev;
+    }
+    return 0;
+}
+
 template <int MT, int NR>
 __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_constant__ GemvParams gp) {
     int pi = 0;
@@ -468,11 +488,9 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
             const int4 sg = pseg == 0 ? segs.part0 : segs.part1;
             const int g = sg.x;
             int kf = 0, kl = 0;
-            unsigned long long cur = 0;
-            if (lane == 0) {  // ahead of the wait: the contributors and the counter word
+            if (lane == 0) {  // ahead of the wait: the group's contributors
                 kf = first_cta(pspan, P.ncta, g);
                 kl = last_cta(pspan, P.ncta, g, P.nb);
-                cur = atomicAdd(P.cnt + g, 0ull);
             }
             if (!warp_wait(&fix_ready[pseg], 0, abort_flag) || *abort_flag) break;
             for (int rr = lane; rr < 128; rr += 32)
@@ -482,24 +500,14 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
             __syncwarp();
             int last = 0;
             if (lane == 0) {
-                const unsigned long long want = (unsigned long long)(kl - kf + 1);
                 unsigned long long *cw = P.cnt + g;
-                bool done = false;
                 asm volatile("fence.acq_rel.gpu;" ::: "memory");
-                for (int it = 0; it < (1 << 20) && !done; ++it) {
-                    const unsigned long long c = (cur >> 16) == gp.tag ? (cur & 0xFFFFull) + 1 : 1;
-                    const unsigned long long prev = atomicCAS(cw, cur, (gp.tag << 16) | c);
-                    if (prev == cur) {
-                        done = true;
-                        last = c == want;
-                    } else {
-                        cur = prev;
-                    }
-                }
-                if (!done) {
+                const unsigned c = arrive_count(cw, gp.tag);
+                if (c == 0) {
                     *abort_flag = 1;
                     atomicExch(&g_gemv_status, MXS_ERR_TIMEOUT);
                 }
+                last = c == (unsigned)(kl - kf + 1);
                 if (last) {
                     asm volatile("fence.acq_rel.gpu;" ::: "memory");
                     // (tag, 0): what a replay of this call expects to find
