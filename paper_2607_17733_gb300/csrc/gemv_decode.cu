@@ -228,6 +228,11 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
 __device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
     return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
 }
+// the 128-byte lines of a 64-byte block (a hint: no data returns)
+__device__ __forceinline__ void prefetch_l2(const uint16_t *p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p + 31));
+}
 __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
     const long long t0 = clock64();
     while (!mbar_poll(bar, parity) && clock64() - t0 < kWaitCycles) {
@@ -555,6 +560,15 @@ __global__ void __launch_bounds__(kGThreads, 1) gemv_decode_kernel(const __grid_
     // int8 codes (mxs_quantize_act's rule), four threads per block of a
     // token; x may come from the kernel before (programmatic dependent launch)
     const int set = tid >> 7, r = tid & 127;
+    // the blocks of x into L2 ahead of the wait: every write lands in L2, so a
+    // block the kernel before still writes is read afresh after the wait,
+    // and the loads below no longer queue behind the weight ring's first
+    // copies in DRAM
+    for (int jt = tid; jt < ns * MT; jt += kCThreads) {
+        const int j = jt / MT, t = jt - j * MT;
+        const int s = q0 + j < P.nb ? q0 + j : q0 + j - P.nb;
+        if (t < M) prefetch_l2(P.x + (int64_t)t * P.ld_x + 32 * (int64_t)sblk[s]);
+    }
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const int nq = ns * MT * 4;
     for (int base = 0; base < nq; base += kCThreads) {  // the same trip count in every thread

@@ -264,6 +264,28 @@ __device__ __forceinline__ void quantize_rows(const Plan &p, const QuantArgs &a)
     }
 }
 
+// Decode shapes (M <= 16): each thread's block of x into L2 before the wait
+// for the kernel before.  Every write lands in L2, so a block that kernel
+// still writes is read afresh after the wait; otherwise the loads after the
+// wait find it there (larger M: the quantizer is bandwidth-bound and the
+// prefetch would only compete with the kernel before for L2).
+template <bool kPlanes, bool kPerm>
+__device__ __forceinline__ void prefetch_x(const Plan &p, const QuantArgs &a) {
+    if (kPerm || a.M > 16) return;
+    const int vs = blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t row = (int64_t)blockIdx.y * blockDim.y + threadIdx.y;
+    if (vs >= a.V || row >= a.M) return;
+    int s = vs;
+    if (kPlanes) {
+        const int j = vs - 4 * p.st4;
+        s = vs < 4 * p.st4 ? (vs < p.n4 ? vs : -1) : (j < p.n68 ? p.n4 + j : -1);
+    }
+    if (s < 0) return;
+    const uint16_t *src = a.x + row * a.ld + kBlock * (int64_t)p.slot_block[s];
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(src));
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(src + kBlock - 1));
+}
+
 // Programmatic dependent launch, both ways: a decode GEMM launched after
 // these kernels may start at once (it waits for them before reading the
 // planes), and they wait for the kernel before them (which may write x or
@@ -272,6 +294,7 @@ template <bool kCodes, bool kPlanes, bool kRhaz, bool kPerm>
 __global__ void __launch_bounds__(kCtaThreads) quantize_act_kernel(const __grid_constant__ Plan p,
                                                                    const __grid_constant__ QuantArgs a) {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    prefetch_x<kPlanes, kPerm>(p, a);
     asm volatile("griddepcontrol.wait;" ::: "memory");
     quantize_rows<kCodes, kPlanes, kRhaz, kPerm>(p, a);
 }
@@ -287,6 +310,7 @@ struct QuantGroup {
 template <bool kRhaz>
 __global__ void __launch_bounds__(kCtaThreads) quantize_act_group_kernel(const __grid_constant__ QuantGroup g) {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    prefetch_x<true, false>(g.p[blockIdx.z], g.a[blockIdx.z]);
     asm volatile("griddepcontrol.wait;" ::: "memory");
     quantize_rows<false, true, kRhaz, false>(g.p[blockIdx.z], g.a[blockIdx.z]);
 }
