@@ -131,21 +131,33 @@ def peaks():
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
 
 
+def code_sha(src: bytes) -> str:
+    """sha256[:16] of a CUDA source with its comments and blank space removed:
+    the same for two versions that differ only in comments or layout."""
+    import hashlib
+    import re
+    text = src.decode("utf-8")
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return hashlib.sha256(" ".join(text.split()).encode()).hexdigest()[:16]
+
+
 def profile_traffic(kernel_file: str, profile_md: str):
     """DRAM bytes per launch recorded in a committed ncu summary, if it was taken
-    on the current source of the kernel (sha256 of the .cu file)."""
+    on the current code of the kernel: the summary's sha is the sha256[:16] of
+    the .cu file, or of its code alone (code_sha)."""
     import hashlib
     try:
         src = open(os.path.join(ROOT, "paper_2607_17733_gb300", "csrc", kernel_file), "rb").read()
         text = open(os.path.join(ROOT, "profiles", profile_md)).read()
     except OSError:
         return None
-    sha = hashlib.sha256(src).hexdigest()[:16]
+    shas = {hashlib.sha256(src).hexdigest()[:16], code_sha(src)}
     for line in text.splitlines():
         if line.startswith("traffic_bytes_per_launch:"):
             parts = line.split()
             # traffic_bytes_per_launch: <bytes> kernel_sha: <sha>
-            if len(parts) >= 4 and parts[3] == sha:
+            if len(parts) >= 4 and parts[3] in shas:
                 return float(parts[1])
     return None
 

@@ -30,8 +30,9 @@
 // problem's weight bytes, cut at plane-stage boundaries; row groups its range
 // covers whole go straight to y, the partial ones at its ends leave per-row
 // partial sums in the workspace for the last of the group's CTAs to arrive,
-// which adds them in CTA order (tagged 64-bit arrival counters: no workspace
-// preparation).
+// which adds them in CTA order (tagged 64-bit arrival counters, as there: no
+// workspace preparation); the sum for a CTA's final segment is done by all
+// its threads once every role is done.
 //
 // Roles (800 threads, one CTA per SM, all of tensor memory):
 //   warp 0      producer: lane 0 the weight bytes of each stage (bulk copy,

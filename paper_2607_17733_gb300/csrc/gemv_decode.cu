@@ -29,8 +29,8 @@
 // a group's CTAs to arrive (an arrival counter in the workspace) adds the
 // partials in CTA order and writes y: deterministic, independent of timing.
 // A CTA takes its partial groups first and hands their sums to a hand-off
-// warp (workspace stores, a release fence, one compare-and-swap, and for the
-// last arriver the ordered sum), so that the latency of that exchange overlaps
+// warp (workspace stores, a release fence, one arrival, and for the last
+// arriver the ordered sum), so that the latency of that exchange overlaps
 // the streaming of the rest of its range.  (Measured on the 70B layers: with
 // one CTA per SM and equal bytes, q/k/v, o, gate/up and down took 18.1, 15.9,
 // 53.8 and 37.0 us against 19.7, 14.7, 53.8 and 38.5 us with whole groups
@@ -40,7 +40,8 @@
 // Per CTA.  Prologue: it quantizes the activations of the slots its range
 // takes (x is bf16; the rule, bit for bit, of mxs_quantize_act; four threads
 // per block, the block maximum by shuffles) into shared memory as int8 codes
-// and scale bytes.  One lane of a producer warp streams the range into a ring
+// and scale bytes, its blocks of x prefetched into L2 before the wait for the
+// kernel before.  One lane of a producer warp streams the range into a ring
 // of shared-memory stages with cp.async.bulk (eighteen 4-bit slots, 39 KB, or
 // six 6/8-bit slots, 25 KB, per stage; four stages in flight), starting
 // before the wait for the kernel before (the weights are static).  Main loop:
@@ -56,12 +57,15 @@
 // copies.
 //
 // Arrival counters are 64-bit words holding a 48-bit tag, a number the host
-// draws afresh for every call, and a 16-bit count.  A CTA that finds another
-// tag takes the count for zero, and the last arriver leaves (tag, 0), so the
-// workspace needs no preparation: garbage, planes of an earlier call with
-// M > 1, or the counters of an earlier call all read as zero (unless a stale
-// word carries this call's 48-bit tag), and a CUDA graph that replays one call
-// finds its own tag with count zero.
+// draws afresh for every call (increasing), and a 16-bit count.  An arrival
+// raises the word to (tag, 0) by an atomic maximum and takes its count by an
+// atomic add (one round trip); a word that still holds another tag (a larger
+// one: prior contents of the workspace) goes through compare-and-swap, which
+// takes it for count zero.  The last arriver leaves (tag, 0), so the workspace
+// needs no preparation: garbage, planes of an earlier call with M > 1, or the
+// counters of an earlier call all read as zero (unless a stale word carries
+// this call's 48-bit tag), and a CUDA graph that replays one call finds its
+// own tag with count zero.
 #include <algorithm>
 #include <atomic>
 #include <cstring>
