@@ -440,9 +440,11 @@ def run_decode(args, spec: Spec):
     capture_stream = torch.cuda.Stream(device=dev)
     groups = [[it for it in items if it[0] == M] for M in spec.Ms]
 
-    def make_step(events=None):
+    def make_step(events=None, grps=None):
+        grps = groups if grps is None else grps
+
         def fn():
-            for gi, grp in enumerate(groups):
+            for gi, grp in enumerate(grps):
                 if args.path not in ("fused", "grouped"):
                     for M, lin, x, bufs in grp:
                         if args.path == "codes":
@@ -545,18 +547,55 @@ def run_decode(args, spec: Spec):
                     "bytes_per_step": gemm_bytes, "gemm_ms_per_step": gemm_ms,
                     "gemm_launches_per_step": gemm_launches, "share_of_step": gemm_ms / ms}
 
-    # ---- end to end through the public API with host buffers
+    # ---- end to end through the public API with host buffers: every step copies
+    # its inputs in from pinned host memory and reads its outputs back, on two
+    # copy streams (in, out) beside the compute stream, over two device buffer
+    # sets, so that step k+1's inputs arrive and step k's outputs leave while
+    # the neighbouring step computes (the copies share the host link and HBM)
+    x_dev2, y_dev2 = torch.empty_like(x_dev), torch.empty_like(y_dev)
+
+    def rebind(it):
+        M, lin, x, bufs = it
+        xo = (x.data_ptr() - x_dev.data_ptr()) // x.element_size()
+        yo = (bufs["y"].data_ptr() - y_dev.data_ptr()) // 4
+        b2 = dict(bufs)
+        b2["y"] = y_dev2[yo:yo + M * lin.N].view(M, lin.N)
+        return (M, lin, x_dev2[xo:xo + M * lin.K].view(M, lin.K), b2)
+
+    plain2 = capture(make_step(grps=[[rebind(it) for it in grp] for grp in groups]))
+    sets = [(x_dev, y_dev, plain), (x_dev2, y_dev2, plain2)]
+    comp, s_in, s_out = torch.cuda.current_stream(), torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    got = [torch.cuda.Event() for _ in sets]   # a set's inputs are in
+    done = [torch.cuda.Event() for _ in sets]  # a set's compute is done
+    out = [torch.cuda.Event() for _ in sets]   # a set's outputs are out
     barrier(ws)
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e2e_steps = max(1, min(args.steps, 50))
-    e0.record()
-    for _ in range(e2e_steps):
-        x_dev.copy_(x_host, non_blocking=True)
-        plain.replay()
-        y_host.copy_(y_dev, non_blocking=True)
-    e1.record()
+    e0.record(comp)
+    s_in.wait_event(e0)
+    s_out.wait_event(e0)
+    for k in range(e2e_steps):
+        b = k % 2
+        xd, yd, g = sets[b]
+        if k >= 2:
+            s_in.wait_event(done[b])  # step k - 2 has read this set's inputs
+        with torch.cuda.stream(s_in):
+            xd.copy_(x_host, non_blocking=True)
+        got[b].record(s_in)
+        comp.wait_event(got[b])
+        if k >= 2:
+            comp.wait_event(out[b])  # step k - 2's outputs have left this set
+        g.replay()
+        done[b].record(comp)
+        s_out.wait_event(done[b])
+        with torch.cuda.stream(s_out):
+            y_host.copy_(yd, non_blocking=True)
+        out[b].record(s_out)
+    comp.wait_stream(s_in)
+    comp.wait_stream(s_out)
+    e1.record(comp)
     torch.cuda.synchronize()
     e2e_ms = allreduce_max(e0.elapsed_time(e1) / e2e_steps, ws)
     e2e = {"value": ws * step_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
