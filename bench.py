@@ -723,7 +723,7 @@ def run_prefill_part(args, spec: Spec):
     q_bytes = sum(2 * M * lin.K + pl.numel() for (lin, _), pl in zip(items, planes))
     n_launch = len(items) + len(items) // nproj * len(STAGES)
 
-    def fn(events=None):
+    def fn(events=None, xs=xs, ys=ys):
         for base in range(0, len(items), nproj):
             for si, stage in enumerate(STAGES):
                 idxs = [base + i for i in stage]
@@ -785,20 +785,44 @@ def run_prefill_part(args, spec: Spec):
 
     probes = probe_peaks(torch) if rank == 0 else {}
 
-    # end to end: the step's activations from pinned host memory, every output back
+    # end to end: every step's activations from pinned host memory and every
+    # output back, on an input and an output copy stream beside the compute
+    # stream over two device buffer sets (as in the decode part)
     x_host = [x.cpu().pin_memory() for x in xs]
     y_host = [torch.empty(tuple(y.shape), dtype=torch.float32).pin_memory() for y in ys]
+    sets = [(xs, ys), ([torch.empty_like(x) for x in xs], [torch.empty_like(y) for y in ys])]
+    comp, s_in, s_out = torch.cuda.current_stream(), torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    got = [torch.cuda.Event() for _ in sets]   # a set's inputs are in
+    done = [torch.cuda.Event() for _ in sets]  # a set's compute is done
+    out = [torch.cuda.Event() for _ in sets]   # a set's outputs are out
     barrier(ws)
     torch.cuda.synchronize()
     e2e_steps = max(1, min(steps, 5))
-    t0.record()
-    for _ in range(e2e_steps):
-        for xh, x in zip(x_host, xs):
-            x.copy_(xh, non_blocking=True)
-        fn()
-        for yh, y in zip(y_host, ys):
-            yh.copy_(y, non_blocking=True)
-    t1.record()
+    t0.record(comp)
+    s_in.wait_event(t0)
+    s_out.wait_event(t0)
+    for k in range(e2e_steps):
+        b = k % 2
+        X, Y = sets[b]
+        if k >= 2:
+            s_in.wait_event(done[b])  # step k - 2 has read this set's inputs
+        with torch.cuda.stream(s_in):
+            for xh, x in zip(x_host, X):
+                x.copy_(xh, non_blocking=True)
+        got[b].record(s_in)
+        comp.wait_event(got[b])
+        if k >= 2:
+            comp.wait_event(out[b])  # step k - 2's outputs have left this set
+        fn(xs=X, ys=Y)
+        done[b].record(comp)
+        s_out.wait_event(done[b])
+        with torch.cuda.stream(s_out):
+            for yh, y in zip(y_host, Y):
+                yh.copy_(y, non_blocking=True)
+        out[b].record(s_out)
+    comp.wait_stream(s_in)
+    comp.wait_stream(s_out)
+    t1.record(comp)
     torch.cuda.synchronize()
     e2e_ms = allreduce_max(t0.elapsed_time(t1) / e2e_steps, ws)
     e2e = {"value": ws * step_ops / (e2e_ms * 1e-3) / 1e12, "unit": "TOPS",
@@ -809,7 +833,7 @@ def run_prefill_part(args, spec: Spec):
         v, dt, threads, desc, unit = oracle_sample(spec)
         cpu = {"value": v, "unit": unit, "cores": threads, "kind": "oracle", "sample": desc, "seconds": dt}
     q_launches = len(items) // nproj * len(STAGES)
-    del items, xs, planes, ys, x_host, y_host
+    del items, xs, planes, ys, x_host, y_host, sets
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
     if rank != 0:
