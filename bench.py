@@ -338,7 +338,8 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * statistics.median(secs), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int64+f64", "data": "synthetic",
-        "config": {"workload": f"{args.workload} (sample)", "layers": 1, "M": list(spec.Ms)},
+        "config": {"workload": args.workload, "M": list(spec.Ms), "layers": spec.layers,
+                   "sample": desc},
         "cpu_baseline": {"value": value, "unit": unit, "cores": threads, "kind": "oracle", "sample": desc},
         "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
