@@ -32,7 +32,11 @@ _lib = None
 
 
 def build(force: bool = False) -> str:
-    """Compile mxo.c with gcc (plain -O2, IEEE semantics, OpenMP over rows)."""
+    """Compile mxo.c with gcc (plain -O2, IEEE semantics, OpenMP over rows).
+    MXO_LIB names an already built copy instead (the planted-mistake tests
+    load altered copies of mxo.c this way)."""
+    if os.environ.get("MXO_LIB"):
+        return os.environ["MXO_LIB"]
     os.makedirs(_BUILD, exist_ok=True)
     if (not force and os.path.exists(_LIB_PATH)
             and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):

@@ -274,15 +274,20 @@ def test_gemm_entries_match_full_gemm_and_transpose_rule():
 
 
 def test_gemm_nan_block_propagates():
+    """An Inf or NaN in a block (scale byte 255) makes every output that block
+    enters NaN, from either operand: an activation block its row, a weight
+    block its column; the other outputs stay finite."""
     bits = np.array([4, 8], np.uint8)
-    a = np.ones((1, 64), np.float32)
+    a = np.ones((2, 64), np.float32)
     a[0, 40] = np.inf
-    w = np.ones((2, 64), np.float32)
+    w = np.ones((3, 64), np.float32)
+    w[2, 5] = np.nan
     as_, ac = mxo.quantize_bf16(I.f32_to_bf16_bits(a), bits)
     ws, wc = mxo.quantize_bf16(I.f32_to_bf16_bits(w), bits)
-    assert as_[0, 1] == 255
+    assert as_[0, 1] == 255 and ws[2, 0] == 255
     y, _ = mxo.gemm(bits, ac, as_, wc, ws)
-    assert np.all(np.isnan(y))
+    assert np.all(np.isnan(y[0])) and np.all(np.isnan(y[:, 2]))
+    assert np.all(np.isfinite(y[1, :2]))
 
 
 # --------------------------------------------------------------- storage format
