@@ -1,9 +1,13 @@
 """Planted mistakes in the oracle (on the CPU): each copy of oracle/mxo.c
-below carries one plausible error -- an exponent off by one, ties to the
-wrong side, a clamp that admits -2^(b-1), a grid one fraction bit off, a
-dropped or misaligned element in the block dot, a scale with the wrong sign,
-a NaN of one operand ignored, a naive sum -- and is built into its own
-library.  The oracle's pins (tests/test_oracle_pins.py, run against that
+below carries one plausible error -- in the arithmetic (an exponent off by
+one, ties to the wrong side, a clamp that admits -2^(b-1), a grid one
+fraction bit off, a dropped or misaligned element in the block dot, a scale
+with the wrong sign, a NaN of one operand ignored, a naive sum) or in the
+storage formats and MMA operands (nibble order, word layout, sign bit, scale
+byte place, width-group order, the e4m3 and bf16 encoders, plane digits, the
+scale-tile layout) -- and is built into its own library.  (Where the
+digits of a 6/8-bit code split is not pinned: any exact split is as good,
+and no kernel reads the digit form; the bf16 form is their operand.)  The oracle's pins (tests/test_oracle_pins.py, run against that
 library) must reject every copy: this is what lets the pins vouch for the
 oracle."""
 import os
@@ -31,6 +35,17 @@ MUTANTS = {
     "a NaN weight block ignored": ("if (as[kb] == 255 || ws[kb] == 255) nan = 1;", "if (as[kb] == 255) nan = 1;"),
     "naive summation": ("*y = mxo_fsum(terms, nb);",
                         "{ double s_ = 0; for (int64_t q_ = 0; q_ < nb; ++q_) s_ += terms[q_]; *y = s_; }"),
+    # storage formats and MMA operands (every altered copy writes inside its buffers)
+    "activation nibbles swapped": ("(i % 2) ? (nib << 4) : nib", "(i % 2) ? nib : (nib << 4)"),
+    "weight nibble word layout": ("4 * i + (within % 4)", "4 * i + (within / 2)"),
+    "6/8-bit weight sign in bit 6": ("(uint8_t)(((c[e] < 0) << 7) | mag)", "(uint8_t)(((c[e] < 0) << 6) | mag)"),
+    "4-bit weight scale byte one place early": ("slot[2048 + rr]", "slot[2047 + rr]"),
+    "8-bit group before the 6-bit group": ("const int widths[3] = {4, 6, 8};", "const int widths[3] = {4, 8, 6};"),
+    "e4m3 exponent bias": ("code = ((E + 7) << 3) | (int)k;", "code = ((E + 6) << 3) | (int)k;"),
+    "bf16 subnormal scale": ("double k = ldexp(a, 133);", "double k = ldexp(a, 132);"),
+    "4-bit plane digit m/2": ("if (b == 4) { *hi = m / 4.0;", "if (b == 4) { *hi = m / 2.0;"),
+    "low digit one bit off": ("*lo = ldexp((double)l, -(b - 2));", "*lo = ldexp((double)l, -(b - 1));"),
+    "scale tile transposed": ("* 16 + w * 4 + q] = scales", "* 16 + q * 4 + w] = scales"),
 }
 
 

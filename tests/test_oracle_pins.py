@@ -378,7 +378,7 @@ def test_pack_weight_round_trip(N):
     sf = buf[sf_off:sf_off + ((N + 127) // 128) * nst * 512]
     s3, c3 = mxformat.decode_planes(bits, pl, sf, bf16_68=True)  # weight planes: 6/8-bit blocks as bf16
     assert np.array_equal(s3, scales) and np.array_equal(c3, codes)
-    pd, sfd = mxo.planes(bits, scales, codes)  # digit form (decode operand)
+    pd, sfd = mxo.planes(bits, scales, codes)  # digit form (the oracle's second encoding; no kernel reads it)
     s4, c4 = mxformat.decode_planes(bits, pd, sfd.reshape(-1))
     assert np.array_equal(s4, scales) and np.array_equal(c4, codes)
 
