@@ -144,3 +144,13 @@ def test_block_flooring_keeps_the_average_at_or_below_b():
     assert avg <= B + 1e-12
     # each layer loses fewer than 64 columns of 6 bits (column floor + block floor)
     assert B - avg < 2 * 64 * len(d) / sum(d)
+
+
+def test_n6_is_the_floor_of_the_product():
+    """Alg. 3 takes the floor of R * S_layer * (d_in - 32) for the 6-bit column
+    count: a fractional part above one half still rounds down."""
+    d = 4096  # d - 32 = 4064
+    assert A.n6_columns(d, 100.75 / 4064, 1.0) == 100
+    assert A.n6_columns(d, 200.6 / 4064, 1.0) == 200
+    assert A.n6_columns(d, 0.9 / 4064, 1.0) == 0
+    assert A.n6_columns(d, 2 * 301.7 / 4064, 0.5) == 301

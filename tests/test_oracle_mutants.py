@@ -79,3 +79,67 @@ def test_the_unaltered_oracle_passes_the_same_run(tmp_path):
                         os.path.join(ROOT, "tests", "test_oracle_pins.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stdout[-2000:]
+
+
+# ------------------------------------------------- the Python oracles
+PY_MUTANTS = {
+    # oracle/alloc.py (Alg. 1, Theorem 1, Alg. 3), pinned by test_oracle_alloc.py
+    "sensitivity as a sum of |x|": ("oracle/alloc.py", "return np.sum(x * x, axis=0)",
+                                    "return np.sum(np.abs(x), axis=0)"),
+    "R without the 8-bit columns": ("oracle/alloc.py", "num = (B - 4.0) * d.sum() - 4.0 * BLOCK * n",
+                                    "num = (B - 4.0) * d.sum()"),
+    "R with the 6-bit gain halved": ("oracle/alloc.py", "den = np.sum(2.0 * s * (d - BLOCK))",
+                                     "den = np.sum(s * (d - BLOCK))"),
+    "N6 rounded": ("oracle/alloc.py", "v = math.floor(R * s_layer * (d_in - BLOCK))",
+                   "v = round(R * s_layer * (d_in - BLOCK))"),
+    "N6 unclamped": ("oracle/alloc.py", "return int(min(max(v, 0), d_in - BLOCK))", "return int(max(v, 0))"),
+    "ties in reverse order": ("oracle/alloc.py", 'np.argsort(-s, kind="stable")',
+                              'np.argsort(s, kind="stable")[::-1]'),
+    "no 8-bit block": ("oracle/alloc.py", "bits[0] = 8", "bits[0] = 6"),
+    "one 6-bit block too many": ("oracle/alloc.py", "bits[1:1 + n6b] = 6", "bits[1:2 + n6b] = 6"),
+    # oracle/attention.py (KV cache, Appendix A.2), pinned by test_oracle_attention.py
+    "query head reads the wrong KV head": ("oracle/attention.py", "c = (h // G) * D", "c = (h % n_kv_heads) * D"),
+    "scores without the scale": ("oracle/attention.py", "s = scale * (kh @ q[h])", "s = kh @ q[h]"),
+    "weights not normalised": ("oracle/attention.py", "out[h] = (p @ vh) / np.sum(p)", "out[h] = (p @ vh)"),
+    "sequence rows at the wrong place": ("oracle/attention.py", "rows = slice(b * T_cap, b * T_cap + T)",
+                                         "rows = slice(b * T, b * T + T)"),
+    "cache values on the 8-bit grid": ("oracle/attention.py", "return mxo.dequantize(codes, scales, bits)",
+                                       "return mxo.dequantize(codes, scales, np.full(len(bits), 8, np.uint8))"),
+}
+PINS = {"oracle/alloc.py": "test_oracle_alloc.py", "oracle/attention.py": "test_oracle_attention.py"}
+
+
+def _py_tree(tmp_path, rel, old, new):
+    """A copy of tests/ and oracle/ with one oracle file altered (the package
+    linked): the copied conftest puts this tree first on the path."""
+    import shutil
+    skip = shutil.ignore_patterns("__pycache__", "_build")
+    shutil.copytree(os.path.join(ROOT, "tests"), tmp_path / "tests", ignore=skip)
+    shutil.copytree(os.path.join(ROOT, "oracle"), tmp_path / "oracle", ignore=skip)
+    os.symlink(os.path.join(ROOT, "paper_2607_17733_gb300"), tmp_path / "paper_2607_17733_gb300")
+    f = tmp_path / rel
+    src = f.read_text()
+    assert src.count(old) == 1, f"the text to alter must occur once in {rel}"
+    f.write_text(src.replace(old, new))
+    return tmp_path
+
+
+def _run_pins(tree, rel):
+    from oracle import mxo
+    env = dict(os.environ, MXO_LIB=mxo.build(), OMP_NUM_THREADS="2")  # the C oracle as built
+    return subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                           str(tree / "tests" / PINS[rel])],
+                          cwd=str(tree), env=env, capture_output=True, text=True, timeout=600)
+
+
+@pytest.mark.parametrize("name", list(PY_MUTANTS))
+def test_python_pins_reject_a_planted_mistake(tmp_path, name):
+    rel, old, new = PY_MUTANTS[name]
+    r = _run_pins(_py_tree(tmp_path, rel, old, new), rel)
+    assert r.returncode == 1, f"{name}: pins returned {r.returncode}\n{r.stdout[-2000:]}"
+
+
+@pytest.mark.parametrize("rel", list(PINS))
+def test_the_unaltered_python_oracles_pass_the_same_run(tmp_path, rel):
+    r = _run_pins(_py_tree(tmp_path, rel, "import numpy as np", "import numpy as np"), rel)
+    assert r.returncode == 0, r.stdout[-2000:]
