@@ -46,6 +46,17 @@ MUTANTS = {
     "4-bit plane digit m/2": ("if (b == 4) { *hi = m / 4.0;", "if (b == 4) { *hi = m / 2.0;"),
     "low digit one bit off": ("*lo = ldexp((double)l, -(b - 2));", "*lo = ldexp((double)l, -(b - 1));"),
     "scale tile transposed": ("* 16 + w * 4 + q] = scales", "* 16 + q * 4 + w] = scales"),
+    # block maximum, exponent range, special values, exact summation
+    "block maximum without the absolute value": ("else if (fabs(x[i]) > amax) amax = fabs(x[i]);",
+                                                 "else if (x[i] > amax) amax = x[i];"),
+    "exponent floor at -120": ("if (E < -127) E = -127;", "if (E < -120) E = -120;"),
+    "scale byte 255 read as a number": ("if (scale == 255) return NAN;", "if (scale == 256) return NAN;"),
+    "activation scales in block order": ("pscales[r * nb + s] = scales[r * nb + kb];",
+                                         "pscales[r * nb + s] = scales[r * nb + s];"),
+    "bf16 NaN block written as Inf": ("S == 255 ? 0x7FC0 :", "S == 255 ? 0x7F80 :"),
+    "two-sum low part with the wrong sign": ("double lo = y - (hi - x);", "double lo = (hi - x) - y;"),
+    "exact sum without the half-way fix": ("if (y == x - hi) hi = x;", "if (0) hi = x;"),
+    "e4m3 subnormal scale": ("double k = ldexp(a, 9);", "double k = ldexp(a, 8);"),
 }
 
 

@@ -305,6 +305,22 @@ def test_e4m3_encoder_matches_torch_and_table():
         assert code == ref, v
         assert mxformat.E4M3_TABLE[code] == v
     assert mxo.e4m3_encode(17.0) == -1 and mxo.e4m3_encode(0.3) == -1
+    # every finite e4m3 value, subnormals and -0 included, encodes to its own code
+    for code in range(256):
+        if code in (0x7F, 0xFF):  # the NaN codes
+            continue
+        v = float(mxformat.E4M3_TABLE[code])
+        if code == 0x80:
+            v = -0.0
+        assert mxo.e4m3_encode(v) == code, hex(code)
+
+
+@pytest.mark.parametrize("b", [4, 6, 8])
+def test_element_value_of_a_nan_block(b):
+    """Reading R5: a block holding Inf or NaN has scale byte 255, and every
+    element of it reads as NaN, whatever its code."""
+    for m in (-(2 ** (b - 1) - 1), -1, 0, 1, 2 ** (b - 1) - 1):
+        assert math.isnan(mxo.element_value(m, 255, b))
 
 
 @pytest.mark.parametrize("b", [6, 8])
