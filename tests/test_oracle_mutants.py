@@ -71,16 +71,24 @@ def _build(tmp_path, name, old, new):
     return str(lib)
 
 
-@pytest.mark.parametrize("name", list(MUTANTS))
-def test_pins_reject_a_planted_mistake(tmp_path, name):
-    lib = _build(tmp_path, name, *MUTANTS[name])
-    env = dict(os.environ, MXO_LIB=lib, OMP_NUM_THREADS="2")
+def _c_pins(tmp_path, name, old, new):
+    d = tmp_path / name.replace(" ", "_").replace("/", "-")
+    d.mkdir()
+    env = dict(os.environ, MXO_LIB=_build(d, name, old, new), OMP_NUM_THREADS="1")
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
                         os.path.join(ROOT, "tests", "test_oracle_pins.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
-    # 1: some pin failed (0 would mean the mistake went unseen; other codes are
-    # errors of the run itself)
-    assert r.returncode == 1, f"{name}: pins returned {r.returncode}\n{r.stdout[-2000:]}"
+    return name, r
+
+
+def test_pins_reject_every_planted_mistake(tmp_path):
+    """Each altered copy must make some pin fail (pytest's return code 1; 0
+    would mean the mistake went unseen, other codes are errors of the run)."""
+    from concurrent.futures import ThreadPoolExecutor
+    with ThreadPoolExecutor(max(1, min(8, os.cpu_count() or 1))) as ex:
+        runs = list(ex.map(lambda kv: _c_pins(tmp_path, kv[0], *kv[1]), MUTANTS.items()))
+    unseen = [f"{name}: {r.returncode}\n{r.stdout[-600:]}" for name, r in runs if r.returncode != 1]
+    assert not unseen, "\n".join(unseen)
 
 
 def test_the_unaltered_oracle_passes_the_same_run(tmp_path):
@@ -137,17 +145,25 @@ def _py_tree(tmp_path, rel, old, new):
 
 def _run_pins(tree, rel):
     from oracle import mxo
-    env = dict(os.environ, MXO_LIB=mxo.build(), OMP_NUM_THREADS="2")  # the C oracle as built
+    env = dict(os.environ, MXO_LIB=mxo.build(), OMP_NUM_THREADS="1")  # the C oracle as built
     return subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
                            str(tree / "tests" / PINS[rel])],
                           cwd=str(tree), env=env, capture_output=True, text=True, timeout=600)
 
 
-@pytest.mark.parametrize("name", list(PY_MUTANTS))
-def test_python_pins_reject_a_planted_mistake(tmp_path, name):
-    rel, old, new = PY_MUTANTS[name]
-    r = _run_pins(_py_tree(tmp_path, rel, old, new), rel)
-    assert r.returncode == 1, f"{name}: pins returned {r.returncode}\n{r.stdout[-2000:]}"
+def test_python_pins_reject_every_planted_mistake(tmp_path):
+    from concurrent.futures import ThreadPoolExecutor
+
+    def one(item):
+        name, (rel, old, new) = item
+        d = tmp_path / name.replace(" ", "_")
+        d.mkdir()
+        return name, _run_pins(_py_tree(d, rel, old, new), rel)
+
+    with ThreadPoolExecutor(max(1, min(8, os.cpu_count() or 1))) as ex:
+        runs = list(ex.map(one, PY_MUTANTS.items()))
+    unseen = [f"{name}: {r.returncode}\n{r.stdout[-600:]}" for name, r in runs if r.returncode != 1]
+    assert not unseen, "\n".join(unseen)
 
 
 @pytest.mark.parametrize("rel", list(PINS))
