@@ -57,6 +57,20 @@ MUTANTS = {
     "two-sum low part with the wrong sign": ("double lo = y - (hi - x);", "double lo = (hi - x) - y;"),
     "exact sum without the half-way fix": ("if (y == x - hi) hi = x;", "if (0) hi = x;"),
     "e4m3 subnormal scale": ("double k = ldexp(a, 9);", "double k = ldexp(a, 8);"),
+    "4-bit weight sign in bit 2": ("const uint8_t nib = (uint8_t)(((c[e] < 0) << 3) | mag);",
+                                   "const uint8_t nib = (uint8_t)(((c[e] < 0) << 2) | mag);"),
+    "4-bit weight nibbles swapped": ("*byte |= (uint8_t)(within < 4 ? nib : (nib << 4));",
+                                     "*byte |= (uint8_t)(within < 4 ? (nib << 4) : nib);"),
+    "6/8-bit weight scale on the next row": ("slot[4096 + rr] = scales[r * nb + kb];",
+                                             "slot[4096 + (rr + 1) % 128] = scales[r * nb + kb];"),
+    "4-bit plane elements reversed": ("planes[r * kp + 32 * s + i] = (uint8_t)ch;",
+                                      "planes[r * kp + 32 * s + (31 - i)] = (uint8_t)ch;"),
+    "bf16 plane low byte from the high": ("planes[r * kp + p68 + 64 * (s - n4) + 2 * i] = (uint8_t)(v & 0xFF);",
+                                          "planes[r * kp + p68 + 64 * (s - n4) + 2 * i] = (uint8_t)((v >> 8) & 0xFF);"),
+    "6/8-bit scale tile slots swapped": ("int64_t j = 2 * (st - st4) + q;", "int64_t j = 2 * (st - st4) + 1 - q;"),
+    "ties away by floor(v + 1/2)": ("? round(v) : nearbyint(v)", "? floor(v + 0.5) : nearbyint(v)"),
+    "error bound from signed terms": ("for (int64_t kb = 0; kb < nb; ++kb) terms[kb] = fabs(terms[kb]);",
+                                      "for (int64_t kb = 0; kb < nb; ++kb) terms[kb] = terms[kb];"),
 }
 
 
@@ -115,6 +129,8 @@ PY_MUTANTS = {
     "ties in reverse order": ("oracle/alloc.py", 'np.argsort(-s, kind="stable")',
                               'np.argsort(s, kind="stable")[::-1]'),
     "no 8-bit block": ("oracle/alloc.py", "bits[0] = 8", "bits[0] = 6"),
+    "bf16 decoded one bit off": ("oracle/alloc.py", "astype(np.uint32) << 16", "astype(np.uint32) << 15"),
+    "average width per block": ("oracle/alloc.py", "* BLOCK for b in bits_per_layer", "for b in bits_per_layer"),
     "one 6-bit block too many": ("oracle/alloc.py", "bits[1:1 + n6b] = 6", "bits[1:2 + n6b] = 6"),
     # oracle/attention.py (KV cache, Appendix A.2), pinned by test_oracle_attention.py
     "query head reads the wrong KV head": ("oracle/attention.py", "c = (h // G) * D", "c = (h % n_kv_heads) * D"),
