@@ -140,6 +140,9 @@ PY_MUTANTS = {
                                          "rows = slice(b * T, b * T + T)"),
     "cache values on the 8-bit grid": ("oracle/attention.py", "return mxo.dequantize(codes, scales, bits)",
                                        "return mxo.dequantize(codes, scales, np.full(len(bits), 8, np.uint8))"),
+    "scores against the value cache": ("oracle/attention.py", "s = scale * (kh @ q[h])", "s = scale * (vh @ q[h])"),
+    "sequence lengths ignored": ("oracle/attention.py", "T = int(lengths[b])", "T = T_cap"),
+    "an empty sequence not read as zeros": ("oracle/attention.py", "if T > 0:", "if T >= 0:"),
 }
 PINS = {"oracle/alloc.py": "test_oracle_alloc.py", "oracle/attention.py": "test_oracle_attention.py"}
 
